@@ -1,0 +1,204 @@
+/*
+ * wt — file-backed weights into GB300 device tensors, and the bandwidth-bound
+ * consumer pass over them.  C ABI.
+ *
+ * The problem this library solves is the one the paper calls the ingestion
+ * tax (Sec. 1; Sec. 2.2): checkpoint bytes that already sit in the page cache
+ * must become ordinary device tensors that a kernel in the caller's stream
+ * consumes.  The calls follow the paper's producer and execution contract:
+ *
+ *   wt_open   guarded open + shared read-only map of each file (Algorithm 1:
+ *             size guard, mmap(PROT_READ, MAP_SHARED), close the descriptor)
+ *             and the device-access route for the mapping (Sec. 6.2: registration
+ *             and direct read are probed separately).
+ *   wt_adopt  moves tensor bytes into caller-owned device memory and returns a
+ *             per-tensor ready event (contract C3: order on the GPU).
+ *   wt_pass   one GEMV per matrix in the caller's stream, each launch gated
+ *             by its tensors' events, outputs kept on the device (C2).
+ *   wt_checksum / wt_checksum_plain  per-tensor FNV-1a-64 digests of device
+ *             bytes (the checksums of Sec. 5.1 that confirm kernels read the
+ *             intended bytes).
+ *   wt_close  waits for the library's own work on the mappings, unregisters,
+ *             unmaps (Algorithm 1's deleter; Sec. 4.1 lifetime rules).
+ *
+ * Conventions
+ *   - Every call returns int: WT_OK (0) or a negative WT_E* code.  No C++
+ *     exception crosses this boundary.  wt_last_error() returns a thread-local
+ *     message for the last failing call on the calling thread.
+ *   - Streams and events are CUDA handles passed as void* (cudaStream_t,
+ *     cudaEvent_t); a NULL stream is the legacy default stream.
+ *   - Device pointers are caller-owned (the library never frees them).  The
+ *     library borrows a destination until the event it returned completes.
+ *   - The library never writes to a mapping.  A destination that lies inside
+ *     one of the handle's mappings is rejected with WT_EINVAL (Sec. 4.1:
+ *     read-only intent must be enforced before dispatch).
+ *   - All kernels run on the device that is current when wt_open is called.
+ */
+#ifndef WT_H_
+#define WT_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes -------------------------------------------------------- */
+#define WT_OK 0
+#define WT_EINVAL (-1)    /* bad argument (null, size, alignment, index, dtype) */
+#define WT_EIO (-2)       /* open/read/mmap failed; errno in the message */
+#define WT_EFORMAT (-3)   /* file violates the container format; file, entry, reason in the message */
+#define WT_ENOMEM (-4)    /* host or device allocation failed */
+#define WT_ECUDA (-5)     /* a CUDA runtime call failed; its error string in the message */
+#define WT_ENOTSUP (-6)   /* route or dtype not available on this device/handle */
+#define WT_ETIMEDOUT (-7) /* a bounded device wait gave up (see wt_device_status) */
+
+/* ---- element types (the container's dtype byte) -------------------------- */
+#define WT_F32 0
+#define WT_BF16 1
+#define WT_F16 2
+#define WT_I8 3
+#define WT_U8 4
+
+/* ---- wt_open flags --------------------------------------------------------
+ * Route for device reads of the mapping (one of the first four; default AUTO):
+ *   AUTO       direct read when the device reads pageable memory through the
+ *              host page tables (Grace ATS), else cudaHostRegister, else NONE.
+ *   REGISTER   cudaHostRegister(Mapped) each whole-file mapping (ReadOnly is
+ *              tried first and dropped if the driver rejects it).
+ *   DIRECT     device reads the pageable mapping in place (no registration).
+ *   NONE       the device never touches the mapping; only WT_ADOPT_STAGED works.
+ * HOST_ONLY    parse and map only; no CUDA call at all (index inspection).
+ * PREFAULT     populate every mapping's page-table entries at open
+ *              (MADV_POPULATE_READ); otherwise wt_adopt populates each batch's
+ *              source range just before it enqueues that batch.
+ */
+#define WT_ROUTE_AUTO 0u
+#define WT_ROUTE_REGISTER 1u
+#define WT_ROUTE_DIRECT 2u
+#define WT_ROUTE_NONE 3u
+#define WT_ROUTE_MASK 3u
+#define WT_OPEN_HOST_ONLY (1u << 4)
+#define WT_OPEN_PREFAULT (1u << 5)
+
+/* ---- wt_adopt modes ---------------------------------------------------------
+ *   GATHER   SM gather kernel: 16-byte vector loads from the device-readable
+ *            mapping, coalesced stores to HBM (the default).
+ *   CE       copy engine: cudaMemcpyAsync from the device-readable mapping.
+ *   STAGED   host threads copy page-cache bytes into a pinned ring, the copy
+ *            engine moves each slot (the paper's staged/overlapped copy arm,
+ *            Table "tab:tax" and Table "tab:gh-endpoints").
+ */
+#define WT_ADOPT_GATHER 0u
+#define WT_ADOPT_CE 1u
+#define WT_ADOPT_STAGED 2u
+
+typedef struct wt_handle wt_handle;
+
+typedef struct {
+  const char *name;     /* NUL-terminated, valid until wt_close */
+  int32_t dtype;        /* WT_F32 ... WT_U8 */
+  int32_t ndim;         /* 1..4 */
+  uint64_t shape[4];    /* unused dims are 0 */
+  uint64_t nbytes;      /* prod(shape) * sizeof(dtype) */
+  uint32_t file;        /* index into the wt_open path list */
+  uint64_t offset;      /* absolute file offset, multiple of 64 */
+  const void *host_ptr; /* address of the blob in the read-only mapping */
+} wt_tensor_meta;
+
+/* One GEMV of wt_pass: y[M] = W[M,K] . x[K], fp32 accumulate (Sec. 3.1 protocol:
+ * one single-token GEMV per matrix).  W is row-major [out, in]; x has W's dtype;
+ * y is fp32.  All pointers are caller-owned device memory.  wait_event (a
+ * cudaEvent_t from wt_adopt, or NULL) gates this GEMV on the GPU. */
+typedef struct {
+  const void *W;
+  int32_t dtype;        /* WT_F32, WT_BF16 or WT_F16 */
+  int32_t reserved;     /* must be 0 */
+  uint64_t M;
+  uint64_t K;
+  const void *x;
+  float *y;
+  void *wait_event;
+} wt_gemv_desc;
+
+/* Thread-local message describing the last failure on this thread ("" if none). */
+const char *wt_last_error(void);
+
+/* ABI version of this header (increments on any incompatible change). */
+int wt_abi_version(void);
+
+/* Open n_paths checkpoint files (n_paths may be 0: a context for wt_pass and
+ * wt_checksum only).  Per file: open(O_RDONLY), fstat, pread the header and the
+ * length-prefixed index, validate every entry (dtype, ndim 1..4, nbytes ==
+ * prod(shape)*sizeof(dtype) without overflow, offset % 64 == 0, blob after the
+ * index, inside the file, in index order, no overlap, unique non-empty names,
+ * index length exactly consumed), mmap(PROT_READ, MAP_SHARED), close the fd,
+ * then set up the route.  On any failure nothing stays open or mapped and
+ * *out is NULL.  Errors: WT_EINVAL, WT_EIO, WT_EFORMAT, WT_ENOMEM, WT_ECUDA,
+ * WT_ENOTSUP (route requested but unavailable). */
+int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **out);
+
+int wt_num_tensors(const wt_handle *h, size_t *n);
+int wt_num_files(const wt_handle *h, size_t *n);
+/* Tensor i in (file, index) order. */
+int wt_tensor_info(const wt_handle *h, size_t i, wt_tensor_meta *out);
+/* First tensor whose name equals `name`; WT_EINVAL if none. */
+int wt_find(const wt_handle *h, const char *name, size_t *i);
+/* Route actually taken for file f (WT_ROUTE_REGISTER / DIRECT / NONE). */
+int wt_file_route(const wt_handle *h, size_t f, unsigned *route);
+
+/* Copy tensors idx[0..n) into device memory dst[0..n) (each at least nbytes of
+ * that tensor, 16-byte aligned for the vector path) on `stream`, in order.
+ * Tensors are grouped into batches of a few MB to a few hundred MB; one event
+ * is recorded after each batch and ready[i] receives the event of tensor i's
+ * batch (several entries may hold the same event).  Events are owned by the
+ * handle and destroyed by wt_close.  Because the batches run in order on one
+ * stream, ready[i] also implies every earlier tensor of this call.  STAGED
+ * mode blocks the calling thread until every byte has left the page cache
+ * (the copy engine may still be draining the last slots).
+ * Errors: WT_EINVAL (index, null, overlap with a mapping), WT_ENOTSUP (mode
+ * needs a device route the file lacks), WT_ENOMEM, WT_ECUDA. */
+int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsigned mode,
+             void *stream, void **ready);
+
+/* Enqueue one GEMV per descriptor on `stream`.  Consecutive descriptors that
+ * carry the same wait_event form one group: the stream waits on that event
+ * (cudaStreamWaitEvent, never a host wait) and one persistent launch streams
+ * every matrix of the group, rows split evenly across the SMs.  Repeated
+ * calls with identical descriptors reuse a cached launch plan.  The result of
+ * a row does not depend on how rows were grouped or split (deterministic, no
+ * floating-point atomics).  Errors: WT_EINVAL (null pointer with M*K > 0,
+ * reserved != 0, dimension > 2^31-1), WT_ENOTSUP (dtype), WT_ENOMEM, WT_ECUDA. */
+int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream);
+
+/* Leaf-tree FNV-1a-64 digest of each device buffer ptr[i] (nbytes[i] bytes),
+ * written to out_dev[i] (device memory, caller-owned).  D_tree = FNV-1a-64 over
+ * the 8-byte little-endian encodings of [nbytes, leaf_0, ..., leaf_{L-1}],
+ * leaf_k = FNV-1a-64 of bytes [4096k, min(4096(k+1), nbytes)).  Temporary leaf
+ * storage is stream-ordered (cudaMallocAsync/cudaFreeAsync on `stream`). */
+int wt_checksum(wt_handle *h, const void *const *ptr, const uint64_t *nbytes, size_t n,
+                uint64_t *out_dev, void *stream);
+
+/* Literal FNV-1a-64 of each device buffer (one serial chain per buffer; meant
+ * for verification).  Buffers above 256 MiB are rejected with WT_EINVAL. */
+int wt_checksum_plain(wt_handle *h, const void *const *ptr, const uint64_t *nbytes, size_t n,
+                      uint64_t *out_dev, void *stream);
+
+/* Device-side status word of the handle: 0, or the first WT_ETIMEDOUT-class
+ * code a bounded wait inside a kernel recorded (reads it synchronously). */
+int wt_device_status(wt_handle *h, int *status);
+
+/* Kernels this handle has launched so far (gather, GEMV, checksum launches). */
+int wt_kernel_launches(const wt_handle *h, uint64_t *n);
+
+/* Wait for the library's own enqueued work that reads the mappings, then
+ * cudaHostUnregister, munmap, destroy events, free library allocations.
+ * NULL is a no-op.  Callable from any thread. */
+int wt_close(wt_handle *h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* WT_H_ */

@@ -1,0 +1,1038 @@
+// Host side of the wt library: the C ABI of include/wt.h.
+//
+//   open     parallel per-file open / fstat / pread index / validate / mmap
+//            (Algorithm 1's guarded shared read-only map), then the device
+//            route for each mapping (Sec. 6.2: registration and direct read are
+//            probed separately; GB300 reads pageable memory through the host
+//            page tables, so a registration is optional there)
+//   adopt    batches tensors into launches of the gather kernel (or copy-engine
+//            copies, or the staged pinned ring) and records one event per
+//            batch: contract C3 (order on the GPU), Table "tab:contract"
+//   pass     plans one persistent GEMV launch per group of descriptors sharing
+//            a wait event; plans are cached and uploaded stream-ordered
+//   close    waits on the handle's own events, unregisters, unmaps
+#include <fcntl.h>
+#include <sys/mman.h>
+#include <sys/stat.h>
+#include <unistd.h>
+
+#include <algorithm>
+#include <atomic>
+#include <cerrno>
+#include <condition_variable>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <functional>
+#include <list>
+#include <mutex>
+#include <new>
+#include <string>
+#include <thread>
+#include <unordered_set>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "../../include/wt.h"
+#include "wt_kernels.h"
+
+#ifndef MADV_POPULATE_READ
+#define MADV_POPULATE_READ 22
+#endif
+
+namespace {
+
+thread_local std::string t_err;
+
+int set_err(int code, const char *fmt, ...) {
+  char buf[1024];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  t_err = buf;
+  return code;
+}
+
+int cuda_err(cudaError_t e, const char *what) {
+  cudaGetLastError();  // clear the sticky-free error so later calls start clean
+  return set_err(WT_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define CU(call)                                        \
+  do {                                                  \
+    cudaError_t e_ = (call);                            \
+    if (e_ != cudaSuccess) return cuda_err(e_, #call);  \
+  } while (0)
+
+constexpr uint64_t kAlign = 64;
+constexpr int kMaxDims = 4;
+
+int elem_bytes(int dtype) {
+  switch (dtype) {
+    case WT_F32: return 4;
+    case WT_BF16: case WT_F16: return 2;
+    case WT_I8: case WT_U8: return 1;
+    default: return 0;
+  }
+}
+
+// ------------------------------------------------------------------ small thread pool
+class Pool {
+ public:
+  explicit Pool(int n) {
+    for (int i = 0; i < n; ++i) th_.emplace_back([this] { run(); });
+  }
+  ~Pool() {
+    {
+      std::lock_guard<std::mutex> g(m_);
+      stop_ = true;
+    }
+    cv_.notify_all();
+    for (auto &t : th_) t.join();
+  }
+  int size() const { return (int)th_.size(); }
+  // Runs fn(i) for i in [0, n) on the pool and the calling thread; returns when all are done.
+  void parallel_for(size_t n, const std::function<void(size_t)> &fn) {
+    if (n == 0) return;
+    std::lock_guard<std::mutex> one_at_a_time(call_mu_);
+    if (th_.empty() || n == 1) {
+      for (size_t i = 0; i < n; ++i) fn(i);
+      return;
+    }
+    std::atomic<size_t> next{0};
+    std::atomic<size_t> done{0};
+    auto body = [&] {
+      size_t i;
+      while ((i = next.fetch_add(1)) < n) {
+        fn(i);
+        done.fetch_add(1);
+      }
+    };
+    {
+      std::lock_guard<std::mutex> g(m_);
+      job_ = body;
+      gen_++;
+    }
+    cv_.notify_all();
+    body();
+    std::unique_lock<std::mutex> lk(m_);
+    done_cv_.wait(lk, [&] { return done.load() == n && active_ == 0; });
+    job_ = nullptr;
+  }
+
+ private:
+  void run() {
+    uint64_t seen = 0;
+    for (;;) {
+      std::function<void()> job;
+      {
+        std::unique_lock<std::mutex> lk(m_);
+        cv_.wait(lk, [&] { return stop_ || (gen_ != seen && job_); });
+        if (stop_) return;
+        seen = gen_;
+        job = job_;
+        active_++;
+      }
+      job();
+      {
+        std::lock_guard<std::mutex> g(m_);
+        active_--;
+      }
+      done_cv_.notify_all();
+    }
+  }
+  std::vector<std::thread> th_;
+  std::mutex call_mu_;
+  std::mutex m_;
+  std::condition_variable cv_, done_cv_;
+  std::function<void()> job_;
+  uint64_t gen_ = 0;
+  int active_ = 0;
+  bool stop_ = false;
+};
+
+Pool &host_pool() {
+  static Pool p([] {
+    unsigned n = std::thread::hardware_concurrency();
+    return (int)std::min(15u, n > 1 ? n - 1 : 0u);
+  }());
+  return p;
+}
+
+// ------------------------------------------------------------------ handle
+struct Tensor {
+  std::string name;
+  int dtype = 0;
+  int ndim = 0;
+  uint64_t shape[kMaxDims] = {0, 0, 0, 0};
+  uint64_t nbytes = 0;
+  uint32_t file = 0;
+  uint64_t offset = 0;
+};
+
+struct File {
+  std::string path;
+  uint8_t *base = nullptr;  // mapping
+  size_t size = 0;
+  unsigned route = WT_ROUTE_NONE;
+  bool registered = false;
+  const uint8_t *dev = nullptr;  // device-readable address of base
+  std::vector<Tensor> tensors;
+};
+
+struct Plan {
+  std::vector<uint8_t> key;
+  struct Launch {
+    int dtype;
+    int grid;
+    size_t mats, pieces, begin;  // byte offsets in the table
+  };
+  struct Generic {
+    int dtype;
+    const uint8_t *W, *x;
+    float *y;
+    uint64_t M, K;
+  };
+  struct Zero {
+    float *y;
+    uint64_t M;
+  };
+  struct Group {
+    cudaEvent_t wait = nullptr;
+    std::vector<Launch> launches;
+    std::vector<Generic> generic;
+    std::vector<Zero> zero;
+  };
+  std::vector<Group> groups;
+  std::vector<uint8_t> table;
+  uint8_t *host = nullptr;  // pinned copy of table
+  uint8_t *dev = nullptr;
+  cudaEvent_t uploaded = nullptr;
+  cudaEvent_t last = nullptr;
+  bool sent = false;
+  cudaStream_t sent_on = nullptr;
+  uint64_t launches = 0;
+};
+
+struct Ring {
+  static constexpr int kSlots = 4;
+  static constexpr size_t kSlotBytes = 64ull << 20;
+  uint8_t *slot[kSlots] = {nullptr, nullptr, nullptr, nullptr};
+  cudaEvent_t done[kSlots] = {nullptr, nullptr, nullptr, nullptr};
+  bool used[kSlots] = {false, false, false, false};
+};
+
+}  // namespace
+
+struct wt_handle {
+  std::vector<File> files;
+  std::vector<std::pair<uint32_t, uint32_t>> order;  // global tensor index -> (file, entry)
+  bool host_only = false;
+  bool prefaulted = false;
+  int device = -1;
+  int *status = nullptr;
+  std::vector<cudaEvent_t> events;
+  std::list<Plan *> plans;
+  Ring ring;
+  bool ring_ready = false;
+  uint64_t kernel_launches = 0;
+  std::mutex mu;
+
+  const Tensor &tensor(size_t i) const {
+    return files[order[i].first].tensors[order[i].second];
+  }
+};
+
+namespace {
+
+// ------------------------------------------------------------------ index parser
+struct Reader {
+  const uint8_t *p;
+  size_t n, pos = 0;
+  bool need(size_t k) const { return pos <= n && k <= n - pos; }
+  uint64_t le(int k) {
+    uint64_t v = 0;
+    for (int i = 0; i < k; ++i) v |= (uint64_t)p[pos + i] << (8 * i);
+    pos += k;
+    return v;
+  }
+};
+
+int parse_file(File &f, int fd, uint64_t fsize) {
+  const char *path = f.path.c_str();
+  if (fsize < 16) return set_err(WT_EFORMAT, "%s: shorter than the 16-byte header", path);
+  uint8_t hdr[16];
+  if (pread(fd, hdr, 16, 0) != 16) return set_err(WT_EIO, "%s: pread header: %s", path, strerror(errno));
+  if (memcmp(hdr, "WTCKPT01", 8) != 0) return set_err(WT_EFORMAT, "%s: bad magic", path);
+  Reader h{hdr, 16, 8};
+  const uint64_t ilen = h.le(8);
+  if (ilen < 4 || ilen > fsize - 16) return set_err(WT_EFORMAT, "%s: index length outside the file", path);
+  std::vector<uint8_t> ix(ilen);
+  if ((uint64_t)pread(fd, ix.data(), ilen, 16) != ilen)
+    return set_err(WT_EIO, "%s: pread index: %s", path, strerror(errno));
+  Reader r{ix.data(), ix.size()};
+  const uint64_t count = r.le(4);
+  constexpr uint64_t kMinEntry = 2 + 1 + 1 + 1 + 8 + 8 + 8;
+  if (count > (ilen - 4) / kMinEntry) return set_err(WT_EFORMAT, "%s: entry count exceeds the index", path);
+  f.tensors.resize(count);
+  const uint64_t first_blob = 16 + ilen;
+  uint64_t end_prev = first_blob;
+  std::unordered_set<std::string> names;
+  for (uint64_t i = 0; i < count; ++i) {
+    Tensor &t = f.tensors[i];
+    if (!r.need(2)) return set_err(WT_EFORMAT, "%s: entry %llu: index ends inside the name length", path, (unsigned long long)i);
+    const uint64_t nl = r.le(2);
+    if (nl == 0) return set_err(WT_EFORMAT, "%s: entry %llu: empty name", path, (unsigned long long)i);
+    if (!r.need(nl + 2)) return set_err(WT_EFORMAT, "%s: entry %llu: index ends inside the name", path, (unsigned long long)i);
+    t.name.assign(reinterpret_cast<const char *>(r.p + r.pos), nl);
+    r.pos += nl;
+    if (t.name.find('\0') != std::string::npos)
+      return set_err(WT_EFORMAT, "%s: entry %llu: NUL byte in name", path, (unsigned long long)i);
+    t.dtype = (int)r.le(1);
+    t.ndim = (int)r.le(1);
+    const int es = elem_bytes(t.dtype);
+    if (es == 0) return set_err(WT_EFORMAT, "%s: entry %llu: unknown dtype %d", path, (unsigned long long)i, t.dtype);
+    if (t.ndim < 1 || t.ndim > kMaxDims)
+      return set_err(WT_EFORMAT, "%s: entry %llu: ndim %d outside 1..4", path, (unsigned long long)i, t.ndim);
+    if (!r.need(8ull * t.ndim + 16)) return set_err(WT_EFORMAT, "%s: entry %llu: index ends inside the shape", path, (unsigned long long)i);
+    unsigned __int128 elems = 1;
+    for (int d = 0; d < t.ndim; ++d) {
+      t.shape[d] = r.le(8);
+      elems *= t.shape[d];
+      if (elems > ((unsigned __int128)1 << 64)) elems = ((unsigned __int128)1 << 64) + 1;  // saturate
+    }
+    const unsigned __int128 bytes = elems * (unsigned)es;
+    t.offset = r.le(8);
+    t.nbytes = r.le(8);
+    if (bytes > UINT64_MAX) return set_err(WT_EFORMAT, "%s: entry %llu: shape product overflows", path, (unsigned long long)i);
+    if ((unsigned __int128)t.nbytes != bytes)
+      return set_err(WT_EFORMAT, "%s: entry %llu: nbytes %llu != prod(shape) * %d", path, (unsigned long long)i,
+                     (unsigned long long)t.nbytes, es);
+    if (t.offset % kAlign) return set_err(WT_EFORMAT, "%s: entry %llu: offset %llu not 64-byte aligned", path, (unsigned long long)i, (unsigned long long)t.offset);
+    if (t.offset < first_blob) return set_err(WT_EFORMAT, "%s: entry %llu: blob overlaps the header/index", path, (unsigned long long)i);
+    if (t.offset > fsize || t.nbytes > fsize - t.offset)
+      return set_err(WT_EFORMAT, "%s: entry %llu: blob runs past the end of the file", path, (unsigned long long)i);
+    if (t.offset < end_prev) return set_err(WT_EFORMAT, "%s: entry %llu: blob overlaps the previous blob", path, (unsigned long long)i);
+    end_prev = t.offset + t.nbytes;
+    if (!names.insert(t.name).second) return set_err(WT_EFORMAT, "%s: entry %llu: duplicate name '%s'", path, (unsigned long long)i, t.name.c_str());
+  }
+  if (r.pos != ilen) return set_err(WT_EFORMAT, "%s: index length does not match its entries", path);
+  return WT_OK;
+}
+
+void unmap_file(File &f) {
+  if (f.registered) {
+    cudaHostUnregister(f.base);
+    f.registered = false;
+  }
+  if (f.base) {
+    munmap(f.base, f.size);
+    f.base = nullptr;
+  }
+}
+
+// open, parse and map one file; closes the fd on every path.
+int open_one(File &f) {
+  const int fd = open(f.path.c_str(), O_RDONLY | O_CLOEXEC);
+  if (fd < 0) return set_err(WT_EIO, "%s: open: %s", f.path.c_str(), strerror(errno));
+  struct stat st;
+  if (fstat(fd, &st) != 0) {
+    int e = errno;
+    close(fd);
+    return set_err(WT_EIO, "%s: fstat: %s", f.path.c_str(), strerror(e));
+  }
+  int rc = parse_file(f, fd, (uint64_t)st.st_size);
+  if (rc == WT_OK) {
+    f.size = (size_t)st.st_size;
+    void *p = mmap(nullptr, f.size, PROT_READ, MAP_SHARED, fd, 0);
+    if (p == MAP_FAILED) rc = set_err(WT_EIO, "%s: mmap: %s", f.path.c_str(), strerror(errno));
+    else f.base = static_cast<uint8_t *>(p);
+  }
+  close(fd);  // Algorithm 1: the mapping outlives the descriptor
+  return rc;
+}
+
+void prefault(const uint8_t *p, size_t n) {
+  if (n == 0) return;
+  const uintptr_t pg = (uintptr_t)sysconf(_SC_PAGESIZE);
+  const uintptr_t a = reinterpret_cast<uintptr_t>(p) & ~(pg - 1);
+  const uintptr_t b = (reinterpret_cast<uintptr_t>(p) + n + pg - 1) & ~(pg - 1);
+  if (madvise(reinterpret_cast<void *>(a), b - a, MADV_POPULATE_READ) != 0) {
+    // older kernels: touch one byte per page
+    volatile uint8_t sink = 0;
+    for (uintptr_t q = a; q < b; q += pg) sink ^= *reinterpret_cast<const volatile uint8_t *>(q);
+    (void)sink;
+  }
+}
+
+std::vector<bool> g_prepared(64, false);
+std::mutex g_prep_mu;
+
+int prepare_device(int dev) {
+  std::lock_guard<std::mutex> g(g_prep_mu);
+  if (dev < 0 || dev >= 64) return set_err(WT_ECUDA, "device index %d out of range", dev);
+  if (!g_prepared[dev]) {
+    CU(wt::gemv_prepare());
+    g_prepared[dev] = true;
+  }
+  return WT_OK;
+}
+
+bool inside_mapping(const wt_handle *h, const void *p, uint64_t n) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(p), b = a + n;
+  for (const File &f : h->files) {
+    const uintptr_t s = reinterpret_cast<uintptr_t>(f.base), e = s + f.size;
+    if (a < e && b > s) return true;
+  }
+  return false;
+}
+
+int new_event(wt_handle *h, cudaEvent_t *ev) {
+  CU(cudaEventCreateWithFlags(ev, cudaEventDisableTiming));
+  h->events.push_back(*ev);
+  return WT_OK;
+}
+
+// ------------------------------------------------------------------ adopt
+struct Range {
+  size_t tensor;  // position in the caller's list
+  const uint8_t *src_host;
+  const uint8_t *src_dev;
+  uint8_t *dst;
+  uint64_t n;
+};
+
+int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cudaStream_t s,
+                 void **ready, uint64_t total) {
+  const uint64_t target = std::min<uint64_t>(128ull << 20, std::max<uint64_t>(2ull << 20, total / 64));
+  const int grid_cap = 2 * wt::num_sms();
+  size_t i = 0;
+  while (i < rs.size()) {
+    size_t j = i;
+    uint64_t bytes = 0;
+    while (j < rs.size() && (j == i || (bytes < target && j - i < (size_t)wt::kMaxGather))) bytes += rs[j++].n;
+    // populate page-table entries of this batch's sources right before it is enqueued
+    if (!h->prefaulted)
+      for (size_t k = i; k < j; ++k) prefault(rs[k].src_host, rs[k].n);
+    if (mode == WT_ADOPT_GATHER) {
+      wt::GatherBatch b;
+      memset(&b, 0, sizeof b);
+      uint64_t chunks = 0;
+      for (size_t k = i; k < j; ++k) {
+        const uint32_t q = b.n++;
+        b.chunk_prefix[q] = chunks;
+        b.src[q] = rs[k].src_dev;
+        b.dst[q] = rs[k].dst;
+        b.nbytes[q] = rs[k].n;
+        chunks += (rs[k].n + (1ull << wt::kGatherChunkLog2) - 1) >> wt::kGatherChunkLog2;
+      }
+      b.chunk_prefix[b.n] = chunks;
+      if (chunks) {
+        CU(wt::launch_gather(b, (int)std::min<uint64_t>(chunks, (uint64_t)grid_cap), s));
+        h->kernel_launches++;
+      }
+    } else {
+      for (size_t k = i; k < j; ++k)
+        if (rs[k].n) CU(cudaMemcpyAsync(rs[k].dst, rs[k].src_dev, rs[k].n, cudaMemcpyDefault, s));
+    }
+    cudaEvent_t ev;
+    int rc = new_event(h, &ev);
+    if (rc) return rc;
+    CU(cudaEventRecord(ev, s));
+    for (size_t k = i; k < j; ++k) ready[rs[k].tensor] = ev;
+    i = j;
+  }
+  return WT_OK;
+}
+
+int ring_setup(wt_handle *h) {
+  if (h->ring_ready) return WT_OK;
+  for (int k = 0; k < Ring::kSlots; ++k) {
+    CU(cudaHostAlloc(reinterpret_cast<void **>(&h->ring.slot[k]), Ring::kSlotBytes, cudaHostAllocDefault));
+    CU(cudaEventCreateWithFlags(&h->ring.done[k], cudaEventDisableTiming));
+  }
+  h->ring_ready = true;
+  return WT_OK;
+}
+
+// Staged: page cache -> pinned slot (host threads) -> HBM (copy engine).
+int adopt_staged(wt_handle *h, const std::vector<Range> &rs, cudaStream_t s, void **ready) {
+  int rc = ring_setup(h);
+  if (rc) return rc;
+  struct PieceCopy {
+    const uint8_t *src;
+    size_t off;  // in slot
+    uint8_t *dst;
+    size_t n;
+  };
+  int slot = 0;
+  size_t r = 0;
+  uint64_t roff = 0;
+  Pool &pool = host_pool();
+  while (r < rs.size()) {
+    if (h->ring.used[slot]) CU(cudaEventSynchronize(h->ring.done[slot]));
+    uint8_t *buf = h->ring.slot[slot];
+    std::vector<PieceCopy> pcs;
+    std::vector<size_t> finished;  // tensors whose last byte is in this slot
+    size_t fill = 0;
+    while (r < rs.size() && fill < Ring::kSlotBytes) {
+      const uint64_t take = std::min<uint64_t>(rs[r].n - roff, Ring::kSlotBytes - fill);
+      if (take) pcs.push_back({rs[r].src_host + roff, fill, rs[r].dst + roff, (size_t)take});
+      fill += take;
+      roff += take;
+      if (roff == rs[r].n) {
+        finished.push_back(rs[r].tensor);
+        ++r;
+        roff = 0;
+      }
+    }
+    // host copy in 4 MiB pieces across the pool
+    std::vector<std::pair<size_t, size_t>> work;  // (piece, sub-offset)
+    constexpr size_t kSub = 4u << 20;
+    for (size_t p = 0; p < pcs.size(); ++p)
+      for (size_t o = 0; o < pcs[p].n; o += kSub) work.push_back({p, o});
+    pool.parallel_for(work.size(), [&](size_t w) {
+      const PieceCopy &pc = pcs[work[w].first];
+      const size_t o = work[w].second;
+      memcpy(buf + pc.off + o, pc.src + o, std::min(kSub, pc.n - o));
+    });
+    for (const PieceCopy &pc : pcs) CU(cudaMemcpyAsync(pc.dst, buf + pc.off, pc.n, cudaMemcpyHostToDevice, s));
+    CU(cudaEventRecord(h->ring.done[slot], s));
+    h->ring.used[slot] = true;
+    if (!finished.empty()) {
+      cudaEvent_t ev;
+      rc = new_event(h, &ev);
+      if (rc) return rc;
+      CU(cudaEventRecord(ev, s));
+      for (size_t t : finished) ready[t] = ev;
+    }
+    slot = (slot + 1) % Ring::kSlots;
+  }
+  return WT_OK;
+}
+
+// ------------------------------------------------------------------ GEMV planning
+uint32_t pow2ceil(uint32_t v) {
+  uint32_t p = 1;
+  while (p < v) p <<= 1;
+  return p;
+}
+
+wt::MatDesc make_mat(const wt_gemv_desc &d) {
+  wt::MatDesc m;
+  memset(&m, 0, sizeof m);
+  const int es = elem_bytes(d.dtype);
+  m.W = static_cast<const uint8_t *>(d.W);
+  m.x = static_cast<const uint8_t *>(d.x);
+  m.y = d.y;
+  m.M = (uint32_t)d.M;
+  m.V = (uint32_t)(d.K * es / 16);
+  const uint32_t rowb = m.V * 16;
+  if (m.V <= 256) {
+    m.mode = wt::kModeWarpRows;
+    m.G = (uint16_t)(m.V <= 32 ? pow2ceil(m.V) : 32);
+    m.rt = wt::kStageBytes / rowb;
+    m.vc = m.V;
+  } else if (rowb <= (uint32_t)wt::kStageBytes) {
+    m.mode = wt::kModeBlockRows;
+    m.rt = std::min<uint32_t>(wt::kRowBlock, wt::kStageBytes / rowb);
+    m.vc = m.V;
+  } else {
+    m.mode = wt::kModeSplitK;
+    m.rt = wt::kRowBlock;
+    m.vc = wt::kStageBytes / (wt::kRowBlock * 16);
+  }
+  return m;
+}
+
+// Split the rows of `mats` (in order) into `grid` contiguous ranges of nearly equal bytes.
+void partition(const std::vector<wt::MatDesc> &mats, int &grid, std::vector<wt::Piece> &pieces,
+               std::vector<uint32_t> &begin) {
+  uint64_t B = 0;
+  std::vector<uint64_t> start(mats.size() + 1, 0);
+  for (size_t i = 0; i < mats.size(); ++i) {
+    start[i] = B;
+    B += (uint64_t)mats[i].M * mats[i].V * 16;
+  }
+  start[mats.size()] = B;
+  constexpr uint64_t kMinCtaBytes = 64 << 10;
+  grid = (int)std::max<uint64_t>(1, std::min<uint64_t>((uint64_t)wt::num_sms(), (B + kMinCtaBytes - 1) / kMinCtaBytes));
+  // cut c (1..grid-1) at the row boundary nearest byte B*c/grid
+  std::vector<std::pair<uint32_t, uint32_t>> cuts;  // (mat, row)
+  cuts.push_back({0, 0});
+  size_t m = 0;
+  for (int c = 1; c < grid; ++c) {
+    const uint64_t T = (uint64_t)((unsigned __int128)B * c / grid);
+    while (m + 1 < mats.size() && start[m + 1] <= T) ++m;
+    const uint64_t rb = (uint64_t)mats[m].V * 16;
+    uint64_t row = (T - start[m] + rb / 2) / rb;
+    std::pair<uint32_t, uint32_t> cut = {(uint32_t)m, (uint32_t)std::min<uint64_t>(row, mats[m].M)};
+    if (cut.second == mats[m].M && m + 1 < mats.size()) cut = {(uint32_t)m + 1, 0};
+    if (cut < cuts.back()) cut = cuts.back();
+    cuts.push_back(cut);
+  }
+  cuts.push_back({(uint32_t)mats.size(), 0});
+  begin.assign(1, 0);
+  for (int c = 0; c < grid; ++c) {
+    auto a = cuts[c], b = cuts[c + 1];
+    while (a < b) {
+      const uint32_t rend = a.first == b.first ? b.second : mats[a.first].M;
+      if (rend > a.second) pieces.push_back({a.first, a.second, rend, 0});
+      if (a.first == b.first) break;
+      a = {a.first + 1, 0};
+    }
+    begin.push_back((uint32_t)pieces.size());
+  }
+}
+
+size_t align16(size_t v) { return (v + 15) & ~(size_t)15; }
+
+template <class T>
+size_t append(std::vector<uint8_t> &tab, const std::vector<T> &v) {
+  const size_t off = align16(tab.size());
+  tab.resize(off + v.size() * sizeof(T));
+  if (!v.empty()) memcpy(tab.data() + off, v.data(), v.size() * sizeof(T));
+  return off;
+}
+
+int validate_desc(const wt_gemv_desc &d, size_t i) {
+  if (d.dtype != WT_F32 && d.dtype != WT_BF16 && d.dtype != WT_F16)
+    return set_err(d.dtype == WT_I8 || d.dtype == WT_U8 ? WT_ENOTSUP : WT_EINVAL, "desc %zu: dtype %d has no GEMV", i, d.dtype);
+  if (d.reserved != 0) return set_err(WT_EINVAL, "desc %zu: reserved field must be 0", i);
+  if (d.M > 0x7fffffffull || d.K > 0x7fffffffull) return set_err(WT_EINVAL, "desc %zu: M or K above 2^31-1", i);
+  if (d.M > 0 && d.y == nullptr) return set_err(WT_EINVAL, "desc %zu: null y", i);
+  if (d.M > 0 && d.K > 0 && (d.W == nullptr || d.x == nullptr)) return set_err(WT_EINVAL, "desc %zu: null W or x", i);
+  return WT_OK;
+}
+
+int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
+  size_t i = 0;
+  while (i < n) {
+    size_t j = i;
+    while (j < n && d[j].wait_event == d[i].wait_event) ++j;
+    Plan::Group g;
+    g.wait = static_cast<cudaEvent_t>(d[i].wait_event);
+    std::vector<wt::MatDesc> by_dt[3];
+    for (size_t k = i; k < j; ++k) {
+      const wt_gemv_desc &q = d[k];
+      if (q.M == 0) continue;
+      const int es = elem_bytes(q.dtype);
+      if (q.K == 0) {
+        g.zero.push_back({q.y, q.M});
+        continue;
+      }
+      const bool fast = ((reinterpret_cast<uintptr_t>(q.W) | reinterpret_cast<uintptr_t>(q.x)) & 15) == 0 &&
+                        (q.K * es) % 16 == 0;
+      if (fast) by_dt[q.dtype].push_back(make_mat(q));
+      else g.generic.push_back({q.dtype, static_cast<const uint8_t *>(q.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K});
+    }
+    for (int dt = 0; dt < 3; ++dt) {
+      if (by_dt[dt].empty()) continue;
+      Plan::Launch L;
+      L.dtype = dt;
+      std::vector<wt::Piece> pieces;
+      std::vector<uint32_t> begin;
+      partition(by_dt[dt], L.grid, pieces, begin);
+      L.mats = append(P->table, by_dt[dt]);
+      L.pieces = append(P->table, pieces);
+      L.begin = append(P->table, begin);
+      g.launches.push_back(L);
+    }
+    P->groups.push_back(std::move(g));
+    i = j;
+  }
+  const size_t bytes = std::max<size_t>(16, align16(P->table.size()));
+  CU(cudaHostAlloc(reinterpret_cast<void **>(&P->host), bytes, cudaHostAllocDefault));
+  memcpy(P->host, P->table.data(), P->table.size());
+  CU(cudaMalloc(reinterpret_cast<void **>(&P->dev), bytes));
+  CU(cudaEventCreateWithFlags(&P->uploaded, cudaEventDisableTiming));
+  CU(cudaEventCreateWithFlags(&P->last, cudaEventDisableTiming));
+  (void)h;
+  return WT_OK;
+}
+
+void destroy_plan(Plan *P) {
+  if (P->last) cudaEventSynchronize(P->last);
+  if (P->dev) cudaFree(P->dev);
+  if (P->host) cudaFreeHost(P->host);
+  if (P->uploaded) cudaEventDestroy(P->uploaded);
+  if (P->last) cudaEventDestroy(P->last);
+  delete P;
+}
+
+int run_plan(wt_handle *h, Plan *P, cudaStream_t s) {
+  if (!P->sent) {
+    CU(cudaMemcpyAsync(P->dev, P->host, std::max<size_t>(16, align16(P->table.size())), cudaMemcpyHostToDevice, s));
+    CU(cudaEventRecord(P->uploaded, s));
+    P->sent = true;
+    P->sent_on = s;
+  } else if (s != P->sent_on) {
+    CU(cudaStreamWaitEvent(s, P->uploaded, 0));
+  }
+  for (const Plan::Group &g : P->groups) {
+    if (g.wait) CU(cudaStreamWaitEvent(s, g.wait, 0));
+    for (const Plan::Zero &z : g.zero) CU(cudaMemsetAsync(z.y, 0, z.M * sizeof(float), s));
+    for (const Plan::Launch &L : g.launches) {
+      wt::GemvLaunch gl;
+      gl.dtype = L.dtype;
+      gl.grid = L.grid;
+      gl.mats = reinterpret_cast<const wt::MatDesc *>(P->dev + L.mats);
+      gl.pieces = reinterpret_cast<const wt::Piece *>(P->dev + L.pieces);
+      gl.begin = reinterpret_cast<const uint32_t *>(P->dev + L.begin);
+      gl.status = h->status;
+      CU(wt::launch_gemv(gl, s));
+      h->kernel_launches++;
+    }
+    for (const Plan::Generic &q : g.generic) {
+      CU(wt::launch_gemv_generic(q.dtype, q.W, q.x, q.y, q.M, q.K, s));
+      h->kernel_launches++;
+    }
+  }
+  CU(cudaEventRecord(P->last, s));
+  return WT_OK;
+}
+
+int close_impl(wt_handle *h) {
+  int rc = WT_OK;
+  if (!h->host_only && h->device >= 0) {
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != h->device) cudaSetDevice(h->device);
+    for (cudaEvent_t e : h->events) cudaEventSynchronize(e);
+    for (Plan *P : h->plans) destroy_plan(P);
+    h->plans.clear();
+    if (h->ring_ready) {
+      for (int k = 0; k < Ring::kSlots; ++k) {
+        if (h->ring.done[k]) {
+          cudaEventSynchronize(h->ring.done[k]);
+          cudaEventDestroy(h->ring.done[k]);
+        }
+        if (h->ring.slot[k]) cudaFreeHost(h->ring.slot[k]);
+      }
+    }
+    for (cudaEvent_t e : h->events) cudaEventDestroy(e);
+    h->events.clear();
+    if (h->status) cudaFree(h->status);
+    h->status = nullptr;
+    for (File &f : h->files) unmap_file(f);
+    if (cur >= 0 && cur != h->device) cudaSetDevice(cur);
+  } else {
+    for (File &f : h->files) unmap_file(f);
+  }
+  delete h;
+  return rc;
+}
+
+}  // namespace
+
+// ====================================================================== C ABI
+#pragma GCC visibility push(default)
+extern "C" {
+
+const char *wt_last_error(void) { return t_err.c_str(); }
+
+int wt_abi_version(void) { return 1; }
+
+int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **out) {
+  if (!out) return set_err(WT_EINVAL, "wt_open: out is NULL");
+  *out = nullptr;
+  if (n_paths < 0 || (n_paths > 0 && !paths)) return set_err(WT_EINVAL, "wt_open: bad path list");
+  const unsigned route_req = flags & WT_ROUTE_MASK;
+  if (flags & ~(WT_ROUTE_MASK | WT_OPEN_HOST_ONLY | WT_OPEN_PREFAULT))
+    return set_err(WT_EINVAL, "wt_open: unknown flag bits 0x%x", flags);
+  wt_handle *h = nullptr;
+  try {
+    h = new wt_handle();
+    h->host_only = (flags & WT_OPEN_HOST_ONLY) != 0;
+    h->files.resize(n_paths);
+    for (int i = 0; i < n_paths; ++i) {
+      if (!paths[i]) {
+        delete h;
+        return set_err(WT_EINVAL, "wt_open: path %d is NULL", i);
+      }
+      h->files[i].path = paths[i];
+    }
+    // parse + map in parallel; keep the first failure in file order
+    std::vector<int> rcs(n_paths, WT_OK);
+    std::vector<std::string> errs(n_paths);
+    host_pool().parallel_for((size_t)n_paths, [&](size_t i) {
+      rcs[i] = open_one(h->files[i]);
+      if (rcs[i]) errs[i] = t_err;
+    });
+    for (int i = 0; i < n_paths; ++i) {
+      if (rcs[i]) {
+        std::string msg = errs[i];
+        close_impl(h);
+        return set_err(rcs[i], "%s", msg.c_str());
+      }
+    }
+    for (int f = 0; f < n_paths; ++f)
+      for (uint32_t e = 0; e < h->files[f].tensors.size(); ++e) h->order.push_back({(uint32_t)f, e});
+    if (flags & WT_OPEN_PREFAULT) {
+      host_pool().parallel_for((size_t)n_paths, [&](size_t i) { prefault(h->files[i].base, h->files[i].size); });
+      h->prefaulted = true;
+    }
+    if (h->host_only) {
+      for (File &f : h->files) f.route = WT_ROUTE_NONE;
+      *out = h;
+      return WT_OK;
+    }
+    cudaError_t ce = cudaGetDevice(&h->device);
+    if (ce != cudaSuccess) {
+      close_impl(h);
+      return cuda_err(ce, "cudaGetDevice");
+    }
+    int rc = prepare_device(h->device);
+    if (rc) {
+      close_impl(h);
+      return rc;
+    }
+    int ats = 0;
+    cudaDeviceGetAttribute(&ats, cudaDevAttrPageableMemoryAccessUsesHostPageTables, h->device);
+    for (File &f : h->files) {
+      unsigned want = route_req;
+      if (want == WT_ROUTE_AUTO) want = ats ? WT_ROUTE_DIRECT : WT_ROUTE_REGISTER;
+      if (want == WT_ROUTE_DIRECT) {
+        if (!ats) {
+          close_impl(h);
+          return set_err(WT_ENOTSUP, "%s: device does not read pageable memory through host page tables", f.path.c_str());
+        }
+        f.route = WT_ROUTE_DIRECT;
+        f.dev = f.base;
+      } else if (want == WT_ROUTE_REGISTER) {
+        cudaError_t e = cudaHostRegister(f.base, f.size, cudaHostRegisterMapped | cudaHostRegisterReadOnly);
+        if (e != cudaSuccess) {
+          cudaGetLastError();
+          e = cudaHostRegister(f.base, f.size, cudaHostRegisterMapped);
+        }
+        if (e == cudaSuccess) {
+          f.registered = true;
+          void *dp = nullptr;
+          e = cudaHostGetDevicePointer(&dp, f.base, 0);
+          if (e != cudaSuccess) {
+            close_impl(h);
+            return cuda_err(e, "cudaHostGetDevicePointer");
+          }
+          f.route = WT_ROUTE_REGISTER;
+          f.dev = static_cast<const uint8_t *>(dp);
+        } else if (route_req == WT_ROUTE_AUTO) {
+          cudaGetLastError();
+          f.route = WT_ROUTE_NONE;
+        } else {
+          close_impl(h);
+          return cuda_err(e, "cudaHostRegister");
+        }
+      } else {
+        f.route = WT_ROUTE_NONE;
+      }
+    }
+    ce = cudaMalloc(reinterpret_cast<void **>(&h->status), 256);
+    if (ce == cudaSuccess) ce = cudaMemset(h->status, 0, 256);
+    if (ce != cudaSuccess) {
+      close_impl(h);
+      return cuda_err(ce, "status word");
+    }
+    *out = h;
+    return WT_OK;
+  } catch (const std::bad_alloc &) {
+    if (h) close_impl(h);
+    return set_err(WT_ENOMEM, "wt_open: out of host memory");
+  } catch (...) {
+    if (h) close_impl(h);
+    return set_err(WT_EINVAL, "wt_open: unexpected failure");
+  }
+}
+
+int wt_num_tensors(const wt_handle *h, size_t *n) {
+  if (!h || !n) return set_err(WT_EINVAL, "wt_num_tensors: NULL argument");
+  *n = h->order.size();
+  return WT_OK;
+}
+
+int wt_num_files(const wt_handle *h, size_t *n) {
+  if (!h || !n) return set_err(WT_EINVAL, "wt_num_files: NULL argument");
+  *n = h->files.size();
+  return WT_OK;
+}
+
+int wt_tensor_info(const wt_handle *h, size_t i, wt_tensor_meta *out) {
+  if (!h || !out) return set_err(WT_EINVAL, "wt_tensor_info: NULL argument");
+  if (i >= h->order.size()) return set_err(WT_EINVAL, "wt_tensor_info: index %zu out of range", i);
+  const Tensor &t = h->tensor(i);
+  out->name = t.name.c_str();
+  out->dtype = t.dtype;
+  out->ndim = t.ndim;
+  for (int d = 0; d < 4; ++d) out->shape[d] = t.shape[d];
+  out->nbytes = t.nbytes;
+  out->file = h->order[i].first;
+  out->offset = t.offset;
+  out->host_ptr = h->files[out->file].base + t.offset;
+  return WT_OK;
+}
+
+int wt_find(const wt_handle *h, const char *name, size_t *i) {
+  if (!h || !name || !i) return set_err(WT_EINVAL, "wt_find: NULL argument");
+  for (size_t k = 0; k < h->order.size(); ++k)
+    if (h->tensor(k).name == name) {
+      *i = k;
+      return WT_OK;
+    }
+  return set_err(WT_EINVAL, "wt_find: no tensor named '%s'", name);
+}
+
+int wt_file_route(const wt_handle *h, size_t f, unsigned *route) {
+  if (!h || !route) return set_err(WT_EINVAL, "wt_file_route: NULL argument");
+  if (f >= h->files.size()) return set_err(WT_EINVAL, "wt_file_route: file %zu out of range", f);
+  *route = h->files[f].route;
+  return WT_OK;
+}
+
+int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsigned mode, void *stream,
+             void **ready) {
+  if (!h) return set_err(WT_EINVAL, "wt_adopt: NULL handle");
+  if (h->host_only) return set_err(WT_ENOTSUP, "wt_adopt: handle was opened host-only");
+  if (n == 0) return WT_OK;
+  if (!idx || !dst || !ready) return set_err(WT_EINVAL, "wt_adopt: NULL array");
+  if (mode > WT_ADOPT_STAGED) return set_err(WT_EINVAL, "wt_adopt: unknown mode %u", mode);
+  std::lock_guard<std::mutex> g(h->mu);
+  try {
+    std::vector<Range> rs;
+    rs.reserve(n);
+    uint64_t total = 0;
+    for (size_t k = 0; k < n; ++k) {
+      if (idx[k] >= h->order.size()) return set_err(WT_EINVAL, "wt_adopt: tensor index %zu out of range", idx[k]);
+      const File &f = h->files[h->order[idx[k]].first];
+      const Tensor &t = h->tensor(idx[k]);
+      if (t.nbytes && !dst[k]) return set_err(WT_EINVAL, "wt_adopt: dst[%zu] is NULL", k);
+      if (t.nbytes && inside_mapping(h, dst[k], t.nbytes))
+        return set_err(WT_EINVAL, "wt_adopt: dst[%zu] lies inside a read-only mapping", k);
+      if (mode != WT_ADOPT_STAGED && f.route == WT_ROUTE_NONE)
+        return set_err(WT_ENOTSUP, "wt_adopt: %s has no device route; use WT_ADOPT_STAGED", f.path.c_str());
+      ready[k] = nullptr;
+      rs.push_back({k, f.base + t.offset, f.dev ? f.dev + t.offset : nullptr, static_cast<uint8_t *>(dst[k]), t.nbytes});
+      total += t.nbytes;
+    }
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int rc = mode == WT_ADOPT_STAGED ? adopt_staged(h, rs, s, ready) : adopt_device(h, rs, mode, s, ready, total);
+    return rc;
+  } catch (const std::bad_alloc &) {
+    return set_err(WT_ENOMEM, "wt_adopt: out of host memory");
+  }
+}
+
+int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream) {
+  if (!h) return set_err(WT_EINVAL, "wt_pass: NULL handle");
+  if (h->host_only) return set_err(WT_ENOTSUP, "wt_pass: handle was opened host-only");
+  if (n == 0) return WT_OK;
+  if (!d) return set_err(WT_EINVAL, "wt_pass: NULL descriptors");
+  for (size_t i = 0; i < n; ++i) {
+    int rc = validate_desc(d[i], i);
+    if (rc) return rc;
+  }
+  std::lock_guard<std::mutex> g(h->mu);
+  try {
+    const uint8_t *kb = reinterpret_cast<const uint8_t *>(d);
+    std::vector<uint8_t> key(kb, kb + n * sizeof(wt_gemv_desc));
+    Plan *P = nullptr;
+    for (auto it = h->plans.begin(); it != h->plans.end(); ++it)
+      if ((*it)->key == key) {
+        P = *it;
+        h->plans.erase(it);
+        h->plans.push_front(P);
+        break;
+      }
+    if (!P) {
+      P = new Plan();
+      P->key = std::move(key);
+      int rc = build_plan(h, d, n, P);
+      if (rc) {
+        destroy_plan(P);
+        return rc;
+      }
+      h->plans.push_front(P);
+      while (h->plans.size() > 32) {
+        destroy_plan(h->plans.back());
+        h->plans.pop_back();
+      }
+    }
+    return run_plan(h, P, static_cast<cudaStream_t>(stream));
+  } catch (const std::bad_alloc &) {
+    return set_err(WT_ENOMEM, "wt_pass: out of host memory");
+  }
+}
+
+static int checksum_impl(wt_handle *h, const void *const *ptr, const uint64_t *nbytes, size_t n,
+                         uint64_t *out_dev, void *stream, bool plain) {
+  if (!h) return set_err(WT_EINVAL, "wt_checksum: NULL handle");
+  if (h->host_only) return set_err(WT_ENOTSUP, "wt_checksum: handle was opened host-only");
+  if (n == 0) return WT_OK;
+  if (!ptr || !nbytes || !out_dev) return set_err(WT_EINVAL, "wt_checksum: NULL array");
+  for (size_t i = 0; i < n; ++i) {
+    if (nbytes[i] && !ptr[i]) return set_err(WT_EINVAL, "wt_checksum: ptr[%zu] is NULL", i);
+    if (plain && nbytes[i] > (256ull << 20)) return set_err(WT_EINVAL, "wt_checksum_plain: buffer %zu above 256 MiB", i);
+  }
+  const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  std::lock_guard<std::mutex> g(h->mu);
+  for (size_t i0 = 0; i0 < n; i0 += wt::kMaxFnv) {
+    const size_t m = std::min<size_t>(wt::kMaxFnv, n - i0);
+    wt::FnvBatch b;
+    memset(&b, 0, sizeof b);
+    b.n = (uint32_t)m;
+    uint64_t leaves = 0;
+    for (size_t k = 0; k < m; ++k) {
+      b.leaf_prefix[k] = leaves;
+      b.ptr[k] = static_cast<const uint8_t *>(ptr[i0 + k]);
+      b.nbytes[k] = nbytes[i0 + k];
+      b.out[k] = out_dev + i0 + k;
+      leaves += (nbytes[i0 + k] + wt::kLeafBytes - 1) / wt::kLeafBytes;
+    }
+    b.leaf_prefix[m] = leaves;
+    if (plain) {
+      CU(wt::launch_fnv_plain(b, s));
+      h->kernel_launches++;
+    } else {
+      uint64_t *lv = nullptr;
+      if (leaves) CU(cudaMallocAsync(reinterpret_cast<void **>(&lv), leaves * 8, s));
+      CU(wt::launch_fnv_tree(b, lv, s));
+      h->kernel_launches += leaves ? 2 : 1;
+      if (lv) CU(cudaFreeAsync(lv, s));
+    }
+  }
+  return WT_OK;
+}
+
+int wt_checksum(wt_handle *h, const void *const *ptr, const uint64_t *nbytes, size_t n, uint64_t *out_dev,
+                void *stream) {
+  return checksum_impl(h, ptr, nbytes, n, out_dev, stream, false);
+}
+
+int wt_checksum_plain(wt_handle *h, const void *const *ptr, const uint64_t *nbytes, size_t n,
+                      uint64_t *out_dev, void *stream) {
+  return checksum_impl(h, ptr, nbytes, n, out_dev, stream, true);
+}
+
+int wt_device_status(wt_handle *h, int *status) {
+  if (!h || !status) return set_err(WT_EINVAL, "wt_device_status: NULL argument");
+  if (h->host_only) {
+    *status = 0;
+    return WT_OK;
+  }
+  CU(cudaMemcpy(status, h->status, sizeof(int), cudaMemcpyDeviceToHost));
+  return WT_OK;
+}
+
+int wt_kernel_launches(const wt_handle *h, uint64_t *n) {
+  if (!h || !n) return set_err(WT_EINVAL, "wt_kernel_launches: NULL argument");
+  *n = h->kernel_launches;
+  return WT_OK;
+}
+
+int wt_close(wt_handle *h) {
+  if (!h) return WT_OK;
+  return close_impl(h);
+}
+
+}  // extern "C"
+#pragma GCC visibility pop

@@ -1,0 +1,637 @@
+// sm_103a kernels of the file-backed weight path.
+//
+//   gather_kernel      host-mapped file bytes -> HBM, 16-byte vector loads and
+//                      stores (the ingest step: the copy the paper calls the
+//                      ingestion tax, Sec. 1 and Sec. 2.2, done once at the
+//                      host-link rate)
+//   gemv_tma_kernel    y = W x per matrix, fp32 accumulate: the bandwidth-bound
+//                      consumer pass (Sec. 3.1: one single-token GEMV per
+//                      matrix).  W streams HBM -> shared memory through 1-D TMA
+//                      bulk copies on an mbarrier ring; warps reduce with
+//                      shuffles.  No tensor cores: ~1 flop per weight byte.
+//   fnv_*              per-buffer FNV-1a-64 digests (plain and 4 KiB leaf tree)
+//                      that prove ingested bytes equal the file's.
+//
+// Every wait on an mbarrier is bounded (clock64 budget); a wait that runs out
+// records WT_ETIMEDOUT in the caller's status word, makes every later wait of
+// the CTA return at once, and the producer drains its own copies in flight
+// before the CTA exits.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "wt_kernels.h"
+
+namespace wt {
+
+namespace {
+
+constexpr int kStatusTimedOut = -7;  // WT_ETIMEDOUT
+constexpr long long kWaitCycles = 1ll << 31;  // ~1 s at 2 GHz
+
+int g_num_sms[64] = {0};
+
+// ------------------------------------------------------------------ PTX helpers
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ uint64_t l2_evict_first_policy() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+// 1-D bulk copy global -> this CTA's shared memory, completion counted on `bar`.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes,
+                                         uint32_t bar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1], %2, [%3], %4;" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar), "l"(pol)
+      : "memory");
+}
+
+__device__ __forceinline__ void named_bar(int id, int n) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
+// Bounded wait.  Returns false (and raises the CTA's abort flag on a timeout)
+// instead of spinning forever.
+__device__ __forceinline__ bool bounded_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag,
+                                             int *status) {
+  if (*abort_flag) return false;
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (*abort_flag) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      *abort_flag = 1;
+      if (status) atomicCAS(status, 0, kStatusTimedOut);
+      return false;
+    }
+  }
+  return true;
+}
+
+// ------------------------------------------------------------------ element math
+template <int DT>
+struct Elem;
+template <>
+struct Elem<0> {  // f32
+  static constexpr int kEPV = 4;
+  __device__ static __forceinline__ void unpack(const uint4 &v, float (&f)[4]) {
+    f[0] = __uint_as_float(v.x);
+    f[1] = __uint_as_float(v.y);
+    f[2] = __uint_as_float(v.z);
+    f[3] = __uint_as_float(v.w);
+  }
+  __device__ static __forceinline__ float scalar(const uint8_t *p, uint64_t i) {
+    uint32_t u = (uint32_t)p[4 * i] | ((uint32_t)p[4 * i + 1] << 8) | ((uint32_t)p[4 * i + 2] << 16) |
+                 ((uint32_t)p[4 * i + 3] << 24);
+    return __uint_as_float(u);
+  }
+};
+template <>
+struct Elem<1> {  // bf16: the high half of an IEEE single
+  static constexpr int kEPV = 8;
+  __device__ static __forceinline__ void unpack(const uint4 &v, float (&f)[8]) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      f[2 * i] = __uint_as_float(w[i] << 16);
+      f[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+    }
+  }
+  __device__ static __forceinline__ float scalar(const uint8_t *p, uint64_t i) {
+    uint32_t u = (uint32_t)p[2 * i] | ((uint32_t)p[2 * i + 1] << 8);
+    return __uint_as_float(u << 16);
+  }
+};
+template <>
+struct Elem<2> {  // f16
+  static constexpr int kEPV = 8;
+  __device__ static __forceinline__ void unpack(const uint4 &v, float (&f)[8]) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      __half2 h = *reinterpret_cast<const __half2 *>(&w[i]);
+      float2 t = __half22float2(h);
+      f[2 * i] = t.x;
+      f[2 * i + 1] = t.y;
+    }
+  }
+  __device__ static __forceinline__ float scalar(const uint8_t *p, uint64_t i) {
+    uint16_t u = (uint16_t)(p[2 * i] | (p[2 * i + 1] << 8));
+    return __half2float(__ushort_as_half(u));
+  }
+};
+
+// acc += <w, x> over one 16-byte vector, in element order.
+template <int DT>
+__device__ __forceinline__ float dot16(const uint4 &w, const float (&xf)[Elem<DT>::kEPV], float acc) {
+  float wf[Elem<DT>::kEPV];
+  Elem<DT>::unpack(w, wf);
+#pragma unroll
+  for (int e = 0; e < Elem<DT>::kEPV; ++e) acc = fmaf(wf[e], xf[e], acc);
+  return acc;
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(addr));
+  return v;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// ------------------------------------------------------------------ gather
+__global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ GatherBatch b) {
+  const uint64_t total = b.chunk_prefix[b.n];
+  for (uint64_t c = blockIdx.x; c < total; c += gridDim.x) {
+    // range holding chunk c (binary search over the prefix in parameter space)
+    uint32_t lo = 0, hi = b.n - 1;
+    while (lo < hi) {
+      uint32_t mid = (lo + hi + 1) >> 1;
+      if (b.chunk_prefix[mid] <= c) lo = mid; else hi = mid - 1;
+    }
+    const uint64_t off = (c - b.chunk_prefix[lo]) << kGatherChunkLog2;
+    const uint64_t n = b.nbytes[lo];
+    const uint64_t len = min((uint64_t)1 << kGatherChunkLog2, n - off);
+    const uint8_t *src = b.src[lo] + off;
+    uint8_t *dst = b.dst[lo] + off;
+    if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0) {
+      const uint4 *s4 = reinterpret_cast<const uint4 *>(src);
+      uint4 *d4 = reinterpret_cast<uint4 *>(dst);
+      const uint32_t n16 = (uint32_t)(len >> 4);
+      uint32_t i = threadIdx.x;
+      const uint32_t st = blockDim.x;
+      for (; i + 3 * st < n16; i += 4 * st) {
+        uint4 a0 = s4[i], a1 = s4[i + st], a2 = s4[i + 2 * st], a3 = s4[i + 3 * st];
+        d4[i] = a0;
+        d4[i + st] = a1;
+        d4[i + 2 * st] = a2;
+        d4[i + 3 * st] = a3;
+      }
+      for (; i < n16; i += st) d4[i] = s4[i];
+      for (uint32_t t = (n16 << 4) + threadIdx.x; t < len; t += st) dst[t] = src[t];
+    } else {
+      for (uint32_t t = threadIdx.x; t < len; t += blockDim.x) dst[t] = src[t];
+    }
+  }
+}
+
+// ------------------------------------------------------------------ GEMV
+constexpr int kConsumers = kConsumerWarps * 32;
+constexpr int kGemvThreads = kConsumers + 32;
+constexpr size_t kBarOff = (size_t)kStages * kStageBytes;
+constexpr size_t kRedOff = kBarOff + 2 * kStages * sizeof(uint64_t);
+constexpr size_t kFlagOff = kRedOff + 2 * kConsumerWarps * kRowBlock * sizeof(float);
+constexpr size_t kGemvSmem = kFlagOff + 16;
+
+template <int DT>
+__device__ __forceinline__ void load_xvec(const uint8_t *x, uint32_t v, bool ok,
+                                          float (&xf)[Elem<DT>::kEPV]) {
+  if (ok) {
+    uint4 t = __ldg(reinterpret_cast<const uint4 *>(x) + v);
+    Elem<DT>::unpack(t, xf);
+  } else {
+#pragma unroll
+    for (int e = 0; e < Elem<DT>::kEPV; ++e) xf[e] = 0.f;
+  }
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kGemvThreads, 1)
+    gemv_tma_kernel(const MatDesc *__restrict__ mats, const Piece *__restrict__ pieces,
+                    const uint32_t *__restrict__ begin, int *status) {
+  constexpr int EPV = Elem<DT>::kEPV;
+  extern __shared__ __align__(128) uint8_t smem[];
+  const uint32_t stage0 = smem_u32(smem);
+  const uint32_t full0 = smem_u32(smem + kBarOff);
+  const uint32_t empty0 = full0 + kStages * 8;
+  float *red = reinterpret_cast<float *>(smem + kRedOff);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + kFlagOff);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t p0 = begin[blockIdx.x];
+  const uint32_t p1 = begin[blockIdx.x + 1];
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, kConsumerWarps);
+    }
+    *abort_flag = 0;
+    mbar_fence_init();
+  }
+  __syncthreads();
+
+  if (warp == kConsumerWarps) {
+    // ---------------- producer: one thread issues every bulk copy of the CTA
+    if (lane == 0) {
+      const uint64_t pol = l2_evict_first_policy();
+      uint32_t it = 0;
+      bool live = true;
+      for (uint32_t pi = p0; pi < p1 && live; ++pi) {
+        const Piece pc = pieces[pi];
+        const MatDesc md = mats[pc.mat];
+        const uint64_t rowb = (uint64_t)md.V * 16;
+        for (uint32_t r = pc.r0; r < pc.r1 && live; r += md.rt) {
+          const uint32_t nr = min(md.rt, pc.r1 - r);
+          const uint32_t nchunk = md.mode == kModeSplitK ? (md.V + md.vc - 1) / md.vc : 1;
+          for (uint32_t c = 0; c < nchunk; ++c) {
+            const uint32_t s = it % kStages;
+            if (it >= kStages &&
+                !bounded_wait(empty0 + 8 * s, ((it / kStages) - 1) & 1, abort_flag, status)) {
+              live = false;
+              break;
+            }
+            const uint32_t dst = stage0 + s * kStageBytes;
+            const uint32_t bar = full0 + 8 * s;
+            if (md.mode != kModeSplitK) {
+              const uint32_t bytes = nr * (uint32_t)rowb;
+              mbar_expect_tx(bar, bytes);
+              bulk_g2s(dst, md.W + (uint64_t)r * rowb, bytes, bar, pol);
+            } else {
+              const uint32_t v0 = c * md.vc;
+              const uint32_t nv = min(md.vc, md.V - v0);
+              mbar_expect_tx(bar, nr * nv * 16);
+              for (uint32_t q = 0; q < nr; ++q)
+                bulk_g2s(dst + q * md.vc * 16, md.W + (uint64_t)(r + q) * rowb + (uint64_t)v0 * 16,
+                         nv * 16, bar, pol);
+            }
+            ++it;
+          }
+        }
+      }
+      if (!live || *abort_flag) {
+        // drain: the copies of the last (up to kStages) issued stages may still be in flight
+        const uint32_t first = it > (uint32_t)kStages ? it - kStages : 0;
+        for (uint32_t j = first; j < it; ++j) {
+          const long long t0 = clock64();
+          while (!mbar_try_wait(full0 + 8 * (j % kStages), (j / kStages) & 1) &&
+                 clock64() - t0 < kWaitCycles) {
+          }
+        }
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---------------- consumers: 8 warps
+    const int ct = threadIdx.x;  // 0..255
+    uint32_t it = 0;
+    int par = 0;
+    float xf[8][EPV];
+    for (uint32_t pi = p0; pi < p1; ++pi) {
+      const Piece pc = pieces[pi];
+      const MatDesc md = mats[pc.mat];
+      const uint32_t V = md.V;
+      if (md.mode == kModeWarpRows) {
+        const uint32_t G = md.G;
+        const uint32_t gl = lane & (G - 1);
+        const uint32_t sub = lane / G;
+        const uint32_t rpw = 32 / G;
+        const uint32_t nj = (V + G - 1) / G;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const uint32_t v = gl + j * G;
+          load_xvec<DT>(md.x, v, j < (int)nj && v < V, xf[j]);
+        }
+        for (uint32_t r = pc.r0; r < pc.r1; r += md.rt) {
+          const uint32_t nr = min(md.rt, pc.r1 - r);
+          const uint32_t s = it % kStages;
+          bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
+          const uint32_t tile = stage0 + s * kStageBytes;
+          for (uint32_t base = warp * rpw; base < nr; base += kConsumerWarps * rpw) {
+            const uint32_t row = base + sub;
+            const bool valid = row < nr;
+            float a0 = 0.f, a1 = 0.f;
+            if (valid) {
+#pragma unroll
+              for (int j = 0; j < 8; j += 2) {
+                const uint32_t v = gl + j * G;
+                if (j < (int)nj && v < V) a0 = dot16<DT>(lds128(tile + (row * V + v) * 16), xf[j], a0);
+                const uint32_t v1 = gl + (j + 1) * G;
+                if (j + 1 < (int)nj && v1 < V)
+                  a1 = dot16<DT>(lds128(tile + (row * V + v1) * 16), xf[j + 1], a1);
+              }
+            }
+            float acc = a0 + a1;
+            for (uint32_t o = G >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+            if (valid && gl == 0) md.y[r + row] = acc;
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(empty0 + 8 * s);
+          ++it;
+        }
+      } else {
+        // block modes: the whole consumer group shares each row
+        const bool split = md.mode == kModeSplitK;
+        const uint32_t nj = split ? 1 : (V + kConsumers - 1) / kConsumers;
+        if (!split) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const uint32_t v = ct + j * kConsumers;
+            load_xvec<DT>(md.x, v, j < (int)nj && v < V, xf[j]);
+          }
+        }
+        const uint32_t vstride = split ? md.vc : V;  // vectors per row inside a stage
+        for (uint32_t r = pc.r0; r < pc.r1; r += md.rt) {
+          const uint32_t nr = min(md.rt, pc.r1 - r);
+          float acc[kRowBlock];
+#pragma unroll
+          for (int q = 0; q < kRowBlock; ++q) acc[q] = 0.f;
+          const uint32_t nchunk = split ? (V + md.vc - 1) / md.vc : 1;
+          for (uint32_t c = 0; c < nchunk; ++c) {
+            const uint32_t v0 = c * md.vc;
+            const uint32_t nv = split ? min(md.vc, V - v0) : V;
+            if (split) load_xvec<DT>(md.x, v0 + ct, ct < nv, xf[0]);
+            const uint32_t s = it % kStages;
+            bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
+            const uint32_t tile = stage0 + s * kStageBytes;
+#pragma unroll
+            for (int q = 0; q < kRowBlock; ++q) {
+              if (q < (int)nr) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                  const uint32_t v = ct + j * kConsumers;
+                  if (j < (int)nj && v < nv) acc[q] = dot16<DT>(lds128(tile + (q * vstride + v) * 16), xf[j], acc[q]);
+                }
+              }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(empty0 + 8 * s);
+            ++it;
+          }
+          // cross-warp reduction in a fixed order: deterministic per row
+          float *rb = red + par * (kConsumerWarps * kRowBlock);
+#pragma unroll
+          for (int q = 0; q < kRowBlock; ++q) {
+            if (q < (int)nr) {
+              const float t = warp_sum(acc[q]);
+              if (lane == 0) rb[warp * kRowBlock + q] = t;
+            }
+          }
+          named_bar(1, kConsumers);
+          if (ct < (int)nr) {
+            float t = 0.f;
+#pragma unroll
+            for (int w = 0; w < kConsumerWarps; ++w) t += rb[w * kRowBlock + ct];
+            md.y[r + ct] = t;
+          }
+          par ^= 1;
+        }
+      }
+    }
+  }
+  __syncthreads();
+}
+
+// Fallback: one warp per row, byte-assembled scalar loads (any alignment).
+template <int DT>
+__global__ void gemv_generic_kernel(const uint8_t *W, const uint8_t *x, float *y, uint64_t M,
+                                    uint64_t K) {
+  const uint64_t warps = (uint64_t)gridDim.x * (blockDim.x >> 5);
+  const int lane = threadIdx.x & 31;
+  for (uint64_t row = (uint64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); row < M;
+       row += warps) {
+    const uint8_t *wr = W + row * K * (uint64_t)(16 / Elem<DT>::kEPV);
+    float acc = 0.f;
+    for (uint64_t k = lane; k < K; k += 32) acc = fmaf(Elem<DT>::scalar(wr, k), Elem<DT>::scalar(x, k), acc);
+    acc = warp_sum(acc);
+    if (lane == 0) y[row] = acc;
+  }
+}
+
+// ------------------------------------------------------------------ FNV-1a-64
+constexpr uint64_t kFnvOffset = 0xcbf29ce484222325ull;
+constexpr uint64_t kFnvPrime = 0x00000100000001b3ull;
+
+__device__ __forceinline__ uint64_t fnv_byte(uint64_t h, uint32_t b) { return (h ^ b) * kFnvPrime; }
+
+__device__ __forceinline__ uint64_t fnv_word(uint64_t h, uint32_t w) {
+  h = fnv_byte(h, w & 0xff);
+  h = fnv_byte(h, (w >> 8) & 0xff);
+  h = fnv_byte(h, (w >> 16) & 0xff);
+  return fnv_byte(h, w >> 24);
+}
+
+__device__ __forceinline__ uint64_t fnv_le64(uint64_t h, uint64_t v) {
+  h = fnv_word(h, (uint32_t)v);
+  return fnv_word(h, (uint32_t)(v >> 32));
+}
+
+__device__ __forceinline__ uint32_t find_buf(const FnvBatch &b, uint64_t leaf) {
+  uint32_t lo = 0, hi = b.n - 1;
+  while (lo < hi) {
+    uint32_t mid = (lo + hi + 1) >> 1;
+    if (b.leaf_prefix[mid] <= leaf) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// One thread per 4 KiB leaf.  A warp stages 256-byte slices of its 32 leaves
+// in shared memory with coalesced 16-byte loads (two leaves per warp load),
+// then each lane hashes its own row.
+constexpr int kFnvWarps = 4;
+constexpr int kSlice = 256;
+constexpr int kSliceStride = kSlice + 16;  // padding: 8 consecutive lanes hit distinct bank groups
+
+__global__ void __launch_bounds__(kFnvWarps * 32) fnv_leaf_kernel(const __grid_constant__ FnvBatch b,
+                                                                   uint64_t *leaves) {
+  __shared__ __align__(16) uint8_t buf[kFnvWarps][32][kSliceStride];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint64_t total = b.leaf_prefix[b.n];
+  const uint64_t nwarps = (uint64_t)gridDim.x * kFnvWarps;
+  for (uint64_t base = ((uint64_t)blockIdx.x * kFnvWarps + warp) * 32; base < total; base += nwarps * 32) {
+    const uint64_t leaf = base + lane;
+    const bool mine = leaf < total;
+    const uint8_t *lp = nullptr;
+    uint32_t llen = 0;
+    if (mine) {
+      const uint32_t t = find_buf(b, leaf);
+      const uint64_t off = (leaf - b.leaf_prefix[t]) * kLeafBytes;
+      lp = b.ptr[t] + off;
+      llen = (uint32_t)min(kLeafBytes, b.nbytes[t] - off);
+    }
+    uint64_t h = kFnvOffset;
+    for (uint32_t s0 = 0; s0 < kLeafBytes; s0 += kSlice) {
+      // cooperative load: lanes 0-15 fetch leaf i, lanes 16-31 leaf i+1, bytes [s0, s0 + 256)
+      for (int i2 = 0; i2 < 32; i2 += 2) {
+        const int src = i2 + (lane >> 4);
+        const uint8_t *p = reinterpret_cast<const uint8_t *>(
+            __shfl_sync(0xffffffffu, (unsigned long long)lp, src));
+        const uint32_t n = __shfl_sync(0xffffffffu, llen, src);
+        const uint32_t o = s0 + (lane & 15) * 16;
+        uint8_t *d = &buf[warp][src][(lane & 15) * 16];
+        if (p != nullptr && o < n) {
+          if (o + 16 <= n && ((reinterpret_cast<uintptr_t>(p) + o) & 15) == 0) {
+            *reinterpret_cast<uint4 *>(d) = *reinterpret_cast<const uint4 *>(p + o);
+          } else {
+            for (uint32_t k = 0; k < 16 && o + k < n; ++k) d[k] = p[o + k];
+          }
+        }
+      }
+      __syncwarp();
+      if (mine && s0 < llen) {
+        const uint32_t m = min((uint32_t)kSlice, llen - s0);
+        const uint8_t *row = buf[warp][lane];
+        uint32_t k = 0;
+        for (; k + 16 <= m; k += 16) {
+          const uint4 v = *reinterpret_cast<const uint4 *>(row + k);
+          h = fnv_word(h, v.x);
+          h = fnv_word(h, v.y);
+          h = fnv_word(h, v.z);
+          h = fnv_word(h, v.w);
+        }
+        for (; k < m; ++k) h = fnv_byte(h, row[k]);
+      }
+      __syncwarp();
+    }
+    if (mine) leaves[leaf] = h;
+  }
+}
+
+// One thread per buffer: FNV-1a over LE64(nbytes) then the LE64 of each leaf.
+__global__ void fnv_combine_kernel(const __grid_constant__ FnvBatch b, const uint64_t *leaves) {
+  const uint32_t t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= b.n) return;
+  uint64_t h = fnv_le64(kFnvOffset, b.nbytes[t]);
+  for (uint64_t l = b.leaf_prefix[t]; l < b.leaf_prefix[t + 1]; ++l) h = fnv_le64(h, leaves[l]);
+  *b.out[t] = h;
+}
+
+// One thread per buffer: the literal serial FNV-1a-64.
+__global__ void fnv_plain_kernel(const __grid_constant__ FnvBatch b) {
+  const uint32_t t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= b.n) return;
+  const uint8_t *p = b.ptr[t];
+  const uint64_t n = b.nbytes[t];
+  uint64_t h = kFnvOffset;
+  uint64_t i = 0;
+  // bytes up to the first 16-byte boundary, then vectors, then the tail
+  while (i < n && ((reinterpret_cast<uintptr_t>(p) + i) & 15) != 0) h = fnv_byte(h, p[i++]);
+  const uint4 *v = reinterpret_cast<const uint4 *>(p + i);
+  const uint64_t nv = (n - i) >> 4;
+  for (uint64_t k = 0; k < nv; ++k) {
+    const uint4 w = v[k];
+    h = fnv_word(h, w.x);
+    h = fnv_word(h, w.y);
+    h = fnv_word(h, w.z);
+    h = fnv_word(h, w.w);
+  }
+  for (i += nv << 4; i < n; ++i) h = fnv_byte(h, p[i]);
+  *b.out[t] = h;
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------ launchers
+int num_sms() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  if (g_num_sms[dev] == 0) {
+    int n = 0;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    g_num_sms[dev] = n > 0 ? n : 1;
+  }
+  return g_num_sms[dev];
+}
+
+cudaError_t launch_gather(const GatherBatch &b, int grid, cudaStream_t s) {
+  if (b.n == 0 || b.chunk_prefix[b.n] == 0) return cudaSuccess;
+  gather_kernel<<<grid, 256, 0, s>>>(b);
+  return cudaGetLastError();
+}
+
+size_t gemv_smem_bytes() { return kGemvSmem; }
+
+cudaError_t gemv_prepare() {
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(gemv_tma_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemvSmem)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(gemv_tma_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemvSmem)) != cudaSuccess) return e;
+  return cudaFuncSetAttribute(gemv_tma_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemvSmem);
+}
+
+cudaError_t launch_gemv(const GemvLaunch &L, cudaStream_t s) {
+  if (L.grid <= 0) return cudaSuccess;
+  switch (L.dtype) {
+    case 0: gemv_tma_kernel<0><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
+    case 1: gemv_tma_kernel<1><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
+    case 2: gemv_tma_kernel<2><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemv_generic(int dtype, const uint8_t *W, const uint8_t *x, float *y, uint64_t M,
+                                uint64_t K, cudaStream_t s) {
+  if (M == 0) return cudaSuccess;
+  const uint64_t blocks64 = (M + 7) / 8;
+  const int grid = (int)(blocks64 < (uint64_t)num_sms() * 8 ? blocks64 : (uint64_t)num_sms() * 8);
+  switch (dtype) {
+    case 0: gemv_generic_kernel<0><<<grid, 256, 0, s>>>(W, x, y, M, K); break;
+    case 1: gemv_generic_kernel<1><<<grid, 256, 0, s>>>(W, x, y, M, K); break;
+    case 2: gemv_generic_kernel<2><<<grid, 256, 0, s>>>(W, x, y, M, K); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fnv_tree(const FnvBatch &b, uint64_t *leaves, cudaStream_t s) {
+  if (b.n == 0) return cudaSuccess;
+  const uint64_t total = b.leaf_prefix[b.n];
+  if (total > 0) {
+    const uint64_t warps = (total + 31) / 32;
+    const uint64_t blocks = (warps + kFnvWarps - 1) / kFnvWarps;
+    const uint64_t cap = (uint64_t)num_sms() * 16;
+    fnv_leaf_kernel<<<(int)(blocks < cap ? blocks : cap), kFnvWarps * 32, 0, s>>>(b, leaves);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  fnv_combine_kernel<<<(b.n + 127) / 128, 128, 0, s>>>(b, leaves);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fnv_plain(const FnvBatch &b, cudaStream_t s) {
+  if (b.n == 0) return cudaSuccess;
+  fnv_plain_kernel<<<(b.n + 63) / 64, 64, 0, s>>>(b);
+  return cudaGetLastError();
+}
+
+}  // namespace wt

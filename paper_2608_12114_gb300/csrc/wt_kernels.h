@@ -1,0 +1,98 @@
+// Internal interface between the host library (wt_host.cpp) and the sm_103a
+// kernels (wt_kernels.cu).  Not part of the public C ABI (include/wt.h).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+namespace wt {
+
+// ---------------------------------------------------------------- ingest gather
+// One launch copies up to kMaxGather (src, dst, nbytes) ranges; the whole
+// descriptor set travels in the kernel's parameter space (no device table).
+constexpr int kMaxGather = 128;
+constexpr int kGatherChunkLog2 = 16;  // 64 KiB of one range per CTA iteration
+
+struct GatherBatch {
+  uint32_t n;
+  uint32_t pad;
+  uint64_t chunk_prefix[kMaxGather + 1];  // first chunk index of range i; [n] = total
+  const uint8_t *src[kMaxGather];
+  uint8_t *dst[kMaxGather];
+  uint64_t nbytes[kMaxGather];
+};
+
+cudaError_t launch_gather(const GatherBatch &b, int grid, cudaStream_t s);
+
+// ---------------------------------------------------------------- GEMV
+// Tile geometry.  A stage is one TMA bulk transfer target in shared memory.
+constexpr int kStageBytes = 32768;
+constexpr int kStages = 6;
+constexpr int kConsumerWarps = 8;
+constexpr int kRowBlock = 8;  // rows of a block-mode tile / split-K row block
+
+enum GemvMode : uint16_t {
+  kModeWarpRows = 0,   // rows of <= 256 vectors: each warp owns whole rows
+  kModeBlockRows = 1,  // 256 < vectors <= kStageBytes/16: whole CTA per row, full-row tiles
+  kModeSplitK = 2,     // longer rows: row blocks of kRowBlock rows x 4 KiB column chunks
+};
+
+struct alignas(16) MatDesc {
+  const uint8_t *W;
+  const uint8_t *x;
+  float *y;
+  uint32_t M;     // rows
+  uint32_t V;     // 16-byte vectors per row (K * sizeof(elem) / 16)
+  uint32_t rt;    // rows per tile (modes 0/1) or per row block (mode 2)
+  uint32_t vc;    // vectors per column chunk (mode 2); V otherwise
+  uint16_t mode;  // GemvMode
+  uint16_t G;     // mode 0: lanes per row (power of two <= 32)
+  uint32_t pad;
+};
+
+struct alignas(16) Piece {
+  uint32_t mat;  // index into the launch's MatDesc table
+  uint32_t r0;   // first row
+  uint32_t r1;   // one past the last row
+  uint32_t pad;
+};
+
+struct GemvLaunch {
+  int dtype;               // WT_F32 / WT_BF16 / WT_F16
+  int grid;                // CTAs; CTA b owns pieces [begin[b], begin[b+1])
+  const MatDesc *mats;     // device
+  const Piece *pieces;     // device
+  const uint32_t *begin;   // device, grid + 1 entries
+  int *status;             // device status word (bounded-wait failures)
+};
+
+cudaError_t gemv_prepare();  // one-time function attributes
+cudaError_t launch_gemv(const GemvLaunch &L, cudaStream_t s);
+size_t gemv_smem_bytes();
+
+// Fallback for operands the tiled kernel cannot take (unaligned W/x or rows
+// whose byte length is not a multiple of 16): one warp per row, scalar loads.
+cudaError_t launch_gemv_generic(int dtype, const uint8_t *W, const uint8_t *x, float *y,
+                                uint64_t M, uint64_t K, cudaStream_t s);
+
+// ---------------------------------------------------------------- FNV-1a-64
+constexpr int kMaxFnv = 256;
+constexpr uint64_t kLeafBytes = 4096;
+
+struct FnvBatch {
+  uint32_t n;
+  uint32_t pad;
+  uint64_t leaf_prefix[kMaxFnv + 1];  // first global leaf of buffer i; [n] = total leaves
+  const uint8_t *ptr[kMaxFnv];
+  uint64_t nbytes[kMaxFnv];
+  uint64_t *out[kMaxFnv];  // device address of the digest of buffer i
+};
+
+cudaError_t launch_fnv_tree(const FnvBatch &b, uint64_t *leaves, cudaStream_t s);
+cudaError_t launch_fnv_plain(const FnvBatch &b, cudaStream_t s);
+
+int num_sms();  // of the current device (cached per device)
+
+}  // namespace wt

@@ -1,0 +1,148 @@
+"""File -> first use, on top of the C ABI (torch supplies device memory and streams only).
+
+    h = wt.Handle(paths)                       # wt_open: parse, map, route
+    mats = matrices(h)                         # 2-D tensors, row blocks joined
+    dev = DeviceCheckpoint.allocate(h, mats)   # one caller-owned buffer per matrix/vector
+    events = dev.adopt(h, mode, stream)        # wt_adopt: per-tensor ready events
+    xs, ys = dev.inputs(), dev.outputs()       # x per inner size K, fp32 y per matrix
+    h.pass_(dev.descs(xs, ys, events), stream) # wt_pass: each GEMV waits on its bytes only
+
+Row blocks: a tensor named "<name>#r<k>" is row block k of matrix <name> (the
+many-small workload splits each matrix's rows across two files); its blocks are
+adopted into one contiguous [M, K] device buffer, in k order, and the GEMV of
+<name> waits on the event of its last-ingested block (the ingest stream is in
+order, so that event implies the earlier blocks).
+"""
+from __future__ import annotations
+
+import re
+from dataclasses import dataclass, field
+from typing import Dict, List, Optional, Sequence
+
+import numpy as np
+
+from . import synth, wt
+
+_BLOCK = re.compile(r"^(.*)#r(\d+)$")
+_ESZ = {wt.WT_F32: 4, wt.WT_BF16: 2, wt.WT_F16: 2, wt.WT_I8: 1, wt.WT_U8: 1}
+_ALIGN = 256
+
+
+@dataclass
+class MatrixRef:
+    name: str
+    dtype: int
+    shape: tuple            # (M, K) for matrices, (n,) / other for non-GEMV tensors
+    parts: List[int]        # tensor indices in row order
+    gemv: bool              # 2-D with a GEMV dtype
+
+
+def matrices(h: wt.Handle) -> List[MatrixRef]:
+    """Group the handle's tensors into logical tensors (row blocks joined), in first-seen order."""
+    out: List[MatrixRef] = []
+    by_name: Dict[str, MatrixRef] = {}
+    blocks: Dict[str, Dict[int, int]] = {}
+    for i, t in enumerate(h.tensors):
+        m = _BLOCK.match(t.name)
+        if not m:
+            ref = MatrixRef(t.name, t.dtype, t.shape, [i],
+                            len(t.shape) == 2 and t.dtype in (wt.WT_F32, wt.WT_BF16, wt.WT_F16))
+            out.append(ref)
+            by_name[t.name] = ref
+            continue
+        base, k = m.group(1), int(m.group(2))
+        blocks.setdefault(base, {})[k] = i
+        if base not in by_name:
+            ref = MatrixRef(base, t.dtype, (), [], False)
+            out.append(ref)
+            by_name[base] = ref
+    for base, parts in blocks.items():
+        ref = by_name[base]
+        idx = [parts[k] for k in sorted(parts)]
+        ts = [h.tensors[i] for i in idx]
+        K = ts[0].shape[1] if len(ts[0].shape) == 2 else None
+        if K is None or any(len(t.shape) != 2 or t.shape[1] != K or t.dtype != ts[0].dtype for t in ts):
+            raise ValueError("row blocks of %s do not stack" % base)
+        ref.parts = idx
+        ref.shape = (sum(t.shape[0] for t in ts), K)
+        ref.gemv = ts[0].dtype in (wt.WT_F32, wt.WT_BF16, wt.WT_F16)
+    return out
+
+
+@dataclass
+class DeviceCheckpoint:
+    mats: List[MatrixRef]
+    bufs: List[object]                   # torch uint8 tensors, one per MatrixRef
+    dst: Dict[int, int] = field(default_factory=dict)  # tensor index -> device address
+    canary: int = 0
+
+    @staticmethod
+    def allocate(h: wt.Handle, mats: Sequence[MatrixRef], device="cuda", canary: int = 0,
+                 slab: bool = True) -> "DeviceCheckpoint":
+        """One device buffer per logical tensor (optionally `canary` spare bytes after each).
+
+        slab=True carves every buffer out of one allocation (256-byte aligned offsets)."""
+        import torch
+        sizes = [sum(h.tensors[i].nbytes for i in m.parts) for m in mats]
+        bufs = []
+        if slab:
+            offs, pos = [], 0
+            for n in sizes:
+                offs.append(pos)
+                pos += -(-(n + canary) // _ALIGN) * _ALIGN
+            big = torch.empty(max(pos, 1), dtype=torch.uint8, device=device)
+            bufs = [big[o:o + n + canary] for o, n in zip(offs, sizes)]
+        else:
+            bufs = [torch.empty(n + canary, dtype=torch.uint8, device=device) for n in sizes]
+        dc = DeviceCheckpoint(list(mats), bufs, canary=canary)
+        for m, b in zip(mats, bufs):
+            off = 0
+            for i in m.parts:
+                dc.dst[i] = b.data_ptr() + off
+                off += h.tensors[i].nbytes
+        return dc
+
+    def adopt(self, h: wt.Handle, mode: int = wt.WT_ADOPT_GATHER, stream: int = 0,
+              order: Optional[Sequence[int]] = None) -> Dict[int, int]:
+        """wt_adopt every tensor (file/index order unless `order`); returns tensor -> event."""
+        idx = list(order) if order is not None else sorted(self.dst)
+        evs = h.adopt(idx, [self.dst[i] for i in idx], mode, stream)
+        return dict(zip(idx, evs))
+
+    def gemv_mats(self) -> List[int]:
+        return [k for k, m in enumerate(self.mats) if m.gemv]
+
+    def inputs(self, device="cuda") -> Dict[tuple, object]:
+        """x per (K, dtype): N(0,1) from the seeded generator, cast to the weight dtype."""
+        import torch
+        xs = {}
+        for k in self.gemv_mats():
+            m = self.mats[k]
+            key = (m.shape[1], m.dtype)
+            if key not in xs:
+                xs[key] = torch.from_numpy(synth.make_x(m.shape[1], m.dtype)).to(device)
+        return xs
+
+    def outputs(self, device="cuda") -> Dict[int, object]:
+        import torch
+        return {k: torch.empty(self.mats[k].shape[0], dtype=torch.float32, device=device)
+                for k in self.gemv_mats()}
+
+    def descs(self, xs, ys, events: Optional[Dict[int, int]] = None,
+              only: Optional[Sequence[int]] = None) -> List[wt.GemvDesc]:
+        out = []
+        pos = {i: n for n, i in enumerate(events)} if events else {}
+        for k in (only if only is not None else self.gemv_mats()):
+            m = self.mats[k]
+            ev = events[max(m.parts, key=pos.__getitem__)] if events else 0
+            out.append(wt.gemv_desc(self.bufs[k].data_ptr(), m.dtype, m.shape[0], m.shape[1],
+                                    xs[(m.shape[1], m.dtype)].data_ptr(), ys[k].data_ptr(), ev))
+        return out
+
+    @property
+    def weight_bytes(self) -> int:
+        return sum(int(np.prod(self.mats[k].shape)) * _ESZ[self.mats[k].dtype] for k in self.gemv_mats())
+
+    @property
+    def data_bytes(self) -> int:
+        return sum(int(b.numel()) - self.canary for b in self.bufs)

@@ -1,0 +1,196 @@
+"""Thin ctypes binding of libwt.so (include/wt.h), same names as the C ABI.
+
+Argument marshalling only: every step of the path runs in the library's C++
+and CUDA code.  Pointers are plain integers (``tensor.data_ptr()``), streams
+are ``torch.cuda.Stream.cuda_stream`` integers; PyTorch supplies device memory
+and streams and nothing else.  There is no fallback: if the library cannot be
+loaded, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+from dataclasses import dataclass
+from typing import List, Optional, Sequence, Tuple
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libwt.so")
+
+WT_OK, WT_EINVAL, WT_EIO, WT_EFORMAT, WT_ENOMEM, WT_ECUDA, WT_ENOTSUP, WT_ETIMEDOUT = 0, -1, -2, -3, -4, -5, -6, -7
+WT_F32, WT_BF16, WT_F16, WT_I8, WT_U8 = 0, 1, 2, 3, 4
+WT_ROUTE_AUTO, WT_ROUTE_REGISTER, WT_ROUTE_DIRECT, WT_ROUTE_NONE = 0, 1, 2, 3
+WT_OPEN_HOST_ONLY, WT_OPEN_PREFAULT = 1 << 4, 1 << 5
+WT_ADOPT_GATHER, WT_ADOPT_CE, WT_ADOPT_STAGED = 0, 1, 2
+ROUTE_NAMES = {WT_ROUTE_REGISTER: "register", WT_ROUTE_DIRECT: "direct", WT_ROUTE_NONE: "none"}
+MODE_NAMES = {WT_ADOPT_GATHER: "gather", WT_ADOPT_CE: "ce", WT_ADOPT_STAGED: "staged"}
+
+# every entry point declared in include/wt.h
+SYMBOLS = ("wt_last_error", "wt_abi_version", "wt_open", "wt_num_tensors", "wt_num_files",
+           "wt_tensor_info", "wt_find", "wt_file_route", "wt_adopt", "wt_pass", "wt_checksum",
+           "wt_checksum_plain", "wt_device_status", "wt_kernel_launches", "wt_close")
+
+
+class WtError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__("wt error %d: %s" % (code, msg))
+        self.code = code
+
+
+class TensorMeta(C.Structure):
+    _fields_ = [("name", C.c_char_p), ("dtype", C.c_int32), ("ndim", C.c_int32),
+                ("shape", C.c_uint64 * 4), ("nbytes", C.c_uint64), ("file", C.c_uint32),
+                ("offset", C.c_uint64), ("host_ptr", C.c_void_p)]
+
+
+class GemvDesc(C.Structure):
+    _fields_ = [("W", C.c_void_p), ("dtype", C.c_int32), ("reserved", C.c_int32),
+                ("M", C.c_uint64), ("K", C.c_uint64), ("x", C.c_void_p), ("y", C.c_void_p),
+                ("wait_event", C.c_void_p)]
+
+
+_lib = None
+
+
+def lib(path: str = LIB_PATH):
+    """Load libwt.so (built by paper_2608_12114_gb300.build).  Raises if it is missing."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError("libwt.so is not built (%s); run paper_2608_12114_gb300.build.build()" % path)
+    L = C.CDLL(path)
+    vp, sz, u64p = C.c_void_p, C.c_size_t, C.POINTER(C.c_uint64)
+    L.wt_last_error.restype = C.c_char_p
+    L.wt_abi_version.restype = C.c_int
+    L.wt_open.argtypes = [C.POINTER(C.c_char_p), C.c_int, C.c_uint, C.POINTER(vp)]
+    L.wt_num_tensors.argtypes = [vp, C.POINTER(sz)]
+    L.wt_num_files.argtypes = [vp, C.POINTER(sz)]
+    L.wt_tensor_info.argtypes = [vp, sz, C.POINTER(TensorMeta)]
+    L.wt_find.argtypes = [vp, C.c_char_p, C.POINTER(sz)]
+    L.wt_file_route.argtypes = [vp, sz, C.POINTER(C.c_uint)]
+    L.wt_adopt.argtypes = [vp, C.POINTER(sz), C.POINTER(vp), sz, C.c_uint, vp, C.POINTER(vp)]
+    L.wt_pass.argtypes = [vp, C.POINTER(GemvDesc), sz, vp]
+    L.wt_checksum.argtypes = [vp, C.POINTER(vp), u64p, sz, vp, vp]
+    L.wt_checksum_plain.argtypes = [vp, C.POINTER(vp), u64p, sz, vp, vp]
+    L.wt_device_status.argtypes = [vp, C.POINTER(C.c_int)]
+    L.wt_kernel_launches.argtypes = [vp, u64p]
+    L.wt_close.argtypes = [vp]
+    for s in SYMBOLS:
+        if s not in ("wt_last_error",):
+            getattr(L, s).restype = C.c_int
+    L.wt_last_error.restype = C.c_char_p
+    _lib = L
+    return L
+
+
+def _check(rc: int):
+    if rc != WT_OK:
+        raise WtError(rc, lib().wt_last_error().decode(errors="replace"))
+
+
+@dataclass
+class TensorInfo:
+    name: str
+    dtype: int
+    shape: Tuple[int, ...]
+    nbytes: int
+    file: int
+    offset: int
+    host_ptr: int
+
+
+class Handle:
+    """An open checkpoint (wt_open ... wt_close)."""
+
+    def __init__(self, paths: Sequence[str], flags: int = 0):
+        L = lib()
+        arr = (C.c_char_p * max(1, len(paths)))(*[p.encode() for p in paths])
+        h = C.c_void_p()
+        _check(L.wt_open(arr, len(paths), flags, C.byref(h)))
+        self._h = h
+        n = C.c_size_t()
+        _check(L.wt_num_tensors(h, C.byref(n)))
+        self.tensors: List[TensorInfo] = []
+        for i in range(n.value):
+            m = TensorMeta()
+            _check(L.wt_tensor_info(h, i, C.byref(m)))
+            self.tensors.append(TensorInfo(m.name.decode(), m.dtype, tuple(m.shape[:m.ndim]), m.nbytes,
+                                           m.file, m.offset, m.host_ptr or 0))
+        nf = C.c_size_t()
+        _check(L.wt_num_files(h, C.byref(nf)))
+        self.n_files = nf.value
+
+    @property
+    def ptr(self):
+        if self._h is None:
+            raise WtError(WT_EINVAL, "handle is closed")
+        return self._h
+
+    def find(self, name: str) -> int:
+        i = C.c_size_t()
+        _check(lib().wt_find(self.ptr, name.encode(), C.byref(i)))
+        return i.value
+
+    def route(self, f: int) -> int:
+        r = C.c_uint()
+        _check(lib().wt_file_route(self.ptr, f, C.byref(r)))
+        return r.value
+
+    def adopt(self, idx: Sequence[int], dst: Sequence[int], mode: int = WT_ADOPT_GATHER,
+              stream: int = 0) -> List[int]:
+        """wt_adopt: returns the ready event (cudaEvent_t as int) of each tensor."""
+        n = len(idx)
+        ia = (C.c_size_t * max(1, n))(*idx)
+        da = (C.c_void_p * max(1, n))(*dst)
+        ra = (C.c_void_p * max(1, n))()
+        _check(lib().wt_adopt(self.ptr, ia, da, n, mode, C.c_void_p(stream), ra))
+        return [ra[i] or 0 for i in range(n)]
+
+    def pass_(self, descs: Sequence[GemvDesc], stream: int = 0):
+        """wt_pass over a list of GemvDesc."""
+        n = len(descs)
+        arr = (GemvDesc * max(1, n))(*descs)
+        _check(lib().wt_pass(self.ptr, arr, n, C.c_void_p(stream)))
+
+    def checksum(self, ptrs: Sequence[int], nbytes: Sequence[int], out_dev: int, stream: int = 0,
+                 plain: bool = False):
+        n = len(ptrs)
+        pa = (C.c_void_p * max(1, n))(*ptrs)
+        na = (C.c_uint64 * max(1, n))(*nbytes)
+        fn = lib().wt_checksum_plain if plain else lib().wt_checksum
+        _check(fn(self.ptr, pa, na, n, C.c_void_p(out_dev), C.c_void_p(stream)))
+
+    def device_status(self) -> int:
+        s = C.c_int()
+        _check(lib().wt_device_status(self.ptr, C.byref(s)))
+        return s.value
+
+    def kernel_launches(self) -> int:
+        v = C.c_uint64()
+        _check(lib().wt_kernel_launches(self.ptr, C.byref(v)))
+        return v.value
+
+    def close(self):
+        if self._h is not None:
+            h, self._h = self._h, None
+            _check(lib().wt_close(h))
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *a):
+        self.close()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def gemv_desc(W: int, dtype: int, M: int, K: int, x: int, y: int, wait_event: int = 0) -> GemvDesc:
+    return GemvDesc(W, dtype, 0, M, K, x, y, wait_event or None)
+
+
+def open(paths: Sequence[str], flags: int = 0) -> Handle:  # noqa: A001 - mirrors wt_open
+    return Handle(paths, flags)

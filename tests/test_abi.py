@@ -1,0 +1,131 @@
+"""The C ABI library loads, exports every entry point of include/wt.h, and its host-side
+parser agrees with the oracle (no GPU needed: WT_OPEN_HOST_ONLY makes no CUDA call)."""
+import os
+import re
+
+import pytest
+
+import oracle
+from paper_2608_12114_gb300 import build, synth, wt
+from tests import _files
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    build.build()
+    return wt.lib()
+
+
+def declared_symbols():
+    src = open(os.path.join(ROOT, "include", "wt.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(wt_[a-z_]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(L):
+    decl = declared_symbols()
+    assert len(decl) >= 15
+    for s in decl:
+        assert hasattr(L, s), s
+    assert sorted(wt.SYMBOLS) == decl
+    assert L.wt_abi_version() == 1
+
+
+def test_only_the_abi_is_exported(L):
+    import subprocess
+    out = subprocess.run(["nm", "-D", "--defined-only", wt.LIB_PATH], capture_output=True, text=True).stdout
+    exported = sorted({l.split()[-1] for l in out.splitlines() if " T " in l})
+    assert exported == declared_symbols()
+
+
+def test_host_only_parse_matches_oracle(L, tmp_path):
+    ck = synth.build("mid", str(tmp_path / "mid"), layers=2, vocab=96)
+    with wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY) as h:
+        assert h.n_files == len(ck.paths)
+        got = [(t.name, t.dtype, t.shape, t.nbytes, t.file, t.offset) for t in h.tensors]
+        want = []
+        for f, p in enumerate(ck.paths):
+            for e in oracle.load(p).entries:
+                want.append((e["name"], e["dtype"], e["shape"], e["nbytes"], f, e["offset"]))
+        assert got == want
+        assert all(h.route(f) == wt.WT_ROUTE_NONE for f in range(h.n_files))
+        assert h.find("layers.1.down") == [t.name for t in h.tensors].index("layers.1.down")
+        with pytest.raises(wt.WtError) as ei:
+            h.find("nope")
+        assert ei.value.code == wt.WT_EINVAL
+
+
+def test_host_ptr_points_at_file_bytes(L, tmp_path):
+    import ctypes
+    ck = synth.build("tiny", str(tmp_path))
+    of = oracle.load(ck.paths[0])
+    with wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY) as h:
+        for i, t in enumerate(h.tensors):
+            assert ctypes.string_at(t.host_ptr, t.nbytes) == of.blob(i).tobytes()
+
+
+@pytest.mark.parametrize("label,img", _files.bad_files(), ids=[b[0] for b in _files.bad_files()])
+def test_rejections_agree_with_oracle(L, tmp_path, label, img):
+    p = str(tmp_path / (label + ".wt"))
+    with open(p, "wb") as f:
+        f.write(img)
+    with pytest.raises(oracle.OracleError):
+        oracle.load(p)
+    with pytest.raises(wt.WtError) as ei:
+        wt.Handle([p], wt.WT_OPEN_HOST_ONLY)
+    assert ei.value.code == wt.WT_EFORMAT
+    assert p in str(ei.value)
+
+
+def test_good_hand_built_file(L, tmp_path):
+    img, (o1, ba), (o2, bb) = _files.good_two_entry()
+    p = str(tmp_path / "g.wt")
+    open(p, "wb").write(img)
+    with wt.Handle([p], wt.WT_OPEN_HOST_ONLY) as h:
+        assert [(t.name, t.shape, t.offset, t.nbytes) for t in h.tensors] == [("a", (2, 4), o1, 16), ("b", (3,), o2, 6)]
+
+
+def test_missing_file_and_bad_arguments(L, tmp_path):
+    with pytest.raises(wt.WtError) as ei:
+        wt.Handle([str(tmp_path / "missing.wt")], wt.WT_OPEN_HOST_ONLY)
+    assert ei.value.code == wt.WT_EIO
+    with pytest.raises(wt.WtError) as ei:
+        wt.Handle([], 1 << 12)
+    assert ei.value.code == wt.WT_EINVAL
+
+
+def test_one_bad_file_leaves_nothing_open(L, tmp_path):
+    ck = synth.build("many", str(tmp_path / "m"), n_matrices=20)
+    bad = str(tmp_path / "bad.wt")
+    open(bad, "wb").write(b"WTCKPT02" + b"\0" * 64)
+    fds0, maps0 = len(os.listdir("/proc/self/fd")), len(open("/proc/self/maps").readlines())
+    for _ in range(5):
+        with pytest.raises(wt.WtError):
+            wt.Handle(ck.paths[:20] + [bad] + ck.paths[20:], wt.WT_OPEN_HOST_ONLY)
+    assert len(os.listdir("/proc/self/fd")) == fds0
+    assert len(open("/proc/self/maps").readlines()) == maps0
+
+
+def test_open_close_cycles_are_flat(L, tmp_path):
+    ck = synth.build("many", str(tmp_path / "c"), n_matrices=10)
+    h = wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY)
+    h.close()
+    fds0, maps0 = len(os.listdir("/proc/self/fd")), len(open("/proc/self/maps").readlines())
+    for _ in range(200):
+        wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY).close()
+    assert len(os.listdir("/proc/self/fd")) == fds0
+    assert len(open("/proc/self/maps").readlines()) == maps0
+
+
+def test_device_calls_refused_on_host_only_handle(L, tmp_path):
+    ck = synth.build("tiny", str(tmp_path))
+    with wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY) as h:
+        with pytest.raises(wt.WtError) as ei:
+            h.adopt([0], [1 << 20])
+        assert ei.value.code == wt.WT_ENOTSUP
+        with pytest.raises(wt.WtError) as ei:
+            h.pass_([wt.gemv_desc(16, wt.WT_F32, 1, 4, 16, 16)])
+        assert ei.value.code == wt.WT_ENOTSUP
+        assert h.device_status() == 0

@@ -1,0 +1,259 @@
+"""GPU parity: the CUDA path, called through the C ABI, against the CPU oracle.
+
+Bytes must match bit for bit (full compare and both FNV digests); every GEMV row
+must satisfy |y - yhat| / sum_j |W_ij x_j| <= 2e-3 (the tolerance the benchmark spec fixes
+for fp32-accumulated bf16 GEMV; fp64 oracle)."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_12114_gb300 import build, pipeline, synth, wt
+
+pytestmark = pytest.mark.gpu
+TOL = 2e-3
+CANARY = 64
+
+
+@pytest.fixture(scope="module")
+def torch():
+    import torch
+    assert torch.cuda.is_available()
+    build.build()
+    wt.lib()
+    torch.cuda.init()
+    return torch
+
+
+def ingest(torch, ck, mode=wt.WT_ADOPT_GATHER, flags=0, stream=None, slab=True):
+    h = wt.Handle(ck.paths, flags)
+    mats = pipeline.matrices(h)
+    dev = pipeline.DeviceCheckpoint.allocate(h, mats, canary=CANARY, slab=slab)
+    for b in dev.bufs:
+        b.fill_(0xA5)
+    torch.cuda.synchronize()
+    s = stream or torch.cuda.Stream()
+    ev = dev.adopt(h, mode, s.cuda_stream)
+    return h, dev, ev, s
+
+
+def check_bytes(torch, h, dev, co):
+    """Full compare of every tensor against the oracle's file bytes, and canaries intact."""
+    for m, b in zip(dev.mats, dev.bufs):
+        got = b.cpu().numpy()
+        want = np.concatenate([co.files[h.tensors[i].file].blob(
+            [e["name"] for e in co.files[h.tensors[i].file].entries].index(h.tensors[i].name)) for i in m.parts]) \
+            if m.parts else np.zeros(0, np.uint8)
+        n = want.size
+        assert np.array_equal(got[:n], want), m.name
+        assert np.all(got[n:n + CANARY] == 0xA5), "canary overwritten after " + m.name
+
+
+def device_digests(torch, h, dev, plain=False):
+    """D_tree (or D_plain) of every tensor, on the device, per tensor index."""
+    idx = sorted(dev.dst)
+    out = torch.zeros(len(idx), dtype=torch.int64, device="cuda")
+    h.checksum([dev.dst[i] for i in idx], [h.tensors[i].nbytes for i in idx], out.data_ptr(), 0, plain=plain)
+    return {i: int(v) & 0xFFFFFFFFFFFFFFFF for i, v in zip(idx, out.cpu().tolist())}
+
+
+def oracle_digests(h, co):
+    d = {}
+    for i, t in enumerate(h.tensors):
+        fo = co.files[t.file]
+        e = [x["name"] for x in fo.entries].index(t.name)
+        d[i] = (oracle.fnv1a64(fo.blob(e)), oracle.fnv_tree(fo.blob(e)))
+    return d
+
+
+def check_gemv(h, dev, co, ys, rows=None):
+    worst = 0.0
+    for k in dev.gemv_mats():
+        m = dev.mats[k]
+        M, K = m.shape
+        W = co.matrix_bytes([h.tensors[i].name for i in m.parts])
+        x = synth.make_x(K, m.dtype)
+        y = ys[k].cpu().numpy().astype(np.float64)
+        if rows is None:
+            yhat, a = oracle.gemv(W, m.dtype, M, K, x)
+            err = oracle.gemv_error(y, yhat, a)
+        else:
+            r = sorted(set([0, M - 1] + [int(v) for v in np.random.default_rng(k).integers(0, M, rows)]))
+            yhat, a = oracle.gemv_rows(W, m.dtype, M, K, x, r)
+            err = oracle.gemv_error(y[r], yhat, a)
+        assert err <= TOL, (m.name, err)
+        worst = max(worst, err)
+    return worst
+
+
+# ----------------------------------------------------------------------------- ingest
+
+@pytest.mark.parametrize("mode", [wt.WT_ADOPT_GATHER, wt.WT_ADOPT_CE, wt.WT_ADOPT_STAGED])
+def test_tiny_ingest_bit_exact_all_modes(torch, tmp_path, mode):
+    ck = synth.build("tiny", str(tmp_path))
+    co = oracle.CheckpointOracle(ck.paths)
+    h, dev, ev, s = ingest(torch, ck, mode)
+    s.synchronize()
+    check_bytes(torch, h, dev, co)
+    assert all(ev[i] for i in ev)
+    od = oracle_digests(h, co)
+    tree, plain = device_digests(torch, h, dev), device_digests(torch, h, dev, plain=True)
+    for i in od:
+        assert (plain[i], tree[i]) == od[i]
+    h.close()
+
+
+@pytest.mark.parametrize("flags", [wt.WT_ROUTE_DIRECT, wt.WT_ROUTE_REGISTER,
+                                   wt.WT_ROUTE_DIRECT | wt.WT_OPEN_PREFAULT])
+def test_routes_give_identical_bytes(torch, tmp_path, flags):
+    ck = synth.build("mid", str(tmp_path), layers=1, vocab=500)
+    co = oracle.CheckpointOracle(ck.paths)
+    h, dev, ev, s = ingest(torch, ck, wt.WT_ADOPT_GATHER, flags)
+    s.synchronize()
+    assert h.route(0) == (flags & 3)
+    check_bytes(torch, h, dev, co)
+    h.close()
+
+
+def test_route_none_needs_staged(torch, tmp_path):
+    ck = synth.build("tiny", str(tmp_path))
+    co = oracle.CheckpointOracle(ck.paths)
+    with pytest.raises(wt.WtError) as ei:
+        ingest(torch, ck, wt.WT_ADOPT_GATHER, wt.WT_ROUTE_NONE)
+    assert ei.value.code == wt.WT_ENOTSUP
+    h, dev, ev, s = ingest(torch, ck, wt.WT_ADOPT_STAGED, wt.WT_ROUTE_NONE)
+    s.synchronize()
+    check_bytes(torch, h, dev, co)
+    h.close()
+
+
+def test_many_halves_land_contiguously(torch, tmp_path):
+    ck = synth.build("many", str(tmp_path), n_matrices=300, workers=4)
+    co = oracle.CheckpointOracle(ck.paths)
+    for mode in (wt.WT_ADOPT_GATHER, wt.WT_ADOPT_CE):
+        h, dev, ev, s = ingest(torch, ck, mode, slab=False)
+        s.synchronize()
+        check_bytes(torch, h, dev, co)
+        od = oracle_digests(h, co)
+        tree = device_digests(torch, h, dev)
+        assert all(tree[i] == od[i][1] for i in od)
+        h.close()
+
+
+def test_destination_inside_mapping_is_refused(torch, tmp_path):
+    ck = synth.build("tiny", str(tmp_path))
+    with wt.Handle(ck.paths) as h:
+        with pytest.raises(wt.WtError) as ei:
+            h.adopt([0], [h.tensors[1].host_ptr])
+        assert ei.value.code == wt.WT_EINVAL
+
+
+# ----------------------------------------------------------------------------- GEMV
+
+SHAPES = [(1, 8), (3, 16), (7, 24), (33, 40), (100, 256), (65, 264), (17, 2048), (9, 2056),
+          (5, 4096), (3, 16384), (10, 16392), (4, 100000), (300, 512), (2, 7), (6, 0), (0, 64)]
+
+
+@pytest.mark.parametrize("dtype", [synth.DT_BF16, synth.DT_F16, synth.DT_F32])
+def test_gemv_shapes_against_oracle(torch, tmp_path, dtype):
+    shapes = SHAPES
+    ck = synth.write_files(synth.custom(str(tmp_path), shapes, dtype=dtype, name="c%d" % dtype))
+    co = oracle.CheckpointOracle(ck.paths)
+    h, dev, ev, s = ingest(torch, ck)
+    xs, ys = dev.inputs(), dev.outputs()
+    for y in ys.values():
+        y.fill_(float("nan"))
+    torch.cuda.synchronize()
+    h.pass_(dev.descs(xs, ys, ev), s.cuda_stream)
+    s.synchronize()
+    check_gemv(h, dev, co, ys)
+    assert h.device_status() == 0
+    h.close()
+
+
+def test_one_hot_x_returns_exact_columns(torch, tmp_path):
+    shapes = [(40, 24), (64, 1024), (9, 2056), (5, 20000)]
+    ck = synth.write_files(synth.custom(str(tmp_path), shapes, dtype=synth.DT_BF16, name="oh"))
+    co = oracle.CheckpointOracle(ck.paths)
+    h, dev, ev, s = ingest(torch, ck)
+    s.synchronize()
+    for k, (M, K) in zip(dev.gemv_mats(), shapes):
+        for j in (0, K // 2 + 3, K - 1):
+            x = torch.zeros(K, dtype=torch.bfloat16, device="cuda")
+            x[j] = 1.0
+            y = torch.empty(M, dtype=torch.float32, device="cuda")
+            h.pass_([wt.gemv_desc(dev.bufs[k].data_ptr(), wt.WT_BF16, M, K, x.data_ptr(), y.data_ptr())], 0)
+            W = co.files[0].blob(k).view("<u2").reshape(M, K)[:, j].astype(np.uint32) << 16
+            assert np.array_equal(y.cpu().numpy().view(np.uint32), W.astype(np.uint32))
+    h.close()
+
+
+def test_grouping_does_not_change_results(torch, tmp_path):
+    ck = synth.build("mid", str(tmp_path), layers=2, vocab=3000)
+    h, dev, ev, s = ingest(torch, ck)
+    xs = dev.inputs()
+    ya, yb = dev.outputs(), dev.outputs()
+    torch.cuda.synchronize()
+    h.pass_(dev.descs(xs, ya, ev), s.cuda_stream)               # grouped by ingest batch
+    for k in dev.gemv_mats():                                     # one matrix per call
+        h.pass_(dev.descs(xs, yb, None, only=[k]), s.cuda_stream)
+    yc = dev.outputs()
+    torch.cuda.synchronize()
+    h.pass_(dev.descs(xs, yc), s.cuda_stream)                     # all in one resident launch
+    s.synchronize()
+    for k in dev.gemv_mats():
+        assert torch.equal(ya[k], yb[k]) and torch.equal(ya[k], yc[k])
+    h.close()
+
+
+def test_first_use_pipeline_mid(torch, tmp_path):
+    """Ingest on one stream, consume on another gated only by per-batch events."""
+    ck = synth.build("mid", str(tmp_path), layers=3, workers=4)
+    co = oracle.CheckpointOracle(ck.paths)
+    ingest_s, consume_s = torch.cuda.Stream(), torch.cuda.Stream()
+    h = wt.Handle(ck.paths)
+    dev = pipeline.DeviceCheckpoint.allocate(h, pipeline.matrices(h))
+    xs, ys = dev.inputs(), dev.outputs()
+    torch.cuda.synchronize()
+    ev = dev.adopt(h, wt.WT_ADOPT_GATHER, ingest_s.cuda_stream)
+    h.pass_(dev.descs(xs, ys, ev), consume_s.cuda_stream)  # no host wait between the two
+    consume_s.synchronize()
+    check_gemv(h, dev, co, ys)
+    yr = dev.outputs()
+    torch.cuda.synchronize()
+    h.pass_(dev.descs(xs, yr), consume_s.cuda_stream)
+    consume_s.synchronize()
+    for k in dev.gemv_mats():
+        assert torch.equal(ys[k], yr[k])
+    h.close()
+
+
+# ----------------------------------------------------------------------------- checksums
+
+def test_checksum_edges(torch):
+    rng = np.random.default_rng(7)
+    data = rng.integers(0, 256, 3 * 4096 + 100, dtype=np.uint8)
+    buf = torch.from_numpy(data).cuda()
+    cases = [(0, 0), (0, 1), (1, 15), (3, 4095), (0, 4096), (0, 4097), (5, 8192 + 17), (16, 3 * 4096 + 84)]
+    base = buf.data_ptr()
+    for plain in (False, True):
+        with wt.Handle([]) as h:
+            out = torch.zeros(len(cases), dtype=torch.int64, device="cuda")
+            h.checksum([base + o for o, n in cases], [n for o, n in cases], out.data_ptr(), 0, plain=plain)
+            got = [int(v) & (2 ** 64 - 1) for v in out.cpu().tolist()]
+        fn = oracle.fnv1a64 if plain else oracle.fnv_tree
+        assert got == [fn(data[o:o + n]) for o, n in cases]
+
+
+def test_checksum_many_buffers(torch):
+    """More buffers than one launch carries (the host splits them into batches)."""
+    n = 600
+    rng = np.random.default_rng(8)
+    sizes = rng.integers(0, 9000, n)
+    data = rng.integers(0, 256, int(sizes.sum()) + 64, dtype=np.uint8)
+    buf = torch.from_numpy(data).cuda()
+    offs = np.concatenate([[0], np.cumsum(sizes)[:-1]])
+    with wt.Handle([]) as h:
+        out = torch.zeros(n, dtype=torch.int64, device="cuda")
+        h.checksum([buf.data_ptr() + int(o) for o in offs], [int(s) for s in sizes], out.data_ptr(), 0)
+        got = [int(v) & (2 ** 64 - 1) for v in out.cpu().tolist()]
+    assert got == [oracle.fnv_tree(data[o:o + s]) for o, s in zip(offs, sizes)]
