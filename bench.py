@@ -1,0 +1,554 @@
+"""Benchmark of the file-backed weight path on GB300 (one JSON line on stdout).
+
+Metric: file -> first-use ingest GB/s, and resident GEMV-pass GB/s against HBM peak.
+
+  value   resident pass: every matrix of the checkpoint through the persistent
+          TMA-fed GEMV (one launch per pass), weights already in HBM; weight
+          bytes / time (the paper's convention: weight bytes counted once).
+  e2e     file -> first use through the C ABI: wt_open (parse, map, route),
+          wt_adopt (host-mapped pages -> HBM, per-batch events), the
+          event-gated first GEMV pass, and the device -> host read of every y;
+          ingested data bytes / wall time.  Page cache warm (the paper's
+          precondition for adoption).
+
+A step is one resident pass over the whole checkpoint.  Inputs (16 GB for the
+default workload) are far larger than L2, so no flush is needed between passes.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload large|mid|many|sweep:I|tiny]
+  python bench.py --impl reference ...   # the CPU oracle on a bounded sample (the reference arm)
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "file→first-use ingest GB/s; resident GEMV-pass GB/s vs HBM peak (%)"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+WORKLOADS = {
+    "large": "large decoder checkpoint, bf16, 4 shards (16.06 GB): 32 layers, d=4096, kv 1024, FFN 14336, vocab 128256",
+    "mid": "mid decoder checkpoint, bf16, 3 shards (5.40 GB): 32 layers, d=2560, FFN 6912, vocab 32000",
+    "many": "many-small: 1253 bf16 matrices split by rows across 2506 files (1.56 GB)",
+    "tiny": "tiny: 8 fp32 256x256 matrices + 8 fp32[256] vectors in one file (2.1 MB)",
+}
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=400, help="timed resident passes")
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="wt", choices=["wt", "reference"])
+    p.add_argument("--workload", default="large")
+    p.add_argument("--layers", type=int, default=None, help="override decoder layer count (small profiling cases)")
+    p.add_argument("--mode", default="gather", choices=["gather", "ce", "staged"])
+    p.add_argument("--e2e-reps", type=int, default=5)
+    p.add_argument("--arms", action="store_true", help="also time the ce/staged/stock-torch ingest arms")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=15.0, help="CPU budget of the oracle sample")
+    p.add_argument("--data-dir", default=None)
+    p.add_argument("--workers", type=int, default=0)
+    return p.parse_args()
+
+
+# ----------------------------------------------------------------------------- workload files
+
+def workload_ck(args, outdir):
+    from paper_2608_12114_gb300 import synth
+    w = args.workload
+    if w.startswith("sweep:"):
+        return synth.sweep(outdir, points=[int(w.split(":")[1])])
+    if w == "tiny":
+        return synth.tiny(outdir)
+    if w == "many":
+        return synth.many(outdir)
+    if w in ("mid", "large"):
+        return synth.decoder(outdir, w, layers=args.layers)
+    raise SystemExit("unknown workload " + w)
+
+
+def workload_desc(args):
+    w = args.workload
+    if w.startswith("sweep:"):
+        i = int(w.split(":")[1])
+        return "size sweep point %d: one bf16 4096x%d matrix (%d MiB)" % (i, 128 << i, 1 << i)
+    d = WORKLOADS[w]
+    if args.layers is not None:
+        d += " (reduced to %d layers)" % args.layers
+    return d
+
+
+def make_files(args, rank, world):
+    """Rank 0 writes the workload (spawned workers, before any CUDA call); all ranks share it."""
+    from paper_2608_12114_gb300 import synth
+    base = args.data_dir or os.path.join(tempfile.gettempdir(), "wt_bench")
+    outdir = os.path.join(base, args.workload.replace(":", "_") + ("_l%d" % args.layers if args.layers else ""))
+    ck = workload_ck(args, outdir)
+    t0 = time.time()
+    if rank == 0:
+        workers = args.workers or min(16, os.cpu_count() or 1)
+        synth.write_files(ck, workers=workers)
+        os.sync()
+    gen_s = time.time() - t0
+    return ck, gen_s
+
+
+# ----------------------------------------------------------------------------- measurement helpers
+
+class Clocks:
+    """nvidia-smi samples of SM clock and throttle reasons, taken while the timed region runs."""
+
+    Q = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, bus_id):
+        self.bus_id = bus_id
+        self.p = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        cmd = ["nvidia-smi", "--query-gpu=" + self.Q, "--format=csv,noheader,nounits", "-lms", "50"]
+        if self.bus_id:
+            cmd += ["-i", self.bus_id]
+        try:
+            self.p = subprocess.Popen(cmd, stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.p = None
+        time.sleep(0.5)
+        self.t0 = time.time()
+        return self
+
+    def __exit__(self, *a):
+        self.t1 = time.time()
+        if self.p:
+            time.sleep(0.15)
+            self.p.terminate()
+            self.p.wait()
+
+    def summary(self):
+        import datetime
+        rows = []
+        if self.path and os.path.exists(self.path):
+            for line in open(self.path):
+                f = [x.strip() for x in line.split(",")]
+                if len(f) < 9:
+                    continue
+                try:
+                    ts = datetime.datetime.strptime(f[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                except ValueError:
+                    continue
+                if self.t0 - 0.05 <= ts <= self.t1 + 0.05:
+                    rows.append(f)
+            os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        def num(v):
+            try:
+                return float(v)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.strip().lower() == "active"})
+        pw = [num(r[3]) for r in rows if num(r[3]) is not None]
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None}
+
+
+def bus_id():
+    try:
+        import torch
+        pr = torch.cuda.get_device_properties(torch.cuda.current_device())
+        return "%08X:%02X:%02X.0" % (pr.pci_domain_id, pr.pci_bus_id, pr.pci_device_id)
+    except Exception:
+        return None
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        try:
+            d = json.load(open(p))
+            return float(d["hbm_gbs"]), "measured"
+        except Exception:
+            pass
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def pinned_h2d_gbs(torch, nbytes=1 << 30, reps=10):
+    """Copy-engine H2D from a pinned (cudaMallocHost) buffer, best of `reps`: the ingest roofline."""
+    h = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+    h.fill_(1)
+    d = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    s = torch.cuda.Stream()
+    best = 1e30
+    with torch.cuda.stream(s):
+        for _ in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(s)
+            d.copy_(h, non_blocking=True)
+            b.record(s)
+            b.synchronize()
+            best = min(best, a.elapsed_time(b))
+    del h, d
+    return nbytes / best / 1e6
+
+
+def kernel_traffic(name):
+    """DRAM bytes per launch from the committed ncu summary, if it matches the current kernels."""
+    p = os.path.join(ROOT, "profiles", name)
+    if not os.path.exists(p):
+        return None
+    try:
+        d = json.load(open(p))
+    except Exception:
+        return None
+    src = os.path.join(ROOT, "paper_2608_12114_gb300", "csrc", "wt_kernels.cu")
+    digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    if d.get("kernel_source_sha256_16") != digest:
+        return None
+    return d
+
+
+# ----------------------------------------------------------------------------- the wt arm
+
+def first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab):
+    """One file -> first-use run; returns (seconds, handle stats)."""
+    t0 = time.perf_counter()
+    h = wt.Handle(ck.paths)
+    mats = pipeline.matrices(h)
+    dev = slab["dev"]
+    ev = dev.adopt(h, mode, ingest_s.cuda_stream)
+    h.pass_(dev.descs(slab["xs"], slab["ys"], ev), consume_s.cuda_stream)
+    with torch.cuda.stream(consume_s):
+        y_host.copy_(slab["yflat"], non_blocking=True)
+    consume_s.synchronize()
+    dt = time.perf_counter() - t0
+    launches = h.kernel_launches()
+    status = h.device_status()
+    h.close()
+    return dt, launches, status, len(mats)
+
+
+def run_wt(args, rank, world):
+    ck, gen_s = make_files(args, rank, world)
+    import torch
+    from paper_2608_12114_gb300 import build, pipeline, wt
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        dist.barrier()
+    if rank == 0:
+        build.build()
+    if dist:
+        dist.barrier()
+    build.build()  # no-op when fresh; loads the same in-tree library on every rank
+    mode = {"gather": wt.WT_ADOPT_GATHER, "ce": wt.WT_ADOPT_CE, "staged": wt.WT_ADOPT_STAGED}[args.mode]
+
+    h2d = pinned_h2d_gbs(torch)
+    log("pinned H2D %.1f GB/s; files %.2f GB generated in %.1f s" % (h2d, ck.data_bytes / 1e9, gen_s))
+
+    # device buffers, x and y are allocated once (a user allocates them once too)
+    h0 = wt.Handle(ck.paths)
+    mats = pipeline.matrices(h0)
+    dev = pipeline.DeviceCheckpoint.allocate(h0, mats)
+    xs = dev.inputs()
+    rows = [mats[k].shape[0] for k in dev.gemv_mats()]
+    yflat = torch.empty(sum(rows), dtype=torch.float32, device="cuda")
+    ys, o = {}, 0
+    for k, r in zip(dev.gemv_mats(), rows):
+        ys[k] = yflat[o:o + r]
+        o += r
+    slab = {"dev": dev, "xs": xs, "ys": ys, "yflat": yflat}
+    y_host = torch.empty(sum(rows), dtype=torch.float32, pin_memory=True)
+    weight_bytes = dev.weight_bytes
+    data_bytes = ck.data_bytes
+    alg_bytes = sum(dev.mats[k].shape[0] * dev.mats[k].shape[1] * 2 + dev.mats[k].shape[1] * 2 + 4 * dev.mats[k].shape[0]
+                    for k in dev.gemv_mats()) if all(dev.mats[k].dtype == wt.WT_BF16 for k in dev.gemv_mats()) else None
+    h0.close()
+    torch.cuda.synchronize()
+
+    ingest_s, consume_s = torch.cuda.Stream(), torch.cuda.Stream()
+
+    # ---------------- e2e: file -> first use (1 warm-up, then timed repetitions)
+    e2e_times, e2e_launches = [], 0
+    for rep in range(1 + args.e2e_reps):
+        if dist:
+            dist.barrier()
+        dt, nl, st, nm = first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab)
+        if st != 0:
+            raise SystemExit("device status %d after first-use run" % st)
+        if rep > 0:
+            e2e_times.append(dt)
+            e2e_launches = nl
+    e2e_s = statistics.median(e2e_times)
+    e2e_gbs = data_bytes / e2e_s / 1e9
+    log("file->first-use: %.1f ms median (%s), %.1f GB/s = %.1f%% of pinned H2D" % (
+        e2e_s * 1e3, ", ".join("%.1f" % (t * 1e3) for t in e2e_times), e2e_gbs, 100 * e2e_gbs / h2d))
+
+    arms = {}
+    if args.arms:
+        for name, m in (("gather", wt.WT_ADOPT_GATHER), ("ce", wt.WT_ADOPT_CE), ("staged", wt.WT_ADOPT_STAGED)):
+            ts = [first_use(torch, wt, pipeline, ck, m, ingest_s, consume_s, y_host, slab)[0] for _ in range(3)]
+            arms[name] = round(data_bytes / min(ts) / 1e9, 1)
+        arms["stock_torch"] = round(stock_torch_arm(torch, ck, wt, pipeline) / 1e9, 1)
+        log("ingest arms GB/s:", arms)
+
+    # ---------------- resident pass: the steady-state consumer
+    h = wt.Handle(ck.paths)
+    ev = dev.adopt(h, mode, ingest_s.cuda_stream)
+    ingest_s.synchronize()
+    descs = dev.descs(xs, ys)
+    s = consume_s
+    for _ in range(args.warmup):
+        h.pass_(descs, s.cuda_stream)
+    s.synchronize()
+    n0 = h.kernel_launches()
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with Clocks(bus_id()) as clk:
+        evs[0].record(s)
+        for i in range(args.steps):
+            h.pass_(descs, s.cuda_stream)
+            evs[i + 1].record(s)
+        s.synchronize()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    launches = h.kernel_launches() - n0
+    per = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
+    total_ms = evs[0].elapsed_time(evs[-1])
+    status = h.device_status()
+    h.close()
+    if status != 0:
+        raise SystemExit("device status %d after resident passes" % status)
+
+    if dist:
+        t = torch.tensor([total_ms, e2e_s], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms, e2e_s_max = t.tolist()
+    else:
+        e2e_s_max = e2e_s
+    ms_per_step = total_ms / args.steps
+    value = weight_bytes * args.steps * world / (total_ms / 1e3) / 1e9
+    launches_per_pass = launches / args.steps
+    avg_launch_ms = statistics.mean(per) if launches_per_pass == 1 else None
+    peak, peak_kind = measured_peaks()
+    roof = None
+    if avg_launch_ms and alg_bytes:
+        achieved = alg_bytes / (avg_launch_ms / 1e3) / 1e9
+        tr = kernel_traffic("gemv_tma_large_traffic.json") if args.workload == "large" else None
+        roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
+                "traffic": (tr["dram_bytes_per_launch_full"] if tr else None),
+                "algorithmic_bytes_per_launch": alg_bytes,
+                "kernel": "gemv_tma_kernel<bf16>",
+                "frac_of_nominal_8TBps": round(achieved / NOMINAL_HBM_GBS, 4)}
+    clocks = clk.summary()
+    out = {
+        "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,0.02) bf16 weights, norms 1.0, x ~ N(0,1))",
+        "config": {"workload": workload_desc(args), "weight_bytes": weight_bytes, "data_bytes": data_bytes,
+                   "files": len(ck.paths), "matrices": len(dev.gemv_mats()), "ingest_mode": args.mode,
+                   "l2": "inputs larger than L2 (no flush)", "parallelism": "replicas" if world > 1 else "1 GPU"},
+        "resident_frac_of_hbm": {"measured": round(value / world / peak, 4), "nominal_8TBps": round(value / world / NOMINAL_HBM_GBS, 4)},
+        "clocks": clocks,
+        "e2e": {"value": round(data_bytes * world / e2e_s_max / 1e9, 1), "unit": "GB/s",
+                "h2d_bytes_per_step": data_bytes, "d2h_bytes_per_step": int(y_host.numel() * 4),
+                "ms": round(e2e_s * 1e3, 2), "pinned_h2d_gbs": round(h2d, 1),
+                "frac_of_pinned_h2d": round(e2e_gbs / h2d, 4), "reps": args.e2e_reps,
+                "what": "wt_open + wt_adopt + event-gated first pass + D2H of all y, page cache warm",
+                "launches_per_run": e2e_launches},
+        "gpu_launches": int(launches),
+        "roofline": roof,
+    }
+    if arms:
+        out["ingest_arms_gbs"] = arms
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(args, ck, args.cpu_seconds)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def stock_torch_arm(torch, ck, wt, pipeline):
+    """The stock path: file bytes -> CPU tensor -> .to('cuda') per tensor, then F.linear."""
+    import numpy as np
+    h = wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    total = 0
+    for f, p in enumerate(ck.paths):
+        mm = np.memmap(p, dtype=np.uint8, mode="r")
+        for t in h.tensors:
+            if t.file != f:
+                continue
+            cpu = torch.from_numpy(np.array(mm[t.offset:t.offset + t.nbytes]))
+            g = cpu.to("cuda")
+            if len(t.shape) == 2 and t.dtype == wt.WT_BF16:
+                W = g.view(torch.bfloat16).view(t.shape)
+                x = torch.ones(t.shape[1], dtype=torch.bfloat16, device="cuda")
+                torch.nn.functional.linear(x, W)
+            total += t.nbytes
+        del mm
+    torch.cuda.synchronize()
+    h.close()
+    return total / (time.perf_counter() - t0)
+
+
+# ----------------------------------------------------------------------------- the oracle (CPU)
+
+class OracleSample:
+    """The oracle, as it stands, walking the workload's matrices in layer order in row blocks.
+
+    Files are parsed (read in full, index decoded) when the walk first reaches them; every
+    block is an fp64 GEMV of up to 1024 rows.  run(budget) stops after `budget_s` of work."""
+
+    BLOCK = 1024
+
+    def __init__(self, ck):
+        import oracle
+        oracle.build()
+        self.oracle = oracle
+        self.ck = ck
+        self.files = {}
+        self.parse_s = 0.0
+        self.parsed = 0
+        self.m = 0
+        self.r = 0
+        self.xs = {}
+
+    def _blob(self, i):
+        t = self.ck.tensors[i]
+        if t.file not in self.files:
+            t0 = time.perf_counter()
+            fo = self.oracle.load(self.ck.paths[t.file])
+            self.parse_s += time.perf_counter() - t0
+            self.parsed += fo.size
+            self.files[t.file] = (fo, {e["name"]: k for k, e in enumerate(fo.entries)})
+        fo, names = self.files[t.file]
+        return fo.blob(names[t.name])
+
+    def run(self, budget_s):
+        """GEMV row blocks until the budget is spent; returns (weight bytes, GEMV seconds)."""
+        import numpy as np
+        from paper_2608_12114_gb300 import synth
+        done_b, gemv_s = 0, 0.0
+        t_end = time.perf_counter() + budget_s
+        while time.perf_counter() < t_end:
+            m = self.ck.matrices[self.m]
+            blobs = [self._blob(i) for i in m.parts]
+            W = blobs[0] if len(blobs) == 1 else np.concatenate(blobs)
+            key = (m.K, m.dtype)
+            if key not in self.xs:
+                self.xs[key] = synth.make_x(m.K, m.dtype)
+            r1 = min(m.M, self.r + self.BLOCK)
+            t0 = time.perf_counter()
+            self.oracle.gemv_rows(W, m.dtype, m.M, m.K, self.xs[key], range(self.r, r1))
+            gemv_s += time.perf_counter() - t0
+            done_b += (r1 - self.r) * m.K * synth.ELEM_SIZE[m.dtype]
+            self.r = r1
+            if self.r == m.M:
+                self.m, self.r = (self.m + 1) % len(self.ck.matrices), 0
+        return done_b, gemv_s
+
+    def close(self):
+        for fo, _ in self.files.values():
+            fo.close()
+        self.files = {}
+
+    def describe(self, wbytes):
+        return ("oracle walk over the workload's matrices in layer order, %.2f GB of weights in "
+                "1024-row blocks (%d of %d files parsed, %.2f GB read at %.2f GB/s)" % (
+                    wbytes / 1e9, len(self.files), len(self.ck.paths), self.parsed / 1e9,
+                    self.parsed / self.parse_s / 1e9 if self.parse_s else 0.0))
+
+
+def cpu_baseline(args, ck, budget_s):
+    """The oracle on the host cores over a bounded sample (about `budget_s` of CPU work)."""
+    o = OracleSample(ck)
+    wb, gs = o.run(budget_s)
+    desc = o.describe(wb)
+    parse_rate = o.parsed / o.parse_s if o.parse_s else None
+    o.close()
+    gemv_rate = wb / gs if gs else None
+    first = (1.0 / (1.0 / parse_rate + 1.0 / gemv_rate)) if parse_rate and gemv_rate else None
+    return {"value": round(gemv_rate / 1e9, 4) if gemv_rate else None, "unit": "GB/s", "cores": 1,
+            "kind": "oracle", "sample": desc + "; value = fp64 GEMV weight GB/s",
+            "cores_available": len(os.sched_getaffinity(0)),
+            "parse_gbs": round(parse_rate / 1e9, 3) if parse_rate else None,
+            "first_use_gbs": round(first / 1e9, 4) if first else None}
+
+
+def run_reference(args, rank, world):
+    """The reference arm: the CPU oracle as it stands, on the same workload, metric and unit.
+    Each step is a bounded slice of the oracle's walk; the run stays within a few minutes."""
+    if rank != 0:
+        return
+    ck, gen_s = make_files(args, 0, 1)
+    steps, warm = max(1, args.steps), max(0, args.warmup)
+    budget = min(10.0, max(0.05, 150.0 / (steps + warm)))
+    o = OracleSample(ck)
+    rates, tot_b, tot_s = [], 0, 0.0
+    for i in range(warm + steps):
+        wb, gs = o.run(budget)
+        if i >= warm and gs > 0:
+            rates.append(wb / gs)
+            tot_b += wb
+            tot_s += gs
+    desc = o.describe(tot_b)
+    parse_rate = o.parsed / o.parse_s if o.parse_s else None
+    o.close()
+    v = statistics.median(rates) / 1e9
+    first = 1.0 / (1.0 / parse_rate + 1.0 / (tot_b / tot_s)) / 1e9 if parse_rate else None
+    cb = {"value": round(v, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+          "sample": "%d steps of %.2f s each: %s" % (steps, budget, desc)}
+    out = {"impl": "reference", "metric": METRIC, "value": round(v, 4), "unit": "GB/s", "n_gpus": 1,
+           "steps": steps, "warmup": warm, "ms_per_step": round(tot_s / max(1, len(rates)) * 1e3, 2),
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic", "config": {"workload": workload_desc(args)}, "cpu_baseline": cb,
+           "e2e": {"value": round(first, 4) if first else None, "unit": "GB/s",
+                   "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0,
+                   "what": "1 / (1/parse GB/s + 1/GEMV GB/s) of the oracle"}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    args = parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    run_wt(args, rank, world)
+
+
+if __name__ == "__main__":
+    main()

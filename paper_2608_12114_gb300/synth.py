@@ -45,7 +45,7 @@ ELEM_SIZE = {DT_F32: 4, DT_BF16: 2, DT_F16: 2, DT_I8: 1, DT_U8: 1}
 
 # spawn-key prefixes for the per-tensor value streams of each workload
 _STREAM_KEY = {"many": 1, "sweep": 2, "mid": 3, "large": 4, "custom": 5}
-_CHUNK = 1 << 22  # values drawn per generator call (fixed so streams are reproducible)
+_CHUNK = 1 << 24  # elements per value stream (each chunk of a tensor has its own stream)
 
 
 @dataclasses.dataclass
@@ -100,20 +100,54 @@ class Checkpoint:
 # --------------------------------------------------------------------------- values
 
 def f32_to_bf16_bits(a: np.ndarray) -> np.ndarray:
-    """Round float32 values to bfloat16 bit patterns, round-to-nearest-even."""
-    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32).astype(np.uint64)
-    r = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    """Round finite float32 values to bfloat16 bit patterns, round-to-nearest-even."""
+    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32)
+    r = (u >> 16) & 1
+    r += 0x7FFF
+    r += u          # finite inputs stay below 2^32
+    r >>= 16
     return r.astype(np.uint16)
 
 
+_BUFS: Dict[str, np.ndarray] = {}
+
+
+def _buf(name: str, dtype, count: int) -> np.ndarray:
+    """Per-process scratch arrays, reused across chunks (fresh pages are slow to fault in)."""
+    b = _BUFS.get(name)
+    if b is None or b.size < count:
+        b = _BUFS[name] = np.empty(max(count, _CHUNK), dtype)
+    return b[:count]
+
+
+def _normal_bf16(rng, count: int, scale: float) -> np.ndarray:
+    """N(0, scale) drawn in float32, rounded to bf16 (RNE), as little-endian bytes; in place."""
+    v = _buf("f32", np.float32, count)
+    rng.standard_normal(out=v, dtype=np.float32)
+    v *= np.float32(scale)
+    u = v.view(np.uint32)
+    r = _buf("u32", np.uint32, count)
+    np.right_shift(u, np.uint32(16), out=r)
+    r &= np.uint32(1)
+    r += np.uint32(0x7FFF)
+    r += u
+    r >>= np.uint32(16)
+    o = _buf("u16", np.uint16, count)
+    np.copyto(o, r, casting="unsafe")
+    return o.view(np.uint8)
+
+
 def _tensor_values(t: TensorSpec, start: int, count: int, rng) -> np.ndarray:
-    """Draw `count` values (the next ones of `rng`) for `t` as raw little-endian element bytes."""
+    """`count` values of `t` starting at element `start`, as raw little-endian element bytes."""
+    if t.fill == "normal" and t.dtype == DT_BF16:
+        return _normal_bf16(rng, count, t.scale)
     if t.fill == "ones":
         v = np.ones(count, dtype=np.float32)
     elif t.fill == "uniform":
-        v = (rng.uniform(-t.scale, t.scale, count)).astype(np.float32)
+        v = rng.uniform(-t.scale, t.scale, count).astype(np.float32)
     elif t.fill == "normal":
-        v = (rng.standard_normal(count) * t.scale).astype(np.float32)
+        v = rng.standard_normal(count, dtype=np.float32)
+        v *= np.float32(t.scale)
     elif t.fill == "array":
         return np.ascontiguousarray(t.array).reshape(-1).view(np.uint8)[
             start * ELEM_SIZE[t.dtype]:(start + count) * ELEM_SIZE[t.dtype]]
@@ -128,8 +162,9 @@ def _tensor_values(t: TensorSpec, start: int, count: int, rng) -> np.ndarray:
     raise ValueError("no value recipe for dtype %d" % t.dtype)
 
 
-def _rng_for(t: TensorSpec):
-    return np.random.Generator(np.random.PCG64(np.random.SeedSequence(0, spawn_key=t.key)))
+def _rng_for(t: TensorSpec, chunk: int):
+    """Value stream of chunk `chunk` (of _CHUNK elements) of tensor `t`."""
+    return np.random.Generator(np.random.PCG64(np.random.SeedSequence(0, spawn_key=t.key + (chunk,))))
 
 
 def make_x(K: int, dtype: int) -> np.ndarray:
@@ -172,24 +207,24 @@ def layout(entries: Sequence[TensorSpec]) -> Tuple[bytes, int]:
     return MAGIC + struct.pack("<Q", idx_len) + idx, end
 
 
-def _write_tensor(path: str, t: TensorSpec) -> None:
+def _write_chunk(path: str, t: TensorSpec, c: int) -> int:
+    """Write elements [c*_CHUNK, (c+1)*_CHUNK) of `t`; each chunk draws from its own stream."""
+    es = ELEM_SIZE[t.dtype]
+    n = t.nbytes // es
+    s = c * _CHUNK
+    cnt = min(_CHUNK, n - s)
+    rng = _rng_for(t, c) if t.fill in ("normal", "uniform") else None
+    buf = np.ascontiguousarray(_tensor_values(t, s, cnt, rng))
     fd = os.open(path, os.O_WRONLY)
     try:
-        n = t.nbytes // ELEM_SIZE[t.dtype] if t.nbytes else 0
-        rng = _rng_for(t) if t.fill in ("normal", "uniform") else None
-        es = ELEM_SIZE[t.dtype]
-        for s in range(0, n, _CHUNK):
-            c = min(_CHUNK, n - s)
-            buf = _tensor_values(t, s, c, rng)
-            os.pwrite(fd, np.ascontiguousarray(buf), t.offset + s * es)
+        os.pwrite(fd, buf, t.offset + s * es)
     finally:
         os.close(fd)
+    return cnt * es
 
 
 def _write_task(args):
-    path, t = args
-    _write_tensor(path, t)
-    return t.nbytes
+    return _write_chunk(*args)
 
 
 def write_files(ck: Checkpoint, workers: int = 0) -> Checkpoint:
@@ -205,12 +240,14 @@ def write_files(ck: Checkpoint, workers: int = 0) -> Checkpoint:
         with open(path, "wb") as fh:
             fh.truncate(size)
             fh.write(head)
-        tasks += [(path, ck.tensors[i]) for i in idxs if ck.tensors[i].nbytes]
-    tasks.sort(key=lambda a: -a[1].nbytes)
+        for i in idxs:
+            t = ck.tensors[i]
+            n = t.nbytes // ELEM_SIZE[t.dtype]
+            tasks += [(path, t, c) for c in range(-(-n // _CHUNK))]
     if workers and workers > 1 and len(tasks) > 1:
         import multiprocessing as mp
         with mp.get_context("spawn").Pool(min(workers, len(tasks))) as pool:
-            for _ in pool.imap_unordered(_write_task, tasks, chunksize=1):
+            for _ in pool.imap_unordered(_write_task, tasks, chunksize=max(1, len(tasks) // (8 * workers))):
                 pass
     else:
         for a in tasks:
