@@ -185,6 +185,23 @@ int wt_checksum(wt_handle *h, const void *const *ptr, const uint64_t *nbytes, si
 int wt_checksum_plain(wt_handle *h, const void *const *ptr, const uint64_t *nbytes, size_t n,
                       uint64_t *out_dev, void *stream);
 
+/* Leaf-tree digests exactly as wt_checksum computes them, for callers that must
+ * not allocate device memory: code inside an allocator hook (it would re-enter
+ * the allocator it serves), programs whose device memory is all handed to
+ * their own pool, and loops that cannot take the device-wide synchronisation
+ * of cudaFree.  The paper has no counterpart; this is a library convenience.
+ * No handle is needed.  The leaf digests live in an 8 MiB array compiled into
+ * the library (every GPU that loads the library keeps it until exit); a call
+ * whose buffers need more than 1,048,576 leaves of 4096 bytes (4 GiB of input
+ * in total) is rejected with WT_EINVAL.  The first call on each device looks
+ * up that array's device address (cudaGetSymbolAddress) with the device
+ * current; make that first call before any stream capture.  Calls share the
+ * array, so two calls whose kernels overlap on the GPU race; calls ordered on
+ * one stream do not.  Nothing in the array needs clearing between calls.
+ * Errors: WT_EINVAL (NULL array or buffer, too large), WT_ECUDA. */
+int wt_checksum_noalloc(const void *const *ptr, const uint64_t *nbytes, size_t n, uint64_t *out_dev,
+                        void *stream);
+
 /* Device-side status word of the handle: 0, or the first WT_ETIMEDOUT-class
  * code a bounded wait inside a kernel recorded (reads it synchronously). */
 int wt_device_status(wt_handle *h, int *status);

@@ -727,6 +727,8 @@ int close_impl(wt_handle *h) {
 
 }  // namespace
 
+int wt::set_error(int code, const char *msg) { return set_err(code, "%s", msg); }
+
 // ====================================================================== C ABI
 #pragma GCC visibility push(default)
 extern "C" {

@@ -95,4 +95,7 @@ cudaError_t launch_fnv_plain(const FnvBatch &b, cudaStream_t s);
 
 int num_sms();  // of the current device (cached per device)
 
+// Records `msg` as this thread's wt_last_error() text and returns `code`.
+int set_error(int code, const char *msg);
+
 }  // namespace wt

@@ -1,0 +1,91 @@
+// wt_checksum_noalloc: the leaf-tree digest of wt_checksum for callers that must
+// not allocate device memory.
+//
+// Some callers cannot call cudaMalloc at the moment they want a digest: code
+// running inside an allocator hook (it would re-enter the allocator it is
+// serving), programs that have handed all device memory to their own pool up
+// front (a serving engine's weight/KV arena), and loops that cannot afford the
+// device-wide synchronisation cudaFree implies.  wt_checksum needs a temporary
+// array of leaf digests and takes it from cudaMallocAsync; this entry point
+// uses a fixed array compiled into the library instead.
+//
+// The array below is a file-scope __device__ object: every GPU that loads this
+// library holds its 8 MiB until the process exits.  Host code cannot use its
+// name as a device address, so the first call on each device (with that device
+// current) asks the runtime for the address with cudaGetSymbolAddress and
+// caches it; that first call should come before any stream capture.  All calls
+// share the array, and nothing in it needs to start at zero: each call writes
+// every leaf slot it later reads.  Two calls whose kernels overlap on the GPU
+// (different streams, no ordering between them) race on the array.
+#include <cstring>
+#include <mutex>
+
+#include "../../include/wt.h"
+#include "wt_kernels.h"
+
+namespace {
+
+constexpr uint64_t kNoAllocMaxLeaves = 1ull << 20;  // 4096-byte leaves: 4 GiB of input per call
+__device__ __align__(256) uint64_t g_noalloc_leaves[kNoAllocMaxLeaves];
+
+std::mutex g_mu;
+uint64_t *g_leaves_addr[64] = {nullptr};
+
+int fail(int code, const char *msg) { return wt::set_error(code, msg); }  // readable via wt_last_error
+
+}  // namespace
+
+extern "C" __attribute__((visibility("default"))) int wt_checksum_noalloc(
+    const void *const *ptr, const uint64_t *nbytes, size_t n, uint64_t *out_dev, void *stream) {
+  if (n == 0) return WT_OK;
+  if (!ptr || !nbytes || !out_dev) return fail(WT_EINVAL, "wt_checksum_noalloc: NULL array");
+  uint64_t leaves = 0;
+  for (size_t i = 0; i < n; ++i) {
+    if (nbytes[i] && !ptr[i]) return fail(WT_EINVAL, "wt_checksum_noalloc: NULL buffer");
+    leaves += (nbytes[i] + wt::kLeafBytes - 1) / wt::kLeafBytes;
+  }
+  if (leaves > kNoAllocMaxLeaves)
+    return fail(WT_EINVAL,
+                "wt_checksum_noalloc: input needs more than 1048576 leaves of 4096 bytes (4 GiB per call); "
+                "split the call or use wt_checksum");
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= 64) return fail(WT_ECUDA, "wt_checksum_noalloc: cudaGetDevice failed");
+  uint64_t *scratch;
+  {
+    std::lock_guard<std::mutex> g(g_mu);
+    if (!g_leaves_addr[dev]) {
+      void *p = nullptr;
+      e = cudaGetSymbolAddress(&p, g_noalloc_leaves);
+      if (e != cudaSuccess || !p) {
+        cudaGetLastError();
+        return fail(WT_ECUDA, "wt_checksum_noalloc: cudaGetSymbolAddress of the leaf array failed");
+      }
+      g_leaves_addr[dev] = static_cast<uint64_t *>(p);
+    }
+    scratch = g_leaves_addr[dev];
+  }
+  // Batches run in order on one stream, so each reuses the array from slot 0.
+  const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  for (size_t i0 = 0; i0 < n; i0 += wt::kMaxFnv) {
+    const size_t m = n - i0 < (size_t)wt::kMaxFnv ? n - i0 : (size_t)wt::kMaxFnv;
+    wt::FnvBatch b;
+    memset(&b, 0, sizeof b);
+    b.n = (uint32_t)m;
+    uint64_t l = 0;
+    for (size_t k = 0; k < m; ++k) {
+      b.leaf_prefix[k] = l;
+      b.ptr[k] = static_cast<const uint8_t *>(ptr[i0 + k]);
+      b.nbytes[k] = nbytes[i0 + k];
+      b.out[k] = out_dev + i0 + k;
+      l += (nbytes[i0 + k] + wt::kLeafBytes - 1) / wt::kLeafBytes;
+    }
+    b.leaf_prefix[m] = l;
+    e = wt::launch_fnv_tree(b, scratch, s);
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      return fail(WT_ECUDA, "wt_checksum_noalloc: kernel launch failed");
+    }
+  }
+  return WT_OK;
+}

@@ -27,7 +27,8 @@ MODE_NAMES = {WT_ADOPT_GATHER: "gather", WT_ADOPT_CE: "ce", WT_ADOPT_STAGED: "st
 # every entry point declared in include/wt.h
 SYMBOLS = ("wt_last_error", "wt_abi_version", "wt_open", "wt_num_tensors", "wt_num_files",
            "wt_tensor_info", "wt_find", "wt_file_route", "wt_adopt", "wt_pass", "wt_checksum",
-           "wt_checksum_plain", "wt_device_status", "wt_kernel_launches", "wt_close")
+           "wt_checksum_plain", "wt_checksum_noalloc", "wt_device_status", "wt_kernel_launches",
+           "wt_close")
 
 
 class WtError(RuntimeError):
@@ -72,6 +73,7 @@ def lib(path: str = LIB_PATH):
     L.wt_pass.argtypes = [vp, C.POINTER(GemvDesc), sz, vp]
     L.wt_checksum.argtypes = [vp, C.POINTER(vp), u64p, sz, vp, vp]
     L.wt_checksum_plain.argtypes = [vp, C.POINTER(vp), u64p, sz, vp, vp]
+    L.wt_checksum_noalloc.argtypes = [C.POINTER(vp), u64p, sz, vp, vp]
     L.wt_device_status.argtypes = [vp, C.POINTER(C.c_int)]
     L.wt_kernel_launches.argtypes = [vp, u64p]
     L.wt_close.argtypes = [vp]
@@ -186,6 +188,14 @@ class Handle:
             self.close()
         except Exception:
             pass
+
+
+def checksum_noalloc(ptrs: Sequence[int], nbytes: Sequence[int], out_dev: int, stream: int = 0):
+    """wt_checksum_noalloc: leaf-tree digests without any device allocation (no handle)."""
+    n = len(ptrs)
+    pa = (C.c_void_p * max(1, n))(*ptrs)
+    na = (C.c_uint64 * max(1, n))(*nbytes)
+    _check(lib().wt_checksum_noalloc(pa, na, n, C.c_void_p(out_dev), C.c_void_p(stream)))
 
 
 def gemv_desc(W: int, dtype: int, M: int, K: int, x: int, y: int, wait_event: int = 0) -> GemvDesc:
