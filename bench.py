@@ -56,6 +56,7 @@ def parse_args():
     p.add_argument("--layers", type=int, default=None, help="override decoder layer count (small profiling cases)")
     p.add_argument("--mode", default="gather", choices=["gather", "ce", "staged"])
     p.add_argument("--e2e-reps", type=int, default=5)
+    p.add_argument("--skip-e2e", action="store_true", help="resident passes only (profiling runs)")
     p.add_argument("--arms", action="store_true", help="also time the ce/staged/stock-torch ingest arms")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="CPU budget of the oracle sample")
@@ -293,7 +294,7 @@ def run_wt(args, rank, world):
 
     # ---------------- e2e: file -> first use (1 warm-up, then timed repetitions)
     e2e_times, e2e_launches = [], 0
-    for rep in range(1 + args.e2e_reps):
+    for rep in range(0 if args.skip_e2e else 1 + args.e2e_reps):
         if dist:
             dist.barrier()
         dt, nl, st, nm = first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab)
@@ -302,7 +303,7 @@ def run_wt(args, rank, world):
         if rep > 0:
             e2e_times.append(dt)
             e2e_launches = nl
-    e2e_s = statistics.median(e2e_times)
+    e2e_s = statistics.median(e2e_times) if e2e_times else float("nan")
     e2e_gbs = data_bytes / e2e_s / 1e9
     log("file->first-use: %.1f ms median (%s), %.1f GB/s = %.1f%% of pinned H2D" % (
         e2e_s * 1e3, ", ".join("%.1f" % (t * 1e3) for t in e2e_times), e2e_gbs, 100 * e2e_gbs / h2d))

@@ -234,6 +234,59 @@ __device__ __forceinline__ void load_xvec(const uint8_t *x, uint32_t v, bool ok,
   }
 }
 
+// Warp-rows tile: each warp owns whole rows, G lanes per row, NJ 16-byte vectors per lane.
+template <int DT, int NJ>
+__device__ __forceinline__ void tile_warp_rows(uint32_t tile, uint32_t V, uint32_t nr, uint32_t G,
+                                               uint32_t gl, uint32_t sub, uint32_t rpw, int warp,
+                                               const float (&xf)[8][Elem<DT>::kEPV], float *y) {
+  for (uint32_t base = warp * rpw; base < nr; base += kConsumerWarps * rpw) {
+    const uint32_t row = base + sub;
+    const bool valid = row < nr;
+    float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+    for (int j = 0; j < NJ; ++j) {
+      const uint32_t v = gl + j * G;
+      if (valid && v < V) {
+        const uint4 w = lds128(tile + (row * V + v) * 16);
+        if (j & 1) a1 = dot16<DT>(w, xf[j], a1);
+        else a0 = dot16<DT>(w, xf[j], a0);
+      }
+    }
+    float acc = a0 + a1;
+    for (uint32_t o = G >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (valid && gl == 0) y[row] = acc;
+  }
+}
+
+// Block-rows tile: all consumer threads share each of the nr rows; thread ct holds
+// vectors ct + 256 j.  Each warp's partial of row q lands in rb[q * warps + warp].
+template <int DT, int NJ>
+__device__ __forceinline__ void tile_block_rows(uint32_t tile, uint32_t V, uint32_t nr, int ct, int warp,
+                                                int lane, const float (&xf)[8][Elem<DT>::kEPV], float *rb) {
+  for (uint32_t q = 0; q < nr; ++q) {
+    float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+    for (int j = 0; j < NJ; ++j) {
+      const uint32_t v = ct + j * kConsumers;
+      if (j + 1 < NJ || v < V) {
+        const uint4 w = lds128(tile + (q * V + v) * 16);
+        if (j & 1) a1 = dot16<DT>(w, xf[j], a1);
+        else a0 = dot16<DT>(w, xf[j], a0);
+      }
+    }
+    const float t = warp_sum(a0 + a1);
+    if (lane == 0) rb[q * kConsumerWarps + warp] = t;
+  }
+}
+
+// Sum of the consumer warps' partials of one row, in warp order (deterministic).
+__device__ __forceinline__ float sum_warps(const float *p) {
+  float t = 0.f;
+#pragma unroll
+  for (int w = 0; w < kConsumerWarps; ++w) t += p[w];
+  return t;
+}
+
 template <int DT>
 __global__ void __launch_bounds__(kGemvThreads, 1)
     gemv_tma_kernel(const MatDesc *__restrict__ mats, const Piece *__restrict__ pieces,
@@ -337,83 +390,86 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
           const uint32_t s = it % kStages;
           bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
           const uint32_t tile = stage0 + s * kStageBytes;
-          for (uint32_t base = warp * rpw; base < nr; base += kConsumerWarps * rpw) {
-            const uint32_t row = base + sub;
-            const bool valid = row < nr;
-            float a0 = 0.f, a1 = 0.f;
-            if (valid) {
-#pragma unroll
-              for (int j = 0; j < 8; j += 2) {
-                const uint32_t v = gl + j * G;
-                if (j < (int)nj && v < V) a0 = dot16<DT>(lds128(tile + (row * V + v) * 16), xf[j], a0);
-                const uint32_t v1 = gl + (j + 1) * G;
-                if (j + 1 < (int)nj && v1 < V)
-                  a1 = dot16<DT>(lds128(tile + (row * V + v1) * 16), xf[j + 1], a1);
-              }
-            }
-            float acc = a0 + a1;
-            for (uint32_t o = G >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-            if (valid && gl == 0) md.y[r + row] = acc;
+          float *y = md.y + r;
+          switch (nj) {
+            case 1: tile_warp_rows<DT, 1>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
+            case 2: tile_warp_rows<DT, 2>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
+            case 3: tile_warp_rows<DT, 3>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
+            case 4: tile_warp_rows<DT, 4>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
+            case 5: tile_warp_rows<DT, 5>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
+            case 6: tile_warp_rows<DT, 6>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
+            case 7: tile_warp_rows<DT, 7>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
+            default: tile_warp_rows<DT, 8>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
           }
           __syncwarp();
           if (lane == 0) mbar_arrive(empty0 + 8 * s);
           ++it;
         }
-      } else {
-        // block modes: the whole consumer group shares each row
-        const bool split = md.mode == kModeSplitK;
-        const uint32_t nj = split ? 1 : (V + kConsumers - 1) / kConsumers;
-        if (!split) {
+      } else if (md.mode == kModeBlockRows) {
+        // whole consumer group shares each row; one tile = up to kRowBlock full rows
+        const uint32_t nj = (V + kConsumers - 1) / kConsumers;
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const uint32_t v = ct + j * kConsumers;
-            load_xvec<DT>(md.x, v, j < (int)nj && v < V, xf[j]);
-          }
+        for (int j = 0; j < 8; ++j) {
+          const uint32_t v = ct + j * kConsumers;
+          load_xvec<DT>(md.x, v, j < (int)nj && v < V, xf[j]);
         }
-        const uint32_t vstride = split ? md.vc : V;  // vectors per row inside a stage
+        for (uint32_t r = pc.r0; r < pc.r1; r += md.rt) {
+          const uint32_t nr = min(md.rt, pc.r1 - r);
+          const uint32_t s = it % kStages;
+          bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
+          const uint32_t tile = stage0 + s * kStageBytes;
+          float *rb = red + par * (kConsumerWarps * kRowBlock);
+          switch (nj) {
+            case 1: tile_block_rows<DT, 1>(tile, V, nr, ct, warp, lane, xf, rb); break;
+            case 2: tile_block_rows<DT, 2>(tile, V, nr, ct, warp, lane, xf, rb); break;
+            case 3: tile_block_rows<DT, 3>(tile, V, nr, ct, warp, lane, xf, rb); break;
+            case 4: tile_block_rows<DT, 4>(tile, V, nr, ct, warp, lane, xf, rb); break;
+            case 5: tile_block_rows<DT, 5>(tile, V, nr, ct, warp, lane, xf, rb); break;
+            case 6: tile_block_rows<DT, 6>(tile, V, nr, ct, warp, lane, xf, rb); break;
+            case 7: tile_block_rows<DT, 7>(tile, V, nr, ct, warp, lane, xf, rb); break;
+            default: tile_block_rows<DT, 8>(tile, V, nr, ct, warp, lane, xf, rb); break;
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(empty0 + 8 * s);
+          ++it;
+          named_bar(1, kConsumers);
+          if (ct < (int)nr) md.y[r + ct] = sum_warps(rb + ct * kConsumerWarps);
+          par ^= 1;
+        }
+      } else {
+        // split-K: row blocks of kRowBlock rows, streamed in column chunks of md.vc vectors
+        const uint32_t nchunk = (V + md.vc - 1) / md.vc;
         for (uint32_t r = pc.r0; r < pc.r1; r += md.rt) {
           const uint32_t nr = min(md.rt, pc.r1 - r);
           float acc[kRowBlock];
 #pragma unroll
           for (int q = 0; q < kRowBlock; ++q) acc[q] = 0.f;
-          const uint32_t nchunk = split ? (V + md.vc - 1) / md.vc : 1;
           for (uint32_t c = 0; c < nchunk; ++c) {
             const uint32_t v0 = c * md.vc;
-            const uint32_t nv = split ? min(md.vc, V - v0) : V;
-            if (split) load_xvec<DT>(md.x, v0 + ct, ct < nv, xf[0]);
+            const uint32_t nv = min(md.vc, V - v0);
+            load_xvec<DT>(md.x, v0 + ct, ct < nv, xf[0]);
             const uint32_t s = it % kStages;
             bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
             const uint32_t tile = stage0 + s * kStageBytes;
+            if (ct < nv) {
 #pragma unroll
-            for (int q = 0; q < kRowBlock; ++q) {
-              if (q < (int)nr) {
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                  const uint32_t v = ct + j * kConsumers;
-                  if (j < (int)nj && v < nv) acc[q] = dot16<DT>(lds128(tile + (q * vstride + v) * 16), xf[j], acc[q]);
-                }
-              }
+              for (int q = 0; q < kRowBlock; ++q)
+                if (q < (int)nr) acc[q] = dot16<DT>(lds128(tile + (q * md.vc + ct) * 16), xf[0], acc[q]);
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(empty0 + 8 * s);
             ++it;
           }
-          // cross-warp reduction in a fixed order: deterministic per row
           float *rb = red + par * (kConsumerWarps * kRowBlock);
 #pragma unroll
           for (int q = 0; q < kRowBlock; ++q) {
             if (q < (int)nr) {
               const float t = warp_sum(acc[q]);
-              if (lane == 0) rb[warp * kRowBlock + q] = t;
+              if (lane == 0) rb[q * kConsumerWarps + warp] = t;
             }
           }
           named_bar(1, kConsumers);
-          if (ct < (int)nr) {
-            float t = 0.f;
-#pragma unroll
-            for (int w = 0; w < kConsumerWarps; ++w) t += rb[w * kRowBlock + ct];
-            md.y[r + ct] = t;
-          }
+          if (ct < (int)nr) md.y[r + ct] = sum_warps(rb + ct * kConsumerWarps);
           par ^= 1;
         }
       }
