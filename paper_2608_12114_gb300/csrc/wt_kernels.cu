@@ -154,16 +154,6 @@ struct Elem<2> {  // f16
   }
 };
 
-// acc += <w, x> over one 16-byte vector, in element order.
-template <int DT>
-__device__ __forceinline__ float dot16(const uint4 &w, const float (&xf)[Elem<DT>::kEPV], float acc) {
-  float wf[Elem<DT>::kEPV];
-  Elem<DT>::unpack(w, wf);
-#pragma unroll
-  for (int e = 0; e < Elem<DT>::kEPV; ++e) acc = fmaf(wf[e], xf[e], acc);
-  return acc;
-}
-
 __device__ __forceinline__ uint4 lds128(uint32_t addr) {
   uint4 v;
   asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
@@ -222,61 +212,169 @@ constexpr size_t kRedOff = kBarOff + 2 * kStages * sizeof(uint64_t);
 constexpr size_t kFlagOff = kRedOff + 2 * kConsumerWarps * kRowBlock * sizeof(float);
 constexpr size_t kGemvSmem = kFlagOff + 16;
 
+// Two fp32 values in one 64-bit register; fma.rn.f32x2 performs two independent
+// round-to-nearest FMAs (the same arithmetic as two fmaf calls) in one instruction.
+__device__ __forceinline__ uint64_t pack2(uint32_t lo, uint32_t hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(lo), "r"(hi));
+  return r;
+}
+__device__ __forceinline__ float sum2(uint64_t v) {
+  uint32_t lo, hi;
+  asm("mov.b64 {%0, %1}, %2;" : "=r"(lo), "=r"(hi) : "l"(v));
+  return __uint_as_float(lo) + __uint_as_float(hi);
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+
+// A 16-byte vector as fp32 pairs (element 2i in the low half, 2i+1 in the high half).
 template <int DT>
-__device__ __forceinline__ void load_xvec(const uint8_t *x, uint32_t v, bool ok,
-                                          float (&xf)[Elem<DT>::kEPV]) {
-  if (ok) {
-    uint4 t = __ldg(reinterpret_cast<const uint4 *>(x) + v);
-    Elem<DT>::unpack(t, xf);
-  } else {
+struct Pairs {
+  static constexpr int N = Elem<DT>::kEPV / 2;
+  __device__ static __forceinline__ uint64_t get(const uint4 &v, int i) {
+    const uint32_t w = i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w;
+    if (DT == 1) return pack2(w << 16, w & 0xffff0000u);  // bf16
+    if (DT == 2) {                                          // f16
+      const float2 t = __half22float2(*reinterpret_cast<const __half2 *>(&w));
+      return pack2(__float_as_uint(t.x), __float_as_uint(t.y));
+    }
+    return i == 0 ? pack2(v.x, v.y) : pack2(v.z, v.w);  // f32
+  }
+};
+
+// Four running fp32 partial sums of one row (two f32x2 registers).
+struct Acc4 {
+  uint64_t a = 0, b = 0;
+  __device__ __forceinline__ float total() const { return sum2(a) + sum2(b); }
+};
+
+template <int DT>
+__device__ __forceinline__ void dot16(const uint4 &w, const uint64_t (&xp)[Pairs<DT>::N], Acc4 &acc) {
 #pragma unroll
-    for (int e = 0; e < Elem<DT>::kEPV; ++e) xf[e] = 0.f;
+  for (int i = 0; i < Pairs<DT>::N; ++i) {
+    if (i & 1) acc.b = fma2(Pairs<DT>::get(w, i), xp[i], acc.b);
+    else acc.a = fma2(Pairs<DT>::get(w, i), xp[i], acc.a);
   }
 }
 
-// Warp-rows tile: each warp owns whole rows, G lanes per row, NJ 16-byte vectors per lane.
+template <int DT>
+__device__ __forceinline__ void load_xpairs(const uint8_t *x, uint32_t v, bool ok, uint64_t (&xp)[Pairs<DT>::N]) {
+  const uint4 t = ok ? __ldg(reinterpret_cast<const uint4 *>(x) + v) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+  for (int i = 0; i < Pairs<DT>::N; ++i) xp[i] = Pairs<DT>::get(t, i);
+}
+
+__device__ __forceinline__ uint4 lds_or_zero(uint32_t addr, bool ok) {
+  return ok ? lds128(addr) : make_uint4(0, 0, 0, 0);
+}
+
+// Sums N per-lane values (N a power of two) over the 32 lanes with N/2 + N/4 + ... + 1
+// halving exchanges, then plain exchanges for the remaining offsets.  Afterwards every
+// lane holds the full sum of value index lane >> (5 - log2 N).  Fixed data flow, so the
+// result is deterministic.
+template <int N>
+__device__ __forceinline__ float transpose_reduce(float (&v)[N], int lane) {
+  int o = 16;
+#pragma unroll
+  for (int n = N; n > 1; n >>= 1, o >>= 1) {
+    const bool up = (lane & o) != 0;
+#pragma unroll
+    for (int k = 0; k < n / 2; ++k) {
+      const float send = up ? v[k] : v[k + n / 2];
+      const float keep = up ? v[k + n / 2] : v[k];
+      v[k] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+    }
+  }
+  float t = v[0];
+  for (; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+  return t;
+}
+
+template <int N>
+struct Log2 {
+  static constexpr int value = N <= 1 ? 0 : 1 + Log2<(N > 1 ? N / 2 : 1)>::value;
+};
+template <>
+struct Log2<1> {
+  static constexpr int value = 0;
+};
+
+// Warp-rows tile: each warp owns whole rows, G lanes per row, NJ 16-byte vectors per
+// lane per row.  U rows are loaded before any is used (latency of shared loads overlaps).
 template <int DT, int NJ>
 __device__ __forceinline__ void tile_warp_rows(uint32_t tile, uint32_t V, uint32_t nr, uint32_t G,
-                                               uint32_t gl, uint32_t sub, uint32_t rpw, int warp,
-                                               const float (&xf)[8][Elem<DT>::kEPV], float *y) {
-  for (uint32_t base = warp * rpw; base < nr; base += kConsumerWarps * rpw) {
-    const uint32_t row = base + sub;
-    const bool valid = row < nr;
-    float a0 = 0.f, a1 = 0.f;
+                                               uint32_t gl, uint32_t sub, uint32_t rpw, int warp, int lane,
+                                               const uint64_t (&xp)[8][Pairs<DT>::N], float *y) {
+  constexpr int U = NJ <= 2 ? 4 : (NJ <= 4 ? 2 : 1);
+  const uint32_t step = kConsumerWarps * rpw;
+  for (uint32_t base = warp * rpw; base < nr; base += U * step) {
+    uint4 w[U][NJ];
 #pragma unroll
-    for (int j = 0; j < NJ; ++j) {
-      const uint32_t v = gl + j * G;
-      if (valid && v < V) {
-        const uint4 w = lds128(tile + (row * V + v) * 16);
-        if (j & 1) a1 = dot16<DT>(w, xf[j], a1);
-        else a0 = dot16<DT>(w, xf[j], a0);
+    for (int u = 0; u < U; ++u) {
+      const uint32_t row = base + u * step + sub;
+#pragma unroll
+      for (int j = 0; j < NJ; ++j) {
+        const uint32_t v = gl + j * G;
+        w[u][j] = lds_or_zero(tile + (row * V + v) * 16, row < nr && v < V);
       }
     }
-    float acc = a0 + a1;
-    for (uint32_t o = G >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (valid && gl == 0) y[row] = acc;
+    float t[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      Acc4 acc;
+#pragma unroll
+      for (int j = 0; j < NJ; ++j) dot16<DT>(w[u][j], xp[j], acc);
+      t[u] = acc.total();
+    }
+    if (G == 32) {
+      const float sum = transpose_reduce<U>(t, lane);
+      constexpr int L = Log2<U>::value;
+      const uint32_t row = base + (uint32_t)(lane >> (5 - L)) * step;
+      if ((lane & ((32 >> L) - 1)) == 0 && row < nr) y[row] = sum;
+    } else {
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        for (uint32_t o = G >> 1; o > 0; o >>= 1) t[u] += __shfl_xor_sync(0xffffffffu, t[u], o);
+        const uint32_t row = base + u * step + sub;
+        if (gl == 0 && row < nr) y[row] = t[u];
+      }
+    }
   }
 }
 
-// Block-rows tile: all consumer threads share each of the nr rows; thread ct holds
-// vectors ct + 256 j.  Each warp's partial of row q lands in rb[q * warps + warp].
-template <int DT, int NJ>
-__device__ __forceinline__ void tile_block_rows(uint32_t tile, uint32_t V, uint32_t nr, int ct, int warp,
-                                                int lane, const float (&xf)[8][Elem<DT>::kEPV], float *rb) {
-  for (uint32_t q = 0; q < nr; ++q) {
-    float a0 = 0.f, a1 = 0.f;
+// Block-rows tile of exactly NR rows: all consumer threads share each row; thread ct
+// holds vectors ct + 256 j.  Warp partials land in rb[q * warps + warp].
+template <int DT, int NJ, int NR>
+__device__ __forceinline__ void tile_block_rows(uint32_t tile, uint32_t V, int ct, int warp, int lane,
+                                                const uint64_t (&xp)[8][Pairs<DT>::N], float *rb) {
+  constexpr int NP = NR <= 1 ? 1 : NR <= 2 ? 2 : NR <= 4 ? 4 : 8;
+  uint4 w[NR][NJ];
+#pragma unroll
+  for (int q = 0; q < NR; ++q) {
 #pragma unroll
     for (int j = 0; j < NJ; ++j) {
       const uint32_t v = ct + j * kConsumers;
-      if (j + 1 < NJ || v < V) {
-        const uint4 w = lds128(tile + (q * V + v) * 16);
-        if (j & 1) a1 = dot16<DT>(w, xf[j], a1);
-        else a0 = dot16<DT>(w, xf[j], a0);
-      }
+      w[q][j] = lds_or_zero(tile + (q * V + v) * 16, j + 1 < NJ || v < V);
     }
-    const float t = warp_sum(a0 + a1);
-    if (lane == 0) rb[q * kConsumerWarps + warp] = t;
   }
+  float t[NP];
+#pragma unroll
+  for (int q = 0; q < NP; ++q) {
+    t[q] = 0.f;
+    if (q < NR) {
+      Acc4 acc;
+#pragma unroll
+      for (int j = 0; j < NJ; ++j) dot16<DT>(w[q < NR ? q : 0][j], xp[j], acc);
+      t[q] = acc.total();
+    }
+  }
+  const float sum = transpose_reduce<NP>(t, lane);
+  constexpr int L = Log2<NP>::value;
+  const int q = lane >> (5 - L);
+  if ((lane & ((32 >> L) - 1)) == 0 && q < NR) rb[q * kConsumerWarps + warp] = sum;
 }
 
 // Sum of the consumer warps' partials of one row, in warp order (deterministic).
@@ -288,10 +386,26 @@ __device__ __forceinline__ float sum_warps(const float *p) {
 }
 
 template <int DT>
+__device__ __forceinline__ bool block_rows_dispatch(uint32_t nj, uint32_t nr, uint32_t tile, uint32_t V, int ct,
+                                                    int warp, int lane, const uint64_t (&xp)[8][Pairs<DT>::N],
+                                                    float *rb) {
+#define WT_BR(NJ, NR) \
+  case NJ * 8 + NR: tile_block_rows<DT, NJ, NR>(tile, V, ct, warp, lane, xp, rb); return true;
+  switch (nj * 8 + nr) {
+    WT_BR(2, 1) WT_BR(2, 2) WT_BR(2, 3) WT_BR(2, 4) WT_BR(2, 5) WT_BR(2, 6) WT_BR(2, 7)
+    WT_BR(3, 1) WT_BR(3, 2) WT_BR(3, 3)
+    WT_BR(4, 1) WT_BR(4, 2)
+    WT_BR(5, 1) WT_BR(6, 1) WT_BR(7, 1) WT_BR(8, 1)
+    default: return false;
+  }
+#undef WT_BR
+}
+
+template <int DT>
 __global__ void __launch_bounds__(kGemvThreads, 1)
     gemv_tma_kernel(const MatDesc *__restrict__ mats, const Piece *__restrict__ pieces,
                     const uint32_t *__restrict__ begin, int *status) {
-  constexpr int EPV = Elem<DT>::kEPV;
+  constexpr int NP = Pairs<DT>::N;
   extern __shared__ __align__(128) uint8_t smem[];
   const uint32_t stage0 = smem_u32(smem);
   const uint32_t full0 = smem_u32(smem + kBarOff);
@@ -369,7 +483,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
     const int ct = threadIdx.x;  // 0..255
     uint32_t it = 0;
     int par = 0;
-    float xf[8][EPV];
+    uint64_t xp[8][NP];
     for (uint32_t pi = p0; pi < p1; ++pi) {
       const Piece pc = pieces[pi];
       const MatDesc md = mats[pc.mat];
@@ -383,7 +497,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           const uint32_t v = gl + j * G;
-          load_xvec<DT>(md.x, v, j < (int)nj && v < V, xf[j]);
+          load_xpairs<DT>(md.x, v, j < (int)nj && v < V, xp[j]);
         }
         for (uint32_t r = pc.r0; r < pc.r1; r += md.rt) {
           const uint32_t nr = min(md.rt, pc.r1 - r);
@@ -392,14 +506,14 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
           const uint32_t tile = stage0 + s * kStageBytes;
           float *y = md.y + r;
           switch (nj) {
-            case 1: tile_warp_rows<DT, 1>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
-            case 2: tile_warp_rows<DT, 2>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
-            case 3: tile_warp_rows<DT, 3>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
-            case 4: tile_warp_rows<DT, 4>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
-            case 5: tile_warp_rows<DT, 5>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
-            case 6: tile_warp_rows<DT, 6>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
-            case 7: tile_warp_rows<DT, 7>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
-            default: tile_warp_rows<DT, 8>(tile, V, nr, G, gl, sub, rpw, warp, xf, y); break;
+            case 1: tile_warp_rows<DT, 1>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
+            case 2: tile_warp_rows<DT, 2>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
+            case 3: tile_warp_rows<DT, 3>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
+            case 4: tile_warp_rows<DT, 4>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
+            case 5: tile_warp_rows<DT, 5>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
+            case 6: tile_warp_rows<DT, 6>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
+            case 7: tile_warp_rows<DT, 7>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
+            default: tile_warp_rows<DT, 8>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
           }
           __syncwarp();
           if (lane == 0) mbar_arrive(empty0 + 8 * s);
@@ -411,7 +525,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           const uint32_t v = ct + j * kConsumers;
-          load_xvec<DT>(md.x, v, j < (int)nj && v < V, xf[j]);
+          load_xpairs<DT>(md.x, v, j < (int)nj && v < V, xp[j]);
         }
         for (uint32_t r = pc.r0; r < pc.r1; r += md.rt) {
           const uint32_t nr = min(md.rt, pc.r1 - r);
@@ -419,16 +533,8 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
           bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
           const uint32_t tile = stage0 + s * kStageBytes;
           float *rb = red + par * (kConsumerWarps * kRowBlock);
-          switch (nj) {
-            case 1: tile_block_rows<DT, 1>(tile, V, nr, ct, warp, lane, xf, rb); break;
-            case 2: tile_block_rows<DT, 2>(tile, V, nr, ct, warp, lane, xf, rb); break;
-            case 3: tile_block_rows<DT, 3>(tile, V, nr, ct, warp, lane, xf, rb); break;
-            case 4: tile_block_rows<DT, 4>(tile, V, nr, ct, warp, lane, xf, rb); break;
-            case 5: tile_block_rows<DT, 5>(tile, V, nr, ct, warp, lane, xf, rb); break;
-            case 6: tile_block_rows<DT, 6>(tile, V, nr, ct, warp, lane, xf, rb); break;
-            case 7: tile_block_rows<DT, 7>(tile, V, nr, ct, warp, lane, xf, rb); break;
-            default: tile_block_rows<DT, 8>(tile, V, nr, ct, warp, lane, xf, rb); break;
-          }
+          if (!block_rows_dispatch<DT>(nj, nr, tile, V, ct, warp, lane, xp, rb) && ct == 0)
+            atomicCAS(status, 0, -1);  // unreachable by construction of the plan
           __syncwarp();
           if (lane == 0) mbar_arrive(empty0 + 8 * s);
           ++it;
@@ -441,33 +547,31 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
         const uint32_t nchunk = (V + md.vc - 1) / md.vc;
         for (uint32_t r = pc.r0; r < pc.r1; r += md.rt) {
           const uint32_t nr = min(md.rt, pc.r1 - r);
-          float acc[kRowBlock];
-#pragma unroll
-          for (int q = 0; q < kRowBlock; ++q) acc[q] = 0.f;
+          Acc4 acc[kRowBlock];
           for (uint32_t c = 0; c < nchunk; ++c) {
             const uint32_t v0 = c * md.vc;
             const uint32_t nv = min(md.vc, V - v0);
-            load_xvec<DT>(md.x, v0 + ct, ct < nv, xf[0]);
+            load_xpairs<DT>(md.x, v0 + ct, ct < nv, xp[0]);
             const uint32_t s = it % kStages;
             bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
             const uint32_t tile = stage0 + s * kStageBytes;
-            if (ct < nv) {
+            uint4 w[kRowBlock];
 #pragma unroll
-              for (int q = 0; q < kRowBlock; ++q)
-                if (q < (int)nr) acc[q] = dot16<DT>(lds128(tile + (q * md.vc + ct) * 16), xf[0], acc[q]);
-            }
+            for (int q = 0; q < kRowBlock; ++q)
+              w[q] = lds_or_zero(tile + (q * md.vc + ct) * 16, q < (int)nr && ct < nv);
+#pragma unroll
+            for (int q = 0; q < kRowBlock; ++q) dot16<DT>(w[q], xp[0], acc[q]);
             __syncwarp();
             if (lane == 0) mbar_arrive(empty0 + 8 * s);
             ++it;
           }
-          float *rb = red + par * (kConsumerWarps * kRowBlock);
+          float t[kRowBlock];
 #pragma unroll
-          for (int q = 0; q < kRowBlock; ++q) {
-            if (q < (int)nr) {
-              const float t = warp_sum(acc[q]);
-              if (lane == 0) rb[q * kConsumerWarps + warp] = t;
-            }
-          }
+          for (int q = 0; q < kRowBlock; ++q) t[q] = acc[q].total();
+          float *rb = red + par * (kConsumerWarps * kRowBlock);
+          const float sum = transpose_reduce<kRowBlock>(t, lane);
+          const int q = lane >> 2;
+          if ((lane & 3) == 0 && q < (int)nr) rb[q * kConsumerWarps + warp] = sum;
           named_bar(1, kConsumers);
           if (ct < (int)nr) md.y[r + ct] = sum_warps(rb + ct * kConsumerWarps);
           par ^= 1;
