@@ -228,6 +228,24 @@ def kernel_traffic(name):
     return d
 
 
+# ----------------------------------------------------------------------------- replicas (N > 1)
+
+def combine_ranks(dist, device, total_ms, e2e_s):
+    """Max over ranks of the timed-region length and of the first-use time: the slowest
+    replica sets the clock.  Without a process group the local values are returned."""
+    if dist is None:
+        return total_ms, e2e_s
+    import torch
+    t = torch.tensor([total_ms, e2e_s], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return tuple(t.tolist())
+
+
+def aggregate_gbs(bytes_per_rank, world, seconds):
+    """Whole-job rate: every replica moves the same bytes, the job takes the slowest time."""
+    return bytes_per_rank * world / seconds / 1e9
+
+
 # ----------------------------------------------------------------------------- the wt arm
 
 def first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab):
@@ -347,14 +365,9 @@ def run_wt(args, rank, world):
     if status != 0:
         raise SystemExit("device status %d after resident passes" % status)
 
-    if dist:
-        t = torch.tensor([total_ms, e2e_s], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms, e2e_s_max = t.tolist()
-    else:
-        e2e_s_max = e2e_s
+    total_ms, e2e_s_max = combine_ranks(dist, "cuda", total_ms, e2e_s)
     ms_per_step = total_ms / args.steps
-    value = weight_bytes * args.steps * world / (total_ms / 1e3) / 1e9
+    value = aggregate_gbs(weight_bytes * args.steps, world, total_ms / 1e3)
     launches_per_pass = launches / args.steps
     avg_launch_ms = statistics.mean(per) if launches_per_pass == 1 else None
     peak, peak_kind = measured_peaks()
@@ -379,7 +392,7 @@ def run_wt(args, rank, world):
                    "l2": "inputs larger than L2 (no flush)", "parallelism": "replicas" if world > 1 else "1 GPU"},
         "resident_frac_of_hbm": {"measured": round(value / world / peak, 4), "nominal_8TBps": round(value / world / NOMINAL_HBM_GBS, 4)},
         "clocks": clocks,
-        "e2e": {"value": round(data_bytes * world / e2e_s_max / 1e9, 1), "unit": "GB/s",
+        "e2e": {"value": round(aggregate_gbs(data_bytes, world, e2e_s_max), 1), "unit": "GB/s",
                 "h2d_bytes_per_step": data_bytes, "d2h_bytes_per_step": int(y_host.numel() * 4),
                 "ms": round(e2e_s * 1e3, 2), "pinned_h2d_gbs": round(h2d, 1),
                 "frac_of_pinned_h2d": round(e2e_gbs / h2d, 4), "reps": args.e2e_reps,

@@ -9,17 +9,17 @@
  *
  *   wt_open   guarded open + shared read-only map of each file (Algorithm 1:
  *             size guard, mmap(PROT_READ, MAP_SHARED), close the descriptor)
- *             and the device-access route for the mapping (Sec. 6.2: registration
+ *             and the device-access route for the mapping (Sec. 7.3: registration
  *             and direct read are probed separately).
  *   wt_adopt  moves tensor bytes into caller-owned device memory and returns a
  *             per-tensor ready event (contract C3: order on the GPU).
  *   wt_pass   one GEMV per matrix in the caller's stream, each launch gated
  *             by its tensors' events, outputs kept on the device (C2).
  *   wt_checksum / wt_checksum_plain  per-tensor FNV-1a-64 digests of device
- *             bytes (the checksums of Sec. 5.1 that confirm kernels read the
+ *             bytes (the checksums of Sec. 6.1 that confirm kernels read the
  *             intended bytes).
  *   wt_close  waits for the library's own work on the mappings, unregisters,
- *             unmaps (Algorithm 1's deleter; Sec. 4.1 lifetime rules).
+ *             unmaps (Algorithm 1's deleter; Sec. 5.1 lifetime rules).
  *
  * Conventions
  *   - Every call returns int: WT_OK (0) or a negative WT_E* code.  No C++
@@ -30,7 +30,7 @@
  *   - Device pointers are caller-owned (the library never frees them).  The
  *     library borrows a destination until the event it returned completes.
  *   - The library never writes to a mapping.  A destination that lies inside
- *     one of the handle's mappings is rejected with WT_EINVAL (Sec. 4.1:
+ *     one of the handle's mappings is rejected with WT_EINVAL (Sec. 5.1:
  *     read-only intent must be enforced before dispatch).
  *   - All kernels run on the device that is current when wt_open is called.
  */

@@ -9,7 +9,7 @@
  *
  *   O1  parse   read() the whole file into a heap buffer; decode the
  *               length-prefixed index byte by byte; apply the producer's
- *               guards (Algorithm 1: size = M*K*sizeof(dtype); Sec. 4.3:
+ *               guards (Algorithm 1: size = M*K*sizeof(dtype); Sec. 5.3:
  *               aligned bases) generalised to the container.
  *   O2  bytes   FNV-1a-64 of every blob (D_plain) and the leaf-tree digest
  *               (D_tree, 4096-byte leaves) defined below.
@@ -198,7 +198,7 @@ int or_load(const char *path, or_file **out) {
     pos += 16;
     /* Algorithm 1's size guard: the blob holds exactly prod(shape) elements */
     if (e->nbytes != count) return fail(f, path, "nbytes != prod(shape) * sizeof(dtype)", i);
-    /* aligned base (Sec. 4.3), after the index, inside the file */
+    /* aligned base (Sec. 5.3), after the index, inside the file */
     if (e->offset % OR_ALIGN != 0) return fail(f, path, "offset not 64-byte aligned", i);
     if (e->offset < data_start) return fail(f, path, "blob overlaps the header or index", i);
     if (e->offset > f->size || e->nbytes > f->size - e->offset)

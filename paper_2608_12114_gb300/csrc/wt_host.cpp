@@ -2,7 +2,7 @@
 //
 //   open     parallel per-file open / fstat / pread index / validate / mmap
 //            (Algorithm 1's guarded shared read-only map), then the device
-//            route for each mapping (Sec. 6.2: registration and direct read are
+//            route for each mapping (Sec. 7.3: registration and direct read are
 //            probed separately; GB300 reads pageable memory through the host
 //            page tables, so a registration is optional there)
 //   adopt    batches tensors into launches of the gather kernel (or copy-engine

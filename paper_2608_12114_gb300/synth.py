@@ -7,7 +7,7 @@ path's arithmetic (no parsing, no checksum, no GEMV); the CUDA library and the
 CPU oracle each decode these files with their own code.
 
 The container stands in for the paper's per-tensor page-aligned files
-(Sec. 4.3 suggests an aligned container as the alternative to one inode per
+(Sec. 5.3 suggests an aligned container as the alternative to one inode per
 tensor; Algorithm 1 guards size = M*K*sizeof(dtype)).
 
 Layout (all integers little-endian):
@@ -23,7 +23,7 @@ Workloads (shapes of the paper's measured cases; values are synthetic):
   tiny   8 fp32 256x256 matrices + 8 fp32[256] vectors, U[-1,1] from PCG64(0)
   sweep  one bf16 4096 x (128*2^i) matrix per file, N(0, 0.02)
   many   1253 bf16 matrices split by rows into 2506 single-tensor files
-         (the 1253-matrix / 2506-file spine shape of Sec. 4.3)
+         (the 1253-matrix / 2506-file spine shape of Sec. 5.3)
   mid    32-layer decoder, d=2560, FFN 6912, vocab 32000, 3 shards
   large  32-layer decoder, d=4096, kv 1024, FFN 14336, vocab 128256, 4 shards
 """
