@@ -187,10 +187,15 @@ class CheckpointOracle:
                     return f, i
         raise KeyError(name)
 
-    def matrix_bytes(self, names: Sequence[str]) -> np.ndarray:
-        """Row blocks named in order, concatenated (the many workload's halves)."""
-        parts = [self.files[f].blob(i) for f, i in (self.find(n) for n in names)]
-        return parts[0] if len(parts) == 1 else np.concatenate(parts)
+    def blob_of(self, f: int, name: str) -> np.ndarray:
+        """Bytes of the entry `name` of file `f` (names are unique within a file only)."""
+        fo = self.files[f]
+        return fo.blob([e["name"] for e in fo.entries].index(name))
+
+    def matrix_bytes(self, parts: Sequence[Tuple[int, str]]) -> np.ndarray:
+        """Row blocks given as (file, name), in row order, concatenated (the many workload's halves)."""
+        blobs = [self.blob_of(f, n) for f, n in parts]
+        return blobs[0] if len(blobs) == 1 else np.concatenate(blobs)
 
     def close(self):
         for fo in self.files:

@@ -71,7 +71,7 @@ def run_and_check(torch, ck, rows=16, plain_limit=256 << 20):
         for k in dev.gemv_mats():
             m = dev.mats[k]
             M, K = m.shape
-            W = co.matrix_bytes([h.tensors[i].name for i in m.parts])
+            W = co.matrix_bytes([(h.tensors[i].file, h.tensors[i].name) for i in m.parts])
             x = synth.make_x(K, m.dtype)
             y = ys[k].cpu().numpy().astype(np.float64)
             if rows is None:

@@ -75,7 +75,7 @@ def test_many_halves_are_row_blocks(tmp_path):
     ck = synth.build("many", str(tmp_path), n_matrices=5)
     co = oracle.CheckpointOracle(ck.paths)
     for m in ck.matrices:
-        W = co.matrix_bytes([ck.tensors[i].name for i in m.parts])
+        W = co.matrix_bytes([(ck.tensors[i].file, ck.tensors[i].name) for i in m.parts])
         assert W.size == m.M * m.K * 2
         assert ck.tensors[m.parts[0]].shape == (m.M // 2, m.K)
         assert ck.tensors[m.parts[1]].shape == (m.M - m.M // 2, m.K)
