@@ -178,6 +178,7 @@ struct File {
   size_t size = 0;
   unsigned route = WT_ROUTE_NONE;
   bool registered = false;
+  bool populated = false;        // page-table entries already filled (registered files)
   const uint8_t *dev = nullptr;  // device-readable address of base
   std::vector<Tensor> tensors;
 };
@@ -402,47 +403,106 @@ struct Range {
   const uint8_t *src_dev;
   uint8_t *dst;
   uint64_t n;
+  bool populated;  // source page-table entries already filled
 };
 
 int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cudaStream_t s,
                  void **ready, uint64_t total) {
   const uint64_t target = std::min<uint64_t>(128ull << 20, std::max<uint64_t>(2ull << 20, total / 64));
   const int grid_cap = 2 * wt::num_sms();
-  size_t i = 0;
-  while (i < rs.size()) {
+  // Tensors larger than a batch are cut into pieces (multiples of 64 KiB, so each piece keeps
+  // its range's alignment): page-table population and transfer then pipeline inside a tensor.
+  // A tensor's event is the event of the batch holding its last piece.
+  const uint64_t piece = std::max<uint64_t>(target & ~((1ull << 16) - 1), 1ull << 16);
+  std::vector<Range> ps;
+  ps.reserve(rs.size());
+  for (const Range &r : rs) {
+    if (r.n <= piece) {
+      ps.push_back(r);
+      continue;
+    }
+    for (uint64_t o = 0; o < r.n; o += piece)
+      ps.push_back({r.tensor, r.src_host + o, r.src_dev ? r.src_dev + o : nullptr, r.dst + o, std::min(piece, r.n - o),
+                    r.populated});
+  }
+  std::vector<std::pair<size_t, size_t>> batches;
+  for (size_t i = 0; i < ps.size();) {
     size_t j = i;
     uint64_t bytes = 0;
-    while (j < rs.size() && (j == i || (bytes < target && j - i < (size_t)wt::kMaxGather))) bytes += rs[j++].n;
-    // populate page-table entries of this batch's sources right before it is enqueued
-    if (!h->prefaulted)
-      for (size_t k = i; k < j; ++k) prefault(rs[k].src_host, rs[k].n);
+    while (j < ps.size() && (j == i || (bytes < target && j - i < (size_t)wt::kMaxGather))) bytes += ps[j++].n;
+    batches.push_back({i, j});
+    i = j;
+  }
+  // A helper thread populates the page-table entries of batch after batch; batch b is
+  // enqueued once its sources are populated, so this host work (about 1 TB/s for large
+  // ranges, a few microseconds per small one) overlaps the transfer of earlier batches.
+  // Concurrent populate calls on one address space contend, so one thread does them all.
+  std::vector<std::vector<std::pair<const uint8_t *, size_t>>> work(batches.size());
+  bool any = false;
+  for (size_t b = 0; b < batches.size(); ++b)
+    for (size_t k = batches[b].first; k < batches[b].second; ++k)
+      if (!ps[k].populated)
+        for (uint64_t o = 0; o < ps[k].n; o += 16ull << 20) {
+          work[b].push_back({ps[k].src_host + o, (size_t)std::min<uint64_t>(16ull << 20, ps[k].n - o)});
+          any = true;
+        }
+  std::mutex mu;
+  std::condition_variable cv;
+  size_t populated = any ? 0 : batches.size();
+  std::atomic<bool> stop{false};
+  std::thread helper;
+  if (any) {
+    helper = std::thread([&] {
+      for (size_t b = 0; b < batches.size() && !stop.load(); ++b) {
+        for (const auto &w : work[b]) prefault(w.first, w.second);
+        {
+          std::lock_guard<std::mutex> g(mu);
+          populated = b + 1;
+        }
+        cv.notify_one();
+      }
+    });
+  }
+  struct Joiner {
+    std::thread &t;
+    std::atomic<bool> &stop;
+    ~Joiner() {
+      stop.store(true);
+      if (t.joinable()) t.join();
+    }
+  } joiner{helper, stop};
+  for (size_t b = 0; b < batches.size(); ++b) {
+    if (any) {
+      std::unique_lock<std::mutex> lk(mu);
+      cv.wait(lk, [&] { return populated > b; });
+    }
+    const size_t i = batches[b].first, j = batches[b].second;
     if (mode == WT_ADOPT_GATHER) {
-      wt::GatherBatch b;
-      memset(&b, 0, sizeof b);
+      wt::GatherBatch gb;
+      memset(&gb, 0, sizeof gb);
       uint64_t chunks = 0;
       for (size_t k = i; k < j; ++k) {
-        const uint32_t q = b.n++;
-        b.chunk_prefix[q] = chunks;
-        b.src[q] = rs[k].src_dev;
-        b.dst[q] = rs[k].dst;
-        b.nbytes[q] = rs[k].n;
-        chunks += (rs[k].n + (1ull << wt::kGatherChunkLog2) - 1) >> wt::kGatherChunkLog2;
+        const uint32_t q = gb.n++;
+        gb.chunk_prefix[q] = chunks;
+        gb.src[q] = ps[k].src_dev;
+        gb.dst[q] = ps[k].dst;
+        gb.nbytes[q] = ps[k].n;
+        chunks += (ps[k].n + (1ull << wt::kGatherChunkLog2) - 1) >> wt::kGatherChunkLog2;
       }
-      b.chunk_prefix[b.n] = chunks;
+      gb.chunk_prefix[gb.n] = chunks;
       if (chunks) {
-        CU(wt::launch_gather(b, (int)std::min<uint64_t>(chunks, (uint64_t)grid_cap), s));
+        CU(wt::launch_gather(gb, (int)std::min<uint64_t>(chunks, (uint64_t)grid_cap), s));
         h->kernel_launches++;
       }
     } else {
       for (size_t k = i; k < j; ++k)
-        if (rs[k].n) CU(cudaMemcpyAsync(rs[k].dst, rs[k].src_dev, rs[k].n, cudaMemcpyDefault, s));
+        if (ps[k].n) CU(cudaMemcpyAsync(ps[k].dst, ps[k].src_dev, ps[k].n, cudaMemcpyDefault, s));
     }
     cudaEvent_t ev;
     int rc = new_event(h, &ev);
     if (rc) return rc;
     CU(cudaEventRecord(ev, s));
-    for (size_t k = i; k < j; ++k) ready[rs[k].tensor] = ev;
-    i = j;
+    for (size_t k = i; k < j; ++k) ready[ps[k].tensor] = ev;
   }
   return WT_OK;
 }
@@ -811,6 +871,7 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
         }
         if (e == cudaSuccess) {
           f.registered = true;
+          f.populated = true;  // registration pins (and so maps) every page
           void *dp = nullptr;
           e = cudaHostGetDevicePointer(&dp, f.base, 0);
           if (e != cudaSuccess) {
@@ -913,7 +974,8 @@ int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsign
       if (mode != WT_ADOPT_STAGED && f.route == WT_ROUTE_NONE)
         return set_err(WT_ENOTSUP, "wt_adopt: %s has no device route; use WT_ADOPT_STAGED", f.path.c_str());
       ready[k] = nullptr;
-      rs.push_back({k, f.base + t.offset, f.dev ? f.dev + t.offset : nullptr, static_cast<uint8_t *>(dst[k]), t.nbytes});
+      rs.push_back({k, f.base + t.offset, f.dev ? f.dev + t.offset : nullptr, static_cast<uint8_t *>(dst[k]), t.nbytes,
+                    f.populated || h->prefaulted});
       total += t.nbytes;
     }
     const cudaStream_t s = static_cast<cudaStream_t>(stream);

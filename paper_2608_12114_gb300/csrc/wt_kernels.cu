@@ -308,7 +308,7 @@ template <int DT, int NJ>
 __device__ __forceinline__ void tile_warp_rows(uint32_t tile, uint32_t V, uint32_t nr, uint32_t G,
                                                uint32_t gl, uint32_t sub, uint32_t rpw, int warp, int lane,
                                                const uint64_t (&xp)[8][Pairs<DT>::N], float *y) {
-  constexpr int U = NJ <= 2 ? 4 : (NJ <= 4 ? 2 : 1);
+  constexpr int U = NJ == 1 ? 8 : NJ == 2 ? 4 : (NJ <= 4 ? 2 : 1);
   const uint32_t step = kConsumerWarps * rpw;
   for (uint32_t base = warp * rpw; base < nr; base += U * step) {
     uint4 w[U][NJ];
@@ -341,6 +341,44 @@ __device__ __forceinline__ void tile_warp_rows(uint32_t tile, uint32_t V, uint32
         const uint32_t row = base + u * step + sub;
         if (gl == 0 && row < nr) y[row] = t[u];
       }
+    }
+  }
+}
+
+// Short-row tile (V <= 16 vectors): G = pow2ceil(V) lanes per row, one vector per lane,
+// 32 / G rows per warp per sweep.  Eight sweeps are loaded before use and their
+// reductions over the G lanes are unrolled, so the eight shuffle chains interleave.
+template <int DT, int G>
+__device__ __forceinline__ void tile_small_rows(uint32_t tile, uint32_t V, uint32_t nr, int warp, int lane,
+                                                const uint64_t (&xp)[Pairs<DT>::N], float *y) {
+  constexpr int RPW = 32 / G;
+  constexpr int U = 8;
+  const uint32_t gl = lane & (G - 1);
+  const uint32_t sub = lane / G;
+  const uint32_t step = kConsumerWarps * RPW;
+  for (uint32_t base = warp * RPW; base < nr; base += U * step) {
+    uint4 w[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const uint32_t row = base + u * step + sub;
+      w[u] = lds_or_zero(tile + (row * V + gl) * 16, row < nr && gl < V);
+    }
+    float t[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      Acc4 acc;
+      dot16<DT>(w[u], xp, acc);
+      t[u] = acc.total();
+    }
+#pragma unroll
+    for (int o = G / 2; o > 0; o >>= 1) {
+#pragma unroll
+      for (int u = 0; u < U; ++u) t[u] += __shfl_xor_sync(0xffffffffu, t[u], o);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const uint32_t row = base + u * step + sub;
+      if (gl == 0 && row < nr) y[row] = t[u];
     }
   }
 }
@@ -505,7 +543,15 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
           bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
           const uint32_t tile = stage0 + s * kStageBytes;
           float *y = md.y + r;
-          switch (nj) {
+          if (G < 32) {
+            switch (G) {
+              case 1: tile_small_rows<DT, 1>(tile, V, nr, warp, lane, xp[0], y); break;
+              case 2: tile_small_rows<DT, 2>(tile, V, nr, warp, lane, xp[0], y); break;
+              case 4: tile_small_rows<DT, 4>(tile, V, nr, warp, lane, xp[0], y); break;
+              case 8: tile_small_rows<DT, 8>(tile, V, nr, warp, lane, xp[0], y); break;
+              default: tile_small_rows<DT, 16>(tile, V, nr, warp, lane, xp[0], y); break;
+            }
+          } else switch (nj) {
             case 1: tile_warp_rows<DT, 1>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
             case 2: tile_warp_rows<DT, 2>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
             case 3: tile_warp_rows<DT, 3>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;

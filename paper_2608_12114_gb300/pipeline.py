@@ -75,6 +75,7 @@ class DeviceCheckpoint:
     bufs: List[object]                   # torch uint8 tensors, one per MatrixRef
     dst: Dict[int, int] = field(default_factory=dict)  # tensor index -> device address
     canary: int = 0
+    _tables: Dict[tuple, object] = field(default_factory=dict)
 
     @staticmethod
     def allocate(h: wt.Handle, mats: Sequence[MatrixRef], device="cuda", canary: int = 0,
@@ -129,14 +130,27 @@ class DeviceCheckpoint:
                 for k in self.gemv_mats()}
 
     def descs(self, xs, ys, events: Optional[Dict[int, int]] = None,
-              only: Optional[Sequence[int]] = None) -> List[wt.GemvDesc]:
-        out = []
-        pos = {i: n for n, i in enumerate(events)} if events else {}
-        for k in (only if only is not None else self.gemv_mats()):
-            m = self.mats[k]
-            ev = events[max(m.parts, key=pos.__getitem__)] if events else 0
-            out.append(wt.gemv_desc(self.bufs[k].data_ptr(), m.dtype, m.shape[0], m.shape[1],
-                                    xs[(m.shape[1], m.dtype)].data_ptr(), ys[k].data_ptr(), ev))
+              only: Optional[Sequence[int]] = None) -> np.ndarray:
+        """wt_pass descriptors (a DESC_DTYPE array) for the GEMV matrices, or for `only`.
+
+        With `events`, matrix k waits on the event of its last-ingested row block."""
+        ks = list(only) if only is not None else self.gemv_mats()
+        key = tuple(ks)
+        base = self._tables.get(key)
+        if base is None:  # the parts that depend only on this checkpoint's buffers
+            base = np.zeros(len(ks), wt.DESC_DTYPE)
+            mats = [self.mats[k] for k in ks]
+            base["W"] = [self.bufs[k].data_ptr() for k in ks]
+            base["dtype"] = [m.dtype for m in mats]
+            base["M"] = [m.shape[0] for m in mats]
+            base["K"] = [m.shape[1] for m in mats]
+            self._tables[key] = base
+        out = base.copy()
+        out["x"] = [xs[(self.mats[k].shape[1], self.mats[k].dtype)].data_ptr() for k in ks]
+        out["y"] = [ys[k].data_ptr() for k in ks]
+        if events:
+            pos = {i: n for n, i in enumerate(events)}
+            out["wait_event"] = [events[max(self.mats[k].parts, key=pos.__getitem__)] for k in ks]
         return out
 
     @property

@@ -13,6 +13,8 @@ import os
 from dataclasses import dataclass
 from typing import List, Optional, Sequence, Tuple
 
+import numpy as np
+
 HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libwt.so")
 
@@ -47,6 +49,12 @@ class GemvDesc(C.Structure):
     _fields_ = [("W", C.c_void_p), ("dtype", C.c_int32), ("reserved", C.c_int32),
                 ("M", C.c_uint64), ("K", C.c_uint64), ("x", C.c_void_p), ("y", C.c_void_p),
                 ("wait_event", C.c_void_p)]
+
+
+# The same 56-byte layout as a numpy record, for building many descriptors at once.
+DESC_DTYPE = np.dtype([("W", "<u8"), ("dtype", "<i4"), ("reserved", "<i4"), ("M", "<u8"), ("K", "<u8"),
+                       ("x", "<u8"), ("y", "<u8"), ("wait_event", "<u8")])
+assert DESC_DTYPE.itemsize == C.sizeof(GemvDesc)
 
 
 _lib = None
@@ -148,10 +156,16 @@ class Handle:
         _check(lib().wt_adopt(self.ptr, ia, da, n, mode, C.c_void_p(stream), ra))
         return [ra[i] or 0 for i in range(n)]
 
-    def pass_(self, descs: Sequence[GemvDesc], stream: int = 0):
-        """wt_pass over a list of GemvDesc."""
-        n = len(descs)
-        arr = (GemvDesc * max(1, n))(*descs)
+    def pass_(self, descs, stream: int = 0):
+        """wt_pass over a list of GemvDesc or a contiguous numpy array of DESC_DTYPE records."""
+        if isinstance(descs, np.ndarray):
+            if descs.dtype != DESC_DTYPE or not descs.flags.c_contiguous:
+                raise ValueError("descriptor array must be a contiguous DESC_DTYPE array")
+            n = descs.size
+            arr = C.cast(descs.ctypes.data if n else 0, C.POINTER(GemvDesc))
+        else:
+            n = len(descs)
+            arr = (GemvDesc * max(1, n))(*descs)
         _check(lib().wt_pass(self.ptr, arr, n, C.c_void_p(stream)))
 
     def checksum(self, ptrs: Sequence[int], nbytes: Sequence[int], out_dev: int, stream: int = 0,
