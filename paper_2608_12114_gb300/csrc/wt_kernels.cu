@@ -209,7 +209,8 @@ constexpr int kConsumers = kConsumerWarps * 32;
 constexpr int kGemvThreads = kConsumers + 32;
 constexpr size_t kBarOff = (size_t)kStages * kStageBytes;
 constexpr size_t kRedOff = kBarOff + 2 * kStages * sizeof(uint64_t);
-constexpr size_t kFlagOff = kRedOff + 2 * kConsumerWarps * kRowBlock * sizeof(float);
+constexpr int kRedRows = 64;  // rows whose warp partials are gathered before one cross-warp sum
+constexpr size_t kFlagOff = kRedOff + 2 * kConsumerWarps * kRedRows * sizeof(float);
 constexpr size_t kGemvSmem = kFlagOff + 16;
 
 // Two fp32 values in one 64-bit register; fma.rn.f32x2 performs two independent
@@ -415,6 +416,15 @@ __device__ __forceinline__ void tile_block_rows(uint32_t tile, uint32_t V, int c
   if ((lane & ((32 >> L) - 1)) == 0 && q < NR) rb[q * kConsumerWarps + warp] = sum;
 }
 
+// Rows per tile for a piece of `rows` rows.  Split-K pieces use balanced row blocks of at
+// most kRowBlock rows (27 rows -> 7, 7, 7, 6), so no stage of the piece runs nearly empty.
+__device__ __forceinline__ uint32_t piece_rows_per_tile(const MatDesc &md, const Piece &pc) {
+  if (md.mode != kModeSplitK) return md.rt;
+  const uint32_t rows = pc.r1 - pc.r0;
+  const uint32_t nblk = (rows + kRowBlock - 1) / kRowBlock;
+  return nblk ? (rows + nblk - 1) / nblk : 1;
+}
+
 // Sum of the consumer warps' partials of one row, in warp order (deterministic).
 __device__ __forceinline__ float sum_warps(const float *p) {
   float t = 0.f;
@@ -476,8 +486,9 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
         const Piece pc = pieces[pi];
         const MatDesc md = mats[pc.mat];
         const uint64_t rowb = (uint64_t)md.V * 16;
-        for (uint32_t r = pc.r0; r < pc.r1 && live; r += md.rt) {
-          const uint32_t nr = min(md.rt, pc.r1 - r);
+        const uint32_t rt = piece_rows_per_tile(md, pc);
+        for (uint32_t r = pc.r0; r < pc.r1 && live; r += rt) {
+          const uint32_t nr = min(rt, pc.r1 - r);
           const uint32_t nchunk = md.mode == kModeSplitK ? (md.V + md.vc - 1) / md.vc : 1;
           for (uint32_t c = 0; c < nchunk; ++c) {
             const uint32_t s = it % kStages;
@@ -573,48 +584,63 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
           const uint32_t v = ct + j * kConsumers;
           load_xpairs<DT>(md.x, v, j < (int)nj && v < V, xp[j]);
         }
+        // Warp partials of up to kRedRows rows collect in one half of `red`; the consumer
+        // group then synchronises once and sums them (one barrier per kRedRows rows).
+        uint32_t g0 = pc.r0, gn = 0;
         for (uint32_t r = pc.r0; r < pc.r1; r += md.rt) {
           const uint32_t nr = min(md.rt, pc.r1 - r);
           const uint32_t s = it % kStages;
           bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
           const uint32_t tile = stage0 + s * kStageBytes;
-          float *rb = red + par * (kConsumerWarps * kRowBlock);
+          float *rb = red + par * (kConsumerWarps * kRedRows) + gn * kConsumerWarps;
           if (!block_rows_dispatch<DT>(nj, nr, tile, V, ct, warp, lane, xp, rb) && ct == 0)
             atomicCAS(status, 0, -1);  // unreachable by construction of the plan
           __syncwarp();
           if (lane == 0) mbar_arrive(empty0 + 8 * s);
           ++it;
-          named_bar(1, kConsumers);
-          if (ct < (int)nr) md.y[r + ct] = sum_warps(rb + ct * kConsumerWarps);
-          par ^= 1;
+          gn += nr;
+          if (r + nr >= pc.r1 || gn + md.rt > (uint32_t)kRedRows) {
+            named_bar(1, kConsumers);
+            const float *gb = red + par * (kConsumerWarps * kRedRows);
+            for (uint32_t q = ct; q < gn; q += kConsumers) md.y[g0 + q] = sum_warps(gb + q * kConsumerWarps);
+            par ^= 1;
+            g0 += gn;
+            gn = 0;
+          }
         }
       } else {
-        // split-K: row blocks of kRowBlock rows, streamed in column chunks of md.vc vectors
+        // split-K: row blocks of up to kRowBlock rows, streamed in column chunks of md.vc
+        // vectors; the x slice of the next chunk is fetched while the current one is used.
         const uint32_t nchunk = (V + md.vc - 1) / md.vc;
-        for (uint32_t r = pc.r0; r < pc.r1; r += md.rt) {
-          const uint32_t nr = min(md.rt, pc.r1 - r);
+        const uint32_t rt = piece_rows_per_tile(md, pc);
+        load_xpairs<DT>(md.x, ct, (uint32_t)ct < min(md.vc, V), xp[0]);
+        for (uint32_t r = pc.r0; r < pc.r1; r += rt) {
+          const uint32_t nr = min(rt, pc.r1 - r);
           Acc4 acc[kRowBlock];
           for (uint32_t c = 0; c < nchunk; ++c) {
-            const uint32_t v0 = c * md.vc;
-            const uint32_t nv = min(md.vc, V - v0);
-            load_xpairs<DT>(md.x, v0 + ct, ct < nv, xp[0]);
+            const uint32_t nv = min(md.vc, V - c * md.vc);
+            const uint32_t c1 = c + 1 < nchunk ? c + 1 : 0;  // next chunk (or chunk 0 of the next block)
+            const uint32_t nv1 = min(md.vc, V - c1 * md.vc);
+            load_xpairs<DT>(md.x, c1 * md.vc + ct, (uint32_t)ct < nv1, xp[1]);
             const uint32_t s = it % kStages;
             bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
             const uint32_t tile = stage0 + s * kStageBytes;
             uint4 w[kRowBlock];
 #pragma unroll
             for (int q = 0; q < kRowBlock; ++q)
-              w[q] = lds_or_zero(tile + (q * md.vc + ct) * 16, q < (int)nr && ct < nv);
+              w[q] = lds_or_zero(tile + (q * md.vc + ct) * 16, q < (int)nr && (uint32_t)ct < nv);
 #pragma unroll
             for (int q = 0; q < kRowBlock; ++q) dot16<DT>(w[q], xp[0], acc[q]);
             __syncwarp();
             if (lane == 0) mbar_arrive(empty0 + 8 * s);
             ++it;
+#pragma unroll
+            for (int i = 0; i < NP; ++i) xp[0][i] = xp[1][i];
           }
           float t[kRowBlock];
 #pragma unroll
           for (int q = 0; q < kRowBlock; ++q) t[q] = acc[q].total();
-          float *rb = red + par * (kConsumerWarps * kRowBlock);
+          float *rb = red + par * (kConsumerWarps * kRedRows);
           const float sum = transpose_reduce<kRowBlock>(t, lane);
           const int q = lane >> 2;
           if ((lane & 3) == 0 && q < (int)nr) rb[q * kConsumerWarps + warp] = sum;
