@@ -62,6 +62,8 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="CPU budget of the oracle sample")
     p.add_argument("--data-dir", default=None)
     p.add_argument("--workers", type=int, default=0)
+    p.add_argument("--policy", action="store_true",
+                   help="measure the map / resident / per-use-copy endpoints and apply Algorithm 2 (one JSON line)")
     return p.parse_args()
 
 
@@ -554,12 +556,32 @@ def run_reference(args, rank, world):
     print(json.dumps(out), flush=True)
 
 
+def run_policy(args):
+    """Algorithm 2 (Sec. 8.1) on this GPU for the workload: a GB300 row of Table "policy"."""
+    ck, gen_s = make_files(args, 0, 1)
+    import torch
+    from paper_2608_12114_gb300 import build, policy
+    build.build()
+    torch.cuda.set_device(0)
+    h2d = pinned_h2d_gbs(torch)
+    out = policy.measure_gb300(ck.paths, reps=max(3, min(args.e2e_reps, 9)))
+    d = out.as_dict()
+    d.update({"metric": "endpoint selection (Algorithm 2): W/B per endpoint", "unit": "ms",
+              "config": {"workload": workload_desc(args)}, "pinned_h2d_gbs": round(h2d, 1),
+              "what": "map = GEMV reads the prefaulted file mapping in place; resident = GEMV over an HBM "
+                      "copy; copy = wt_adopt into HBM then the event-gated GEMV, every pass"})
+    print(json.dumps(d), flush=True)
+
+
 def main():
     args = parse_args()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     if args.impl == "reference":
         run_reference(args, rank, world)
+        return
+    if args.policy:
+        run_policy(args)
         return
     run_wt(args, rank, world)
 

@@ -162,7 +162,11 @@ int wt_file_route(const wt_handle *h, size_t f, unsigned *route);
 int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsigned mode,
              void *stream, void **ready);
 
-/* Enqueue one GEMV per descriptor on `stream`.  Consecutive descriptors that
+/* Enqueue one GEMV per descriptor on `stream`.  W may be device memory (the resident
+ * endpoint: TMA-fed kernel streaming HBM) or lie inside one of this handle's file mappings
+ * (the map endpoint of Sec. 8.1, contract C1: the kernel reads the mapped rows in place over
+ * the host link, no copy; the rows are populated once when the plan is built and must stay
+ * resident, Algorithm 2's precondition).  y must not lie inside a mapping.  Consecutive descriptors that
  * carry the same wait_event form one group: the stream waits on that event
  * (cudaStreamWaitEvent, never a host wait) and one persistent launch streams
  * every matrix of the group, rows split evenly across the SMs.  Repeated
@@ -205,6 +209,13 @@ int wt_checksum_noalloc(const void *const *ptr, const uint64_t *nbytes, size_t n
 /* Device-side status word of the handle: 0, or the first WT_ETIMEDOUT-class
  * code a bounded wait inside a kernel recorded (reads it synchronously). */
 int wt_device_status(wt_handle *h, int *status);
+
+/* Bytes of the handle's file mappings that are resident in the page cache right now
+ * (mincore over every mapping, page granular, clipped to the file sizes) and their total.
+ * Algorithm 2 stops with "storage-bound" when the mapped set is not resident (Sec. 8.1);
+ * Table "controls" queries residency before and after a measurement.  Host-only handles
+ * work too.  Errors: WT_EINVAL, WT_EIO. */
+int wt_residency(const wt_handle *h, uint64_t *resident, uint64_t *total);
 
 /* Kernels this handle has launched so far (gather, GEMV, checksum launches). */
 int wt_kernel_launches(const wt_handle *h, uint64_t *n);

@@ -201,8 +201,9 @@ struct Plan {
     uint64_t M;
   };
   struct Group {
-    cudaEvent_t wait = nullptr;
+    size_t first = 0;  // index of the group's first descriptor (its wait_event is read per call)
     std::vector<Launch> launches;
+    std::vector<Launch> mapped;  // W read in place from a file mapping (map endpoint)
     std::vector<Generic> generic;
     std::vector<Zero> zero;
   };
@@ -667,14 +668,24 @@ int validate_desc(const wt_gemv_desc &d, size_t i) {
   return WT_OK;
 }
 
+// The mapping holding [p, p + n) (whole range inside one file mapping), or nullptr.
+const File *mapping_of(const wt_handle *h, const void *p, uint64_t n) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+  for (const File &f : h->files) {
+    const uintptr_t s = reinterpret_cast<uintptr_t>(f.base);
+    if (a >= s && a + n <= s + f.size && a + n >= a) return &f;
+  }
+  return nullptr;
+}
+
 int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
   size_t i = 0;
   while (i < n) {
     size_t j = i;
     while (j < n && d[j].wait_event == d[i].wait_event) ++j;
     Plan::Group g;
-    g.wait = static_cast<cudaEvent_t>(d[i].wait_event);
-    std::vector<wt::MatDesc> by_dt[3];
+    g.first = i;
+    std::vector<wt::MatDesc> by_dt[3], mapped_dt[3];
     for (size_t k = i; k < j; ++k) {
       const wt_gemv_desc &q = d[k];
       if (q.M == 0) continue;
@@ -685,20 +696,39 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
       }
       const bool fast = ((reinterpret_cast<uintptr_t>(q.W) | reinterpret_cast<uintptr_t>(q.x)) & 15) == 0 &&
                         (q.K * es) % 16 == 0;
-      if (fast) by_dt[q.dtype].push_back(make_mat(q));
-      else g.generic.push_back({q.dtype, static_cast<const uint8_t *>(q.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K});
+      const File *f = mapping_of(h, q.W, q.M * q.K * es);
+      if (!f && inside_mapping(h, q.W, q.M * q.K * es))
+        return set_err(WT_EINVAL, "wt_pass: W of desc %zu straddles the end of a mapping", k);
+      if (f) {
+        // map endpoint: the kernel reads the mapped rows in place over the host link
+        if (f->route == WT_ROUTE_NONE || !f->dev)
+          return set_err(WT_ENOTSUP, "wt_pass: W of desc %zu lies in %s, which has no device route", k, f->path.c_str());
+        const uint64_t off = reinterpret_cast<const uint8_t *>(q.W) - f->base;
+        if (!h->prefaulted && !f->populated) prefault(f->base + off, q.M * q.K * es);
+        wt_gemv_desc qd = q;
+        qd.W = f->dev + off;
+        if (fast) mapped_dt[q.dtype].push_back(make_mat(qd));
+        else g.generic.push_back({q.dtype, static_cast<const uint8_t *>(qd.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K});
+      } else if (fast) {
+        by_dt[q.dtype].push_back(make_mat(q));
+      } else {
+        g.generic.push_back({q.dtype, static_cast<const uint8_t *>(q.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K});
+      }
     }
-    for (int dt = 0; dt < 3; ++dt) {
-      if (by_dt[dt].empty()) continue;
-      Plan::Launch L;
-      L.dtype = dt;
-      std::vector<wt::Piece> pieces;
-      std::vector<uint32_t> begin;
-      partition(by_dt[dt], L.grid, pieces, begin);
-      L.mats = append(P->table, by_dt[dt]);
-      L.pieces = append(P->table, pieces);
-      L.begin = append(P->table, begin);
-      g.launches.push_back(L);
+    for (int pass = 0; pass < 2; ++pass) {
+      for (int dt = 0; dt < 3; ++dt) {
+        std::vector<wt::MatDesc> &ms = pass == 0 ? by_dt[dt] : mapped_dt[dt];
+        if (ms.empty()) continue;
+        Plan::Launch L;
+        L.dtype = dt;
+        std::vector<wt::Piece> pieces;
+        std::vector<uint32_t> begin;
+        partition(ms, L.grid, pieces, begin);
+        L.mats = append(P->table, ms);
+        L.pieces = append(P->table, pieces);
+        L.begin = append(P->table, begin);
+        (pass == 0 ? g.launches : g.mapped).push_back(L);
+      }
     }
     P->groups.push_back(std::move(g));
     i = j;
@@ -709,7 +739,6 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
   CU(cudaMalloc(reinterpret_cast<void **>(&P->dev), bytes));
   CU(cudaEventCreateWithFlags(&P->uploaded, cudaEventDisableTiming));
   CU(cudaEventCreateWithFlags(&P->last, cudaEventDisableTiming));
-  (void)h;
   return WT_OK;
 }
 
@@ -722,7 +751,7 @@ void destroy_plan(Plan *P) {
   delete P;
 }
 
-int run_plan(wt_handle *h, Plan *P, cudaStream_t s) {
+int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s) {
   if (!P->sent) {
     CU(cudaMemcpyAsync(P->dev, P->host, std::max<size_t>(16, align16(P->table.size())), cudaMemcpyHostToDevice, s));
     CU(cudaEventRecord(P->uploaded, s));
@@ -732,7 +761,8 @@ int run_plan(wt_handle *h, Plan *P, cudaStream_t s) {
     CU(cudaStreamWaitEvent(s, P->uploaded, 0));
   }
   for (const Plan::Group &g : P->groups) {
-    if (g.wait) CU(cudaStreamWaitEvent(s, g.wait, 0));
+    cudaEvent_t wait = static_cast<cudaEvent_t>(d[g.first].wait_event);
+    if (wait) CU(cudaStreamWaitEvent(s, wait, 0));
     for (const Plan::Zero &z : g.zero) CU(cudaMemsetAsync(z.y, 0, z.M * sizeof(float), s));
     for (const Plan::Launch &L : g.launches) {
       wt::GemvLaunch gl;
@@ -743,6 +773,17 @@ int run_plan(wt_handle *h, Plan *P, cudaStream_t s) {
       gl.begin = reinterpret_cast<const uint32_t *>(P->dev + L.begin);
       gl.status = h->status;
       CU(wt::launch_gemv(gl, s));
+      h->kernel_launches++;
+    }
+    for (const Plan::Launch &L : g.mapped) {
+      wt::GemvLaunch gl;
+      gl.dtype = L.dtype;
+      gl.grid = L.grid;
+      gl.mats = reinterpret_cast<const wt::MatDesc *>(P->dev + L.mats);
+      gl.pieces = reinterpret_cast<const wt::Piece *>(P->dev + L.pieces);
+      gl.begin = reinterpret_cast<const uint32_t *>(P->dev + L.begin);
+      gl.status = h->status;
+      CU(wt::launch_gemv_mapped(gl, s));
       h->kernel_launches++;
     }
     for (const Plan::Generic &q : g.generic) {
@@ -994,10 +1035,20 @@ int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream) {
   for (size_t i = 0; i < n; ++i) {
     int rc = validate_desc(d[i], i);
     if (rc) return rc;
+    if (d[i].M && inside_mapping(h, d[i].y, d[i].M * sizeof(float)))
+      return set_err(WT_EINVAL, "wt_pass: y of desc %zu lies inside a read-only mapping", i);
   }
   std::lock_guard<std::mutex> g(h->mu);
   try {
-    const uint8_t *kb = reinterpret_cast<const uint8_t *>(d);
+    // Plans are keyed by the descriptors with each wait_event replaced by its group's
+    // ordinal: calls that differ only in which events they wait on share one plan.
+    std::vector<wt_gemv_desc> kd(d, d + n);
+    uintptr_t ordinal = 0;
+    for (size_t i = 0; i < n; ++i) {
+      if (i == 0 || d[i].wait_event != d[i - 1].wait_event) ++ordinal;
+      kd[i].wait_event = d[i].wait_event ? reinterpret_cast<void *>(ordinal) : nullptr;
+    }
+    const uint8_t *kb = reinterpret_cast<const uint8_t *>(kd.data());
     std::vector<uint8_t> key(kb, kb + n * sizeof(wt_gemv_desc));
     Plan *P = nullptr;
     for (auto it = h->plans.begin(); it != h->plans.end(); ++it)
@@ -1021,7 +1072,7 @@ int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream) {
         h->plans.pop_back();
       }
     }
-    return run_plan(h, P, static_cast<cudaStream_t>(stream));
+    return run_plan(h, P, d, static_cast<cudaStream_t>(stream));
   } catch (const std::bad_alloc &) {
     return set_err(WT_ENOMEM, "wt_pass: out of host memory");
   }
@@ -1084,6 +1135,25 @@ int wt_device_status(wt_handle *h, int *status) {
     return WT_OK;
   }
   CU(cudaMemcpy(status, h->status, sizeof(int), cudaMemcpyDeviceToHost));
+  return WT_OK;
+}
+
+int wt_residency(const wt_handle *h, uint64_t *resident, uint64_t *total) {
+  if (!h || !resident || !total) return set_err(WT_EINVAL, "wt_residency: NULL argument");
+  const size_t pg = (size_t)sysconf(_SC_PAGESIZE);
+  uint64_t res = 0, tot = 0;
+  std::vector<unsigned char> vec;
+  for (const File &f : h->files) {
+    const size_t pages = (f.size + pg - 1) / pg;
+    vec.assign(pages, 0);
+    if (pages && mincore(f.base, f.size, vec.data()) != 0)
+      return set_err(WT_EIO, "wt_residency: mincore(%s): %s", f.path.c_str(), strerror(errno));
+    for (size_t i = 0; i < pages; ++i)
+      if (vec[i] & 1) res += std::min<uint64_t>(pg, f.size - i * pg);
+    tot += f.size;
+  }
+  *resident = res;
+  *total = tot;
   return WT_OK;
 }
 

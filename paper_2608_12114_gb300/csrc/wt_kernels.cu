@@ -654,6 +654,49 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
   __syncthreads();
 }
 
+// Map endpoint: one lane group per row (G = pow2ceil(V) lanes for rows shorter than 32
+// vectors, the whole warp otherwise); each lane keeps four 16-byte loads of the mapped rows
+// in flight; x comes from L1/L2.  Link-bound by design (the weights never enter HBM).
+template <int DT>
+__global__ void __launch_bounds__(256) gemv_mapped_kernel(const MatDesc *__restrict__ mats,
+                                                          const Piece *__restrict__ pieces,
+                                                          const uint32_t *__restrict__ begin) {
+  constexpr int NP = Pairs<DT>::N;
+  constexpr int kWarps = 8;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (uint32_t pi = begin[blockIdx.x]; pi < begin[blockIdx.x + 1]; ++pi) {
+    const Piece pc = pieces[pi];
+    const MatDesc md = mats[pc.mat];
+    const uint32_t V = md.V;
+    const uint32_t G = V >= 32 ? 32u : (V <= 1 ? 1u : 1u << (32 - __clz(V - 1)));
+    const uint32_t gl = lane & (G - 1), sub = lane / G, rpw = 32 / G;
+    for (uint32_t base = pc.r0 + warp * rpw; base < pc.r1; base += kWarps * rpw) {
+      const uint32_t row = base + sub;
+      const bool valid = row < pc.r1;
+      const uint4 *w4 = reinterpret_cast<const uint4 *>(md.W + (uint64_t)(valid ? row : pc.r0) * V * 16);
+      Acc4 acc;
+      for (uint32_t v = gl; v < V; v += 4 * G) {
+        uint4 w[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const uint32_t vv = v + u * G;
+          w[u] = (valid && vv < V) ? w4[vv] : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const uint32_t vv = v + u * G;
+          uint64_t xp[NP];
+          load_xpairs<DT>(md.x, vv, vv < V, xp);
+          dot16<DT>(w[u], xp, acc);
+        }
+      }
+      float t = acc.total();
+      for (uint32_t o = G >> 1; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+      if (valid && gl == 0) md.y[row] = t;
+    }
+  }
+}
+
 // Fallback: one warp per row, byte-assembled scalar loads (any alignment).
 template <int DT>
 __global__ void gemv_generic_kernel(const uint8_t *W, const uint8_t *x, float *y, uint64_t M,
@@ -826,6 +869,17 @@ cudaError_t launch_gemv(const GemvLaunch &L, cudaStream_t s) {
     case 0: gemv_tma_kernel<0><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
     case 1: gemv_tma_kernel<1><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
     case 2: gemv_tma_kernel<2><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemv_mapped(const GemvLaunch &L, cudaStream_t s) {
+  if (L.grid <= 0) return cudaSuccess;
+  switch (L.dtype) {
+    case 0: gemv_mapped_kernel<0><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
+    case 1: gemv_mapped_kernel<1><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
+    case 2: gemv_mapped_kernel<2><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();

@@ -72,6 +72,11 @@ cudaError_t gemv_prepare();  // one-time function attributes
 cudaError_t launch_gemv(const GemvLaunch &L, cudaStream_t s);
 size_t gemv_smem_bytes();
 
+// Map endpoint (the paper's adoption, contract C1): W is read in place from a file mapping
+// the device reaches over the host link, with 16-byte loads and no TMA; same tables as
+// launch_gemv (MatDesc.W holds the device-readable address of the mapped rows).
+cudaError_t launch_gemv_mapped(const GemvLaunch &L, cudaStream_t s);
+
 // Fallback for operands the tiled kernel cannot take (unaligned W/x or rows
 // whose byte length is not a multiple of 16): one warp per row, scalar loads.
 cudaError_t launch_gemv_generic(int dtype, const uint8_t *W, const uint8_t *x, float *y,

@@ -29,8 +29,8 @@ MODE_NAMES = {WT_ADOPT_GATHER: "gather", WT_ADOPT_CE: "ce", WT_ADOPT_STAGED: "st
 # every entry point declared in include/wt.h
 SYMBOLS = ("wt_last_error", "wt_abi_version", "wt_open", "wt_num_tensors", "wt_num_files",
            "wt_tensor_info", "wt_find", "wt_file_route", "wt_adopt", "wt_pass", "wt_checksum",
-           "wt_checksum_plain", "wt_checksum_noalloc", "wt_device_status", "wt_kernel_launches",
-           "wt_close")
+           "wt_checksum_plain", "wt_checksum_noalloc", "wt_device_status", "wt_residency",
+           "wt_kernel_launches", "wt_close")
 
 
 class WtError(RuntimeError):
@@ -84,6 +84,7 @@ def lib(path: str = LIB_PATH):
     L.wt_checksum_noalloc.argtypes = [C.POINTER(vp), u64p, sz, vp, vp]
     L.wt_device_status.argtypes = [vp, C.POINTER(C.c_int)]
     L.wt_kernel_launches.argtypes = [vp, u64p]
+    L.wt_residency.argtypes = [vp, u64p, u64p]
     L.wt_close.argtypes = [vp]
     for s in SYMBOLS:
         if s not in ("wt_last_error",):
@@ -180,6 +181,12 @@ class Handle:
         s = C.c_int()
         _check(lib().wt_device_status(self.ptr, C.byref(s)))
         return s.value
+
+    def residency(self) -> Tuple[int, int]:
+        """wt_residency: (bytes resident in the page cache, total mapped bytes)."""
+        r, t = C.c_uint64(), C.c_uint64()
+        _check(lib().wt_residency(self.ptr, C.byref(r), C.byref(t)))
+        return r.value, t.value
 
     def kernel_launches(self) -> int:
         v = C.c_uint64()
