@@ -230,6 +230,7 @@ struct Ring {
 
 struct wt_handle {
   std::vector<File> files;
+  std::vector<std::pair<uintptr_t, uint32_t>> by_base;  // (mapping start, file), sorted: address lookups
   std::vector<std::pair<uint32_t, uint32_t>> order;  // global tensor index -> (file, entry)
   bool host_only = false;
   bool prefaulted = false;
@@ -382,13 +383,15 @@ int prepare_device(int dev) {
   return WT_OK;
 }
 
+// Mappings never overlap, so sorted by start, a range [a, b) meets a mapping iff it meets the
+// last mapping starting before b.
 bool inside_mapping(const wt_handle *h, const void *p, uint64_t n) {
-  const uintptr_t a = reinterpret_cast<uintptr_t>(p), b = a + n;
-  for (const File &f : h->files) {
-    const uintptr_t s = reinterpret_cast<uintptr_t>(f.base), e = s + f.size;
-    if (a < e && b > s) return true;
-  }
-  return false;
+  const uintptr_t a = reinterpret_cast<uintptr_t>(p), b = a + (n ? n : 1);
+  auto it = std::lower_bound(h->by_base.begin(), h->by_base.end(), std::make_pair(b, (uint32_t)0));
+  if (it == h->by_base.begin()) return false;
+  const File &f = h->files[std::prev(it)->second];
+  const uintptr_t s = reinterpret_cast<uintptr_t>(f.base), e = s + f.size;
+  return a < e && b > s;
 }
 
 int new_event(wt_handle *h, cudaEvent_t *ev) {
@@ -671,11 +674,11 @@ int validate_desc(const wt_gemv_desc &d, size_t i) {
 // The mapping holding [p, p + n) (whole range inside one file mapping), or nullptr.
 const File *mapping_of(const wt_handle *h, const void *p, uint64_t n) {
   const uintptr_t a = reinterpret_cast<uintptr_t>(p);
-  for (const File &f : h->files) {
-    const uintptr_t s = reinterpret_cast<uintptr_t>(f.base);
-    if (a >= s && a + n <= s + f.size && a + n >= a) return &f;
-  }
-  return nullptr;
+  auto it = std::upper_bound(h->by_base.begin(), h->by_base.end(), std::make_pair(a, UINT32_MAX));
+  if (it == h->by_base.begin()) return nullptr;
+  const File &f = h->files[std::prev(it)->second];
+  const uintptr_t s = reinterpret_cast<uintptr_t>(f.base);
+  return (a >= s && a + n <= s + f.size && a + n >= a) ? &f : nullptr;
 }
 
 int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
@@ -873,6 +876,8 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
     }
     for (int f = 0; f < n_paths; ++f)
       for (uint32_t e = 0; e < h->files[f].tensors.size(); ++e) h->order.push_back({(uint32_t)f, e});
+    for (int f = 0; f < n_paths; ++f) h->by_base.push_back({reinterpret_cast<uintptr_t>(h->files[f].base), (uint32_t)f});
+    std::sort(h->by_base.begin(), h->by_base.end());
     if (flags & WT_OPEN_PREFAULT) {
       host_pool().parallel_for((size_t)n_paths, [&](size_t i) { prefault(h->files[i].base, h->files[i].size); });
       h->prefaulted = true;
