@@ -39,6 +39,7 @@ WORKLOADS = {
     "mid": "mid decoder checkpoint, bf16, 3 shards (5.40 GB): 32 layers, d=2560, FFN 6912, vocab 32000",
     "many": "many-small: 1253 bf16 matrices split by rows across 2506 files (1.56 GB)",
     "tiny": "tiny: 8 fp32 256x256 matrices + 8 fp32[256] vectors in one file (2.1 MB)",
+    "protocol": "matched protocol by bytes: 12 files of one bf16 12288x3584 matrix (88.1 MB each, 1.06 GB)",
 }
 
 
@@ -62,6 +63,8 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="CPU budget of the oracle sample")
     p.add_argument("--data-dir", default=None)
     p.add_argument("--workers", type=int, default=0)
+    p.add_argument("--cube", action="store_true",
+                   help="the C1/C2/C3 contract ablation and ordering mechanisms on the protocol workload")
     p.add_argument("--policy", action="store_true",
                    help="measure the map / resident / per-use-copy endpoints and apply Algorithm 2 (one JSON line)")
     return p.parse_args()
@@ -76,6 +79,8 @@ def workload_ck(args, outdir):
         return synth.sweep(outdir, points=[int(w.split(":")[1])])
     if w == "tiny":
         return synth.tiny(outdir)
+    if w == "protocol":
+        return synth.protocol(outdir)
     if w == "many":
         return synth.many(outdir)
     if w in ("mid", "large"):
@@ -556,6 +561,22 @@ def run_reference(args, rank, world):
     print(json.dumps(out), flush=True)
 
 
+def run_cube(args):
+    """Table "cube" and the ordering figure (Sec. 4) on this GPU, protocol workload by default."""
+    if args.workload == "large":
+        args.workload = "protocol"
+    ck, gen_s = make_files(args, 0, 1)
+    import torch
+    from paper_2608_12114_gb300 import build, contract
+    build.build()
+    torch.cuda.set_device(0)
+    out = contract.measure(ck.paths, reps=max(3, min(args.e2e_reps, 9)))
+    out.update({"metric": "execution-contract ablation: idle GB/s per cell, excess ms per pass over an "
+                          "in-flight framework workload", "config": {"workload": workload_desc(args)},
+                "cells": "(weights, activations, ordering): map = C1 on, device = C2 on, stream = C3 on"})
+    print(json.dumps(out), flush=True)
+
+
 def run_policy(args):
     """Algorithm 2 (Sec. 8.1) on this GPU for the workload: a GB300 row of Table "policy"."""
     ck, gen_s = make_files(args, 0, 1)
@@ -582,6 +603,9 @@ def main():
         return
     if args.policy:
         run_policy(args)
+        return
+    if args.cube:
+        run_cube(args)
         return
     run_wt(args, rank, world)
 

@@ -44,7 +44,7 @@ DTYPE_NAMES = {DT_F32: "f32", DT_BF16: "bf16", DT_F16: "f16", DT_I8: "i8", DT_U8
 ELEM_SIZE = {DT_F32: 4, DT_BF16: 2, DT_F16: 2, DT_I8: 1, DT_U8: 1}
 
 # spawn-key prefixes for the per-tensor value streams of each workload
-_STREAM_KEY = {"many": 1, "sweep": 2, "mid": 3, "large": 4, "custom": 5}
+_STREAM_KEY = {"many": 1, "sweep": 2, "mid": 3, "large": 4, "custom": 5, "protocol": 6}
 _CHUNK = 1 << 24  # elements per value stream (each chunk of a tensor has its own stream)
 
 
@@ -363,10 +363,24 @@ def custom(outdir: str, shapes: Sequence[Tuple[int, int]], dtype: int = DT_BF16,
     return Checkpoint(name, [os.path.join(outdir, name + ".wt")], tensors, mats)
 
 
+def protocol(outdir: str, matrices: int = 12, rows: int = 12288, cols: int = 3584) -> Checkpoint:
+    """The paper's matched protocol by bytes (Sec. 3.1): a pass visits 12 page-cache-resident
+    files of 88.1 MB each (there 12288x7168 int8 with fp16 row scales; here 12288x3584 bf16,
+    the same weight bytes per file)."""
+    tensors, mats, paths = [], [], []
+    for f in range(matrices):
+        tensors.append(TensorSpec("w", DT_BF16, (rows, cols), f, key=(_STREAM_KEY["protocol"], f)))
+        mats.append(Matrix("p%d" % f, DT_BF16, rows, cols, [f]))
+        paths.append(os.path.join(outdir, "protocol_%02d.wt" % f))
+    return Checkpoint("protocol", paths, tensors, mats)
+
+
 def build(workload: str, outdir: str, workers: int = 0, **kw) -> Checkpoint:
     """Describe and write a workload; returns the Checkpoint (paths, tensors, matrices)."""
     if workload == "tiny":
         ck = tiny(outdir)
+    elif workload == "protocol":
+        ck = protocol(outdir, **kw)
     elif workload == "sweep":
         ck = sweep(outdir, **kw)
     elif workload == "many":
