@@ -58,6 +58,8 @@ def lib():
                               C.c_void_p, C.c_void_p]
         L.or_gemv_rows.argtypes = [C.c_void_p, C.c_int, C.c_uint64, C.c_uint64, C.c_void_p,
                                    C.c_void_p, C.c_uint64, C.c_void_p, C.c_void_p]
+        L.or_gemv_q8.argtypes = [C.c_void_p, C.c_void_p, C.c_uint64, C.c_uint64, C.c_void_p, C.c_void_p,
+                                 C.c_uint64, C.c_void_p, C.c_void_p]
         _lib = L
     return _lib
 
@@ -149,6 +151,23 @@ def gemv_rows(W: np.ndarray, dtype: int, M: int, K: int, x: np.ndarray,
     if r.size and lib().or_gemv_rows(_ptr(W), dtype, M, K, _ptr(x), _ptr(r), r.size,
                                      _ptr(yhat), _ptr(a)) != 0:
         raise OracleError("gemv_rows: bad dtype or row")
+    return yhat, a
+
+
+def gemv_q8(W: np.ndarray, s: np.ndarray, M: int, K: int, x: np.ndarray,
+            rows: Optional[Sequence[int]] = None) -> Tuple[np.ndarray, np.ndarray]:
+    """(yhat, a) for int8 W [M, K] with fp16 row scales s [M] and fp16 x [K] (O3, int8 form):
+    yhat_i = s_i * sum_j W_ij x_j, a_i = |s_i| * sum_j |W_ij x_j|; all rows or the given rows."""
+    W = np.ascontiguousarray(W).view(np.uint8)
+    s = np.ascontiguousarray(s).view(np.uint8)
+    x = np.ascontiguousarray(x).view(np.uint8)
+    r = None if rows is None else np.ascontiguousarray(rows, dtype=np.uint64)
+    n = M if r is None else r.size
+    yhat = np.zeros(n, np.float64)
+    a = np.zeros(n, np.float64)
+    if n and lib().or_gemv_q8(_ptr(W), _ptr(s), M, K, _ptr(x), None if r is None else _ptr(r), n,
+                              _ptr(yhat), _ptr(a)) != 0:
+        raise OracleError("gemv_q8: bad row")
     return yhat, a
 
 

@@ -314,6 +314,28 @@ int or_gemv(const uint8_t *W, int dtype, uint64_t M, uint64_t K, const uint8_t *
   return 0;
 }
 
+/* O3 for int8 weights with fp16 row scales (the paper's single-token kernel, Sec. 3.1 and
+ * Table "tab:tax"): yhat_i = s_i * sum_j W_ij x_j and a_i = |s_i| * sum_j |W_ij x_j| in fp64,
+ * j in index order; W is int8 [M, K], s is fp16 [M], x is fp16 [K]. */
+int or_gemv_q8(const uint8_t *W, const uint8_t *s, uint64_t M, uint64_t K, const uint8_t *x,
+               const uint64_t *rows, uint64_t nrows, double *yhat, double *a) {
+  for (uint64_t i = 0; i < nrows; ++i) {
+    const uint64_t r = rows ? rows[i] : i;
+    if (r >= M) return -1;
+    const uint8_t *row = W + r * K;
+    double acc = 0.0, abs_acc = 0.0;
+    for (uint64_t j = 0; j < K; ++j) {
+      const double p = (double)(int8_t)row[j] * elem(x, 2, j);
+      acc += p;
+      abs_acc += fabs(p);
+    }
+    const double sc = elem(s, 2, r);
+    yhat[i] = sc * acc;
+    a[i] = fabs(sc) * abs_acc;
+  }
+  return 0;
+}
+
 /* O3 for a chosen set of rows (full-size checks sample rows). */
 int or_gemv_rows(const uint8_t *W, int dtype, uint64_t M, uint64_t K, const uint8_t *x,
                  const uint64_t *rows, uint64_t nrows, double *yhat, double *a) {

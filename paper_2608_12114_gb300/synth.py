@@ -44,7 +44,7 @@ DTYPE_NAMES = {DT_F32: "f32", DT_BF16: "bf16", DT_F16: "f16", DT_I8: "i8", DT_U8
 ELEM_SIZE = {DT_F32: 4, DT_BF16: 2, DT_F16: 2, DT_I8: 1, DT_U8: 1}
 
 # spawn-key prefixes for the per-tensor value streams of each workload
-_STREAM_KEY = {"many": 1, "sweep": 2, "mid": 3, "large": 4, "custom": 5, "protocol": 6}
+_STREAM_KEY = {"many": 1, "sweep": 2, "mid": 3, "large": 4, "custom": 5, "protocol": 6, "protocol_q8": 7}
 _CHUNK = 1 << 24  # elements per value stream (each chunk of a tensor has its own stream)
 
 
@@ -56,7 +56,8 @@ class TensorSpec:
     dtype: int
     shape: Tuple[int, ...]
     file: int
-    fill: str = "normal"          # "normal" (std=scale), "uniform" (+-scale), "ones", "array"
+    fill: str = "normal"          # "normal" (std=scale), "uniform" (+-scale), "ones", "array",
+                                  # "int8" (uniform integers in [-127, 127]), "rowscale" (U[scale, 10*scale])
     scale: float = 0.02
     key: Tuple[int, ...] = ()     # spawn key of the value stream
     offset: int = 0               # absolute file offset (filled by layout())
@@ -76,6 +77,7 @@ class Matrix:
     M: int
     K: int
     parts: List[int]              # tensor indices, in row order
+    scale: Optional[int] = None   # tensor index of the fp16 row scales (int8 weights)
 
 
 @dataclasses.dataclass
@@ -151,6 +153,10 @@ def _tensor_values(t: TensorSpec, start: int, count: int, rng) -> np.ndarray:
     elif t.fill == "array":
         return np.ascontiguousarray(t.array).reshape(-1).view(np.uint8)[
             start * ELEM_SIZE[t.dtype]:(start + count) * ELEM_SIZE[t.dtype]]
+    elif t.fill == "int8":
+        return rng.integers(-127, 128, count, dtype=np.int8).view(np.uint8)
+    elif t.fill == "rowscale":
+        v = rng.uniform(t.scale, 10 * t.scale, count).astype(np.float32)
     else:
         raise ValueError(t.fill)
     if t.dtype == DT_F32:
@@ -169,10 +175,13 @@ def _rng_for(t: TensorSpec, chunk: int):
 
 def make_x(K: int, dtype: int) -> np.ndarray:
     """GEMV input for inner size K: N(0,1) from PCG64(1000003 + K), cast fp64->fp32->dtype (RNE).
+    int8 weights take fp16 activations, so DT_I8 returns fp16 x.
 
     Returned as the raw little-endian element bytes (uint8)."""
     rng = np.random.Generator(np.random.PCG64(1000003 + K))
     v = rng.standard_normal(K).astype(np.float32)
+    if dtype == DT_I8:
+        dtype = DT_F16
     if dtype == DT_F32:
         return v.astype("<f4").view(np.uint8).copy()
     if dtype == DT_BF16:
@@ -213,7 +222,7 @@ def _write_chunk(path: str, t: TensorSpec, c: int) -> int:
     n = t.nbytes // es
     s = c * _CHUNK
     cnt = min(_CHUNK, n - s)
-    rng = _rng_for(t, c) if t.fill in ("normal", "uniform") else None
+    rng = _rng_for(t, c) if t.fill in ("normal", "uniform", "int8", "rowscale") else None
     buf = np.ascontiguousarray(_tensor_values(t, s, cnt, rng))
     fd = os.open(path, os.O_WRONLY)
     try:
@@ -375,12 +384,38 @@ def protocol(outdir: str, matrices: int = 12, rows: int = 12288, cols: int = 358
     return Checkpoint("protocol", paths, tensors, mats)
 
 
+def protocol_q8(outdir: str, matrices: int = 12, rows: int = 12288, cols: int = 7168) -> Checkpoint:
+    """The paper's matched protocol (Sec. 3.1): 12 files, each one int8 rows x cols matrix "w"
+    (88.1 MB at 12288x7168) and its fp16 row scales "w.scale"."""
+    tensors, mats, paths = [], [], []
+    for f in range(matrices):
+        tensors.append(TensorSpec("w", DT_I8, (rows, cols), f, fill="int8", key=(_STREAM_KEY["protocol_q8"], 2 * f)))
+        tensors.append(TensorSpec("w.scale", DT_F16, (rows,), f, fill="rowscale", scale=0.002,
+                                  key=(_STREAM_KEY["protocol_q8"], 2 * f + 1)))
+        mats.append(Matrix("p%d" % f, DT_I8, rows, cols, [2 * f], scale=2 * f + 1))
+        paths.append(os.path.join(outdir, "protocol_q8_%02d.wt" % f))
+    return Checkpoint("protocol_q8", paths, tensors, mats)
+
+
+def custom_q8(outdir: str, shapes: Sequence[Tuple[int, int]], name: str = "custom_q8") -> Checkpoint:
+    """One file holding, per shape, an int8 [M, K] matrix "w<i>" and its fp16 scales "w<i>.scale"."""
+    tensors, mats = [], []
+    for i, (M, K) in enumerate(shapes):
+        tensors.append(TensorSpec(f"w{i}", DT_I8, (M, K), 0, fill="int8", key=(_STREAM_KEY["custom"], 1000 + 2 * i)))
+        tensors.append(TensorSpec(f"w{i}.scale", DT_F16, (M,), 0, fill="rowscale", scale=0.002,
+                                  key=(_STREAM_KEY["custom"], 1001 + 2 * i)))
+        mats.append(Matrix(f"w{i}", DT_I8, M, K, [2 * i], scale=2 * i + 1))
+    return Checkpoint(name, [os.path.join(outdir, name + ".wt")], tensors, mats)
+
+
 def build(workload: str, outdir: str, workers: int = 0, **kw) -> Checkpoint:
     """Describe and write a workload; returns the Checkpoint (paths, tensors, matrices)."""
     if workload == "tiny":
         ck = tiny(outdir)
     elif workload == "protocol":
         ck = protocol(outdir, **kw)
+    elif workload == "protocol_q8":
+        ck = protocol_q8(outdir, **kw)
     elif workload == "sweep":
         ck = sweep(outdir, **kw)
     elif workload == "many":

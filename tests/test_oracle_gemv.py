@@ -138,3 +138,42 @@ def test_empty_shapes():
     assert y.size == 0
     y, a = oracle.gemv(np.zeros(0, np.uint8), BF16, 4, 0, np.zeros(0, np.uint8))
     assert not y.any() and not a.any()
+
+
+# ----------------------------------------------------------------------------- int8 + fp16 row scales
+
+def _f16(v):
+    return np.asarray(v, np.float16).astype("<f2").view(np.uint8)
+
+
+def test_q8_integer_exact_with_power_of_two_scales():
+    rng = np.random.default_rng(11)
+    M, K = 11, 53
+    W = rng.integers(-128, 128, (M, K)).astype(np.int8)
+    x = rng.integers(-3, 4, K)
+    s = 2.0 ** rng.integers(-6, 2, M)
+    yhat, a = oracle.gemv_q8(W.view(np.uint8), _f16(s), M, K, _f16(x))
+    for i in range(M):
+        exact = sum(int(W[i, j]) * int(x[j]) for j in range(K))
+        assert yhat[i] == s[i] * exact
+        assert a[i] == abs(s[i]) * sum(abs(int(W[i, j]) * int(x[j])) for j in range(K))
+
+
+def test_q8_one_hot_gives_scaled_column_and_matches_numpy():
+    rng = np.random.default_rng(12)
+    M, K = 40, 96
+    W = rng.integers(-128, 128, (M, K)).astype(np.int8)
+    s = rng.uniform(0.001, 0.02, M).astype(np.float16)
+    for j in (0, 17, K - 1):
+        x = np.zeros(K, np.float16)
+        x[j] = 1.0
+        yhat, _ = oracle.gemv_q8(W.view(np.uint8), s.view(np.uint8), M, K, x.view(np.uint8))
+        assert np.array_equal(yhat, s.astype(np.float64) * W[:, j].astype(np.float64))
+    xv = rng.standard_normal(K).astype(np.float16)
+    yhat, a = oracle.gemv_q8(W.view(np.uint8), s.view(np.uint8), M, K, xv.view(np.uint8))
+    ref = s.astype(np.float64) * (W.astype(np.float64) @ xv.astype(np.float64))
+    assert np.allclose(yhat, ref, rtol=1e-12, atol=0)
+    yr, ar = oracle.gemv_q8(W.view(np.uint8), s.view(np.uint8), M, K, xv.view(np.uint8), rows=[5, 0, 39])
+    assert list(yr) == [yhat[5], yhat[0], yhat[39]] and list(ar) == [a[5], a[0], a[39]]
+    with pytest.raises(oracle.OracleError):
+        oracle.gemv_q8(W.view(np.uint8), s.view(np.uint8), M, K, xv.view(np.uint8), rows=[M])
