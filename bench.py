@@ -40,6 +40,7 @@ WORKLOADS = {
     "many": "many-small: 1253 bf16 matrices split by rows across 2506 files (1.56 GB)",
     "tiny": "tiny: 8 fp32 256x256 matrices + 8 fp32[256] vectors in one file (2.1 MB)",
     "protocol": "matched protocol by bytes: 12 files of one bf16 12288x3584 matrix (88.1 MB each, 1.06 GB)",
+    "protocol_q8": "matched protocol: 12 files of one int8 12288x7168 matrix (88.1 MB) + fp16 row scales; fp16 x",
 }
 
 
@@ -81,6 +82,8 @@ def workload_ck(args, outdir):
         return synth.tiny(outdir)
     if w == "protocol":
         return synth.protocol(outdir)
+    if w == "protocol_q8":
+        return synth.protocol_q8(outdir)
     if w == "many":
         return synth.many(outdir)
     if w in ("mid", "large"):

@@ -108,18 +108,22 @@ typedef struct {
 } wt_tensor_meta;
 
 /* One GEMV of wt_pass: y[M] = W[M,K] . x[K], fp32 accumulate (Sec. 3.1 protocol:
- * one single-token GEMV per matrix).  W is row-major [out, in]; x has W's dtype;
- * y is fp32.  All pointers are caller-owned device memory.  wait_event (a
- * cudaEvent_t from wt_adopt, or NULL) gates this GEMV on the GPU. */
+ * one single-token GEMV per matrix).  W is row-major [out, in]; y is fp32.  For WT_F32,
+ * WT_BF16 and WT_F16 weights x has W's dtype and scale is NULL.  For WT_I8 weights (the
+ * paper's packed-int8 kernel with fp16 row scales, Sec. 3.1 and Table "tab:tax") x is
+ * fp16 and scale points at M fp16 row scales: y_i = scale_i * sum_j W_ij x_j.  All
+ * pointers are caller-owned device memory (or, for W, the handle's mapping: see
+ * wt_pass).  wait_event (a cudaEvent_t from wt_adopt, or NULL) gates this GEMV on the GPU. */
 typedef struct {
   const void *W;
-  int32_t dtype;        /* WT_F32, WT_BF16 or WT_F16 */
+  int32_t dtype;        /* WT_F32, WT_BF16, WT_F16 or WT_I8 */
   int32_t reserved;     /* must be 0 */
   uint64_t M;
   uint64_t K;
   const void *x;
   float *y;
   void *wait_event;
+  const void *scale;    /* WT_I8: fp16 [M] row scales; otherwise NULL */
 } wt_gemv_desc;
 
 /* Thread-local message describing the last failure on this thread ("" if none). */

@@ -195,6 +195,7 @@ struct Plan {
     const uint8_t *W, *x;
     float *y;
     uint64_t M, K;
+    const uint8_t *scale;
   };
   struct Zero {
     float *y;
@@ -591,15 +592,19 @@ wt::MatDesc make_mat(const wt_gemv_desc &d) {
   m.W = static_cast<const uint8_t *>(d.W);
   m.x = static_cast<const uint8_t *>(d.x);
   m.y = d.y;
+  m.s = static_cast<const uint8_t *>(d.scale);
   m.M = (uint32_t)d.M;
   m.V = (uint32_t)(d.K * es / 16);
   const uint32_t rowb = m.V * 16;
-  if (m.V <= 256) {
+  // a consumer thread keeps at most 8 (bf16/f16/f32) or 4 (int8: 16 f16 activations per
+  // weight vector) x vectors in registers; the mode limits follow from that
+  const uint32_t xj = d.dtype == WT_I8 ? 4 : 8;
+  if (m.V <= 32 * xj) {
     m.mode = wt::kModeWarpRows;
     m.G = (uint16_t)(m.V <= 32 ? pow2ceil(m.V) : 32);
     m.rt = wt::kStageBytes / rowb;
     m.vc = m.V;
-  } else if (rowb <= (uint32_t)wt::kStageBytes) {
+  } else if (rowb <= (uint32_t)wt::kStageBytes && m.V <= 256 * xj) {
     m.mode = wt::kModeBlockRows;
     m.rt = std::min<uint32_t>(wt::kRowBlock, wt::kStageBytes / rowb);
     m.vc = m.V;
@@ -662,8 +667,11 @@ size_t append(std::vector<uint8_t> &tab, const std::vector<T> &v) {
 }
 
 int validate_desc(const wt_gemv_desc &d, size_t i) {
-  if (d.dtype != WT_F32 && d.dtype != WT_BF16 && d.dtype != WT_F16)
-    return set_err(d.dtype == WT_I8 || d.dtype == WT_U8 ? WT_ENOTSUP : WT_EINVAL, "desc %zu: dtype %d has no GEMV", i, d.dtype);
+  if (d.dtype != WT_F32 && d.dtype != WT_BF16 && d.dtype != WT_F16 && d.dtype != WT_I8)
+    return set_err(d.dtype == WT_U8 ? WT_ENOTSUP : WT_EINVAL, "desc %zu: dtype %d has no GEMV", i, d.dtype);
+  if (d.dtype == WT_I8 && d.M > 0 && d.K > 0 && d.scale == nullptr)
+    return set_err(WT_EINVAL, "desc %zu: int8 weights need fp16 row scales", i);
+  if (d.dtype != WT_I8 && d.scale != nullptr) return set_err(WT_EINVAL, "desc %zu: scale is for int8 weights only", i);
   if (d.reserved != 0) return set_err(WT_EINVAL, "desc %zu: reserved field must be 0", i);
   if (d.M > 0x7fffffffull || d.K > 0x7fffffffull) return set_err(WT_EINVAL, "desc %zu: M or K above 2^31-1", i);
   if (d.M > 0 && d.y == nullptr) return set_err(WT_EINVAL, "desc %zu: null y", i);
@@ -688,7 +696,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
     while (j < n && d[j].wait_event == d[i].wait_event) ++j;
     Plan::Group g;
     g.first = i;
-    std::vector<wt::MatDesc> by_dt[3], mapped_dt[3];
+    std::vector<wt::MatDesc> by_dt[4], mapped_dt[4];
     for (size_t k = i; k < j; ++k) {
       const wt_gemv_desc &q = d[k];
       if (q.M == 0) continue;
@@ -711,15 +719,17 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         wt_gemv_desc qd = q;
         qd.W = f->dev + off;
         if (fast) mapped_dt[q.dtype].push_back(make_mat(qd));
-        else g.generic.push_back({q.dtype, static_cast<const uint8_t *>(qd.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K});
+        else g.generic.push_back({q.dtype, static_cast<const uint8_t *>(qd.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
+                                  static_cast<const uint8_t *>(q.scale)});
       } else if (fast) {
         by_dt[q.dtype].push_back(make_mat(q));
       } else {
-        g.generic.push_back({q.dtype, static_cast<const uint8_t *>(q.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K});
+        g.generic.push_back({q.dtype, static_cast<const uint8_t *>(q.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
+                             static_cast<const uint8_t *>(q.scale)});
       }
     }
     for (int pass = 0; pass < 2; ++pass) {
-      for (int dt = 0; dt < 3; ++dt) {
+      for (int dt = 0; dt < 4; ++dt) {
         std::vector<wt::MatDesc> &ms = pass == 0 ? by_dt[dt] : mapped_dt[dt];
         if (ms.empty()) continue;
         Plan::Launch L;
@@ -790,7 +800,7 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s) {
       h->kernel_launches++;
     }
     for (const Plan::Generic &q : g.generic) {
-      CU(wt::launch_gemv_generic(q.dtype, q.W, q.x, q.y, q.M, q.K, s));
+      CU(wt::launch_gemv_generic(q.dtype, q.W, q.x, q.y, q.M, q.K, q.scale, s));
       h->kernel_launches++;
     }
   }
@@ -839,7 +849,7 @@ extern "C" {
 
 const char *wt_last_error(void) { return t_err.c_str(); }
 
-int wt_abi_version(void) { return 1; }
+int wt_abi_version(void) { return 2; }
 
 int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **out) {
   if (!out) return set_err(WT_EINVAL, "wt_open: out is NULL");

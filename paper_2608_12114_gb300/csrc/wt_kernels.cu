@@ -154,6 +154,35 @@ struct Elem<2> {  // f16
   }
 };
 
+template <>
+struct Elem<3> {  // int8 weights (their activations are f16, their rows carry f16 scales)
+  static constexpr int kEPV = 16;
+  __device__ static __forceinline__ float scalar(const uint8_t *p, uint64_t i) { return (float)(int8_t)p[i]; }
+};
+
+// Element type of x for weights of type DT: int8 weights take f16 activations.
+template <int DT>
+struct XElem {
+  static constexpr int value = DT == 3 ? 2 : DT;
+};
+
+// x vectors a consumer thread keeps in registers (16-byte weight vectors it covers).
+template <int DT>
+struct XJ {
+  static constexpr int value = DT == 3 ? 4 : 8;
+};
+
+// Vector counts above XJ never reach a kernel of that type (the planner keeps them out);
+// clamping keeps every template instantiation inside the register array.
+#define WT_NJC(n) ((n) <= XJ<DT>::value ? (n) : XJ<DT>::value)
+
+// Row scale applied at the store: f16 per row for int8 weights, 1 otherwise.
+template <int DT>
+__device__ __forceinline__ float row_scale(const uint8_t *s, uint64_t row) {
+  if constexpr (DT == 3) return __half2float(reinterpret_cast<const __half *>(s)[row]);
+  return 1.f;
+}
+
 __device__ __forceinline__ uint4 lds128(uint32_t addr) {
   uint4 v;
   asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
@@ -236,13 +265,23 @@ template <int DT>
 struct Pairs {
   static constexpr int N = Elem<DT>::kEPV / 2;
   __device__ static __forceinline__ uint64_t get(const uint4 &v, int i) {
-    const uint32_t w = i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w;
-    if (DT == 1) return pack2(w << 16, w & 0xffff0000u);  // bf16
-    if (DT == 2) {                                          // f16
-      const float2 t = __half22float2(*reinterpret_cast<const __half2 *>(&w));
-      return pack2(__float_as_uint(t.x), __float_as_uint(t.y));
+    if constexpr (DT == 3) {
+      // int8 pair (bytes 2i, 2i+1): with u = b ^ 0x80 = b + 128, the float with bits
+      // 0x4B000000 | u is exactly 2^23 + u; one f32x2 FMA subtracts 2^23 + 128, exactly.
+      const uint32_t w = (i >> 1) == 0 ? v.x : (i >> 1) == 1 ? v.y : (i >> 1) == 2 ? v.z : v.w;
+      const uint32_t u = w ^ 0x80808080u;
+      const uint32_t k = (uint32_t)(i & 1) * 2;
+      const uint64_t biased = pack2(__byte_perm(u, 0x4B000000u, 0x7540u | k), __byte_perm(u, 0x4B000000u, 0x7540u | (k + 1)));
+      return fma2(biased, 0x3F8000003F800000ull, 0xCB000080CB000080ull);  // x 1.0 - 8388736.0
+    } else {
+      const uint32_t w = i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w;
+      if (DT == 1) return pack2(w << 16, w & 0xffff0000u);  // bf16
+      if (DT == 2) {                                          // f16
+        const float2 t = __half22float2(*reinterpret_cast<const __half2 *>(&w));
+        return pack2(__float_as_uint(t.x), __float_as_uint(t.y));
+      }
+      return i == 0 ? pack2(v.x, v.y) : pack2(v.z, v.w);  // f32
     }
-    return i == 0 ? pack2(v.x, v.y) : pack2(v.z, v.w);  // f32
   }
 };
 
@@ -263,9 +302,20 @@ __device__ __forceinline__ void dot16(const uint4 &w, const uint64_t (&xp)[Pairs
 
 template <int DT>
 __device__ __forceinline__ void load_xpairs(const uint8_t *x, uint32_t v, bool ok, uint64_t (&xp)[Pairs<DT>::N]) {
-  const uint4 t = ok ? __ldg(reinterpret_cast<const uint4 *>(x) + v) : make_uint4(0, 0, 0, 0);
+  if constexpr (DT == 3) {
+    // the 16 f16 activations of weight vector v: 32 bytes
+    const uint4 a = ok ? __ldg(reinterpret_cast<const uint4 *>(x) + 2 * v) : make_uint4(0, 0, 0, 0);
+    const uint4 b = ok ? __ldg(reinterpret_cast<const uint4 *>(x) + 2 * v + 1) : make_uint4(0, 0, 0, 0);
 #pragma unroll
-  for (int i = 0; i < Pairs<DT>::N; ++i) xp[i] = Pairs<DT>::get(t, i);
+    for (int i = 0; i < 4; ++i) {
+      xp[i] = Pairs<2>::get(a, i);
+      xp[4 + i] = Pairs<2>::get(b, i);
+    }
+  } else {
+    const uint4 t = ok ? __ldg(reinterpret_cast<const uint4 *>(x) + v) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+    for (int i = 0; i < Pairs<DT>::N; ++i) xp[i] = Pairs<DT>::get(t, i);
+  }
 }
 
 __device__ __forceinline__ uint4 lds_or_zero(uint32_t addr, bool ok) {
@@ -308,7 +358,8 @@ struct Log2<1> {
 template <int DT, int NJ>
 __device__ __forceinline__ void tile_warp_rows(uint32_t tile, uint32_t V, uint32_t nr, uint32_t G,
                                                uint32_t gl, uint32_t sub, uint32_t rpw, int warp, int lane,
-                                               const uint64_t (&xp)[8][Pairs<DT>::N], float *y) {
+                                               const uint64_t (&xp)[XJ<DT>::value][Pairs<DT>::N], float *y,
+                                               const uint8_t *sr) {
   constexpr int U = NJ == 1 ? 8 : NJ == 2 ? 4 : (NJ <= 4 ? 2 : 1);
   const uint32_t step = kConsumerWarps * rpw;
   for (uint32_t base = warp * rpw; base < nr; base += U * step) {
@@ -334,13 +385,13 @@ __device__ __forceinline__ void tile_warp_rows(uint32_t tile, uint32_t V, uint32
       const float sum = transpose_reduce<U>(t, lane);
       constexpr int L = Log2<U>::value;
       const uint32_t row = base + (uint32_t)(lane >> (5 - L)) * step;
-      if ((lane & ((32 >> L) - 1)) == 0 && row < nr) y[row] = sum;
+      if ((lane & ((32 >> L) - 1)) == 0 && row < nr) y[row] = sum * row_scale<DT>(sr, row);
     } else {
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         for (uint32_t o = G >> 1; o > 0; o >>= 1) t[u] += __shfl_xor_sync(0xffffffffu, t[u], o);
         const uint32_t row = base + u * step + sub;
-        if (gl == 0 && row < nr) y[row] = t[u];
+        if (gl == 0 && row < nr) y[row] = t[u] * row_scale<DT>(sr, row);
       }
     }
   }
@@ -351,7 +402,7 @@ __device__ __forceinline__ void tile_warp_rows(uint32_t tile, uint32_t V, uint32
 // reductions over the G lanes are unrolled, so the eight shuffle chains interleave.
 template <int DT, int G>
 __device__ __forceinline__ void tile_small_rows(uint32_t tile, uint32_t V, uint32_t nr, int warp, int lane,
-                                                const uint64_t (&xp)[Pairs<DT>::N], float *y) {
+                                                const uint64_t (&xp)[Pairs<DT>::N], float *y, const uint8_t *sr) {
   constexpr int RPW = 32 / G;
   constexpr int U = 8;
   const uint32_t gl = lane & (G - 1);
@@ -379,7 +430,7 @@ __device__ __forceinline__ void tile_small_rows(uint32_t tile, uint32_t V, uint3
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const uint32_t row = base + u * step + sub;
-      if (gl == 0 && row < nr) y[row] = t[u];
+      if (gl == 0 && row < nr) y[row] = t[u] * row_scale<DT>(sr, row);
     }
   }
 }
@@ -388,7 +439,7 @@ __device__ __forceinline__ void tile_small_rows(uint32_t tile, uint32_t V, uint3
 // holds vectors ct + 256 j.  Warp partials land in rb[q * warps + warp].
 template <int DT, int NJ, int NR>
 __device__ __forceinline__ void tile_block_rows(uint32_t tile, uint32_t V, int ct, int warp, int lane,
-                                                const uint64_t (&xp)[8][Pairs<DT>::N], float *rb) {
+                                                const uint64_t (&xp)[XJ<DT>::value][Pairs<DT>::N], float *rb) {
   constexpr int NP = NR <= 1 ? 1 : NR <= 2 ? 2 : NR <= 4 ? 4 : 8;
   uint4 w[NR][NJ];
 #pragma unroll
@@ -435,11 +486,12 @@ __device__ __forceinline__ float sum_warps(const float *p) {
 
 template <int DT>
 __device__ __forceinline__ bool block_rows_dispatch(uint32_t nj, uint32_t nr, uint32_t tile, uint32_t V, int ct,
-                                                    int warp, int lane, const uint64_t (&xp)[8][Pairs<DT>::N],
+                                                    int warp, int lane, const uint64_t (&xp)[XJ<DT>::value][Pairs<DT>::N],
                                                     float *rb) {
 #define WT_BR(NJ, NR) \
-  case NJ * 8 + NR: tile_block_rows<DT, NJ, NR>(tile, V, ct, warp, lane, xp, rb); return true;
+  case NJ * 8 + NR: tile_block_rows<DT, WT_NJC(NJ), NR>(tile, V, ct, warp, lane, xp, rb); return true;
   switch (nj * 8 + nr) {
+    WT_BR(1, 1) WT_BR(1, 2) WT_BR(1, 3) WT_BR(1, 4) WT_BR(1, 5) WT_BR(1, 6) WT_BR(1, 7) WT_BR(1, 8)
     WT_BR(2, 1) WT_BR(2, 2) WT_BR(2, 3) WT_BR(2, 4) WT_BR(2, 5) WT_BR(2, 6) WT_BR(2, 7)
     WT_BR(3, 1) WT_BR(3, 2) WT_BR(3, 3)
     WT_BR(4, 1) WT_BR(4, 2)
@@ -532,7 +584,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
     const int ct = threadIdx.x;  // 0..255
     uint32_t it = 0;
     int par = 0;
-    uint64_t xp[8][NP];
+    uint64_t xp[XJ<DT>::value][NP];
     for (uint32_t pi = p0; pi < p1; ++pi) {
       const Piece pc = pieces[pi];
       const MatDesc md = mats[pc.mat];
@@ -544,7 +596,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
         const uint32_t rpw = 32 / G;
         const uint32_t nj = (V + G - 1) / G;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < XJ<DT>::value; ++j) {
           const uint32_t v = gl + j * G;
           load_xpairs<DT>(md.x, v, j < (int)nj && v < V, xp[j]);
         }
@@ -554,23 +606,24 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
           bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
           const uint32_t tile = stage0 + s * kStageBytes;
           float *y = md.y + r;
+          const uint8_t *sr = md.s ? md.s + 2ull * r : nullptr;  // f16 row scales (int8 weights)
           if (G < 32) {
             switch (G) {
-              case 1: tile_small_rows<DT, 1>(tile, V, nr, warp, lane, xp[0], y); break;
-              case 2: tile_small_rows<DT, 2>(tile, V, nr, warp, lane, xp[0], y); break;
-              case 4: tile_small_rows<DT, 4>(tile, V, nr, warp, lane, xp[0], y); break;
-              case 8: tile_small_rows<DT, 8>(tile, V, nr, warp, lane, xp[0], y); break;
-              default: tile_small_rows<DT, 16>(tile, V, nr, warp, lane, xp[0], y); break;
+              case 1: tile_small_rows<DT, 1>(tile, V, nr, warp, lane, xp[0], y, sr); break;
+              case 2: tile_small_rows<DT, 2>(tile, V, nr, warp, lane, xp[0], y, sr); break;
+              case 4: tile_small_rows<DT, 4>(tile, V, nr, warp, lane, xp[0], y, sr); break;
+              case 8: tile_small_rows<DT, 8>(tile, V, nr, warp, lane, xp[0], y, sr); break;
+              default: tile_small_rows<DT, 16>(tile, V, nr, warp, lane, xp[0], y, sr); break;
             }
           } else switch (nj) {
-            case 1: tile_warp_rows<DT, 1>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
-            case 2: tile_warp_rows<DT, 2>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
-            case 3: tile_warp_rows<DT, 3>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
-            case 4: tile_warp_rows<DT, 4>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
-            case 5: tile_warp_rows<DT, 5>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
-            case 6: tile_warp_rows<DT, 6>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
-            case 7: tile_warp_rows<DT, 7>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
-            default: tile_warp_rows<DT, 8>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y); break;
+            case 1: tile_warp_rows<DT, WT_NJC(1)>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y, sr); break;
+            case 2: tile_warp_rows<DT, WT_NJC(2)>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y, sr); break;
+            case 3: tile_warp_rows<DT, WT_NJC(3)>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y, sr); break;
+            case 4: tile_warp_rows<DT, WT_NJC(4)>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y, sr); break;
+            case 5: tile_warp_rows<DT, WT_NJC(5)>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y, sr); break;
+            case 6: tile_warp_rows<DT, WT_NJC(6)>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y, sr); break;
+            case 7: tile_warp_rows<DT, WT_NJC(7)>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y, sr); break;
+            default: tile_warp_rows<DT, WT_NJC(8)>(tile, V, nr, G, gl, sub, rpw, warp, lane, xp, y, sr); break;
           }
           __syncwarp();
           if (lane == 0) mbar_arrive(empty0 + 8 * s);
@@ -580,7 +633,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
         // whole consumer group shares each row; one tile = up to kRowBlock full rows
         const uint32_t nj = (V + kConsumers - 1) / kConsumers;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < XJ<DT>::value; ++j) {
           const uint32_t v = ct + j * kConsumers;
           load_xpairs<DT>(md.x, v, j < (int)nj && v < V, xp[j]);
         }
@@ -602,7 +655,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
           if (r + nr >= pc.r1 || gn + md.rt > (uint32_t)kRedRows) {
             named_bar(1, kConsumers);
             const float *gb = red + par * (kConsumerWarps * kRedRows);
-            for (uint32_t q = ct; q < gn; q += kConsumers) md.y[g0 + q] = sum_warps(gb + q * kConsumerWarps);
+            for (uint32_t q = ct; q < gn; q += kConsumers) md.y[g0 + q] = sum_warps(gb + q * kConsumerWarps) * row_scale<DT>(md.s, g0 + q);
             par ^= 1;
             g0 += gn;
             gn = 0;
@@ -645,7 +698,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
           const int q = lane >> 2;
           if ((lane & 3) == 0 && q < (int)nr) rb[q * kConsumerWarps + warp] = sum;
           named_bar(1, kConsumers);
-          if (ct < (int)nr) md.y[r + ct] = sum_warps(rb + ct * kConsumerWarps);
+          if (ct < (int)nr) md.y[r + ct] = sum_warps(rb + ct * kConsumerWarps) * row_scale<DT>(md.s, r + ct);
           par ^= 1;
         }
       }
@@ -692,7 +745,7 @@ __global__ void __launch_bounds__(256) gemv_mapped_kernel(const MatDesc *__restr
       }
       float t = acc.total();
       for (uint32_t o = G >> 1; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-      if (valid && gl == 0) md.y[row] = t;
+      if (valid && gl == 0) md.y[row] = t * row_scale<DT>(md.s, row);
     }
   }
 }
@@ -700,16 +753,17 @@ __global__ void __launch_bounds__(256) gemv_mapped_kernel(const MatDesc *__restr
 // Fallback: one warp per row, byte-assembled scalar loads (any alignment).
 template <int DT>
 __global__ void gemv_generic_kernel(const uint8_t *W, const uint8_t *x, float *y, uint64_t M,
-                                    uint64_t K) {
+                                    uint64_t K, const uint8_t *s) {
   const uint64_t warps = (uint64_t)gridDim.x * (blockDim.x >> 5);
   const int lane = threadIdx.x & 31;
   for (uint64_t row = (uint64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); row < M;
        row += warps) {
     const uint8_t *wr = W + row * K * (uint64_t)(16 / Elem<DT>::kEPV);
     float acc = 0.f;
-    for (uint64_t k = lane; k < K; k += 32) acc = fmaf(Elem<DT>::scalar(wr, k), Elem<DT>::scalar(x, k), acc);
+    for (uint64_t k = lane; k < K; k += 32)
+      acc = fmaf(Elem<DT>::scalar(wr, k), Elem<XElem<DT>::value>::scalar(x, k), acc);
     acc = warp_sum(acc);
-    if (lane == 0) y[row] = acc;
+    if (lane == 0) y[row] = acc * row_scale<DT>(s, row);
   }
 }
 
@@ -860,7 +914,8 @@ cudaError_t gemv_prepare() {
   cudaError_t e;
   if ((e = cudaFuncSetAttribute(gemv_tma_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemvSmem)) != cudaSuccess) return e;
   if ((e = cudaFuncSetAttribute(gemv_tma_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemvSmem)) != cudaSuccess) return e;
-  return cudaFuncSetAttribute(gemv_tma_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemvSmem);
+  if ((e = cudaFuncSetAttribute(gemv_tma_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemvSmem)) != cudaSuccess) return e;
+  return cudaFuncSetAttribute(gemv_tma_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemvSmem);
 }
 
 cudaError_t launch_gemv(const GemvLaunch &L, cudaStream_t s) {
@@ -869,6 +924,7 @@ cudaError_t launch_gemv(const GemvLaunch &L, cudaStream_t s) {
     case 0: gemv_tma_kernel<0><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
     case 1: gemv_tma_kernel<1><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
     case 2: gemv_tma_kernel<2><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
+    case 3: gemv_tma_kernel<3><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();
@@ -880,20 +936,22 @@ cudaError_t launch_gemv_mapped(const GemvLaunch &L, cudaStream_t s) {
     case 0: gemv_mapped_kernel<0><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
     case 1: gemv_mapped_kernel<1><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
     case 2: gemv_mapped_kernel<2><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
+    case 3: gemv_mapped_kernel<3><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();
 }
 
 cudaError_t launch_gemv_generic(int dtype, const uint8_t *W, const uint8_t *x, float *y, uint64_t M,
-                                uint64_t K, cudaStream_t s) {
+                                uint64_t K, const uint8_t *sc, cudaStream_t s) {
   if (M == 0) return cudaSuccess;
   const uint64_t blocks64 = (M + 7) / 8;
   const int grid = (int)(blocks64 < (uint64_t)num_sms() * 8 ? blocks64 : (uint64_t)num_sms() * 8);
   switch (dtype) {
-    case 0: gemv_generic_kernel<0><<<grid, 256, 0, s>>>(W, x, y, M, K); break;
-    case 1: gemv_generic_kernel<1><<<grid, 256, 0, s>>>(W, x, y, M, K); break;
-    case 2: gemv_generic_kernel<2><<<grid, 256, 0, s>>>(W, x, y, M, K); break;
+    case 0: gemv_generic_kernel<0><<<grid, 256, 0, s>>>(W, x, y, M, K, sc); break;
+    case 1: gemv_generic_kernel<1><<<grid, 256, 0, s>>>(W, x, y, M, K, sc); break;
+    case 2: gemv_generic_kernel<2><<<grid, 256, 0, s>>>(W, x, y, M, K, sc); break;
+    case 3: gemv_generic_kernel<3><<<grid, 256, 0, s>>>(W, x, y, M, K, sc); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();

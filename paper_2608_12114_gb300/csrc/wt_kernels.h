@@ -43,6 +43,7 @@ struct alignas(16) MatDesc {
   const uint8_t *W;
   const uint8_t *x;
   float *y;
+  const uint8_t *s;  // f16 row scales (int8 weights), else null
   uint32_t M;     // rows
   uint32_t V;     // 16-byte vectors per row (K * sizeof(elem) / 16)
   uint32_t rt;    // rows per tile (modes 0/1) or per row block (mode 2)
@@ -60,7 +61,7 @@ struct alignas(16) Piece {
 };
 
 struct GemvLaunch {
-  int dtype;               // WT_F32 / WT_BF16 / WT_F16
+  int dtype;               // WT_F32 / WT_BF16 / WT_F16 / WT_I8 (x f16, f16 row scales)
   int grid;                // CTAs; CTA b owns pieces [begin[b], begin[b+1])
   const MatDesc *mats;     // device
   const Piece *pieces;     // device
@@ -80,7 +81,7 @@ cudaError_t launch_gemv_mapped(const GemvLaunch &L, cudaStream_t s);
 // Fallback for operands the tiled kernel cannot take (unaligned W/x or rows
 // whose byte length is not a multiple of 16): one warp per row, scalar loads.
 cudaError_t launch_gemv_generic(int dtype, const uint8_t *W, const uint8_t *x, float *y,
-                                uint64_t M, uint64_t K, cudaStream_t s);
+                                uint64_t M, uint64_t K, const uint8_t *scale, cudaStream_t s);
 
 // ---------------------------------------------------------------- FNV-1a-64
 constexpr int kMaxFnv = 256;

@@ -35,6 +35,7 @@ class MatrixRef:
     shape: tuple            # (M, K) for matrices, (n,) / other for non-GEMV tensors
     parts: List[int]        # tensor indices in row order
     gemv: bool              # 2-D with a GEMV dtype
+    scale: Optional[int] = None  # tensor index of the fp16 row scales of int8 weights ("<name>.scale")
 
 
 def matrices(h: wt.Handle) -> List[MatrixRef]:
@@ -66,6 +67,13 @@ def matrices(h: wt.Handle) -> List[MatrixRef]:
         ref.parts = idx
         ref.shape = (sum(t.shape[0] for t in ts), K)
         ref.gemv = ts[0].dtype in (wt.WT_F32, wt.WT_BF16, wt.WT_F16)
+    # int8 matrices are GEMV matrices when their fp16 row scales "<name>.scale" are present
+    names = {t.name: i for i, t in enumerate(h.tensors)}
+    for ref in out:
+        if ref.dtype == wt.WT_I8 and len(ref.shape) == 2 and len(ref.parts) == 1:
+            si = names.get(ref.name + ".scale")
+            if si is not None and h.tensors[si].dtype == wt.WT_F16 and h.tensors[si].shape == (ref.shape[0],):
+                ref.scale, ref.gemv = si, True
     return out
 
 
@@ -144,14 +152,19 @@ class DeviceCheckpoint:
             base["dtype"] = [m.dtype for m in mats]
             base["M"] = [m.shape[0] for m in mats]
             base["K"] = [m.shape[1] for m in mats]
+            base["scale"] = [self.dst[m.scale] if m.scale is not None else 0 for m in mats]
             self._tables[key] = base
         out = base.copy()
         out["x"] = [xs[(self.mats[k].shape[1], self.mats[k].dtype)].data_ptr() for k in ks]
         out["y"] = [ys[k].data_ptr() for k in ks]
         if events:
             pos = {i: n for n, i in enumerate(events)}
-            out["wait_event"] = [events[max(self.mats[k].parts, key=pos.__getitem__)] for k in ks]
+            out["wait_event"] = [events[max(self.mats[k].parts + ([self.mats[k].scale] if self.mats[k].scale is not None else []),
+                                            key=pos.__getitem__)] for k in ks]
         return out
+
+    def x_dtype(self, k) -> int:
+        return wt.WT_F16 if self.mats[k].dtype == wt.WT_I8 else self.mats[k].dtype
 
     @property
     def weight_bytes(self) -> int:

@@ -124,3 +124,35 @@ def test_sweep_points_full_size(torch, tmp_path):
         run_and_check(torch, ck)
     finally:
         shutil.rmtree(str(tmp_path), ignore_errors=True)
+
+
+def test_matched_protocol_int8_full_size(torch, tmp_path):
+    """The paper's matched protocol: 12 files of 12288x7168 int8 (88.1 MB) with fp16 row scales."""
+    ck = synth.build("protocol_q8", str(tmp_path), workers=16)
+    co = oracle.CheckpointOracle(ck.paths)
+    h = wt.Handle(ck.paths)
+    try:
+        dev = pipeline.DeviceCheckpoint.allocate(h, pipeline.matrices(h))
+        xs, ys = dev.inputs(), dev.outputs()
+        ingest_s, consume_s = torch.cuda.Stream(), torch.cuda.Stream()
+        torch.cuda.synchronize()
+        ev = dev.adopt(h, wt.WT_ADOPT_GATHER, ingest_s.cuda_stream)
+        h.pass_(dev.descs(xs, ys, ev), consume_s.cuda_stream)
+        consume_s.synchronize()
+        ingest_s.synchronize()
+        first = {k: y.clone() for k, y in ys.items()}
+        h.pass_(dev.descs(xs, ys), consume_s.cuda_stream)
+        consume_s.synchronize()
+        assert len(ys) == 12 and all(torch.equal(first[k], ys[k]) for k in ys)
+        for k in dev.gemv_mats():
+            m = dev.mats[k]
+            t, sc = h.tensors[m.parts[0]], h.tensors[m.scale]
+            r = sorted({0, 12287} | {int(v) for v in np.random.default_rng(k).integers(0, 12288, 16)})
+            yhat, a = oracle.gemv_q8(co.blob_of(t.file, t.name), co.blob_of(sc.file, sc.name), 12288, 7168,
+                                     synth.make_x(7168, synth.DT_I8), rows=r)
+            assert oracle.gemv_error(ys[k].cpu().numpy()[r], yhat, a) <= TOL
+        assert h.device_status() == 0
+    finally:
+        h.close()
+        co.close()
+        shutil.rmtree(str(tmp_path), ignore_errors=True)
