@@ -91,6 +91,21 @@ def workload_ck(args, outdir):
     raise SystemExit("unknown workload " + w)
 
 
+DT_NAME = {0: "f32", 1: "bf16", 2: "f16", 3: "int8"}
+DATA_DESC = {
+    "bf16": "synthetic (seeded N(0,0.02) bf16 weights, norms 1.0, x ~ N(0,1))",
+    "int8": "synthetic (seeded uniform int8 weights in [-127, 127], fp16 row scales, fp16 x ~ N(0,1))",
+}
+
+
+def gemv_alg_bytes(dtype, M, K):
+    """Bytes one GEMV must move at minimum: W once, x once, y once (+ the fp16 row scales
+    of int8 weights, whose activations are fp16)."""
+    es = {0: 4, 1: 2, 2: 2, 3: 1}[dtype]
+    xes = 2 if dtype == 3 else es
+    return M * K * es + K * xes + 4 * M + (2 * M if dtype == 3 else 0)
+
+
 def workload_desc(args):
     w = args.workload
     if w.startswith("sweep:"):
@@ -313,8 +328,10 @@ def run_wt(args, rank, world):
     y_host = torch.empty(sum(rows), dtype=torch.float32, pin_memory=True)
     weight_bytes = dev.weight_bytes
     data_bytes = ck.data_bytes
-    alg_bytes = sum(dev.mats[k].shape[0] * dev.mats[k].shape[1] * 2 + dev.mats[k].shape[1] * 2 + 4 * dev.mats[k].shape[0]
-                    for k in dev.gemv_mats()) if all(dev.mats[k].dtype == wt.WT_BF16 for k in dev.gemv_mats()) else None
+    gdt = {dev.mats[k].dtype for k in dev.gemv_mats()}
+    alg_bytes = sum(gemv_alg_bytes(dev.mats[k].dtype, *dev.mats[k].shape) for k in dev.gemv_mats()) \
+        if len(gdt) == 1 else None
+    wdt = DT_NAME[gdt.pop()] if len(gdt) == 1 else "mixed"
     h0.close()
     torch.cuda.synchronize()
 
@@ -389,14 +406,14 @@ def run_wt(args, rank, world):
                 "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
                 "traffic": (tr["dram_bytes_per_launch_full"] if tr else None),
                 "algorithmic_bytes_per_launch": alg_bytes,
-                "kernel": "gemv_tma_kernel<bf16>",
+                "kernel": "gemv_tma_kernel<%s>" % wdt,
                 "frac_of_nominal_8TBps": round(achieved / NOMINAL_HBM_GBS, 4)}
     clocks = clk.summary()
     out = {
         "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic (seeded N(0,0.02) bf16 weights, norms 1.0, x ~ N(0,1))",
+        "scaling": "weak", "vs_baseline": None, "dtype": wdt,
+        "data": DATA_DESC.get(wdt, "synthetic"),
         "config": {"workload": workload_desc(args), "weight_bytes": weight_bytes, "data_bytes": data_bytes,
                    "files": len(ck.paths), "matrices": len(dev.gemv_mats()), "ingest_mode": args.mode,
                    "l2": "inputs larger than L2 (no flush)", "parallelism": "replicas" if world > 1 else "1 GPU"},

@@ -261,29 +261,44 @@ __device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
 }
 
 // A 16-byte vector as fp32 pairs (element 2i in the low half, 2i+1 in the high half).
+// For int8 weights (DT 3) the unit is a quad instead: x is held as four f16 per 64-bit
+// register, matching one 32-bit word of four weights (see dot16).
 template <int DT>
 struct Pairs {
-  static constexpr int N = Elem<DT>::kEPV / 2;
+  static constexpr int N = DT == 3 ? 4 : Elem<DT>::kEPV / 2;
   __device__ static __forceinline__ uint64_t get(const uint4 &v, int i) {
-    if constexpr (DT == 3) {
-      // int8 pair (bytes 2i, 2i+1): with u = b ^ 0x80 = b + 128, the float with bits
-      // 0x4B000000 | u is exactly 2^23 + u; one f32x2 FMA subtracts 2^23 + 128, exactly.
-      const uint32_t w = (i >> 1) == 0 ? v.x : (i >> 1) == 1 ? v.y : (i >> 1) == 2 ? v.z : v.w;
-      const uint32_t u = w ^ 0x80808080u;
-      const uint32_t k = (uint32_t)(i & 1) * 2;
-      const uint64_t biased = pack2(__byte_perm(u, 0x4B000000u, 0x7540u | k), __byte_perm(u, 0x4B000000u, 0x7540u | (k + 1)));
-      return fma2(biased, 0x3F8000003F800000ull, 0xCB000080CB000080ull);  // x 1.0 - 8388736.0
-    } else {
-      const uint32_t w = i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w;
-      if (DT == 1) return pack2(w << 16, w & 0xffff0000u);  // bf16
-      if (DT == 2) {                                          // f16
-        const float2 t = __half22float2(*reinterpret_cast<const __half2 *>(&w));
-        return pack2(__float_as_uint(t.x), __float_as_uint(t.y));
-      }
-      return i == 0 ? pack2(v.x, v.y) : pack2(v.z, v.w);  // f32
+    const uint32_t w = i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w;
+    if (DT == 1) return pack2(w << 16, w & 0xffff0000u);  // bf16
+    if (DT == 2) {                                          // f16
+      const float2 t = __half22float2(*reinterpret_cast<const __half2 *>(&w));
+      return pack2(__float_as_uint(t.x), __float_as_uint(t.y));
     }
+    return i == 0 ? pack2(v.x, v.y) : pack2(v.z, v.w);  // f32
   }
 };
+
+// c + a.lo * b.lo + a.hi * b.hi: fp16 operands, fp32 products and sums (fma.rn.f32.f16:
+// the product of two f16 values is exact in fp32, one rounding per FMA).
+__device__ __forceinline__ float fma_h2(uint32_t a, uint32_t b, float c) {
+  float d;
+  asm("{\n\t.reg .f16 al, ah, bl, bh;\n\t"
+      "mov.b32 {al, ah}, %1;\n\t"
+      "mov.b32 {bl, bh}, %2;\n\t"
+      "fma.rn.f32.f16 %0, al, bl, %3;\n\t"
+      "fma.rn.f32.f16 %0, ah, bh, %0;\n\t}"
+      : "=f"(d)
+      : "r"(a), "r"(b), "f"(c));
+  return d;
+}
+
+// Two int8 weights as exact f16x2.  With u = b ^ 0x80 (0..255) in the low byte and 0x64 in
+// the high byte, a half holds 1024 + u (f16 has unit spacing on [1024, 2048)); subtracting
+// 1152 = 1024 + 128 leaves b, an integer in [-128, 127], exactly.
+__device__ __forceinline__ uint32_t i8x2_to_f16x2(uint32_t u, uint32_t sel) {
+  uint32_t h;
+  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(h) : "r"(__byte_perm(u, 0x64646464u, sel)), "r"(0x64806480u));
+  return h;
+}
 
 // Four running fp32 partial sums of one row (two f32x2 registers).
 struct Acc4 {
@@ -293,10 +308,30 @@ struct Acc4 {
 
 template <int DT>
 __device__ __forceinline__ void dot16(const uint4 &w, const uint64_t (&xp)[Pairs<DT>::N], Acc4 &acc) {
+  if constexpr (DT == 3) {
+    // one word = four int8 weights -> two exact f16x2 words -> four mixed-precision FMAs
+    uint32_t f[4];
+    asm("mov.b64 {%0, %1}, %2;" : "=r"(f[0]), "=r"(f[1]) : "l"(acc.a));
+    asm("mov.b64 {%0, %1}, %2;" : "=r"(f[2]), "=r"(f[3]) : "l"(acc.b));
+    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
-  for (int i = 0; i < Pairs<DT>::N; ++i) {
-    if (i & 1) acc.b = fma2(Pairs<DT>::get(w, i), xp[i], acc.b);
-    else acc.a = fma2(Pairs<DT>::get(w, i), xp[i], acc.a);
+    for (int i = 0; i < 4; ++i) {
+      const uint32_t u = ws[i] ^ 0x80808080u;
+      const uint32_t h01 = i8x2_to_f16x2(u, 0x4140u);
+      const uint32_t h23 = i8x2_to_f16x2(u, 0x4342u);
+      float c = __uint_as_float(f[i]);
+      c = fma_h2(h01, (uint32_t)xp[i], c);
+      c = fma_h2(h23, (uint32_t)(xp[i] >> 32), c);
+      f[i] = __float_as_uint(c);
+    }
+    acc.a = pack2(f[0], f[1]);
+    acc.b = pack2(f[2], f[3]);
+  } else {
+#pragma unroll
+    for (int i = 0; i < Pairs<DT>::N; ++i) {
+      if (i & 1) acc.b = fma2(Pairs<DT>::get(w, i), xp[i], acc.b);
+      else acc.a = fma2(Pairs<DT>::get(w, i), xp[i], acc.a);
+    }
   }
 }
 
@@ -306,11 +341,10 @@ __device__ __forceinline__ void load_xpairs(const uint8_t *x, uint32_t v, bool o
     // the 16 f16 activations of weight vector v: 32 bytes
     const uint4 a = ok ? __ldg(reinterpret_cast<const uint4 *>(x) + 2 * v) : make_uint4(0, 0, 0, 0);
     const uint4 b = ok ? __ldg(reinterpret_cast<const uint4 *>(x) + 2 * v + 1) : make_uint4(0, 0, 0, 0);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      xp[i] = Pairs<2>::get(a, i);
-      xp[4 + i] = Pairs<2>::get(b, i);
-    }
+    xp[0] = pack2(a.x, a.y);
+    xp[1] = pack2(a.z, a.w);
+    xp[2] = pack2(b.x, b.y);
+    xp[3] = pack2(b.z, b.w);
   } else {
     const uint4 t = ok ? __ldg(reinterpret_cast<const uint4 *>(x) + v) : make_uint4(0, 0, 0, 0);
 #pragma unroll

@@ -109,3 +109,39 @@ def test_int8_descriptor_rules(torch, tmp_path):
             h.pass_([wt.gemv_desc(W.data_ptr(), wt.WT_BF16, 8, 32, x.data_ptr(), y.data_ptr(),
                                   scale=x.data_ptr())], 0)
         assert ei.value.code == wt.WT_EINVAL
+
+
+def test_int8_structured_rows(torch):
+    """Rows that stress the int8 -> f16 decode: all zero (y must be exactly 0), sparse +-1,
+    all -128, all 127, alternating extremes and uniform bytes, in every tile mode."""
+    rng = np.random.default_rng(21)
+    for K in (48, 2048, 7168, 20000):
+        M = 30
+        W = np.zeros((M, K), np.int8)
+        for r in range(M):
+            kind = r % 6
+            if kind == 1:
+                W[r, rng.choice(K, 8, replace=False)] = rng.choice([-1, 1], 8)
+            elif kind == 2:
+                W[r] = -128
+            elif kind == 3:
+                W[r] = 127
+            elif kind == 4:
+                W[r, 0::2], W[r, 1::2] = 127, -128
+            elif kind == 5:
+                W[r] = rng.integers(-128, 128, K)
+        s = rng.uniform(0.001, 0.02, M).astype(np.float16)
+        x = synth.make_x(K, synth.DT_I8)
+        Wd = torch.from_numpy(W.view(np.uint8).reshape(-1).copy()).cuda()
+        sd = torch.from_numpy(s.view(np.uint8).copy()).cuda()
+        xd = torch.from_numpy(x.copy()).cuda()
+        y = torch.full((M,), float("nan"), dtype=torch.float32, device="cuda")
+        with wt.Handle([]) as h:  # a handle without files: W is plain device memory
+            h.pass_([wt.gemv_desc(Wd.data_ptr(), wt.WT_I8, M, K, xd.data_ptr(), y.data_ptr(),
+                                  scale=sd.data_ptr())], 0)
+            torch.cuda.synchronize()
+            assert h.device_status() == 0
+        got = y.cpu().numpy()
+        yhat, a = oracle.gemv_q8(W.view(np.uint8).reshape(-1), s.view(np.uint8), M, K, x)
+        assert np.all(got[0::6] == 0.0), K
+        assert oracle.gemv_error(got, yhat, a) <= TOL, K
