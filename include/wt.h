@@ -113,11 +113,18 @@ typedef struct {
  * paper's packed-int8 kernel with fp16 row scales, Sec. 3.1 and Table "tab:tax") x is
  * fp16 and scale points at M fp16 row scales: y_i = scale_i * sum_j W_ij x_j.  All
  * pointers are caller-owned device memory (or, for W, the handle's mapping: see
- * wt_pass).  wait_event (a cudaEvent_t from wt_adopt, or NULL) gates this GEMV on the GPU. */
+ * wt_pass).  wait_event (a cudaEvent_t from wt_adopt, or NULL) gates this GEMV on the GPU.
+ *
+ * cols = T in 1..16 selects the multi-column kernel (the paper's multi-column packed-int8
+ * GEMV of the T-sweep, Sec. 4.3; each weight read serves all T activation columns):
+ * x is X[T, K] row-major (column t = activation vector t, row pitch K elements) and y is
+ * Y[T, M] row-major fp32, Y[t] = diag(scale) W X[t].  It runs on the tensor cores (fp16 or
+ * bf16 products, fp32 accumulate) for WT_BF16, WT_F16 and WT_I8 weights; WT_F32 weights
+ * with cols > 0 are WT_ENOTSUP.  cols = 0 is the one-column GEMV above. */
 typedef struct {
   const void *W;
   int32_t dtype;        /* WT_F32, WT_BF16, WT_F16 or WT_I8 */
-  int32_t reserved;     /* must be 0 */
+  int32_t cols;         /* 0: y = W x; 1..16: Y[T, M] from X[T, K] (see above) */
   uint64_t M;
   uint64_t K;
   const void *x;
@@ -177,7 +184,7 @@ int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsign
  * calls with identical descriptors reuse a cached launch plan.  The result of
  * a row does not depend on how rows were grouped or split (deterministic, no
  * floating-point atomics).  Errors: WT_EINVAL (null pointer with M*K > 0,
- * reserved != 0, dimension > 2^31-1), WT_ENOTSUP (dtype), WT_ENOMEM, WT_ECUDA. */
+ * cols outside 0..16, dimension > 2^31-1), WT_ENOTSUP (dtype), WT_ENOMEM, WT_ECUDA. */
 int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream);
 
 /* Leaf-tree FNV-1a-64 digest of each device buffer ptr[i] (nbytes[i] bytes),

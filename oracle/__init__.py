@@ -171,6 +171,31 @@ def gemv_q8(W: np.ndarray, s: np.ndarray, M: int, K: int, x: np.ndarray,
     return yhat, a
 
 
+def gemv_cols(W: np.ndarray, dtype: int, M: int, K: int, X: np.ndarray, T: int,
+              scale: Optional[np.ndarray] = None,
+              rows: Optional[Sequence[int]] = None) -> Tuple[np.ndarray, np.ndarray]:
+    """(Yhat, A), each [T, n], for the multi-column GEMV of the T-sweep (Sec. 4.3): X holds T
+    activation vectors as rows of [T, K] (fp16 for int8 weights, else W's dtype) and column t
+    of the result is the one-column GEMV of X[t]:  Yhat[t] = diag(scale) W X[t] (scale only
+    for int8 weights, dtype 3), A[t] = the matching sum of |products|.  All rows or `rows`."""
+    X = np.ascontiguousarray(X).view(np.uint8).reshape(-1)
+    xes = 2 if dtype == 3 else {0: 4, 1: 2, 2: 2}[dtype]
+    if X.size != T * K * xes:
+        raise OracleError("gemv_cols: X holds %d bytes, want T*K*%d = %d" % (X.size, xes, T * K * xes))
+    n = M if rows is None else len(rows)
+    Y = np.zeros((T, n), np.float64)
+    A = np.zeros((T, n), np.float64)
+    for t in range(T):
+        xt = X[t * K * xes:(t + 1) * K * xes]
+        if dtype == 3:
+            Y[t], A[t] = gemv_q8(W, scale, M, K, xt, rows=rows)
+        elif rows is None:
+            Y[t], A[t] = gemv(W, dtype, M, K, xt)
+        else:
+            Y[t], A[t] = gemv_rows(W, dtype, M, K, xt, rows)
+    return Y, A
+
+
 def gemv_error(y: np.ndarray, yhat: np.ndarray, a: np.ndarray) -> float:
     """max_i |y_i - yhat_i| / a_i; a row with a_i = 0 must give y_i == 0 exactly (else inf)."""
     y = np.asarray(y, np.float64)

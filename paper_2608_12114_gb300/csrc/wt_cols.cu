@@ -1,0 +1,328 @@
+// Multi-column GEMV: Y[t, :] = diag(s) W X[t, :] for t < T <= 16 activation columns, every
+// weight read once per pass and reused by all T columns (the paper's multi-column packed-int8
+// kernel and its T-sweep, Sec. 4.3 / Sec. 6; speculative batches reuse each weight read).
+//
+// W streams HBM -> shared memory on the same 1-D TMA bulk-copy ring as the one-column GEMV.
+// One stage holds a tile of 16 rows x up to kColVecMax 16-byte vectors of each row (one bulk
+// copy per row; the row pitch in shared memory is 64 bytes past a multiple of 128, so the two
+// rows a quarter-warp reads fall in different banks).  Eight consumer warps split each tile
+// along K and multiply on the tensor cores with warp-level m16n8k16 MMAs (fp32 accumulate):
+//
+//   A (16 x 16)  16 weight rows, decoded in registers (int8 -> exact f16; bf16/f16 as is)
+//   B (16 x 8)   8 activation columns (two MMAs per A for T > 8)
+//
+// The sum over k does not depend on the order of k, so each thread's four k values of one
+// MMA are four consecutive elements of one 16-byte weight vector, and its B values are the
+// same four k of X: A and B fragments come straight from whole vector loads, and an int8
+// word decodes into exactly the two f16x2 registers a fragment needs.
+//
+// Four 16-row tiles form a super block whose X registers are loaded once per K chunk.  At
+// the end of a super block the warps' partial tiles meet in shared memory and are summed in
+// warp order (deterministic; rows never depend on the partition across CTAs).
+//
+// Why warp-level MMAs and not tcgen05: the A operand is decoded from int8 in registers and
+// goes to the MMA from there; tcgen05 takes A only from shared or tensor memory, which would
+// add a store and a fence per decoded tile, and for T <= 16 the tensor rate is far from the
+// bound either way (2 * 16 flops per weight byte at most).
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "wt_device.cuh"
+#include "wt_kernels.h"
+
+namespace wt {
+
+namespace {
+
+constexpr int kColWarps = kConsumerWarps;
+constexpr int kColConsumers = kColWarps * 32;
+constexpr int kColThreads = kColConsumers + 32;  // + one producer warp
+constexpr int kColRows = 16;                     // rows of one stage (one MMA tile)
+constexpr int kColBlocks = 4;                    // tiles per super block
+constexpr int kColSuper = kColRows * kColBlocks;
+constexpr int kColGroups = kColVecMax / (4 * kColWarps);  // 4-vector groups per warp per stage
+constexpr uint32_t kColStride = kColVecMax * 16 + 64;    // row pitch in a stage
+constexpr int kColStages = 6;
+constexpr uint32_t kColStageBytes = kColRows * kColStride;
+constexpr size_t kColRedOff = (size_t)kColStages * kColStageBytes;
+constexpr size_t kColBarOff = kColRedOff + (size_t)kColBlocks * kColWarps * 256 * sizeof(float);
+constexpr size_t kColFlagOff = kColBarOff + 2 * kColStages * sizeof(uint64_t);
+constexpr size_t kColSmem = kColFlagOff + 16;
+static_assert(kColGroups * 4 * kColWarps == kColVecMax, "a stage row splits into whole groups");
+static_assert(kColStride % 128 == 64, "two rows of a quarter-warp must fall in different banks");
+static_assert(kColSmem <= 232448, "shared memory of one CTA");
+
+// 32-bit words of X per weight vector: 16 fp16 activations for an int8 vector, else 8.
+template <int DT>
+struct ColX {
+  static constexpr int W = DT == 3 ? 8 : 4;
+};
+
+template <int DT>
+__device__ __forceinline__ float col_scale(const uint8_t *s, uint64_t row) {
+  if constexpr (DT == 3) return __half2float(reinterpret_cast<const __half *>(s)[row]);
+  return 1.f;
+}
+
+// d += A B on one 16x8x16 tile; bf16 operands for DT 1, f16 otherwise.
+template <int DT>
+__device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+  if constexpr (DT == 1) {
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+  } else {
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+  }
+}
+
+// The activations of weight vector `vec` (global vector index col * V + v) of one column.
+template <int DT>
+__device__ __forceinline__ void load_xvec(const uint8_t *X, uint64_t vec, bool ok, uint32_t (&xr)[ColX<DT>::W]) {
+  const uint4 *p = reinterpret_cast<const uint4 *>(X) + (DT == 3 ? 2 * vec : vec);
+  const uint4 a = ok ? __ldg(p) : make_uint4(0, 0, 0, 0);
+  xr[0] = a.x;
+  xr[1] = a.y;
+  xr[2] = a.z;
+  xr[3] = a.w;
+  if constexpr (DT == 3) {
+    const uint4 b = ok ? __ldg(p + 1) : make_uint4(0, 0, 0, 0);
+    xr[4] = b.x;
+    xr[5] = b.y;
+    xr[6] = b.z;
+    xr[7] = b.w;
+  }
+}
+
+// One stage: rows g and g + 8 of the tile against this warp's vectors of the chunk.
+// Thread (g, t) takes vector (q * warps + warp) * 4 + t of group q.
+template <int DT, int NT>
+__device__ __forceinline__ void cols_stage(uint32_t tile, uint32_t nr, uint32_t nv, int warp, uint32_t g, uint32_t t,
+                                           const uint32_t (&xr)[kColGroups][NT][ColX<DT>::W], float (&acc)[NT][4]) {
+#pragma unroll
+  for (int q = 0; q < kColGroups; ++q) {
+    const uint32_t v0 = (uint32_t)(q * kColWarps + warp) * 4;
+    if (v0 >= nv) continue;  // warp-uniform: the chunk ends before this group
+    const uint32_t v = v0 + t;
+    const uint4 w0 = lds_or_zero(tile + g * kColStride + v * 16, v < nv && g < nr);
+    const uint4 w1 = lds_or_zero(tile + (g + 8) * kColStride + v * 16, v < nv && g + 8 < nr);
+    const uint32_t ra[4] = {w0.x, w0.y, w0.z, w0.w};
+    const uint32_t rb[4] = {w1.x, w1.y, w1.z, w1.w};
+    if constexpr (DT == 3) {
+      // word j = weights k 4j..4j+3 of the vector; its activations are x words 2j, 2j+1
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t u0 = ra[j] ^ 0x80808080u, u1 = rb[j] ^ 0x80808080u;
+        const uint32_t a0 = i8x2_to_f16x2(u0, 0x4140u), a2 = i8x2_to_f16x2(u0, 0x4342u);
+        const uint32_t a1 = i8x2_to_f16x2(u1, 0x4140u), a3 = i8x2_to_f16x2(u1, 0x4342u);
+#pragma unroll
+        for (int n = 0; n < NT; ++n) mma16816<2>(acc[n], a0, a1, a2, a3, xr[q][n][2 * j], xr[q][n][2 * j + 1]);
+      }
+    } else {
+      // words 2s, 2s+1 = elements 4s..4s+3 of the vector
+#pragma unroll
+      for (int s = 0; s < 2; ++s) {
+#pragma unroll
+        for (int n = 0; n < NT; ++n)
+          mma16816<DT>(acc[n], ra[2 * s], rb[2 * s], ra[2 * s + 1], rb[2 * s + 1], xr[q][n][2 * s],
+                       xr[q][n][2 * s + 1]);
+      }
+    }
+  }
+}
+
+struct Ring {
+  uint32_t stage0, full0, empty0;
+  volatile int *abort_flag;
+  int *status;
+};
+
+// Consumer side of one piece (rows [r0, r1) of one matrix), NT = 8-column MMA tiles.
+template <int DT, int NT>
+__device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, const Ring &R, float *red,
+                                           uint32_t &it, int warp, int lane) {
+  const uint32_t V = md.V, vc = md.vc, T = md.G;
+  const uint32_t nchunk = (V + vc - 1) / vc;
+  const uint32_t g = lane >> 2, t = lane & 3;
+  const int ct = threadIdx.x;
+  for (uint32_t sb = pc.r0; sb < pc.r1; sb += kColSuper) {
+    const uint32_t rows = min((uint32_t)kColSuper, pc.r1 - sb);
+    const uint32_t nrb = (rows + kColRows - 1) / kColRows;
+    float acc[kColBlocks][NT][4];
+#pragma unroll
+    for (int b = 0; b < kColBlocks; ++b)
+#pragma unroll
+      for (int n = 0; n < NT; ++n) acc[b][n][0] = acc[b][n][1] = acc[b][n][2] = acc[b][n][3] = 0.f;
+    for (uint32_t c = 0; c < nchunk; ++c) {
+      const uint32_t nv = min(vc, V - c * vc);
+      uint32_t xr[kColGroups][NT][ColX<DT>::W];
+#pragma unroll
+      for (int q = 0; q < kColGroups; ++q) {
+        const uint32_t v = (uint32_t)(q * kColWarps + warp) * 4 + t;
+#pragma unroll
+        for (int n = 0; n < NT; ++n) {
+          const uint32_t col = g + 8 * n;
+          load_xvec<DT>(md.x, (uint64_t)col * V + (uint64_t)c * vc + v, v < nv && col < T, xr[q][n]);
+        }
+      }
+#pragma unroll
+      for (int b = 0; b < kColBlocks; ++b) {
+        if ((uint32_t)b < nrb) {
+          const uint32_t s = it % kColStages;
+          bounded_wait(R.full0 + 8 * s, (it / kColStages) & 1, R.abort_flag, R.status);
+          const uint32_t nr = min((uint32_t)kColRows, rows - b * kColRows);
+          cols_stage<DT, NT>(R.stage0 + s * kColStageBytes, nr, nv, warp, g, t, xr, acc[b]);
+          __syncwarp();
+          if (lane == 0) mbar_arrive(R.empty0 + 8 * s);
+          ++it;
+        }
+      }
+    }
+    // warp partials -> red[b][warp][col][row]; C fragment: (g, 2t), (g, 2t+1), (g+8, 2t), (g+8, 2t+1)
+#pragma unroll
+    for (int b = 0; b < kColBlocks; ++b) {
+      if ((uint32_t)b < nrb) {
+        float *r = red + (b * kColWarps + warp) * 256;
+#pragma unroll
+        for (int n = 0; n < NT; ++n) {
+          const uint32_t c0 = 2 * t + 8 * n;
+          r[c0 * 16 + g] = acc[b][n][0];
+          r[(c0 + 1) * 16 + g] = acc[b][n][1];
+          r[c0 * 16 + g + 8] = acc[b][n][2];
+          r[(c0 + 1) * 16 + g + 8] = acc[b][n][3];
+        }
+      }
+    }
+    named_bar(1, kColConsumers);
+    for (uint32_t o = ct; o < nrb * 256; o += kColConsumers) {
+      const uint32_t b = o >> 8, e = o & 255, col = e >> 4, row = b * kColRows + (e & 15);
+      if (col < T && row < rows) {
+        const float *r = red + b * kColWarps * 256 + e;
+        float sum = 0.f;
+#pragma unroll
+        for (int w = 0; w < kColWarps; ++w) sum += r[w * 256];
+        md.y[(uint64_t)col * md.M + sb + row] = sum * col_scale<DT>(md.s, sb + row);
+      }
+    }
+    named_bar(1, kColConsumers);  // red is rewritten by the next super block
+  }
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kColThreads, 1)
+    gemm_cols_kernel(const MatDesc *__restrict__ mats, const Piece *__restrict__ pieces,
+                     const uint32_t *__restrict__ begin, int *status) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  Ring R;
+  R.stage0 = smem_u32(smem);
+  R.full0 = smem_u32(smem + kColBarOff);
+  R.empty0 = R.full0 + kColStages * 8;
+  R.abort_flag = reinterpret_cast<volatile int *>(smem + kColFlagOff);
+  R.status = status;
+  float *red = reinterpret_cast<float *>(smem + kColRedOff);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t p0 = begin[blockIdx.x];
+  const uint32_t p1 = begin[blockIdx.x + 1];
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kColStages; ++s) {
+      mbar_init(R.full0 + 8 * s, 1);
+      mbar_init(R.empty0 + 8 * s, kColWarps);
+    }
+    *R.abort_flag = 0;
+    mbar_fence_init();
+  }
+  __syncthreads();
+
+  if (warp == kColWarps) {
+    // ---------------- producer: one thread issues every bulk copy of the CTA
+    if (lane == 0) {
+      const uint64_t pol = l2_evict_first_policy();
+      uint32_t it = 0;
+      bool live = true;
+      for (uint32_t pi = p0; pi < p1 && live; ++pi) {
+        const Piece pc = pieces[pi];
+        const MatDesc md = mats[pc.mat];
+        const uint64_t rowb = (uint64_t)md.V * 16;
+        const uint32_t nchunk = (md.V + md.vc - 1) / md.vc;
+        for (uint32_t sb = pc.r0; sb < pc.r1 && live; sb += kColSuper) {
+          const uint32_t rows = min((uint32_t)kColSuper, pc.r1 - sb);
+          const uint32_t nrb = (rows + kColRows - 1) / kColRows;
+          for (uint32_t c = 0; c < nchunk && live; ++c) {
+            const uint32_t v0 = c * md.vc;
+            const uint32_t nv = min(md.vc, md.V - v0);
+            for (uint32_t b = 0; b < nrb; ++b) {
+              const uint32_t s = it % kColStages;
+              if (it >= kColStages &&
+                  !bounded_wait(R.empty0 + 8 * s, ((it / kColStages) - 1) & 1, R.abort_flag, status)) {
+                live = false;
+                break;
+              }
+              const uint32_t nr = min((uint32_t)kColRows, rows - b * kColRows);
+              const uint32_t dst = R.stage0 + s * kColStageBytes;
+              const uint32_t bar = R.full0 + 8 * s;
+              mbar_expect_tx(bar, nr * nv * 16);
+              const uint8_t *src = md.W + (uint64_t)(sb + b * kColRows) * rowb + (uint64_t)v0 * 16;
+              for (uint32_t q = 0; q < nr; ++q) bulk_g2s(dst + q * kColStride, src + q * rowb, nv * 16, bar, pol);
+              ++it;
+            }
+          }
+        }
+      }
+      if (!live || *R.abort_flag) {
+        // drain: the copies of the last (up to kColStages) issued stages may still be in flight
+        const uint32_t first = it > (uint32_t)kColStages ? it - kColStages : 0;
+        for (uint32_t j = first; j < it; ++j) {
+          const long long t0 = clock64();
+          while (!mbar_try_wait(R.full0 + 8 * (j % kColStages), (j / kColStages) & 1) &&
+                 clock64() - t0 < kWaitCycles) {
+          }
+        }
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---------------- consumers: 8 warps
+    uint32_t it = 0;
+    for (uint32_t pi = p0; pi < p1; ++pi) {
+      const Piece pc = pieces[pi];
+      const MatDesc md = mats[pc.mat];
+      if (md.G > 8) cols_piece<DT, 2>(md, pc, R, red, it, warp, lane);
+      else cols_piece<DT, 1>(md, pc, R, red, it, warp, lane);
+    }
+  }
+  __syncthreads();
+}
+
+}  // namespace
+
+size_t gemm_cols_smem_bytes() { return kColSmem; }
+
+cudaError_t gemm_cols_prepare() {
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(gemm_cols_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kColSmem)) !=
+      cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(gemm_cols_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kColSmem)) !=
+      cudaSuccess)
+    return e;
+  return cudaFuncSetAttribute(gemm_cols_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kColSmem);
+}
+
+cudaError_t launch_gemm_cols(const GemvLaunch &L, cudaStream_t s) {
+  switch (L.dtype) {
+    case 1: gemm_cols_kernel<1><<<L.grid, kColThreads, kColSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
+    case 2: gemm_cols_kernel<2><<<L.grid, kColThreads, kColSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
+    case 3: gemm_cols_kernel<3><<<L.grid, kColThreads, kColSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace wt

@@ -196,6 +196,7 @@ struct Plan {
     float *y;
     uint64_t M, K;
     const uint8_t *scale;
+    uint32_t cols;
   };
   struct Zero {
     float *y;
@@ -205,6 +206,7 @@ struct Plan {
     size_t first = 0;  // index of the group's first descriptor (its wait_event is read per call)
     std::vector<Launch> launches;
     std::vector<Launch> mapped;  // W read in place from a file mapping (map endpoint)
+    std::vector<Launch> cols;    // multi-column kernel (tensor cores)
     std::vector<Generic> generic;
     std::vector<Zero> zero;
   };
@@ -379,6 +381,7 @@ int prepare_device(int dev) {
   if (dev < 0 || dev >= 64) return set_err(WT_ECUDA, "device index %d out of range", dev);
   if (!g_prepared[dev]) {
     CU(wt::gemv_prepare());
+    CU(wt::gemm_cols_prepare());
     g_prepared[dev] = true;
   }
   return WT_OK;
@@ -616,6 +619,25 @@ wt::MatDesc make_mat(const wt_gemv_desc &d) {
   return m;
 }
 
+// Multi-column kernel: chunks of at most kColVecMax vectors per row, evened out over the row
+// (448 vectors -> 92, 92, 92, 92, 80) and kept a multiple of 4 (whole 4-vector groups).
+wt::MatDesc make_cols_mat(const wt_gemv_desc &d) {
+  wt::MatDesc m;
+  memset(&m, 0, sizeof m);
+  m.W = static_cast<const uint8_t *>(d.W);
+  m.x = static_cast<const uint8_t *>(d.x);
+  m.y = d.y;
+  m.s = static_cast<const uint8_t *>(d.scale);
+  m.M = (uint32_t)d.M;
+  m.V = (uint32_t)(d.K * elem_bytes(d.dtype) / 16);
+  m.mode = wt::kModeCols;
+  m.G = (uint16_t)d.cols;
+  m.rt = 16;
+  const uint32_t nchunk = (m.V + wt::kColVecMax - 1) / wt::kColVecMax;
+  m.vc = ((m.V + nchunk - 1) / nchunk + 3) / 4 * 4;
+  return m;
+}
+
 // Split the rows of `mats` (in order) into `grid` contiguous ranges of nearly equal bytes.
 void partition(const std::vector<wt::MatDesc> &mats, int &grid, std::vector<wt::Piece> &pieces,
                std::vector<uint32_t> &begin) {
@@ -672,7 +694,9 @@ int validate_desc(const wt_gemv_desc &d, size_t i) {
   if (d.dtype == WT_I8 && d.M > 0 && d.K > 0 && d.scale == nullptr)
     return set_err(WT_EINVAL, "desc %zu: int8 weights need fp16 row scales", i);
   if (d.dtype != WT_I8 && d.scale != nullptr) return set_err(WT_EINVAL, "desc %zu: scale is for int8 weights only", i);
-  if (d.reserved != 0) return set_err(WT_EINVAL, "desc %zu: reserved field must be 0", i);
+  if (d.cols < 0 || d.cols > 16) return set_err(WT_EINVAL, "desc %zu: cols %d outside 0..16", i, (int)d.cols);
+  if (d.cols > 0 && d.dtype == WT_F32)
+    return set_err(WT_ENOTSUP, "desc %zu: the multi-column kernel takes bf16, f16 or int8 weights", i);
   if (d.M > 0x7fffffffull || d.K > 0x7fffffffull) return set_err(WT_EINVAL, "desc %zu: M or K above 2^31-1", i);
   if (d.M > 0 && d.y == nullptr) return set_err(WT_EINVAL, "desc %zu: null y", i);
   if (d.M > 0 && d.K > 0 && (d.W == nullptr || d.x == nullptr)) return set_err(WT_EINVAL, "desc %zu: null W or x", i);
@@ -696,13 +720,14 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
     while (j < n && d[j].wait_event == d[i].wait_event) ++j;
     Plan::Group g;
     g.first = i;
-    std::vector<wt::MatDesc> by_dt[4], mapped_dt[4];
+    std::vector<wt::MatDesc> by_dt[4], mapped_dt[4], cols_dt[4];
     for (size_t k = i; k < j; ++k) {
       const wt_gemv_desc &q = d[k];
       if (q.M == 0) continue;
       const int es = elem_bytes(q.dtype);
+      const uint32_t ncol = q.cols > 0 ? (uint32_t)q.cols : 1;
       if (q.K == 0) {
-        g.zero.push_back({q.y, q.M});
+        g.zero.push_back({q.y, q.M * ncol});
         continue;
       }
       const bool fast = ((reinterpret_cast<uintptr_t>(q.W) | reinterpret_cast<uintptr_t>(q.x)) & 15) == 0 &&
@@ -718,19 +743,21 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         if (!h->prefaulted && !f->populated) prefault(f->base + off, q.M * q.K * es);
         wt_gemv_desc qd = q;
         qd.W = f->dev + off;
-        if (fast) mapped_dt[q.dtype].push_back(make_mat(qd));
+        if (fast && q.cols == 0) mapped_dt[q.dtype].push_back(make_mat(qd));
         else g.generic.push_back({q.dtype, static_cast<const uint8_t *>(qd.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
-                                  static_cast<const uint8_t *>(q.scale)});
+                                  static_cast<const uint8_t *>(q.scale), ncol});
+      } else if (fast && q.cols > 0) {
+        cols_dt[q.dtype].push_back(make_cols_mat(q));
       } else if (fast) {
         by_dt[q.dtype].push_back(make_mat(q));
       } else {
         g.generic.push_back({q.dtype, static_cast<const uint8_t *>(q.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
-                             static_cast<const uint8_t *>(q.scale)});
+                             static_cast<const uint8_t *>(q.scale), ncol});
       }
     }
-    for (int pass = 0; pass < 2; ++pass) {
+    for (int pass = 0; pass < 3; ++pass) {
       for (int dt = 0; dt < 4; ++dt) {
-        std::vector<wt::MatDesc> &ms = pass == 0 ? by_dt[dt] : mapped_dt[dt];
+        std::vector<wt::MatDesc> &ms = pass == 0 ? by_dt[dt] : pass == 1 ? mapped_dt[dt] : cols_dt[dt];
         if (ms.empty()) continue;
         Plan::Launch L;
         L.dtype = dt;
@@ -740,7 +767,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         L.mats = append(P->table, ms);
         L.pieces = append(P->table, pieces);
         L.begin = append(P->table, begin);
-        (pass == 0 ? g.launches : g.mapped).push_back(L);
+        (pass == 0 ? g.launches : pass == 1 ? g.mapped : g.cols).push_back(L);
       }
     }
     P->groups.push_back(std::move(g));
@@ -799,8 +826,19 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s) {
       CU(wt::launch_gemv_mapped(gl, s));
       h->kernel_launches++;
     }
+    for (const Plan::Launch &L : g.cols) {
+      wt::GemvLaunch gl;
+      gl.dtype = L.dtype;
+      gl.grid = L.grid;
+      gl.mats = reinterpret_cast<const wt::MatDesc *>(P->dev + L.mats);
+      gl.pieces = reinterpret_cast<const wt::Piece *>(P->dev + L.pieces);
+      gl.begin = reinterpret_cast<const uint32_t *>(P->dev + L.begin);
+      gl.status = h->status;
+      CU(wt::launch_gemm_cols(gl, s));
+      h->kernel_launches++;
+    }
     for (const Plan::Generic &q : g.generic) {
-      CU(wt::launch_gemv_generic(q.dtype, q.W, q.x, q.y, q.M, q.K, q.scale, s));
+      CU(wt::launch_gemv_generic(q.dtype, q.W, q.x, q.y, q.M, q.K, q.scale, q.cols, s));
       h->kernel_launches++;
     }
   }
@@ -849,7 +887,7 @@ extern "C" {
 
 const char *wt_last_error(void) { return t_err.c_str(); }
 
-int wt_abi_version(void) { return 2; }
+int wt_abi_version(void) { return 3; }
 
 int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **out) {
   if (!out) return set_err(WT_EINVAL, "wt_open: out is NULL");
@@ -1050,7 +1088,7 @@ int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream) {
   for (size_t i = 0; i < n; ++i) {
     int rc = validate_desc(d[i], i);
     if (rc) return rc;
-    if (d[i].M && inside_mapping(h, d[i].y, d[i].M * sizeof(float)))
+    if (d[i].M && inside_mapping(h, d[i].y, d[i].M * std::max<int32_t>(1, d[i].cols) * sizeof(float)))
       return set_err(WT_EINVAL, "wt_pass: y of desc %zu lies inside a read-only mapping", i);
   }
   std::lock_guard<std::mutex> g(h->mu);

@@ -19,87 +19,14 @@
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
+#include "wt_device.cuh"
 #include "wt_kernels.h"
 
 namespace wt {
 
 namespace {
 
-constexpr int kStatusTimedOut = -7;  // WT_ETIMEDOUT
-constexpr long long kWaitCycles = 1ll << 31;  // ~1 s at 2 GHz
-
 int g_num_sms[64] = {0};
-
-// ------------------------------------------------------------------ PTX helpers
-__device__ __forceinline__ uint32_t smem_u32(const void *p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_fence_init() {
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-               : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
-__device__ __forceinline__ uint64_t l2_evict_first_policy() {
-  uint64_t pol;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
-  return pol;
-}
-
-// 1-D bulk copy global -> this CTA's shared memory, completion counted on `bar`.
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes,
-                                         uint32_t bar, uint64_t pol) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1], %2, [%3], %4;" ::"r"(dst),
-      "l"(src), "r"(bytes), "r"(bar), "l"(pol)
-      : "memory");
-}
-
-__device__ __forceinline__ void named_bar(int id, int n) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
-}
-
-// Bounded wait.  Returns false (and raises the CTA's abort flag on a timeout)
-// instead of spinning forever.
-__device__ __forceinline__ bool bounded_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag,
-                                             int *status) {
-  if (*abort_flag) return false;
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity)) {
-    if (*abort_flag) return false;
-    if (clock64() - t0 > kWaitCycles) {
-      *abort_flag = 1;
-      if (status) atomicCAS(status, 0, kStatusTimedOut);
-      return false;
-    }
-  }
-  return true;
-}
 
 // ------------------------------------------------------------------ element math
 template <int DT>
@@ -181,14 +108,6 @@ template <int DT>
 __device__ __forceinline__ float row_scale(const uint8_t *s, uint64_t row) {
   if constexpr (DT == 3) return __half2float(reinterpret_cast<const __half *>(s)[row]);
   return 1.f;
-}
-
-__device__ __forceinline__ uint4 lds128(uint32_t addr) {
-  uint4 v;
-  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "r"(addr));
-  return v;
 }
 
 __device__ __forceinline__ float warp_sum(float v) {
@@ -291,15 +210,6 @@ __device__ __forceinline__ float fma_h2(uint32_t a, uint32_t b, float c) {
   return d;
 }
 
-// Two int8 weights as exact f16x2.  With u = b ^ 0x80 (0..255) in the low byte and 0x64 in
-// the high byte, a half holds 1024 + u (f16 has unit spacing on [1024, 2048)); subtracting
-// 1152 = 1024 + 128 leaves b, an integer in [-128, 127], exactly.
-__device__ __forceinline__ uint32_t i8x2_to_f16x2(uint32_t u, uint32_t sel) {
-  uint32_t h;
-  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(h) : "r"(__byte_perm(u, 0x64646464u, sel)), "r"(0x64806480u));
-  return h;
-}
-
 // Four running fp32 partial sums of one row (two f32x2 registers).
 struct Acc4 {
   uint64_t a = 0, b = 0;
@@ -350,10 +260,6 @@ __device__ __forceinline__ void load_xpairs(const uint8_t *x, uint32_t v, bool o
 #pragma unroll
     for (int i = 0; i < Pairs<DT>::N; ++i) xp[i] = Pairs<DT>::get(t, i);
   }
-}
-
-__device__ __forceinline__ uint4 lds_or_zero(uint32_t addr, bool ok) {
-  return ok ? lds128(addr) : make_uint4(0, 0, 0, 0);
 }
 
 // Sums N per-lane values (N a power of two) over the 32 lanes with N/2 + N/4 + ... + 1
@@ -784,20 +690,25 @@ __global__ void __launch_bounds__(256) gemv_mapped_kernel(const MatDesc *__restr
   }
 }
 
-// Fallback: one warp per row, byte-assembled scalar loads (any alignment).
+// Fallback: one warp per row, byte-assembled scalar loads (any alignment).  Column c of a
+// multi-column call reads x + c * K elements and writes y + c * M.
 template <int DT>
 __global__ void gemv_generic_kernel(const uint8_t *W, const uint8_t *x, float *y, uint64_t M,
-                                    uint64_t K, const uint8_t *s) {
+                                    uint64_t K, const uint8_t *s, uint32_t cols) {
   const uint64_t warps = (uint64_t)gridDim.x * (blockDim.x >> 5);
   const int lane = threadIdx.x & 31;
+  constexpr int kXes = 16 / Elem<XElem<DT>::value>::kEPV;
   for (uint64_t row = (uint64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); row < M;
        row += warps) {
     const uint8_t *wr = W + row * K * (uint64_t)(16 / Elem<DT>::kEPV);
-    float acc = 0.f;
-    for (uint64_t k = lane; k < K; k += 32)
-      acc = fmaf(Elem<DT>::scalar(wr, k), Elem<XElem<DT>::value>::scalar(x, k), acc);
-    acc = warp_sum(acc);
-    if (lane == 0) y[row] = acc * row_scale<DT>(s, row);
+    for (uint32_t c = 0; c < cols; ++c) {
+      const uint8_t *xc = x + (uint64_t)c * K * kXes;
+      float acc = 0.f;
+      for (uint64_t k = lane; k < K; k += 32)
+        acc = fmaf(Elem<DT>::scalar(wr, k), Elem<XElem<DT>::value>::scalar(xc, k), acc);
+      acc = warp_sum(acc);
+      if (lane == 0) y[(uint64_t)c * M + row] = acc * row_scale<DT>(s, row);
+    }
   }
 }
 
@@ -977,15 +888,16 @@ cudaError_t launch_gemv_mapped(const GemvLaunch &L, cudaStream_t s) {
 }
 
 cudaError_t launch_gemv_generic(int dtype, const uint8_t *W, const uint8_t *x, float *y, uint64_t M,
-                                uint64_t K, const uint8_t *sc, cudaStream_t s) {
+                                uint64_t K, const uint8_t *sc, uint32_t cols, cudaStream_t s) {
   if (M == 0) return cudaSuccess;
+  if (cols == 0) cols = 1;
   const uint64_t blocks64 = (M + 7) / 8;
   const int grid = (int)(blocks64 < (uint64_t)num_sms() * 8 ? blocks64 : (uint64_t)num_sms() * 8);
   switch (dtype) {
-    case 0: gemv_generic_kernel<0><<<grid, 256, 0, s>>>(W, x, y, M, K, sc); break;
-    case 1: gemv_generic_kernel<1><<<grid, 256, 0, s>>>(W, x, y, M, K, sc); break;
-    case 2: gemv_generic_kernel<2><<<grid, 256, 0, s>>>(W, x, y, M, K, sc); break;
-    case 3: gemv_generic_kernel<3><<<grid, 256, 0, s>>>(W, x, y, M, K, sc); break;
+    case 0: gemv_generic_kernel<0><<<grid, 256, 0, s>>>(W, x, y, M, K, sc, cols); break;
+    case 1: gemv_generic_kernel<1><<<grid, 256, 0, s>>>(W, x, y, M, K, sc, cols); break;
+    case 2: gemv_generic_kernel<2><<<grid, 256, 0, s>>>(W, x, y, M, K, sc, cols); break;
+    case 3: gemv_generic_kernel<3><<<grid, 256, 0, s>>>(W, x, y, M, K, sc, cols); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();

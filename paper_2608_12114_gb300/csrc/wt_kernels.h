@@ -37,7 +37,10 @@ enum GemvMode : uint16_t {
   kModeWarpRows = 0,   // rows of <= 256 vectors: each warp owns whole rows
   kModeBlockRows = 1,  // 256 < vectors <= kStageBytes/16: whole CTA per row, full-row tiles
   kModeSplitK = 2,     // longer rows: row blocks of kRowBlock rows x 4 KiB column chunks
+  kModeCols = 3,       // multi-column kernel (G = T columns): 16-row tiles x vc-vector chunks
 };
+
+constexpr int kColVecMax = 96;  // multi-column kernel: 16-byte vectors of a row per stage
 
 struct alignas(16) MatDesc {
   const uint8_t *W;
@@ -49,7 +52,7 @@ struct alignas(16) MatDesc {
   uint32_t rt;    // rows per tile (modes 0/1) or per row block (mode 2)
   uint32_t vc;    // vectors per column chunk (mode 2); V otherwise
   uint16_t mode;  // GemvMode
-  uint16_t G;     // mode 0: lanes per row (power of two <= 32)
+  uint16_t G;     // mode 0: lanes per row (power of two <= 32); kModeCols: columns T
   uint32_t pad;
 };
 
@@ -78,10 +81,20 @@ size_t gemv_smem_bytes();
 // launch_gemv (MatDesc.W holds the device-readable address of the mapped rows).
 cudaError_t launch_gemv_mapped(const GemvLaunch &L, cudaStream_t s);
 
-// Fallback for operands the tiled kernel cannot take (unaligned W/x or rows
-// whose byte length is not a multiple of 16): one warp per row, scalar loads.
+// Multi-column GEMV Y[t] = diag(s) W X[t] (t < T <= 16; X [T, K] and Y [T, M] row-major) on the
+// tensor cores (wt_cols.cu); dtype WT_BF16 / WT_F16 / WT_I8, tables as for launch_gemv with
+// MatDesc.mode = kModeCols, MatDesc.G = T and MatDesc.vc = vectors per chunk (<= kColVecMax,
+// a multiple of 4).
+cudaError_t gemm_cols_prepare();
+cudaError_t launch_gemm_cols(const GemvLaunch &L, cudaStream_t s);
+size_t gemm_cols_smem_bytes();
+
+// Fallback for operands the tiled kernels cannot take (unaligned W/x, rows whose byte length
+// is not a multiple of 16, or multi-column W read in place from a mapping): one warp per
+// row, scalar loads.  cols = 0 or 1: y = W x; cols = T > 1: Y [T, M] from X [T, K].
 cudaError_t launch_gemv_generic(int dtype, const uint8_t *W, const uint8_t *x, float *y,
-                                uint64_t M, uint64_t K, const uint8_t *scale, cudaStream_t s);
+                                uint64_t M, uint64_t K, const uint8_t *scale, uint32_t cols,
+                                cudaStream_t s);
 
 // ---------------------------------------------------------------- FNV-1a-64
 constexpr int kMaxFnv = 256;

@@ -46,13 +46,13 @@ class TensorMeta(C.Structure):
 
 
 class GemvDesc(C.Structure):
-    _fields_ = [("W", C.c_void_p), ("dtype", C.c_int32), ("reserved", C.c_int32),
+    _fields_ = [("W", C.c_void_p), ("dtype", C.c_int32), ("cols", C.c_int32),
                 ("M", C.c_uint64), ("K", C.c_uint64), ("x", C.c_void_p), ("y", C.c_void_p),
                 ("wait_event", C.c_void_p), ("scale", C.c_void_p)]
 
 
 # The same 64-byte layout as a numpy record, for building many descriptors at once.
-DESC_DTYPE = np.dtype([("W", "<u8"), ("dtype", "<i4"), ("reserved", "<i4"), ("M", "<u8"), ("K", "<u8"),
+DESC_DTYPE = np.dtype([("W", "<u8"), ("dtype", "<i4"), ("cols", "<i4"), ("M", "<u8"), ("K", "<u8"),
                        ("x", "<u8"), ("y", "<u8"), ("wait_event", "<u8"), ("scale", "<u8")])
 assert DESC_DTYPE.itemsize == C.sizeof(GemvDesc)
 
@@ -220,9 +220,10 @@ def checksum_noalloc(ptrs: Sequence[int], nbytes: Sequence[int], out_dev: int, s
 
 
 def gemv_desc(W: int, dtype: int, M: int, K: int, x: int, y: int, wait_event: int = 0,
-              scale: int = 0) -> GemvDesc:
-    """One wt_gemv_desc; int8 weights (WT_I8) take fp16 x and `scale` = fp16 [M] row scales."""
-    return GemvDesc(W, dtype, 0, M, K, x, y, wait_event or None, scale or None)
+              scale: int = 0, cols: int = 0) -> GemvDesc:
+    """One wt_gemv_desc; int8 weights (WT_I8) take fp16 x and `scale` = fp16 [M] row scales.
+    cols = T in 1..16: x is X[T, K], y is Y[T, M] (the multi-column tensor-core kernel)."""
+    return GemvDesc(W, dtype, cols, M, K, x, y, wait_event or None, scale or None)
 
 
 def open(paths: Sequence[str], flags: int = 0) -> Handle:  # noqa: A001 - mirrors wt_open

@@ -1,0 +1,163 @@
+"""Multi-column GEMV (cols = T in 1..16; the paper's multi-column packed-int8 kernel and its
+T-sweep, Sec. 4.3): Y[t] = diag(s) W X[t] on the tensor cores, against the oracle's
+gemv_cols on every output, max |Y - Yhat| / A <= 2e-3."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_12114_gb300 import build, synth, wt
+
+pytestmark = pytest.mark.gpu
+TOL = 2e-3
+BF16, F16, I8 = wt.WT_BF16, wt.WT_F16, wt.WT_I8
+
+# (dtype, M, K): ragged row counts around the 16-row tile and 64-row super block; K from one
+# 4-vector group to many uneven chunks; K not a multiple of 16 bytes -> generic fallback
+SHAPES = [(I8, 1, 16), (I8, 15, 64), (I8, 16, 1536), (I8, 17, 1552), (I8, 65, 7168), (I8, 130, 20000),
+          (I8, 33, 24), (BF16, 1, 8), (BF16, 63, 768), (BF16, 64, 4096), (BF16, 100, 776), (BF16, 7, 12),
+          (F16, 40, 2048), (F16, 9, 136)]
+TS = [1, 2, 3, 7, 8, 9, 15, 16]
+
+
+@pytest.fixture(scope="module")
+def torch():
+    import torch
+    assert torch.cuda.is_available()
+    build.build()
+    wt.lib()
+    return torch
+
+
+def make(torch, rng, dtype, M, K, T):
+    """Host bytes and device copies of W, X (and s for int8)."""
+    if dtype == I8:
+        W = rng.integers(-128, 128, (M, K)).astype(np.int8).view(np.uint8)
+        s = rng.uniform(0.001, 0.02, M).astype(np.float16).view(np.uint8)
+        X = rng.standard_normal((T, K)).astype(np.float16).view(np.uint8)
+    elif dtype == BF16:
+        W = synth.f32_to_bf16_bits((0.02 * rng.standard_normal((M, K))).astype(np.float32)).view(np.uint8)
+        X = synth.f32_to_bf16_bits(rng.standard_normal((T, K)).astype(np.float32)).view(np.uint8)
+        s = None
+    else:
+        W = (0.02 * rng.standard_normal((M, K))).astype(np.float16).view(np.uint8)
+        X = rng.standard_normal((T, K)).astype(np.float16).view(np.uint8)
+        s = None
+    dev = lambda a: None if a is None else torch.from_numpy(np.ascontiguousarray(a).reshape(-1)).cuda()  # noqa: E731
+    return dict(dtype=dtype, M=M, K=K, T=T, W=W, X=X, s=s, Wd=dev(W), Xd=dev(X), sd=dev(s),
+                Y=torch.full((T * max(M, 1),), float("nan"), dtype=torch.float32, device="cuda"))
+
+
+def desc(c, y=None):
+    return wt.gemv_desc(c["Wd"].data_ptr(), c["dtype"], c["M"], c["K"], c["Xd"].data_ptr(),
+                        (y if y is not None else c["Y"]).data_ptr(),
+                        scale=c["sd"].data_ptr() if c["sd"] is not None else 0, cols=c["T"])
+
+
+def check(c, Y):
+    Yhat, A = oracle.gemv_cols(c["W"].reshape(-1), c["dtype"], c["M"], c["K"], c["X"].reshape(-1), c["T"],
+                               scale=None if c["s"] is None else c["s"])
+    got = Y[:c["T"] * c["M"]].cpu().numpy().astype(np.float64).reshape(c["T"], c["M"])
+    err = oracle.gemv_error(got.reshape(-1), Yhat.reshape(-1), A.reshape(-1))
+    assert err <= TOL, (c["dtype"], c["M"], c["K"], c["T"], err)
+    return err
+
+
+@pytest.mark.parametrize("T", TS)
+def test_cols_against_oracle_and_grouping(torch, T):
+    rng = np.random.default_rng(100 + T)
+    cases = [make(torch, rng, d, M, K, T) for d, M, K in SHAPES]
+    with wt.Handle([]) as h:
+        h.pass_([desc(c) for c in cases], 0)          # every matrix in one group
+        torch.cuda.synchronize()
+        assert h.device_status() == 0
+        for c in cases:
+            check(c, c["Y"])
+        for c in cases:                                # one matrix per call: same bits
+            y2 = torch.full_like(c["Y"], float("nan"))
+            h.pass_([desc(c, y2)], 0)
+            torch.cuda.synchronize()
+            assert torch.equal(y2[:T * c["M"]], c["Y"][:T * c["M"]]), (c["dtype"], c["M"], c["K"])
+
+
+def test_cols_one_hot_columns_are_exact(torch):
+    """X[t] = e_{k_t}: Y[t] = s * W[:, k_t] rounded once (products of integers and ones are
+    exact on the tensor cores)."""
+    rng = np.random.default_rng(7)
+    for M, K in ((70, 7168), (17, 1552), (33, 64)):
+        T = 16
+        W = rng.integers(-128, 128, (M, K)).astype(np.int8)
+        s = rng.uniform(0.001, 0.02, M).astype(np.float16)
+        ks = rng.choice(K, T, replace=False)
+        X = np.zeros((T, K), np.float16)
+        X[np.arange(T), ks] = 1.0
+        Wd = torch.from_numpy(W.view(np.uint8).reshape(-1).copy()).cuda()
+        sd = torch.from_numpy(s.view(np.uint8).copy()).cuda()
+        Xd = torch.from_numpy(X.view(np.uint8).reshape(-1).copy()).cuda()
+        Y = torch.empty(T * M, dtype=torch.float32, device="cuda")
+        with wt.Handle([]) as h:
+            h.pass_([wt.gemv_desc(Wd.data_ptr(), I8, M, K, Xd.data_ptr(), Y.data_ptr(), scale=sd.data_ptr(),
+                                  cols=T)], 0)
+            torch.cuda.synchronize()
+        want = (s.astype(np.float32)[None, :] * W[:, ks].T.astype(np.float32))
+        assert np.array_equal(Y.cpu().numpy().reshape(T, M), want)
+
+
+def test_cols_zero_rows_and_zero_k(torch):
+    rng = np.random.default_rng(8)
+    M, K, T = 40, 3072, 5
+    W = rng.integers(-128, 128, (M, K)).astype(np.int8)
+    W[::3] = 0
+    s = rng.uniform(0.001, 0.02, M).astype(np.float16)
+    X = rng.standard_normal((T, K)).astype(np.float16)
+    Wd = torch.from_numpy(W.view(np.uint8).reshape(-1).copy()).cuda()
+    sd = torch.from_numpy(s.view(np.uint8).copy()).cuda()
+    Xd = torch.from_numpy(X.view(np.uint8).reshape(-1).copy()).cuda()
+    Y = torch.full((T * M,), float("nan"), dtype=torch.float32, device="cuda")
+    Y0 = torch.full((T * M,), float("nan"), dtype=torch.float32, device="cuda")
+    with wt.Handle([]) as h:
+        h.pass_([wt.gemv_desc(Wd.data_ptr(), I8, M, K, Xd.data_ptr(), Y.data_ptr(), scale=sd.data_ptr(), cols=T),
+                 wt.gemv_desc(Wd.data_ptr(), I8, M, 0, Xd.data_ptr(), Y0.data_ptr(), scale=sd.data_ptr(), cols=T)],
+                0)
+        torch.cuda.synchronize()
+    got = Y.cpu().numpy().reshape(T, M)
+    assert np.all(got[:, ::3] == 0.0)
+    Yhat, A = oracle.gemv_cols(W.view(np.uint8), 3, M, K, X.view(np.uint8), T, scale=s.view(np.uint8))
+    assert oracle.gemv_error(got.reshape(-1), Yhat.reshape(-1), A.reshape(-1)) <= TOL
+    assert torch.count_nonzero(Y0) == 0
+
+
+def test_cols_descriptor_rules(torch):
+    x = torch.zeros(64 * 17, dtype=torch.float16, device="cuda")
+    y = torch.zeros(8 * 17, dtype=torch.float32, device="cuda")
+    W = torch.zeros(8 * 64 * 4, dtype=torch.uint8, device="cuda")
+    with wt.Handle([]) as h:
+        for bad in (-1, 17):
+            with pytest.raises(wt.WtError) as ei:
+                h.pass_([wt.gemv_desc(W.data_ptr(), BF16, 8, 64, x.data_ptr(), y.data_ptr(), cols=bad)], 0)
+            assert ei.value.code == wt.WT_EINVAL
+        with pytest.raises(wt.WtError) as ei:
+            h.pass_([wt.gemv_desc(W.data_ptr(), wt.WT_F32, 8, 64, x.data_ptr(), y.data_ptr(), cols=2)], 0)
+        assert ei.value.code == wt.WT_ENOTSUP
+
+
+def test_cols_map_endpoint_reads_in_place(torch, tmp_path):
+    """W inside the handle's mapping with cols > 0 (plain loads through the host page tables)."""
+    shapes = [(33, 2048), (9, 7168)]
+    ck = synth.write_files(synth.custom_q8(str(tmp_path), shapes, name="mc8"))
+    co = oracle.CheckpointOracle(ck.paths)
+    T = 6
+    with wt.Handle(ck.paths) as h:
+        for i, (M, K) in enumerate(shapes):
+            t = h.tensors[h.find("w%d" % i)]
+            sc = h.tensors[h.find("w%d.scale" % i)]
+            s = co.blob_of(sc.file, sc.name)
+            sd = torch.from_numpy(s.copy()).cuda()
+            X = np.random.default_rng(M).standard_normal((T, K)).astype(np.float16)
+            Xd = torch.from_numpy(X.view(np.uint8).reshape(-1).copy()).cuda()
+            Y = torch.full((T * M,), float("nan"), dtype=torch.float32, device="cuda")
+            h.pass_([wt.gemv_desc(t.host_ptr, I8, M, K, Xd.data_ptr(), Y.data_ptr(), scale=sd.data_ptr(),
+                                  cols=T)], 0)
+            torch.cuda.synchronize()
+            Yhat, A = oracle.gemv_cols(co.blob_of(t.file, t.name), 3, M, K, X.view(np.uint8), T, scale=s)
+            assert oracle.gemv_error(Y.cpu().numpy().astype(np.float64), Yhat.reshape(-1), A.reshape(-1)) <= TOL
+        assert h.device_status() == 0

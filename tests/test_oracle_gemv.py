@@ -177,3 +177,51 @@ def test_q8_one_hot_gives_scaled_column_and_matches_numpy():
     assert list(yr) == [yhat[5], yhat[0], yhat[39]] and list(ar) == [a[5], a[0], a[39]]
     with pytest.raises(oracle.OracleError):
         oracle.gemv_q8(W.view(np.uint8), s.view(np.uint8), M, K, xv.view(np.uint8), rows=[M])
+
+
+# ----------------------------------------------------------------------------- T activation columns
+
+def test_cols_integer_exact_and_orientation():
+    """X is [T, K] row-major: column t of the result uses row t of X.  Distinct integer
+    columns make a transposed or shared X fail."""
+    rng = np.random.default_rng(31)
+    M, K, T = 6, 40, 5
+    W = rng.integers(-8, 9, (M, K))
+    X = rng.integers(-4, 5, (T, K))
+    Y, A = oracle.gemv_cols(enc(W, BF16), BF16, M, K, enc(X, BF16), T)
+    assert Y.shape == (T, M)
+    for t in range(T):
+        for i in range(M):
+            assert Y[t, i] == sum(int(W[i, j]) * int(X[t, j]) for j in range(K))
+            assert A[t, i] == sum(abs(int(W[i, j]) * int(X[t, j])) for j in range(K))
+
+
+def test_cols_int8_scaled_exact_and_matches_numpy():
+    rng = np.random.default_rng(32)
+    M, K, T = 9, 64, 3
+    W = rng.integers(-128, 128, (M, K)).astype(np.int8)
+    X = rng.integers(-3, 4, (T, K))
+    s = 2.0 ** rng.integers(-5, 2, M)
+    Y, _ = oracle.gemv_cols(W.view(np.uint8), 3, M, K, _f16(X), T, scale=_f16(s))
+    for t in range(T):
+        for i in range(M):
+            assert Y[t, i] == s[i] * sum(int(W[i, j]) * int(X[t, j]) for j in range(K))
+    Xf = rng.standard_normal((T, K)).astype(np.float16)
+    sf = rng.uniform(0.001, 0.02, M).astype(np.float16)
+    Y, _ = oracle.gemv_cols(W.view(np.uint8), 3, M, K, Xf.view(np.uint8), T, scale=sf.view(np.uint8))
+    ref = (W.astype(np.float64) @ Xf.astype(np.float64).T).T * sf.astype(np.float64)[None, :]
+    assert np.allclose(Y, ref, rtol=1e-12, atol=0)
+
+
+def test_cols_rows_subset_and_single_column():
+    rng = np.random.default_rng(33)
+    M, K, T = 20, 48, 4
+    Wb = synth.f32_to_bf16_bits(rng.standard_normal((M, K)).astype(np.float32)).view(np.uint8)
+    X = synth.f32_to_bf16_bits(rng.standard_normal((T, K)).astype(np.float32)).view(np.uint8)
+    Y, A = oracle.gemv_cols(Wb, BF16, M, K, X, T)
+    Ys, As = oracle.gemv_cols(Wb, BF16, M, K, X, T, rows=[3, 19, 0])
+    assert np.array_equal(Ys, Y[:, [3, 19, 0]]) and np.array_equal(As, A[:, [3, 19, 0]])
+    y1, a1 = oracle.gemv(Wb, BF16, M, K, X.reshape(T, -1)[2])
+    assert np.array_equal(Y[2], y1) and np.array_equal(A[2], a1)
+    with pytest.raises(oracle.OracleError):
+        oracle.gemv_cols(Wb, BF16, M, K, X[:-2], T)
