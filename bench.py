@@ -66,6 +66,9 @@ def parse_args():
     p.add_argument("--workers", type=int, default=0)
     p.add_argument("--cube", action="store_true",
                    help="the C1/C2/C3 contract ablation and ordering mechanisms on the protocol workload")
+    p.add_argument("--tsweep", default=None, metavar="T,T,...",
+                   help="multi-column T-sweep (e.g. 0,1,2,4,8,16; 0 = the one-column kernel) on the "
+                        "int8 matched protocol by default (one JSON line)")
     p.add_argument("--policy", action="store_true",
                    help="measure the map / resident / per-use-copy endpoints and apply Algorithm 2 (one JSON line)")
     return p.parse_args()
@@ -614,6 +617,86 @@ def run_policy(args):
     print(json.dumps(d), flush=True)
 
 
+def run_tsweep(args):
+    """The T-sweep (Sec. 4.3): one multi-column pass over every matrix with T activation
+    columns, resident in HBM (CUDA events over `steps` passes) and per-use copy (wt_adopt +
+    the event-gated pass, wall time per rep)."""
+    if args.workload == "large":
+        args.workload = "protocol_q8"
+    ts = [int(v) for v in args.tsweep.split(",")]
+    ck, gen_s = make_files(args, 0, 1)
+    import torch
+    from paper_2608_12114_gb300 import build, pipeline, wt
+    build.build()
+    torch.cuda.set_device(0)
+    h = wt.Handle(ck.paths)
+    mats = pipeline.matrices(h)
+    dev = pipeline.DeviceCheckpoint.allocate(h, mats)
+    ks = dev.gemv_mats()
+    s = torch.cuda.Stream()
+    ingest = torch.cuda.Stream()
+    dev.adopt(h, wt.WT_ADOPT_GATHER, s.cuda_stream)
+    s.synchronize()
+    wbytes = dev.weight_bytes
+    peak, peak_kind = measured_peaks()
+    g = torch.Generator(device="cpu").manual_seed(1234)
+    rows = []
+    with Clocks(bus_id()) as clk:
+        for T in ts:
+            n = max(T, 1)
+            xs = {}
+            for k in ks:
+                m = dev.mats[k]
+                key = (m.shape[1], m.dtype)
+                if key not in xs:
+                    xdt = torch.bfloat16 if m.dtype == wt.WT_BF16 else torch.float16
+                    xs[key] = torch.randn(n, m.shape[1], generator=g).to(xdt).cuda()
+            ys = {k: torch.empty(n * dev.mats[k].shape[0], dtype=torch.float32, device="cuda") for k in ks}
+            d = dev.descs(xs, ys)
+            d["cols"] = T
+            for _ in range(args.warmup):
+                h.pass_(d, s.cuda_stream)
+            s.synchronize()
+            n0 = h.kernel_launches()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(s)
+            for _ in range(args.steps):
+                h.pass_(d, s.cuda_stream)
+            e1.record(s)
+            s.synchronize()
+            ms = e0.elapsed_time(e1) / args.steps
+            launches = (h.kernel_launches() - n0) / args.steps
+            if h.device_status() != 0:
+                raise SystemExit("device status %d in the T-sweep" % h.device_status())
+            copy_ms = []
+            for rep in range(max(2, args.e2e_reps) + 1):
+                torch.cuda.synchronize()
+                t0 = time.perf_counter()
+                evs = dev.adopt(h, wt.WT_ADOPT_GATHER, ingest.cuda_stream)
+                dc = dev.descs(xs, ys, evs)
+                dc["cols"] = T
+                h.pass_(dc, s.cuda_stream)
+                s.synchronize()
+                ingest.synchronize()
+                if rep:
+                    copy_ms.append((time.perf_counter() - t0) * 1e3)
+            cm = statistics.median(copy_ms)
+            flops = 2.0 * sum(dev.mats[k].shape[0] * dev.mats[k].shape[1] for k in ks) * n
+            rows.append({"T": T, "kernel": "gemv_tma (one column)" if T == 0 else "gemm_cols (mma.sync m16n8k16)",
+                         "ms": round(ms, 4), "weight_gbs": round(wbytes / ms / 1e6, 1),
+                         "logical_gbs": round(n * wbytes / ms / 1e6, 1), "tflops": round(flops / ms / 1e9, 2),
+                         "frac_of_hbm": round(wbytes / ms / 1e6 / peak, 4), "launches_per_pass": launches,
+                         "copy_ms": round(cm, 3), "resident_over_copy": round(cm / ms, 2)})
+            log("T=%d: %.4f ms, %.1f GB/s weights (%.1f%% of %s HBM), copy %.3f ms" % (
+                T, ms, wbytes / ms / 1e6, 100 * wbytes / ms / 1e6 / peak, peak_kind, cm))
+    h.close()
+    out = {"metric": "multi-column T-sweep: resident pass time and weight GB/s per T", "unit": "GB/s",
+           "config": {"workload": workload_desc(args), "weight_bytes": wbytes, "matrices": len(ks),
+                      "steps": args.steps, "warmup": args.warmup, "l2": "inputs larger than L2 (no flush)"},
+           "peak_hbm_gbs": peak, "peak_kind": peak_kind, "tsweep": rows, "clocks": clk.summary()}
+    print(json.dumps(out), flush=True)
+
+
 def main():
     args = parse_args()
     rank = int(os.environ.get("RANK", "0"))
@@ -623,6 +706,9 @@ def main():
         return
     if args.policy:
         run_policy(args)
+        return
+    if args.tsweep:
+        run_tsweep(args)
         return
     if args.cube:
         run_cube(args)

@@ -2,10 +2,12 @@
 // weight read once per pass and reused by all T columns (the paper's multi-column packed-int8
 // kernel and its T-sweep, Sec. 4.3 / Sec. 6; speculative batches reuse each weight read).
 //
-// W streams HBM -> shared memory on the same 1-D TMA bulk-copy ring as the one-column GEMV.
-// One stage holds a tile of 16 rows x up to kColVecMax 16-byte vectors of each row (one bulk
-// copy per row; the row pitch in shared memory is 64 bytes past a multiple of 128, so the two
-// rows a quarter-warp reads fall in different banks).  Eight consumer warps split each tile
+// W streams HBM -> shared memory on an mbarrier ring of 2-D TMA tensor copies: one copy per
+// stage brings a tile of 16 rows x vc 16-byte vectors (a box of the matrix seen as
+// [M, 2V] 8-byte elements; rows and vectors past the end arrive as zeros).  Per-row 1-D
+// copies of 1.5 KB were issue-bound near 3.4 TB/s; one box per 16 rows is not.  The row
+// pitch vc * 16 is 64 bytes past a multiple of 128, so the two rows a quarter-warp reads
+// fall in different banks.  Eight consumer warps split each tile
 // along K and multiply on the tensor cores with warp-level m16n8k16 MMAs (fp32 accumulate):
 //
 //   A (16 x 16)  16 weight rows, decoded in registers (int8 -> exact f16; bf16/f16 as is)
@@ -37,19 +39,18 @@ namespace {
 constexpr int kColWarps = kConsumerWarps;
 constexpr int kColConsumers = kColWarps * 32;
 constexpr int kColThreads = kColConsumers + 32;  // + one producer warp
-constexpr int kColRows = 16;                     // rows of one stage (one MMA tile)
+constexpr int kColRows = kColTileRows;           // rows of one stage (one MMA tile)
 constexpr int kColBlocks = 4;                    // tiles per super block
 constexpr int kColSuper = kColRows * kColBlocks;
-constexpr int kColGroups = kColVecMax / (4 * kColWarps);  // 4-vector groups per warp per stage
-constexpr uint32_t kColStride = kColVecMax * 16 + 64;    // row pitch in a stage
+constexpr int kColGroups = (kColVecMax / 4 + kColWarps - 1) / kColWarps;  // 4-vector groups per warp
 constexpr int kColStages = 6;
-constexpr uint32_t kColStageBytes = kColRows * kColStride;
+constexpr uint32_t kColStageBytes = kColRows * kColVecMax * 16;
 constexpr size_t kColRedOff = (size_t)kColStages * kColStageBytes;
 constexpr size_t kColBarOff = kColRedOff + (size_t)kColBlocks * kColWarps * 256 * sizeof(float);
 constexpr size_t kColFlagOff = kColBarOff + 2 * kColStages * sizeof(uint64_t);
 constexpr size_t kColSmem = kColFlagOff + 16;
-static_assert(kColGroups * 4 * kColWarps == kColVecMax, "a stage row splits into whole groups");
-static_assert(kColStride % 128 == 64, "two rows of a quarter-warp must fall in different banks");
+static_assert(kColVecMax % 8 == 4, "row pitch 64 bytes past a multiple of 128");
+static_assert(kColStageBytes % 128 == 0, "stages stay 128-byte aligned for the tensor copies");
 static_assert(kColSmem <= 232448, "shared memory of one CTA");
 
 // 32-bit words of X per weight vector: 16 fp16 activations for an int8 vector, else 8.
@@ -99,18 +100,32 @@ __device__ __forceinline__ void load_xvec(const uint8_t *X, uint64_t vec, bool o
   }
 }
 
+// 2-D tensor copy of one box into this CTA's shared memory, completion counted on `bar`.
+// x (in 8-byte elements) is always a multiple of 2: 16-byte aligned.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *tmap, int32_t x, int32_t y, uint32_t bar,
+                                            uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"(tmap), "r"(x), "r"(y), "r"(bar), "l"(pol)
+      : "memory");
+}
+
 // One stage: rows g and g + 8 of the tile against this warp's vectors of the chunk.
 // Thread (g, t) takes vector (q * warps + warp) * 4 + t of group q.
+// The box holds vc vectors per row at pitch vc * 16; rows and vectors past the matrix are
+// zeros, so only whole groups past vc are skipped.
 template <int DT, int NT>
-__device__ __forceinline__ void cols_stage(uint32_t tile, uint32_t nr, uint32_t nv, int warp, uint32_t g, uint32_t t,
+__device__ __forceinline__ void cols_stage(uint32_t tile, uint32_t vc, int warp, uint32_t g, uint32_t t,
                                            const uint32_t (&xr)[kColGroups][NT][ColX<DT>::W], float (&acc)[NT][4]) {
+  const uint32_t pitch = vc * 16;
 #pragma unroll
   for (int q = 0; q < kColGroups; ++q) {
     const uint32_t v0 = (uint32_t)(q * kColWarps + warp) * 4;
-    if (v0 >= nv) continue;  // warp-uniform: the chunk ends before this group
+    if (v0 >= vc) continue;  // warp-uniform: the box ends before this group
     const uint32_t v = v0 + t;
-    const uint4 w0 = lds_or_zero(tile + g * kColStride + v * 16, v < nv && g < nr);
-    const uint4 w1 = lds_or_zero(tile + (g + 8) * kColStride + v * 16, v < nv && g + 8 < nr);
+    const uint4 w0 = lds128(tile + g * pitch + v * 16);
+    const uint4 w1 = lds128(tile + (g + 8) * pitch + v * 16);
     const uint32_t ra[4] = {w0.x, w0.y, w0.z, w0.w};
     const uint32_t rb[4] = {w1.x, w1.y, w1.z, w1.w};
     if constexpr (DT == 3) {
@@ -175,8 +190,7 @@ __device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, c
         if ((uint32_t)b < nrb) {
           const uint32_t s = it % kColStages;
           bounded_wait(R.full0 + 8 * s, (it / kColStages) & 1, R.abort_flag, R.status);
-          const uint32_t nr = min((uint32_t)kColRows, rows - b * kColRows);
-          cols_stage<DT, NT>(R.stage0 + s * kColStageBytes, nr, nv, warp, g, t, xr, acc[b]);
+          cols_stage<DT, NT>(R.stage0 + s * kColStageBytes, vc, warp, g, t, xr, acc[b]);
           __syncwarp();
           if (lane == 0) mbar_arrive(R.empty0 + 8 * s);
           ++it;
@@ -216,7 +230,7 @@ __device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, c
 template <int DT>
 __global__ void __launch_bounds__(kColThreads, 1)
     gemm_cols_kernel(const MatDesc *__restrict__ mats, const Piece *__restrict__ pieces,
-                     const uint32_t *__restrict__ begin, int *status) {
+                     const uint32_t *__restrict__ begin, int *status, const uint8_t *__restrict__ maps) {
   extern __shared__ __align__(128) uint8_t smem[];
   Ring R;
   R.stage0 = smem_u32(smem);
@@ -249,14 +263,12 @@ __global__ void __launch_bounds__(kColThreads, 1)
       for (uint32_t pi = p0; pi < p1 && live; ++pi) {
         const Piece pc = pieces[pi];
         const MatDesc md = mats[pc.mat];
-        const uint64_t rowb = (uint64_t)md.V * 16;
+        const uint8_t *tmap = maps + (size_t)pc.mat * kTensorMapBytes;
         const uint32_t nchunk = (md.V + md.vc - 1) / md.vc;
         for (uint32_t sb = pc.r0; sb < pc.r1 && live; sb += kColSuper) {
           const uint32_t rows = min((uint32_t)kColSuper, pc.r1 - sb);
           const uint32_t nrb = (rows + kColRows - 1) / kColRows;
           for (uint32_t c = 0; c < nchunk && live; ++c) {
-            const uint32_t v0 = c * md.vc;
-            const uint32_t nv = min(md.vc, md.V - v0);
             for (uint32_t b = 0; b < nrb; ++b) {
               const uint32_t s = it % kColStages;
               if (it >= kColStages &&
@@ -264,12 +276,10 @@ __global__ void __launch_bounds__(kColThreads, 1)
                 live = false;
                 break;
               }
-              const uint32_t nr = min((uint32_t)kColRows, rows - b * kColRows);
-              const uint32_t dst = R.stage0 + s * kColStageBytes;
               const uint32_t bar = R.full0 + 8 * s;
-              mbar_expect_tx(bar, nr * nv * 16);
-              const uint8_t *src = md.W + (uint64_t)(sb + b * kColRows) * rowb + (uint64_t)v0 * 16;
-              for (uint32_t q = 0; q < nr; ++q) bulk_g2s(dst + q * kColStride, src + q * rowb, nv * 16, bar, pol);
+              mbar_expect_tx(bar, kColRows * md.vc * 16);  // the whole box, zero fill included
+              tma_load_2d(R.stage0 + s * kColStageBytes, tmap, (int32_t)(2 * c * md.vc),
+                          (int32_t)(sb + b * kColRows), bar, pol);
               ++it;
             }
           }
@@ -316,10 +326,11 @@ cudaError_t gemm_cols_prepare() {
 }
 
 cudaError_t launch_gemm_cols(const GemvLaunch &L, cudaStream_t s) {
+  if (L.maps == nullptr) return cudaErrorInvalidValue;
   switch (L.dtype) {
-    case 1: gemm_cols_kernel<1><<<L.grid, kColThreads, kColSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
-    case 2: gemm_cols_kernel<2><<<L.grid, kColThreads, kColSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
-    case 3: gemm_cols_kernel<3><<<L.grid, kColThreads, kColSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
+    case 1: gemm_cols_kernel<1><<<L.grid, kColThreads, kColSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.maps); break;
+    case 2: gemm_cols_kernel<2><<<L.grid, kColThreads, kColSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.maps); break;
+    case 3: gemm_cols_kernel<3><<<L.grid, kColThreads, kColSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.maps); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();

@@ -32,6 +32,7 @@
 #include <unordered_set>
 #include <vector>
 
+#include <cuda.h>  // CUtensorMap and its encoder's signature (resolved through the runtime)
 #include <cuda_runtime.h>
 
 #include "../../include/wt.h"
@@ -189,6 +190,7 @@ struct Plan {
     int dtype;
     int grid;
     size_t mats, pieces, begin;  // byte offsets in the table
+    size_t maps = SIZE_MAX;      // multi-column launches: tensor maps (128-byte aligned)
   };
   struct Generic {
     int dtype;
@@ -620,7 +622,8 @@ wt::MatDesc make_mat(const wt_gemv_desc &d) {
 }
 
 // Multi-column kernel: chunks of at most kColVecMax vectors per row, evened out over the row
-// (448 vectors -> 92, 92, 92, 92, 80) and kept a multiple of 4 (whole 4-vector groups).
+// and rounded up to 4 (mod 8): 448 vectors -> 5 chunks of 92 (the last box zero-filled past
+// the row's end).
 wt::MatDesc make_cols_mat(const wt_gemv_desc &d) {
   wt::MatDesc m;
   memset(&m, 0, sizeof m);
@@ -634,13 +637,51 @@ wt::MatDesc make_cols_mat(const wt_gemv_desc &d) {
   m.G = (uint16_t)d.cols;
   m.rt = 16;
   const uint32_t nchunk = (m.V + wt::kColVecMax - 1) / wt::kColVecMax;
-  m.vc = ((m.V + nchunk - 1) / nchunk + 3) / 4 * 4;
+  m.vc = ((m.V + nchunk - 1) / nchunk + 3) / 8 * 8 + 4;
   return m;
+}
+
+// cuTensorMapEncodeTiled, looked up once through the runtime (no link against libcuda).
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// The tensor map of a multi-column matrix: W as [M rows, 2V] 8-byte elements (row pitch
+// V * 16 bytes), box {2 vc, kColTileRows}, no swizzle, zero fill outside the matrix.
+int encode_cols_map(const wt::MatDesc &m, uint8_t *out) {
+  static_assert(sizeof(CUtensorMap) == wt::kTensorMapBytes, "tensor map size");
+  EncodeTiledFn fn = encode_tiled();
+  if (!fn) return set_err(WT_ECUDA, "wt_pass: cuTensorMapEncodeTiled is not available from the driver");
+  const cuuint64_t dims[2] = {(cuuint64_t)m.V * 2, (cuuint64_t)m.M};
+  const cuuint64_t strides[1] = {(cuuint64_t)m.V * 16};
+  const cuuint32_t box[2] = {m.vc * 2, (cuuint32_t)wt::kColTileRows};
+  const cuuint32_t estr[2] = {1, 1};
+  CUtensorMap map;
+  const CUresult r = fn(&map, CU_TENSOR_MAP_DATA_TYPE_UINT64, 2, const_cast<uint8_t *>(m.W), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS)
+    return set_err(WT_ECUDA, "wt_pass: cuTensorMapEncodeTiled failed (%d) for a %u x %u-vector matrix", (int)r, m.M, m.V);
+  memcpy(out, &map, sizeof map);
+  return WT_OK;
 }
 
 // Split the rows of `mats` (in order) into `grid` contiguous ranges of nearly equal bytes.
 void partition(const std::vector<wt::MatDesc> &mats, int &grid, std::vector<wt::Piece> &pieces,
-               std::vector<uint32_t> &begin) {
+               std::vector<uint32_t> &begin, uint32_t row_align = 1) {
   uint64_t B = 0;
   std::vector<uint64_t> start(mats.size() + 1, 0);
   for (size_t i = 0; i < mats.size(); ++i) {
@@ -659,6 +700,7 @@ void partition(const std::vector<wt::MatDesc> &mats, int &grid, std::vector<wt::
     while (m + 1 < mats.size() && start[m + 1] <= T) ++m;
     const uint64_t rb = (uint64_t)mats[m].V * 16;
     uint64_t row = (T - start[m] + rb / 2) / rb;
+    row = (row + row_align / 2) / row_align * row_align;  // whole tiles per CTA
     std::pair<uint32_t, uint32_t> cut = {(uint32_t)m, (uint32_t)std::min<uint64_t>(row, mats[m].M)};
     if (cut.second == mats[m].M && m + 1 < mats.size()) cut = {(uint32_t)m + 1, 0};
     if (cut < cuts.back()) cut = cuts.back();
@@ -763,10 +805,18 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         L.dtype = dt;
         std::vector<wt::Piece> pieces;
         std::vector<uint32_t> begin;
-        partition(ms, L.grid, pieces, begin);
+        partition(ms, L.grid, pieces, begin, pass == 2 ? (uint32_t)wt::kColTileRows : 1u);
         L.mats = append(P->table, ms);
         L.pieces = append(P->table, pieces);
         L.begin = append(P->table, begin);
+        if (pass == 2) {
+          L.maps = (P->table.size() + 127) & ~(size_t)127;
+          P->table.resize(L.maps + ms.size() * wt::kTensorMapBytes);
+          for (size_t k = 0; k < ms.size(); ++k) {
+            int rc = encode_cols_map(ms[k], P->table.data() + L.maps + k * wt::kTensorMapBytes);
+            if (rc) return rc;
+          }
+        }
         (pass == 0 ? g.launches : pass == 1 ? g.mapped : g.cols).push_back(L);
       }
     }
@@ -834,6 +884,7 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s) {
       gl.pieces = reinterpret_cast<const wt::Piece *>(P->dev + L.pieces);
       gl.begin = reinterpret_cast<const uint32_t *>(P->dev + L.begin);
       gl.status = h->status;
+      gl.maps = P->dev + L.maps;
       CU(wt::launch_gemm_cols(gl, s));
       h->kernel_launches++;
     }

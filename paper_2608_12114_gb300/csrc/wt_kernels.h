@@ -40,7 +40,12 @@ enum GemvMode : uint16_t {
   kModeCols = 3,       // multi-column kernel (G = T columns): 16-row tiles x vc-vector chunks
 };
 
-constexpr int kColVecMax = 96;  // multi-column kernel: 16-byte vectors of a row per stage
+// Multi-column kernel: at most kColVecMax 16-byte vectors of a row per stage, and a chunk
+// length vc = 4 (mod 8) so that the stage's row pitch vc * 16 is 64 bytes past a multiple
+// of 128 (the two rows a quarter-warp reads fall in different banks).
+constexpr int kColVecMax = 92;
+constexpr int kColTileRows = 16;
+constexpr int kTensorMapBytes = 128;  // one CUtensorMap
 
 struct alignas(16) MatDesc {
   const uint8_t *W;
@@ -70,6 +75,8 @@ struct GemvLaunch {
   const Piece *pieces;     // device
   const uint32_t *begin;   // device, grid + 1 entries
   int *status;             // device status word (bounded-wait failures)
+  const uint8_t *maps = nullptr;  // multi-column kernel: one TMA tensor map per MatDesc
+                                  // (kTensorMapBytes each, 128-byte aligned, device)
 };
 
 cudaError_t gemv_prepare();  // one-time function attributes
@@ -84,7 +91,9 @@ cudaError_t launch_gemv_mapped(const GemvLaunch &L, cudaStream_t s);
 // Multi-column GEMV Y[t] = diag(s) W X[t] (t < T <= 16; X [T, K] and Y [T, M] row-major) on the
 // tensor cores (wt_cols.cu); dtype WT_BF16 / WT_F16 / WT_I8, tables as for launch_gemv with
 // MatDesc.mode = kModeCols, MatDesc.G = T and MatDesc.vc = vectors per chunk (<= kColVecMax,
-// a multiple of 4).
+// vc = 4 mod 8), plus GemvLaunch.maps: per matrix a 2-D tensor map of W viewed as
+// [M, 2V] 8-byte elements with box {2 vc, kColTileRows} (rows and columns past the end
+// arrive as zeros).
 cudaError_t gemm_cols_prepare();
 cudaError_t launch_gemm_cols(const GemvLaunch &L, cudaStream_t s);
 size_t gemm_cols_smem_bytes();
