@@ -46,7 +46,8 @@ constexpr int kColGroups = (kColVecMax / 4 + kColWarps - 1) / kColWarps;  // 4-v
 constexpr int kColStages = 6;
 constexpr uint32_t kColStageBytes = kColRows * kColVecMax * 16;
 constexpr size_t kColRedOff = (size_t)kColStages * kColStageBytes;
-constexpr size_t kColBarOff = kColRedOff + (size_t)kColBlocks * kColWarps * 256 * sizeof(float);
+constexpr size_t kColRedFloats = (size_t)kColBlocks * kColWarps * 256;  // one of two halves
+constexpr size_t kColBarOff = kColRedOff + 2 * kColRedFloats * sizeof(float);
 constexpr size_t kColFlagOff = kColBarOff + 2 * kColStages * sizeof(uint64_t);
 constexpr size_t kColSmem = kColFlagOff + 16;
 static_assert(kColVecMax % 8 == 4, "row pitch 64 bytes past a multiple of 128");
@@ -117,7 +118,7 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *tmap, int3
 // zeros, so only whole groups past vc are skipped.
 template <int DT, int NT>
 __device__ __forceinline__ void cols_stage(uint32_t tile, uint32_t vc, int warp, uint32_t g, uint32_t t,
-                                           const uint32_t (&xr)[kColGroups][NT][ColX<DT>::W], float (&acc)[NT][4]) {
+                                           const uint32_t (&xr)[kColGroups][NT][ColX<DT>::W], float (&acc)[2][NT][4]) {
   const uint32_t pitch = vc * 16;
 #pragma unroll
   for (int q = 0; q < kColGroups; ++q) {
@@ -136,7 +137,8 @@ __device__ __forceinline__ void cols_stage(uint32_t tile, uint32_t vc, int warp,
         const uint32_t a0 = i8x2_to_f16x2(u0, 0x4140u), a2 = i8x2_to_f16x2(u0, 0x4342u);
         const uint32_t a1 = i8x2_to_f16x2(u1, 0x4140u), a3 = i8x2_to_f16x2(u1, 0x4342u);
 #pragma unroll
-        for (int n = 0; n < NT; ++n) mma16816<2>(acc[n], a0, a1, a2, a3, xr[q][n][2 * j], xr[q][n][2 * j + 1]);
+        for (int n = 0; n < NT; ++n)
+          mma16816<2>(acc[j & 1][n], a0, a1, a2, a3, xr[q][n][2 * j], xr[q][n][2 * j + 1]);
       }
     } else {
       // words 2s, 2s+1 = elements 4s..4s+3 of the vector
@@ -144,7 +146,7 @@ __device__ __forceinline__ void cols_stage(uint32_t tile, uint32_t vc, int warp,
       for (int s = 0; s < 2; ++s) {
 #pragma unroll
         for (int n = 0; n < NT; ++n)
-          mma16816<DT>(acc[n], ra[2 * s], rb[2 * s], ra[2 * s + 1], rb[2 * s + 1], xr[q][n][2 * s],
+          mma16816<DT>(acc[s][n], ra[2 * s], rb[2 * s], ra[2 * s + 1], rb[2 * s + 1], xr[q][n][2 * s],
                        xr[q][n][2 * s + 1]);
       }
     }
@@ -159,8 +161,8 @@ struct Ring {
 
 // Consumer side of one piece (rows [r0, r1) of one matrix), NT = 8-column MMA tiles.
 template <int DT, int NT>
-__device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, const Ring &R, float *red,
-                                           uint32_t &it, int warp, int lane) {
+__device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, const Ring &R, float *red_base,
+                                           uint32_t &it, uint32_t &par, int warp, int lane) {
   const uint32_t V = md.V, vc = md.vc, T = md.G;
   const uint32_t nchunk = (V + vc - 1) / vc;
   const uint32_t g = lane >> 2, t = lane & 3;
@@ -168,11 +170,13 @@ __device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, c
   for (uint32_t sb = pc.r0; sb < pc.r1; sb += kColSuper) {
     const uint32_t rows = min((uint32_t)kColSuper, pc.r1 - sb);
     const uint32_t nrb = (rows + kColRows - 1) / kColRows;
-    float acc[kColBlocks][NT][4];
+    float acc[kColBlocks][2][NT][4];  // two accumulator sets (even / odd k16 steps): shorter MMA chains
 #pragma unroll
     for (int b = 0; b < kColBlocks; ++b)
 #pragma unroll
-      for (int n = 0; n < NT; ++n) acc[b][n][0] = acc[b][n][1] = acc[b][n][2] = acc[b][n][3] = 0.f;
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int n = 0; n < NT; ++n) acc[b][h][n][0] = acc[b][h][n][1] = acc[b][h][n][2] = acc[b][h][n][3] = 0.f;
     for (uint32_t c = 0; c < nchunk; ++c) {
       const uint32_t nv = min(vc, V - c * vc);
       uint32_t xr[kColGroups][NT][ColX<DT>::W];
@@ -197,7 +201,11 @@ __device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, c
         }
       }
     }
-    // warp partials -> red[b][warp][col][row]; C fragment: (g, 2t), (g, 2t+1), (g+8, 2t), (g+8, 2t+1)
+    // warp partials -> red[b][warp][col][row]; C fragment: (g, 2t), (g, 2t+1), (g+8, 2t), (g+8, 2t+1).
+    // Two halves alternate, so one barrier per super block suffices: a half is rewritten
+    // only after every thread has passed the next super block's barrier.
+    float *red = red_base + par * kColRedFloats;
+    par ^= 1;
 #pragma unroll
     for (int b = 0; b < kColBlocks; ++b) {
       if ((uint32_t)b < nrb) {
@@ -205,10 +213,10 @@ __device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, c
 #pragma unroll
         for (int n = 0; n < NT; ++n) {
           const uint32_t c0 = 2 * t + 8 * n;
-          r[c0 * 16 + g] = acc[b][n][0];
-          r[(c0 + 1) * 16 + g] = acc[b][n][1];
-          r[c0 * 16 + g + 8] = acc[b][n][2];
-          r[(c0 + 1) * 16 + g + 8] = acc[b][n][3];
+          r[c0 * 16 + g] = acc[b][0][n][0] + acc[b][1][n][0];
+          r[(c0 + 1) * 16 + g] = acc[b][0][n][1] + acc[b][1][n][1];
+          r[c0 * 16 + g + 8] = acc[b][0][n][2] + acc[b][1][n][2];
+          r[(c0 + 1) * 16 + g + 8] = acc[b][0][n][3] + acc[b][1][n][3];
         }
       }
     }
@@ -223,7 +231,6 @@ __device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, c
         md.y[(uint64_t)col * md.M + sb + row] = sum * col_scale<DT>(md.s, sb + row);
       }
     }
-    named_bar(1, kColConsumers);  // red is rewritten by the next super block
   }
 }
 
@@ -299,12 +306,12 @@ __global__ void __launch_bounds__(kColThreads, 1)
     __syncwarp();
   } else {
     // ---------------- consumers: 8 warps
-    uint32_t it = 0;
+    uint32_t it = 0, par = 0;
     for (uint32_t pi = p0; pi < p1; ++pi) {
       const Piece pc = pieces[pi];
       const MatDesc md = mats[pc.mat];
-      if (md.G > 8) cols_piece<DT, 2>(md, pc, R, red, it, warp, lane);
-      else cols_piece<DT, 1>(md, pc, R, red, it, warp, lane);
+      if (md.G > 8) cols_piece<DT, 2>(md, pc, R, red, it, par, warp, lane);
+      else cols_piece<DT, 1>(md, pc, R, red, it, par, warp, lane);
     }
   }
   __syncthreads();
