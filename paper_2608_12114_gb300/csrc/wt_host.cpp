@@ -36,6 +36,7 @@
 #include <cuda_runtime.h>
 
 #include "../../include/wt.h"
+#include "../../include/wt_dlpack.h"
 #include "wt_kernels.h"
 
 #ifndef MADV_POPULATE_READ
@@ -169,7 +170,6 @@ struct Tensor {
   int ndim = 0;
   uint64_t shape[kMaxDims] = {0, 0, 0, 0};
   uint64_t nbytes = 0;
-  uint32_t file = 0;
   uint64_t offset = 0;
 };
 
@@ -745,6 +745,22 @@ int validate_desc(const wt_gemv_desc &d, size_t i) {
   return WT_OK;
 }
 
+// Where W lives: 0 = device memory (cudaMalloc, a memory pool, managed): the TMA kernels
+// stream from there; 1 = host memory the device can load from (pinned or registered, or
+// pageable where the device reads through the host page tables); -1 = neither.
+int memory_class(const void *p, int device) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return -1;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return 0;
+  if (a.type == cudaMemoryTypeHost) return 1;
+  int ats = 0;
+  cudaDeviceGetAttribute(&ats, cudaDevAttrPageableMemoryAccessUsesHostPageTables, device);
+  return ats ? 1 : -1;
+}
+
 // The mapping holding [p, p + n) (whole range inside one file mapping), or nullptr.
 const File *mapping_of(const wt_handle *h, const void *p, uint64_t n) {
   const uintptr_t a = reinterpret_cast<uintptr_t>(p);
@@ -787,6 +803,13 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         qd.W = f->dev + off;
         if (fast && q.cols == 0) mapped_dt[q.dtype].push_back(make_mat(qd));
         else g.generic.push_back({q.dtype, static_cast<const uint8_t *>(qd.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
+                                  static_cast<const uint8_t *>(q.scale), ncol});
+      } else if (const int mc = memory_class(q.W, h->device); mc != 0) {
+        if (mc < 0) return set_err(WT_ENOTSUP, "wt_pass: W of desc %zu is host memory this device cannot read", k);
+        // host memory outside this handle (another mapping, a file-backed DLPack tensor, a
+        // pinned buffer): plain loads only, as for the map endpoint; TMA streams device memory
+        if (fast && q.cols == 0) mapped_dt[q.dtype].push_back(make_mat(q));
+        else g.generic.push_back({q.dtype, static_cast<const uint8_t *>(q.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
                                   static_cast<const uint8_t *>(q.scale), ncol});
       } else if (fast && q.cols > 0) {
         cols_dt[q.dtype].push_back(make_cols_mat(q));
@@ -1057,6 +1080,18 @@ int wt_num_tensors(const wt_handle *h, size_t *n) {
   if (!h || !n) return set_err(WT_EINVAL, "wt_num_tensors: NULL argument");
   *n = h->order.size();
   return WT_OK;
+}
+
+int wt_dlpack_tensor(const wt_handle *h, size_t i, unsigned flags, DLManagedTensorVersioned **out) {
+  if (!out) return set_err(WT_EINVAL, "wt_dlpack_tensor: out is NULL");
+  *out = nullptr;
+  if (!h) return set_err(WT_EINVAL, "wt_dlpack_tensor: NULL handle");
+  if (i >= h->order.size()) return set_err(WT_EINVAL, "wt_dlpack_tensor: tensor %zu out of range", i);
+  if (h->host_only && !(flags & WT_DLPACK_HOST))
+    return set_err(WT_EINVAL, "wt_dlpack_tensor: host-only handle: ask for WT_DLPACK_HOST");
+  const Tensor &t = h->tensor(i);
+  const File &f = h->files[h->order[i].first];
+  return wt::dlpack_map(f.path.c_str(), t.offset, t.nbytes, t.dtype, t.ndim, t.shape, flags, out);
 }
 
 int wt_num_files(const wt_handle *h, size_t *n) {

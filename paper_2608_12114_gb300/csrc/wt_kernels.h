@@ -127,3 +127,15 @@ int num_sms();  // of the current device (cached per device)
 int set_error(int code, const char *msg);
 
 }  // namespace wt
+
+struct DLManagedTensorVersioned;
+
+namespace wt {
+
+// The producer's core (wt_dlpack.cpp): maps bytes [off, off + nbytes) of `path` read-only and
+// shared (whole pages), exposes them per WT_DLPACK_* flags and returns a capsule of shape
+// shape[0..ndim) with compact strides.
+int dlpack_map(const char *path, uint64_t off, uint64_t nbytes, int32_t dtype, int ndim, const uint64_t *shape,
+               unsigned flags, DLManagedTensorVersioned **out);
+
+}  // namespace wt

@@ -30,7 +30,11 @@ MODE_NAMES = {WT_ADOPT_GATHER: "gather", WT_ADOPT_CE: "ce", WT_ADOPT_STAGED: "st
 SYMBOLS = ("wt_last_error", "wt_abi_version", "wt_open", "wt_num_tensors", "wt_num_files",
            "wt_tensor_info", "wt_find", "wt_file_route", "wt_adopt", "wt_pass", "wt_checksum",
            "wt_checksum_plain", "wt_checksum_noalloc", "wt_device_status", "wt_residency",
-           "wt_kernel_launches", "wt_close")
+           "wt_kernel_launches", "wt_close",
+           # include/wt_dlpack.h
+           "wt_dlpack_file", "wt_dlpack_tensor", "wt_dlpack_release", "wt_dlpack_live")
+WT_DLPACK_DEVICE, WT_DLPACK_HOST = 0, 1
+kDLCPU, kDLCUDA = 1, 2
 
 
 class WtError(RuntimeError):
@@ -86,9 +90,14 @@ def lib(path: str = LIB_PATH):
     L.wt_kernel_launches.argtypes = [vp, u64p]
     L.wt_residency.argtypes = [vp, u64p, u64p]
     L.wt_close.argtypes = [vp]
+    L.wt_dlpack_file.argtypes = [C.c_char_p, C.c_int32, C.c_uint64, C.c_uint64, C.c_uint, C.POINTER(vp)]
+    L.wt_dlpack_tensor.argtypes = [vp, sz, C.c_uint, C.POINTER(vp)]
+    L.wt_dlpack_release.argtypes = [vp]
+    L.wt_dlpack_live.argtypes = [C.POINTER(C.c_int64)]
     for s in SYMBOLS:
-        if s not in ("wt_last_error",):
+        if s not in ("wt_last_error", "wt_dlpack_release"):
             getattr(L, s).restype = C.c_int
+    L.wt_dlpack_release.restype = None
     L.wt_last_error.restype = C.c_char_p
     _lib = L
     return L
@@ -224,6 +233,141 @@ def gemv_desc(W: int, dtype: int, M: int, K: int, x: int, y: int, wait_event: in
     """One wt_gemv_desc; int8 weights (WT_I8) take fp16 x and `scale` = fp16 [M] row scales.
     cols = T in 1..16: x is X[T, K], y is Y[T, M] (the multi-column tensor-core kernel)."""
     return GemvDesc(W, dtype, cols, M, K, x, y, wait_event or None, scale or None)
+
+
+# ----------------------------------------------------------------------------- DLPack producer
+
+class DLDevice(C.Structure):
+    _fields_ = [("device_type", C.c_int32), ("device_id", C.c_int32)]
+
+
+class DLDataType(C.Structure):
+    _fields_ = [("code", C.c_uint8), ("bits", C.c_uint8), ("lanes", C.c_uint16)]
+
+
+class DLTensor(C.Structure):
+    _fields_ = [("data", C.c_void_p), ("device", DLDevice), ("ndim", C.c_int32), ("dtype", DLDataType),
+                ("shape", C.POINTER(C.c_int64)), ("strides", C.POINTER(C.c_int64)), ("byte_offset", C.c_uint64)]
+
+
+class DLPackVersion(C.Structure):
+    _fields_ = [("major", C.c_uint32), ("minor", C.c_uint32)]
+
+
+class DLManagedTensorVersioned(C.Structure):
+    _fields_ = [("version", DLPackVersion), ("manager_ctx", C.c_void_p), ("deleter", C.c_void_p),
+                ("flags", C.c_uint64), ("dl_tensor", DLTensor)]
+
+
+DLPACK_FLAG_BITMASK_READ_ONLY = 1
+_CAPSULE_NAME = b"dltensor_versioned"  # must outlive every capsule: module constant
+_capsule_new = C.pythonapi.PyCapsule_New
+_capsule_new.restype = C.py_object
+_capsule_new.argtypes = [C.c_void_p, C.c_char_p, C.c_void_p]
+_capsule_is_valid = C.pythonapi.PyCapsule_IsValid
+_capsule_is_valid.restype = C.c_int
+_capsule_is_valid.argtypes = [C.c_void_p, C.c_char_p]
+_capsule_get = C.pythonapi.PyCapsule_GetPointer
+_capsule_get.restype = C.c_void_p
+_capsule_get.argtypes = [C.c_void_p, C.c_char_p]
+
+
+@C.CFUNCTYPE(None, C.c_void_p)
+def _capsule_destructor(cap):
+    # A capsule nobody adopted still carries its original name: run the producer's deleter.
+    # A consumer renames the capsule it adopts and owns the deleter from then on.
+    try:
+        if _capsule_is_valid(cap, _CAPSULE_NAME):
+            lib().wt_dlpack_release(_capsule_get(cap, _CAPSULE_NAME))
+    except Exception:  # noqa: BLE001 - a destructor must not raise
+        pass
+
+
+class FileTensor:
+    """One producer result (Algorithm 1): a read-only, file-backed DLManagedTensorVersioned
+    awaiting adoption.  ``torch.from_dlpack(ft)`` makes a framework tensor over the file's
+    pages with no copy; its storage then owns the mapping.  An instance exports once; if
+    it is never exported, dropping it (or ``release()``) runs the deleter."""
+
+    def __init__(self, ptr: int):
+        self._p = ptr
+
+    @classmethod
+    def from_file(cls, path: str, dtype: int, M: int, K: int, flags: int = WT_DLPACK_DEVICE) -> "FileTensor":
+        out = C.c_void_p()
+        _check(lib().wt_dlpack_file(path.encode(), dtype, M, K, flags, C.byref(out)))
+        return cls(out.value)
+
+    @classmethod
+    def from_handle(cls, h: "Handle", i: int, flags: int = WT_DLPACK_DEVICE) -> "FileTensor":
+        out = C.c_void_p()
+        _check(lib().wt_dlpack_tensor(h.ptr, i, flags, C.byref(out)))
+        return cls(out.value)
+
+    def _managed(self) -> DLManagedTensorVersioned:
+        if self._p is None:
+            raise BufferError("this FileTensor was already exported or released")
+        return DLManagedTensorVersioned.from_address(self._p)
+
+    @property
+    def data_ptr(self) -> int:
+        return self._managed().dl_tensor.data or 0
+
+    @property
+    def shape(self) -> Tuple[int, ...]:
+        t = self._managed().dl_tensor
+        return tuple(t.shape[k] for k in range(t.ndim))
+
+    @property
+    def strides(self) -> Tuple[int, ...]:
+        t = self._managed().dl_tensor
+        return tuple(t.strides[k] for k in range(t.ndim))
+
+    @property
+    def flags(self) -> int:
+        return self._managed().flags
+
+    @property
+    def version(self) -> Tuple[int, int]:
+        v = self._managed().version
+        return (v.major, v.minor)
+
+    def __dlpack_device__(self) -> Tuple[int, int]:
+        d = self._managed().dl_tensor.device
+        return (d.device_type, d.device_id)
+
+    def __dlpack__(self, *, stream=None, max_version=None, dl_device=None, copy=None):
+        """A "dltensor_versioned" capsule (DLPack 1.0, read-only flag set).  The pages hold no
+        pending GPU work, so `stream` needs no synchronisation."""
+        if max_version is None or tuple(max_version)[0] < 1:
+            raise BufferError("the file-backed producer exports versioned (DLPack >= 1.0) capsules only")
+        if copy:
+            raise BufferError("the file-backed producer never copies")
+        if dl_device is not None and tuple(dl_device) != self.__dlpack_device__():
+            raise BufferError("the file-backed tensor lives on %s, not %s" % (self.__dlpack_device__(), tuple(dl_device)))
+        p = self._p
+        if p is None:
+            raise BufferError("this FileTensor was already exported or released")
+        cap = _capsule_new(p, _CAPSULE_NAME, C.cast(_capsule_destructor, C.c_void_p))
+        self._p = None
+        return cap
+
+    def release(self):
+        if self._p is not None:
+            lib().wt_dlpack_release(self._p)
+            self._p = None
+
+    def __del__(self):
+        try:
+            self.release()
+        except Exception:  # noqa: BLE001 - interpreter shutdown
+            pass
+
+
+def dlpack_live() -> int:
+    n = C.c_int64()
+    _check(lib().wt_dlpack_live(C.byref(n)))
+    return n.value
 
 
 def open(paths: Sequence[str], flags: int = 0) -> Handle:  # noqa: A001 - mirrors wt_open

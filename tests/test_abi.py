@@ -19,7 +19,9 @@ def L():
 
 
 def declared_symbols():
-    src = open(os.path.join(ROOT, "include", "wt.h")).read()
+    """Every wt_* function declared in include/*.h."""
+    inc = os.path.join(ROOT, "include")
+    src = "".join(open(os.path.join(inc, f)).read() for f in sorted(os.listdir(inc)) if f.endswith(".h"))
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
     return sorted(set(re.findall(r"\b(wt_[a-z_]+)\s*\(", src)))
 
