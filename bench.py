@@ -240,6 +240,15 @@ def pinned_h2d_gbs(torch, nbytes=1 << 30, reps=10):
     return nbytes / best / 1e6
 
 
+def kernel_source_digest():
+    """First 16 hex digits of the SHA-256 over the GEMV kernel's sources (kernel file, shared
+    device helpers, tile geometry header): a captured traffic figure is valid only for them."""
+    h = hashlib.sha256()
+    for f in ("wt_kernels.cu", "wt_device.cuh", "wt_kernels.h"):
+        h.update(open(os.path.join(ROOT, "paper_2608_12114_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
 def kernel_traffic(name):
     """DRAM bytes per launch from the committed ncu summary, if it matches the current kernels."""
     p = os.path.join(ROOT, "profiles", name)
@@ -249,8 +258,7 @@ def kernel_traffic(name):
         d = json.load(open(p))
     except Exception:
         return None
-    src = os.path.join(ROOT, "paper_2608_12114_gb300", "csrc", "wt_kernels.cu")
-    digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    digest = kernel_source_digest()
     if d.get("kernel_source_sha256_16") != digest:
         return None
     return d
