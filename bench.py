@@ -60,6 +60,8 @@ def parse_args():
     p.add_argument("--e2e-reps", type=int, default=5)
     p.add_argument("--skip-e2e", action="store_true", help="resident passes only (profiling runs)")
     p.add_argument("--arms", action="store_true", help="also time the ce/staged/stock-torch ingest arms")
+    p.add_argument("--cold-reps", type=int, default=0,
+                   help="also time N file -> first-use runs with the files evicted from the page cache")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="CPU budget of the oracle sample")
     p.add_argument("--data-dir", default=None)
@@ -284,22 +286,51 @@ def aggregate_gbs(bytes_per_rank, world, seconds):
 
 # ----------------------------------------------------------------------------- the wt arm
 
-def first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab):
-    """One file -> first-use run; returns (seconds, handle stats)."""
+def first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, phases=None):
+    """One file -> first-use run; returns (seconds, handle stats).  With `phases` (a dict),
+    also records host-side phase times in ms: open (wt_open: parse, map, route), enqueue
+    (wt_adopt + wt_pass return; includes page-table population), drain (until y is on the
+    host), and the route of the first file."""
     t0 = time.perf_counter()
     h = wt.Handle(ck.paths)
     mats = pipeline.matrices(h)
+    t1 = time.perf_counter()
     dev = slab["dev"]
     ev = dev.adopt(h, mode, ingest_s.cuda_stream)
     h.pass_(dev.descs(slab["xs"], slab["ys"], ev), consume_s.cuda_stream)
     with torch.cuda.stream(consume_s):
         y_host.copy_(slab["yflat"], non_blocking=True)
+    t2 = time.perf_counter()
     consume_s.synchronize()
     dt = time.perf_counter() - t0
+    if phases is not None:
+        phases.setdefault("open_ms", []).append((t1 - t0) * 1e3)
+        phases.setdefault("enqueue_ms", []).append((t2 - t1) * 1e3)
+        phases.setdefault("drain_ms", []).append((t0 + dt - t2) * 1e3)
+        phases["route"] = wt.ROUTE_NAMES.get(h.route(0), "?") if h.n_files else None
     launches = h.kernel_launches()
     status = h.device_status()
     h.close()
     return dt, launches, status, len(mats)
+
+
+def evict_page_cache(paths):
+    """Drop the files' pages from the page cache (posix_fadvise DONTNEED on each file only)."""
+    for p in paths:
+        fd = os.open(p, os.O_RDONLY)
+        try:
+            os.fdatasync(fd)
+            os.posix_fadvise(fd, 0, 0, os.POSIX_FADV_DONTNEED)
+        finally:
+            os.close(fd)
+
+
+def quartiles(v):
+    """(q1, q3) of a sample (inclusive method; the sample itself when shorter than 2)."""
+    if len(v) < 2:
+        return (v[0], v[0]) if v else (float("nan"), float("nan"))
+    q = statistics.quantiles(v, n=4, method="inclusive")
+    return q[0], q[2]
 
 
 def run_wt(args, rank, world):
@@ -349,11 +380,12 @@ def run_wt(args, rank, world):
     ingest_s, consume_s = torch.cuda.Stream(), torch.cuda.Stream()
 
     # ---------------- e2e: file -> first use (1 warm-up, then timed repetitions)
-    e2e_times, e2e_launches = [], 0
+    e2e_times, e2e_launches, phases = [], 0, {}
     for rep in range(0 if args.skip_e2e else 1 + args.e2e_reps):
         if dist:
             dist.barrier()
-        dt, nl, st, nm = first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab)
+        dt, nl, st, nm = first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab,
+                                   phases if rep > 0 else None)
         if st != 0:
             raise SystemExit("device status %d after first-use run" % st)
         if rep > 0:
@@ -364,13 +396,32 @@ def run_wt(args, rank, world):
     log("file->first-use: %.1f ms median (%s), %.1f GB/s = %.1f%% of pinned H2D" % (
         e2e_s * 1e3, ", ".join("%.1f" % (t * 1e3) for t in e2e_times), e2e_gbs, 100 * e2e_gbs / h2d))
 
+    cold = None
+    if args.cold_reps and not args.skip_e2e:
+        # storage-bound variant (the precondition of Algorithm 2 fails): the files' pages are
+        # evicted before each run; reported apart from the warm-cache headline
+        ct = []
+        for _ in range(args.cold_reps):
+            evict_page_cache(ck.paths)
+            ct.append(first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab)[0])
+        cold = {"value": round(aggregate_gbs(data_bytes, world, statistics.median(ct)), 1), "unit": "GB/s",
+                "ms": [round(t * 1e3, 1) for t in ct],
+                "what": "file -> first use after posix_fadvise(DONTNEED) on the checkpoint files: storage-bound"}
+        log("cold file->first-use: %s ms" % cold["ms"])
+
     arms = {}
     if args.arms:
-        for name, m in (("gather", wt.WT_ADOPT_GATHER), ("ce", wt.WT_ADOPT_CE), ("staged", wt.WT_ADOPT_STAGED)):
-            ts = [first_use(torch, wt, pipeline, ck, m, ingest_s, consume_s, y_host, slab)[0] for _ in range(3)]
-            arms[name] = round(data_bytes / min(ts) / 1e9, 1)
-        arms["stock_torch"] = round(stock_torch_arm(torch, ck, wt, pipeline) / 1e9, 1)
-        log("ingest arms GB/s:", arms)
+        # the mode order rotates across repetitions so no arm always runs first
+        names = [("gather", wt.WT_ADOPT_GATHER), ("ce", wt.WT_ADOPT_CE), ("staged", wt.WT_ADOPT_STAGED), ("stock_torch", None)]
+        ts = {n: [] for n, _ in names}
+        for r in range(3):
+            for n, m in names[r:] + names[:r]:
+                if m is None:
+                    ts[n].append(data_bytes / stock_torch_arm(torch, ck, wt, pipeline))
+                else:
+                    ts[n].append(first_use(torch, wt, pipeline, ck, m, ingest_s, consume_s, y_host, slab)[0])
+        arms = {n: round(data_bytes / statistics.median(v) / 1e9, 1) for n, v in ts.items()}
+        log("ingest arms GB/s (median of 3, rotated order):", arms)
 
     # ---------------- resident pass: the steady-state consumer
     h = wt.Handle(ck.paths)
@@ -435,12 +486,17 @@ def run_wt(args, rank, world):
                 "ms": round(e2e_s * 1e3, 2), "pinned_h2d_gbs": round(h2d, 1),
                 "frac_of_pinned_h2d": round(e2e_gbs / h2d, 4), "reps": args.e2e_reps,
                 "what": "wt_open + wt_adopt + event-gated first pass + D2H of all y, page cache warm",
-                "launches_per_run": e2e_launches},
+                "launches_per_run": e2e_launches,
+                "iqr_ms": [round(v * 1e3, 2) for v in quartiles(e2e_times)] if e2e_times else None,
+                "phases_ms_median": {k: round(statistics.median(v), 2) for k, v in phases.items() if k.endswith("_ms")},
+                "route": phases.get("route")},
         "gpu_launches": int(launches),
         "roofline": roof,
     }
     if arms:
         out["ingest_arms_gbs"] = arms
+    if cold:
+        out["e2e_cold"] = cold
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(args, ck, args.cpu_seconds)
     if rank == 0:

@@ -161,3 +161,52 @@ def test_cols_map_endpoint_reads_in_place(torch, tmp_path):
             Yhat, A = oracle.gemv_cols(co.blob_of(t.file, t.name), 3, M, K, X.view(np.uint8), T, scale=s)
             assert oracle.gemv_error(Y.cpu().numpy().astype(np.float64), Yhat.reshape(-1), A.reshape(-1)) <= TOL
         assert h.device_status() == 0
+
+
+def test_cols_mixed_column_counts_and_dtypes_in_one_pass(torch):
+    """One wt_pass whose matrices ask for different T (one- and two-tile MMA paths in the same
+    launch) and different dtypes (separate launches of one group)."""
+    rng = np.random.default_rng(9)
+    spec = [(I8, 40, 1536, 3), (I8, 70, 4096, 12), (BF16, 33, 2048, 16), (I8, 17, 7168, 1), (BF16, 50, 768, 9),
+            (F16, 20, 512, 8)]
+    cases = [make(torch, rng, d, M, K, T) for d, M, K, T in spec]
+    with wt.Handle([]) as h:
+        h.pass_([desc(c) for c in cases], 0)
+        torch.cuda.synchronize()
+        assert h.device_status() == 0
+    for c in cases:
+        check(c, c["Y"])
+
+
+def test_cols_full_size_matched_protocol(torch, tmp_path):
+    """The T-sweep's launch configuration at full size: 12 matrices of 12288 x 7168 int8 with
+    fp16 row scales in one pass, T = 8 and 16; first, last and 16 seeded rows per matrix."""
+    from paper_2608_12114_gb300 import pipeline
+    ck = synth.build("protocol_q8", str(tmp_path), workers=16)
+    co = oracle.CheckpointOracle(ck.paths)
+    try:
+        with wt.Handle(ck.paths) as h:
+            dev = pipeline.DeviceCheckpoint.allocate(h, pipeline.matrices(h))
+            torch.cuda.synchronize()
+            dev.adopt(h, wt.WT_ADOPT_GATHER, 0)
+            torch.cuda.synchronize()
+            ks = dev.gemv_mats()
+            for T in (8, 16):
+                X = np.random.default_rng(T).standard_normal((T, 7168)).astype(np.float16)
+                Xd = torch.from_numpy(X.view(np.uint8).reshape(-1).copy()).cuda()
+                ys = {k: torch.full((T * 12288,), float("nan"), dtype=torch.float32, device="cuda") for k in ks}
+                d = dev.descs({(7168, wt.WT_I8): Xd}, ys)
+                d["cols"] = T
+                h.pass_(d, 0)
+                torch.cuda.synchronize()
+                assert h.device_status() == 0
+                for k in ks:
+                    m = dev.mats[k]
+                    t, sc = h.tensors[m.parts[0]], h.tensors[m.scale]
+                    r = sorted({0, 12287} | {int(v) for v in np.random.default_rng(k).integers(0, 12288, 16)})
+                    Yhat, A = oracle.gemv_cols(co.blob_of(t.file, t.name), 3, 12288, 7168, X.view(np.uint8), T,
+                                               scale=co.blob_of(sc.file, sc.name), rows=r)
+                    got = ys[k].cpu().numpy().reshape(T, 12288)[:, r]
+                    assert oracle.gemv_error(got.reshape(-1), Yhat.reshape(-1), A.reshape(-1)) <= TOL, (T, m.name)
+    finally:
+        co.close()
