@@ -60,6 +60,8 @@ def parse_args():
     p.add_argument("--e2e-reps", type=int, default=5)
     p.add_argument("--skip-e2e", action="store_true", help="resident passes only (profiling runs)")
     p.add_argument("--arms", action="store_true", help="also time the ce/staged/stock-torch ingest arms")
+    p.add_argument("--graph", action="store_true",
+                   help="time the resident pass as replays of one captured CUDA graph")
     p.add_argument("--cold-reps", type=int, default=0,
                    help="also time N file -> first-use runs with the files evicted from the page cache")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -97,6 +99,7 @@ def workload_ck(args, outdir):
 
 
 DT_NAME = {0: "f32", 1: "bf16", 2: "f16", 3: "int8"}
+L2_BYTES = 129 * 10 ** 6  # GB300 L2
 DATA_DESC = {
     "bf16": "synthetic (seeded N(0,0.02) bf16 weights, norms 1.0, x ~ N(0,1))",
     "int8": "synthetic (seeded uniform int8 weights in [-127, 127], fp16 row scales, fp16 x ~ N(0,1))",
@@ -432,6 +435,18 @@ def run_wt(args, rank, world):
     for _ in range(args.warmup):
         h.pass_(descs, s.cuda_stream)
     s.synchronize()
+    graph, graph_launches = None, 0
+    if args.graph:
+        # one resident pass captured into a CUDA graph; each step replays it (no host work)
+        n_cap = h.kernel_launches()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=s):
+            h.pass_(descs, torch.cuda.current_stream().cuda_stream)
+        graph_launches = h.kernel_launches() - n_cap
+        with torch.cuda.stream(s):
+            for _ in range(args.warmup):
+                graph.replay()
+        s.synchronize()
     n0 = h.kernel_launches()
     evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
     if dist:
@@ -439,14 +454,20 @@ def run_wt(args, rank, world):
     torch.cuda.synchronize()
     with Clocks(bus_id()) as clk:
         evs[0].record(s)
-        for i in range(args.steps):
-            h.pass_(descs, s.cuda_stream)
-            evs[i + 1].record(s)
+        if graph is not None:
+            with torch.cuda.stream(s):
+                for i in range(args.steps):
+                    graph.replay()
+                    evs[i + 1].record(s)
+        else:
+            for i in range(args.steps):
+                h.pass_(descs, s.cuda_stream)
+                evs[i + 1].record(s)
         s.synchronize()
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
-    launches = h.kernel_launches() - n0
+    launches = h.kernel_launches() - n0 + graph_launches * args.steps
     per = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
     total_ms = evs[0].elapsed_time(evs[-1])
     status = h.device_status()
@@ -478,7 +499,10 @@ def run_wt(args, rank, world):
         "data": DATA_DESC.get(wdt, "synthetic"),
         "config": {"workload": workload_desc(args), "weight_bytes": weight_bytes, "data_bytes": data_bytes,
                    "files": len(ck.paths), "matrices": len(dev.gemv_mats()), "ingest_mode": args.mode,
-                   "l2": "inputs larger than L2 (no flush)", "parallelism": "replicas" if world > 1 else "1 GPU"},
+                   "l2": ("inputs larger than L2 (no flush)" if weight_bytes > L2_BYTES else
+                          "inputs smaller than L2, no flush: passes may hit L2 (a dispatch-overhead point)"),
+                   "parallelism": "replicas" if world > 1 else "1 GPU",
+                   "cuda_graph": bool(args.graph)},
         "resident_frac_of_hbm": {"measured": round(value / world / peak, 4), "nominal_8TBps": round(value / world / NOMINAL_HBM_GBS, 4)},
         "clocks": clocks,
         "e2e": {"value": round(aggregate_gbs(data_bytes, world, e2e_s_max), 1), "unit": "GB/s",

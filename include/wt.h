@@ -183,8 +183,17 @@ int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsign
  * every matrix of the group, rows split evenly across the SMs.  Repeated
  * calls with identical descriptors reuse a cached launch plan.  The result of
  * a row does not depend on how rows were grouped or split (deterministic, no
- * floating-point atomics).  Errors: WT_EINVAL (null pointer with M*K > 0,
- * cols outside 0..16, dimension > 2^31-1), WT_ENOTSUP (dtype), WT_ENOMEM, WT_ECUDA. */
+ * floating-point atomics).
+ *
+ * Stream capture: a wt_pass issued on a stream that is being captured into a CUDA graph
+ * records the pass's launches into the graph (replays then cost no host work).  The same
+ * descriptors must have run through wt_pass once before, outside the capture, and that
+ * stream must have been synchronised since (the plan's tables must be in device memory);
+ * otherwise the call returns WT_EINVAL before issuing any CUDA call.  The captured plan is
+ * kept until wt_close; every replay must complete before wt_close.
+ *
+ * Errors: WT_EINVAL (null pointer with M*K > 0, cols outside 0..16, dimension > 2^31-1, a
+ * capture without the warm-up call), WT_ENOTSUP (dtype), WT_ENOMEM, WT_ECUDA. */
 int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream);
 
 /* Leaf-tree FNV-1a-64 digest of each device buffer ptr[i] (nbytes[i] bytes),

@@ -220,6 +220,7 @@ struct Plan {
   cudaEvent_t last = nullptr;
   bool sent = false;
   cudaStream_t sent_on = nullptr;
+  bool pinned = false;  // used inside a captured CUDA graph: kept until wt_close
   uint64_t launches = 0;
 };
 
@@ -864,8 +865,28 @@ void destroy_plan(Plan *P) {
   delete P;
 }
 
-int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s) {
-  if (!P->sent) {
+// True if the tables of P are in device memory: the stream-ordered upload of its first use
+// has completed.  Queried in relaxed capture mode, so it is legal while a graph is captured.
+bool plan_resident(const Plan *P) {
+  if (!P->sent) return false;
+  cudaStreamCaptureMode m = cudaStreamCaptureModeRelaxed;
+  cudaThreadExchangeStreamCaptureMode(&m);
+  const cudaError_t q = cudaEventQuery(P->uploaded);
+  cudaThreadExchangeStreamCaptureMode(&m);
+  if (q != cudaSuccess && q != cudaErrorNotReady) cudaGetLastError();
+  return q == cudaSuccess;
+}
+
+int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool capturing = false) {
+  if (capturing) {
+    // Inside a stream capture the graph replays later, on its own schedule: the tables must
+    // already be resident, and nothing here may depend on events outside the capture.
+    if (!plan_resident(P))
+      return set_err(WT_EINVAL,
+                     "wt_pass: capturing a pass needs the same descriptors run once outside the capture, "
+                     "with that stream synchronised, before the capture begins");
+    P->pinned = true;
+  } else if (!P->sent) {
     CU(cudaMemcpyAsync(P->dev, P->host, std::max<size_t>(16, align16(P->table.size())), cudaMemcpyHostToDevice, s));
     CU(cudaEventRecord(P->uploaded, s));
     P->sent = true;
@@ -916,7 +937,7 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s) {
       h->kernel_launches++;
     }
   }
-  CU(cudaEventRecord(P->last, s));
+  if (!capturing) CU(cudaEventRecord(P->last, s));
   return WT_OK;
 }
 
@@ -1177,6 +1198,12 @@ int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream) {
     if (d[i].M && inside_mapping(h, d[i].y, d[i].M * std::max<int32_t>(1, d[i].cols) * sizeof(float)))
       return set_err(WT_EINVAL, "wt_pass: y of desc %zu lies inside a read-only mapping", i);
   }
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(static_cast<cudaStream_t>(stream), &cs) != cudaSuccess) {
+    cudaGetLastError();
+    cs = cudaStreamCaptureStatusNone;
+  }
+  const bool capturing = cs == cudaStreamCaptureStatusActive;
   std::lock_guard<std::mutex> g(h->mu);
   try {
     // Plans are keyed by the descriptors with each wait_event replaced by its group's
@@ -1197,6 +1224,10 @@ int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream) {
         h->plans.push_front(P);
         break;
       }
+    if (!P && capturing)  // building a plan allocates: not allowed inside a capture
+      return set_err(WT_EINVAL,
+                     "wt_pass: capturing a pass needs the same descriptors run once outside the capture, "
+                     "with that stream synchronised, before the capture begins");
     if (!P) {
       P = new Plan();
       P->key = std::move(key);
@@ -1206,12 +1237,17 @@ int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream) {
         return rc;
       }
       h->plans.push_front(P);
-      while (h->plans.size() > 32) {
-        destroy_plan(h->plans.back());
-        h->plans.pop_back();
+      // least recently used plans beyond 32 go, except those a captured graph refers to
+      size_t live = h->plans.size();
+      for (auto it = std::prev(h->plans.end()); live > 32 && it != h->plans.begin();) {
+        auto cur = it--;
+        if ((*cur)->pinned) continue;
+        destroy_plan(*cur);
+        h->plans.erase(cur);
+        --live;
       }
     }
-    return run_plan(h, P, d, static_cast<cudaStream_t>(stream));
+    return run_plan(h, P, d, static_cast<cudaStream_t>(stream), capturing);
   } catch (const std::bad_alloc &) {
     return set_err(WT_ENOMEM, "wt_pass: out of host memory");
   }
