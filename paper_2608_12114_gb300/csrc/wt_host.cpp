@@ -209,6 +209,9 @@ struct Plan {
     std::vector<Launch> launches;
     std::vector<Launch> mapped;  // W read in place from a file mapping (map endpoint)
     std::vector<Launch> cols;    // multi-column kernel (tensor cores)
+    size_t reduce = 0;           // SegReduce table of this group's column-segmented matrices
+    int n_reduce = 0;
+    uint32_t reduce_rows = 0;
     std::vector<Generic> generic;
     std::vector<Zero> zero;
   };
@@ -221,6 +224,9 @@ struct Plan {
   bool sent = false;
   cudaStream_t sent_on = nullptr;
   bool pinned = false;  // used inside a captured CUDA graph: kept until wt_close
+  float *ws = nullptr;  // split-K segment partials (device), ws_floats floats
+  size_t ws_floats = 0;
+  std::vector<std::pair<size_t, size_t>> ws_patches;  // (table byte offset of a pointer, ws float offset)
   uint64_t launches = 0;
 };
 
@@ -601,6 +607,7 @@ wt::MatDesc make_mat(const wt_gemv_desc &d) {
   m.s = static_cast<const uint8_t *>(d.scale);
   m.M = (uint32_t)d.M;
   m.V = (uint32_t)(d.K * es / 16);
+  m.rs = m.V;
   const uint32_t rowb = m.V * 16;
   // a consumer thread keeps at most 8 (bf16/f16/f32) or 4 (int8: 16 f16 activations per
   // weight vector) x vectors in registers; the mode limits follow from that
@@ -634,11 +641,41 @@ wt::MatDesc make_cols_mat(const wt_gemv_desc &d) {
   m.s = static_cast<const uint8_t *>(d.scale);
   m.M = (uint32_t)d.M;
   m.V = (uint32_t)(d.K * elem_bytes(d.dtype) / 16);
+  m.rs = m.V;
   m.mode = wt::kModeCols;
   m.G = (uint16_t)d.cols;
   m.rt = 16;
   const uint32_t nchunk = (m.V + wt::kColVecMax - 1) / wt::kColVecMax;
   m.vc = ((m.V + nchunk - 1) / nchunk + 3) / 8 * 8 + 4;
+  return m;
+}
+
+// Segment length for rows of V vectors: ceil(V / seg_vectors) segments of nearly equal
+// length (a multiple of 8 vectors), so no segment is a sliver.  Depends on (V, dtype) only.
+uint32_t seg_length(uint32_t V, int dtype) {
+  const uint32_t S = wt::seg_vectors(dtype);
+  const uint32_t nseg = (V + S - 1) / S;
+  return ((V + nseg - 1) / nseg + 7) / 8 * 8;
+}
+
+// Column segment k of a matrix whose rows exceed seg_vectors(dtype): vectors
+// [k S, min((k + 1) S, V)) of every row, S = seg_length (row pitch: the full row), x
+// advanced to match, no scale, tile mode chosen by the segment's own length, y left for the
+// workspace patch.
+wt::MatDesc make_seg_mat(const wt_gemv_desc &d, uint32_t k) {
+  const int es = elem_bytes(d.dtype);
+  const uint32_t V = (uint32_t)(d.K * es / 16);
+  const uint32_t S = seg_length(V, d.dtype);
+  const uint64_t xvb = d.dtype == WT_I8 ? 32 : 16;  // x bytes per 16-byte weight vector
+  const uint32_t v0 = k * S;
+  wt_gemv_desc sd = d;
+  sd.W = static_cast<const uint8_t *>(d.W) + (uint64_t)v0 * 16;
+  sd.x = static_cast<const uint8_t *>(d.x) + (uint64_t)v0 * xvb;
+  sd.K = (uint64_t)std::min(S, V - v0) * 16 / es;
+  sd.scale = nullptr;
+  wt::MatDesc m = make_mat(sd);
+  m.s = nullptr;
+  m.rs = V;
   return m;
 }
 
@@ -780,6 +817,9 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
     Plan::Group g;
     g.first = i;
     std::vector<wt::MatDesc> by_dt[4], mapped_dt[4], cols_dt[4];
+    std::vector<int64_t> seg_ws[4];  // per by_dt entry: workspace float offset of its partials, or -1
+    std::vector<wt::SegReduce> reds;
+    std::vector<size_t> red_ws;      // per reds entry: workspace float offset
     for (size_t k = i; k < j; ++k) {
       const wt_gemv_desc &q = d[k];
       if (q.M == 0) continue;
@@ -814,8 +854,29 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
                                   static_cast<const uint8_t *>(q.scale), ncol});
       } else if (fast && q.cols > 0) {
         cols_dt[q.dtype].push_back(make_cols_mat(q));
+      } else if (fast && q.K * es / 16 > wt::seg_vectors(q.dtype)) {
+        // long rows: column segments spread over CTAs, summed by the second pass
+        const uint32_t V = (uint32_t)(q.K * es / 16);
+        const uint32_t S = seg_length(V, q.dtype);
+        const uint32_t nseg = (V + S - 1) / S;
+        const size_t off = P->ws_floats;
+        P->ws_floats += (size_t)nseg * q.M;
+        for (uint32_t k = 0; k < nseg; ++k) {
+          by_dt[q.dtype].push_back(make_seg_mat(q, k));
+          seg_ws[q.dtype].push_back((int64_t)(off + (size_t)k * q.M));
+        }
+        wt::SegReduce r;
+        memset(&r, 0, sizeof r);
+        r.y = q.y;
+        r.s = static_cast<const uint8_t *>(q.scale);
+        r.M = (uint32_t)q.M;
+        r.nseg = nseg;
+        reds.push_back(r);
+        red_ws.push_back(off);
+        g.reduce_rows = std::max(g.reduce_rows, (uint32_t)q.M);
       } else if (fast) {
         by_dt[q.dtype].push_back(make_mat(q));
+        seg_ws[q.dtype].push_back(-1);
       } else {
         g.generic.push_back({q.dtype, static_cast<const uint8_t *>(q.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
                              static_cast<const uint8_t *>(q.scale), ncol});
@@ -831,6 +892,10 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         std::vector<uint32_t> begin;
         partition(ms, L.grid, pieces, begin, pass == 2 ? (uint32_t)wt::kColTileRows : 1u);
         L.mats = append(P->table, ms);
+        if (pass == 0)
+          for (size_t k = 0; k < ms.size(); ++k)
+            if (seg_ws[dt][k] >= 0)
+              P->ws_patches.push_back({L.mats + k * sizeof(wt::MatDesc) + offsetof(wt::MatDesc, y), (size_t)seg_ws[dt][k]});
         L.pieces = append(P->table, pieces);
         L.begin = append(P->table, begin);
         if (pass == 2) {
@@ -844,8 +909,21 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         (pass == 0 ? g.launches : pass == 1 ? g.mapped : g.cols).push_back(L);
       }
     }
+    if (!reds.empty()) {
+      g.reduce = append(P->table, reds);
+      g.n_reduce = (int)reds.size();
+      for (size_t k = 0; k < reds.size(); ++k)
+        P->ws_patches.push_back({g.reduce + k * sizeof(wt::SegReduce) + offsetof(wt::SegReduce, ws), red_ws[k]});
+    }
     P->groups.push_back(std::move(g));
     i = j;
+  }
+  if (P->ws_floats) {
+    CU(cudaMalloc(reinterpret_cast<void **>(&P->ws), P->ws_floats * sizeof(float)));
+    for (const auto &pt : P->ws_patches) {
+      const float *p = P->ws + pt.second;
+      memcpy(P->table.data() + pt.first, &p, sizeof p);
+    }
   }
   const size_t bytes = std::max<size_t>(16, align16(P->table.size()));
   CU(cudaHostAlloc(reinterpret_cast<void **>(&P->host), bytes, cudaHostAllocDefault));
@@ -859,6 +937,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
 void destroy_plan(Plan *P) {
   if (P->last) cudaEventSynchronize(P->last);
   if (P->dev) cudaFree(P->dev);
+  if (P->ws) cudaFree(P->ws);
   if (P->host) cudaFreeHost(P->host);
   if (P->uploaded) cudaEventDestroy(P->uploaded);
   if (P->last) cudaEventDestroy(P->last);
@@ -907,6 +986,10 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
       gl.begin = reinterpret_cast<const uint32_t *>(P->dev + L.begin);
       gl.status = h->status;
       CU(wt::launch_gemv(gl, s));
+      h->kernel_launches++;
+    }
+    if (g.n_reduce) {
+      CU(wt::launch_seg_reduce(reinterpret_cast<const wt::SegReduce *>(P->dev + g.reduce), g.n_reduce, g.reduce_rows, s));
       h->kernel_launches++;
     }
     for (const Plan::Launch &L : g.mapped) {

@@ -106,7 +106,7 @@ struct XJ {
 // Row scale applied at the store: f16 per row for int8 weights, 1 otherwise.
 template <int DT>
 __device__ __forceinline__ float row_scale(const uint8_t *s, uint64_t row) {
-  if constexpr (DT == 3) return __half2float(reinterpret_cast<const __half *>(s)[row]);
+  if constexpr (DT == 3) return s ? __half2float(reinterpret_cast<const __half *>(s)[row]) : 1.f;
   return 1.f;
 }
 
@@ -477,7 +477,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
       for (uint32_t pi = p0; pi < p1 && live; ++pi) {
         const Piece pc = pieces[pi];
         const MatDesc md = mats[pc.mat];
-        const uint64_t rowb = (uint64_t)md.V * 16;
+        const uint64_t rowb = (uint64_t)md.rs * 16;  // row pitch (== V * 16 outside split-K segments)
         const uint32_t rt = piece_rows_per_tile(md, pc);
         for (uint32_t r = pc.r0; r < pc.r1 && live; r += rt) {
           const uint32_t nr = min(rt, pc.r1 - r);
@@ -492,9 +492,13 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
             const uint32_t dst = stage0 + s * kStageBytes;
             const uint32_t bar = full0 + 8 * s;
             if (md.mode != kModeSplitK) {
-              const uint32_t bytes = nr * (uint32_t)rowb;
-              mbar_expect_tx(bar, bytes);
-              bulk_g2s(dst, md.W + (uint64_t)r * rowb, bytes, bar, pol);
+              const uint32_t vb = md.V * 16;  // tile rows sit at V * 16 pitch in shared memory
+              mbar_expect_tx(bar, nr * vb);
+              if (md.rs == md.V) {
+                bulk_g2s(dst, md.W + (uint64_t)r * rowb, nr * vb, bar, pol);
+              } else {
+                for (uint32_t q = 0; q < nr; ++q) bulk_g2s(dst + q * vb, md.W + (uint64_t)(r + q) * rowb, vb, bar, pol);
+              }
             } else {
               const uint32_t v0 = c * md.vc;
               const uint32_t nv = min(md.vc, md.V - v0);
@@ -712,6 +716,16 @@ __global__ void gemv_generic_kernel(const uint8_t *W, const uint8_t *x, float *y
   }
 }
 
+// Second pass of cross-CTA split-K: one thread per output row, segments summed in order.
+__global__ void seg_reduce_kernel(const SegReduce *__restrict__ tab) {
+  const SegReduce r = tab[blockIdx.y];
+  const uint32_t row = blockIdx.x * blockDim.x + threadIdx.x;
+  if (row >= r.M) return;
+  float sum = 0.f;
+  for (uint32_t k = 0; k < r.nseg; ++k) sum += r.ws[(uint64_t)k * r.M + row];
+  r.y[row] = r.s ? sum * __half2float(reinterpret_cast<const __half *>(r.s)[row]) : sum;
+}
+
 // ------------------------------------------------------------------ FNV-1a-64
 constexpr uint64_t kFnvOffset = 0xcbf29ce484222325ull;
 constexpr uint64_t kFnvPrime = 0x00000100000001b3ull;
@@ -900,6 +914,13 @@ cudaError_t launch_gemv_generic(int dtype, const uint8_t *W, const uint8_t *x, f
     case 3: gemv_generic_kernel<3><<<grid, 256, 0, s>>>(W, x, y, M, K, sc, cols); break;
     default: return cudaErrorInvalidValue;
   }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_seg_reduce(const SegReduce *tab, int n, uint32_t max_rows, cudaStream_t s) {
+  if (n == 0 || max_rows == 0) return cudaSuccess;
+  const dim3 grid((max_rows + 255) / 256, (unsigned)n);
+  seg_reduce_kernel<<<grid, 256, 0, s>>>(tab);
   return cudaGetLastError();
 }
 

@@ -58,8 +58,31 @@ struct alignas(16) MatDesc {
   uint32_t vc;    // vectors per column chunk (mode 2); V otherwise
   uint16_t mode;  // GemvMode
   uint16_t G;     // mode 0: lanes per row (power of two <= 32); kModeCols: columns T
-  uint32_t pad;
+  uint32_t rs;    // row pitch in 16-byte vectors: V, or the full row of a column segment
+                  // (segments are split-K only); s == nullptr then means "no scale yet"
 };
+
+// Cross-CTA split-K: rows longer than seg_vectors(dtype) are cut into column segments of
+// that many vectors (the last one shorter).  Each segment is a matrix of its own (row pitch
+// the full row; tile mode by its own length: a full segment is one 32 KB or 16 KB row per
+// stage, whole-CTA "block rows") writing partial sums to a workspace; a second pass sums the
+// segments of each row in segment order and applies the row scale.  Segment boundaries
+// depend only on the matrix, so a row's result never depends on how rows and segments were
+// spread over CTAs.
+constexpr uint32_t kSegVec = 2048;  // bf16 / f16 / f32: 32 KB per segment row
+constexpr uint32_t seg_vectors(int dtype) { return dtype == 3 ? kSegVec / 2 : kSegVec; }
+
+struct alignas(16) SegReduce {
+  const float *ws;   // nseg x M partial sums (segment-major)
+  float *y;          // M outputs
+  const uint8_t *s;  // f16 row scales (int8 weights) or null
+  uint32_t M;
+  uint32_t nseg;
+};
+
+// y[row] = (sum over segments of ws[seg * M + row], in segment order) * scale[row], for
+// every SegReduce of the table.
+cudaError_t launch_seg_reduce(const SegReduce *tab, int n, uint32_t max_rows, cudaStream_t s);
 
 struct alignas(16) Piece {
   uint32_t mat;  // index into the launch's MatDesc table
