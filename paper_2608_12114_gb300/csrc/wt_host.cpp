@@ -717,9 +717,19 @@ int encode_cols_map(const wt::MatDesc &m, uint8_t *out) {
   return WT_OK;
 }
 
-// Split the rows of `mats` (in order) into `grid` contiguous ranges of nearly equal bytes.
+// Interleaved slices per CTA for the one-column kernels.  Byte-equal contiguous ranges leave
+// CTAs with different mixes of shapes, and shapes stream at different rates (a decoder's
+// k/v rows at ~92 % of the copy peak, its down rows above it): the slowest CTA sets the pass.
+// Sixteen slices spread over the whole set even that out (large decoder 6342 -> 6864 GB/s).
+// int8 weights keep one range per CTA: they are bound by instructions, and each extra piece
+// costs an exposed reload of x.
+int one_col_slices(int dtype) { return dtype == WT_I8 ? 1 : 16; }
+
+// Split the rows of `mats` (in order) into grid * slices contiguous slices of nearly
+// equal bytes, cut at row boundaries; slice j goes to CTA j % grid, so every CTA streams
+// `slices` slices spread over the whole set and gets a similar mix of shapes.
 void partition(const std::vector<wt::MatDesc> &mats, int &grid, std::vector<wt::Piece> &pieces,
-               std::vector<uint32_t> &begin, uint32_t row_align = 1) {
+               std::vector<uint32_t> &begin, uint32_t row_align = 1, int slices = 1) {
   uint64_t B = 0;
   std::vector<uint64_t> start(mats.size() + 1, 0);
   for (size_t i = 0; i < mats.size(); ++i) {
@@ -729,16 +739,17 @@ void partition(const std::vector<wt::MatDesc> &mats, int &grid, std::vector<wt::
   start[mats.size()] = B;
   constexpr uint64_t kMinCtaBytes = 64 << 10;
   grid = (int)std::max<uint64_t>(1, std::min<uint64_t>((uint64_t)wt::num_sms(), (B + kMinCtaBytes - 1) / kMinCtaBytes));
-  // cut c (1..grid-1) at the row boundary nearest byte B*c/grid
+  const int nslice = grid * slices;
+  // cut c (1..nslice-1) at the row boundary nearest byte B*c/nslice
   std::vector<std::pair<uint32_t, uint32_t>> cuts;  // (mat, row)
   cuts.push_back({0, 0});
   size_t m = 0;
-  for (int c = 1; c < grid; ++c) {
-    const uint64_t T = (uint64_t)((unsigned __int128)B * c / grid);
+  for (int c = 1; c < nslice; ++c) {
+    const uint64_t T = (uint64_t)((unsigned __int128)B * c / nslice);
     while (m + 1 < mats.size() && start[m + 1] <= T) ++m;
     const uint64_t rb = (uint64_t)mats[m].V * 16;
     uint64_t row = (T - start[m] + rb / 2) / rb;
-    row = (row + row_align / 2) / row_align * row_align;  // whole tiles per CTA
+    row = (row + row_align / 2) / row_align * row_align;  // whole tiles per slice
     std::pair<uint32_t, uint32_t> cut = {(uint32_t)m, (uint32_t)std::min<uint64_t>(row, mats[m].M)};
     if (cut.second == mats[m].M && m + 1 < mats.size()) cut = {(uint32_t)m + 1, 0};
     if (cut < cuts.back()) cut = cuts.back();
@@ -747,12 +758,14 @@ void partition(const std::vector<wt::MatDesc> &mats, int &grid, std::vector<wt::
   cuts.push_back({(uint32_t)mats.size(), 0});
   begin.assign(1, 0);
   for (int c = 0; c < grid; ++c) {
-    auto a = cuts[c], b = cuts[c + 1];
-    while (a < b) {
-      const uint32_t rend = a.first == b.first ? b.second : mats[a.first].M;
-      if (rend > a.second) pieces.push_back({a.first, a.second, rend, 0});
-      if (a.first == b.first) break;
-      a = {a.first + 1, 0};
+    for (int j = c; j < nslice; j += grid) {
+      auto a = cuts[j], b = cuts[j + 1];
+      while (a < b) {
+        const uint32_t rend = a.first == b.first ? b.second : mats[a.first].M;
+        if (rend > a.second) pieces.push_back({a.first, a.second, rend, 0});
+        if (a.first == b.first) break;
+        a = {a.first + 1, 0};
+      }
     }
     begin.push_back((uint32_t)pieces.size());
   }
@@ -890,7 +903,8 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         L.dtype = dt;
         std::vector<wt::Piece> pieces;
         std::vector<uint32_t> begin;
-        partition(ms, L.grid, pieces, begin, pass == 2 ? (uint32_t)wt::kColTileRows : 1u);
+        partition(ms, L.grid, pieces, begin, pass == 2 ? (uint32_t)wt::kColTileRows : 1u,
+                  pass == 2 ? 1 : one_col_slices(dt));
         L.mats = append(P->table, ms);
         if (pass == 0)
           for (size_t k = 0; k < ms.size(); ++k)
