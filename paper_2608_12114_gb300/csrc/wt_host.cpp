@@ -739,6 +739,10 @@ void partition(const std::vector<wt::MatDesc> &mats, int &grid, std::vector<wt::
   start[mats.size()] = B;
   constexpr uint64_t kMinCtaBytes = 64 << 10;
   grid = (int)std::max<uint64_t>(1, std::min<uint64_t>((uint64_t)wt::num_sms(), (B + kMinCtaBytes - 1) / kMinCtaBytes));
+  // slices of at least kMinSliceBytes: a slice costs the consumers a reload of x, and a
+  // slice shorter than a tile makes its stages partial
+  constexpr uint64_t kMinSliceBytes = 2ull << 20;
+  slices = (int)std::max<uint64_t>(1, std::min<uint64_t>((uint64_t)slices, B / ((uint64_t)grid * kMinSliceBytes)));
   const int nslice = grid * slices;
   // cut c (1..nslice-1) at the row boundary nearest byte B*c/nslice
   std::vector<std::pair<uint32_t, uint32_t>> cuts;  // (mat, row)
