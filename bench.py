@@ -770,7 +770,12 @@ def run_tsweep(args):
                     copy_ms.append((time.perf_counter() - t0) * 1e3)
             cm = statistics.median(copy_ms)
             flops = 2.0 * sum(dev.mats[k].shape[0] * dev.mats[k].shape[1] for k in ks) * n
-            rows.append({"T": T, "kernel": "gemv_tma (one column)" if T == 0 else "gemm_cols (mma.sync m16n8k16)",
+            two_byte = all(dev.mats[k].dtype in (wt.WT_BF16, wt.WT_F16) for k in ks)
+            force = os.environ.get("WT_COLS_KERNEL")
+            on_umma = two_byte and (force == "umma" or (force != "mma" and T > 8))
+            kname = ("gemv_tma (one column)" if T == 0 else
+                     "gemm_cols_umma (tcgen05, M128 N16 K16)" if on_umma else "gemm_cols (mma.sync m16n8k16)")
+            rows.append({"T": T, "kernel": kname,
                          "ms": round(ms, 4), "weight_gbs": round(wbytes / ms / 1e6, 1),
                          "logical_gbs": round(n * wbytes / ms / 1e6, 1), "tflops": round(flops / ms / 1e9, 2),
                          "frac_of_hbm": round(wbytes / ms / 1e6 / peak, 4), "launches_per_pass": launches,

@@ -191,6 +191,8 @@ struct Plan {
     int grid;
     size_t mats, pieces, begin;  // byte offsets in the table
     size_t maps = SIZE_MAX;      // multi-column launches: tensor maps (128-byte aligned)
+    bool umma = false;           // multi-column launch on tcgen05 (wt_umma.cu)
+    uint32_t nmat = 0, ntiles = 0;
   };
   struct Generic {
     int dtype;
@@ -391,6 +393,7 @@ int prepare_device(int dev) {
   if (!g_prepared[dev]) {
     CU(wt::gemv_prepare());
     CU(wt::gemm_cols_prepare());
+    CU(wt::gemm_cols_umma_prepare());
     g_prepared[dev] = true;
   }
   return WT_OK;
@@ -725,6 +728,54 @@ int encode_cols_map(const wt::MatDesc &m, uint8_t *out) {
 // costs an exposed reload of x.
 int one_col_slices(int dtype) { return dtype == WT_I8 ? 1 : 16; }
 
+// Which multi-column kernel runs a matrix: tcgen05 (wt_umma.cu) for 2-byte weights with more
+// than 8 columns, where its T-independent tensor time wins (bf16 protocol, T = 16: 6529
+// against 6370 GB/s); the warp-level MMA kernel (wt_cols.cu) otherwise (T = 1: 6958 against
+// 6580; int8 decodes in registers there).  WT_COLS_KERNEL=mma or =umma forces one kernel
+// (umma still only for 2-byte weights).
+bool cols_on_umma(int dtype, int cols) {
+  static const int force = [] {
+    const char *e = getenv("WT_COLS_KERNEL");
+    if (e && strcmp(e, "umma") == 0) return 1;
+    if (e && strcmp(e, "mma") == 0) return 2;
+    return 0;
+  }();
+  if (dtype != WT_BF16 && dtype != WT_F16) return false;
+  return force == 1 || (force == 0 && cols > 8);
+}
+
+// The two tensor maps of a tcgen05 multi-column matrix (see wt::UmmaLaunch).
+int encode_umma_maps(const wt::MatDesc &m, int dtype, uint8_t *out) {
+  EncodeTiledFn fn = encode_tiled();
+  if (!fn) return set_err(WT_ECUDA, "wt_pass: cuTensorMapEncodeTiled is not available from the driver");
+  (void)dtype;  // 2-byte weights only
+  const uint64_t K = (uint64_t)m.V * 8;
+  CUtensorMap mw, mx;
+  {
+    const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)m.M};
+    const cuuint64_t strides[1] = {(cuuint64_t)m.V * 16};
+    const cuuint32_t box[2] = {64, 128};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = fn(&mw, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<uint8_t *>(m.W), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return set_err(WT_ECUDA, "wt_pass: tensor map of W failed (%d)", (int)r);
+  }
+  {
+    const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)m.G};
+    const cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+    const cuuint32_t box[2] = {64, 16};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = fn(&mx, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<uint8_t *>(m.x), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return set_err(WT_ECUDA, "wt_pass: tensor map of X failed (%d)", (int)r);
+  }
+  memcpy(out, &mw, sizeof mw);
+  memcpy(out + wt::kTensorMapBytes, &mx, sizeof mx);
+  return WT_OK;
+}
+
 // Split the rows of `mats` (in order) into grid * slices contiguous slices of nearly
 // equal bytes, cut at row boundaries; slice j goes to CTA j % grid, so every CTA streams
 // `slices` slices spread over the whole set and gets a similar mix of shapes.
@@ -833,7 +884,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
     while (j < n && d[j].wait_event == d[i].wait_event) ++j;
     Plan::Group g;
     g.first = i;
-    std::vector<wt::MatDesc> by_dt[4], mapped_dt[4], cols_dt[4];
+    std::vector<wt::MatDesc> by_dt[4], mapped_dt[4], cols_dt[4], umma_dt[4];
     std::vector<int64_t> seg_ws[4];  // per by_dt entry: workspace float offset of its partials, or -1
     std::vector<wt::SegReduce> reds;
     std::vector<size_t> red_ws;      // per reds entry: workspace float offset
@@ -870,7 +921,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         else g.generic.push_back({q.dtype, static_cast<const uint8_t *>(q.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
                                   static_cast<const uint8_t *>(q.scale), ncol});
       } else if (fast && q.cols > 0) {
-        cols_dt[q.dtype].push_back(make_cols_mat(q));
+        (cols_on_umma(q.dtype, q.cols) ? umma_dt : cols_dt)[q.dtype].push_back(make_cols_mat(q));
       } else if (fast && q.K * es / 16 > wt::seg_vectors(q.dtype)) {
         // long rows: column segments spread over CTAs, summed by the second pass
         const uint32_t V = (uint32_t)(q.K * es / 16);
@@ -899,14 +950,39 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
                              static_cast<const uint8_t *>(q.scale), ncol});
       }
     }
-    for (int pass = 0; pass < 3; ++pass) {
+    for (int pass = 0; pass < 4; ++pass) {
       for (int dt = 0; dt < 4; ++dt) {
-        std::vector<wt::MatDesc> &ms = pass == 0 ? by_dt[dt] : pass == 1 ? mapped_dt[dt] : cols_dt[dt];
+        std::vector<wt::MatDesc> &ms =
+            pass == 0 ? by_dt[dt] : pass == 1 ? mapped_dt[dt] : pass == 2 ? cols_dt[dt] : umma_dt[dt];
         if (ms.empty()) continue;
         Plan::Launch L;
         L.dtype = dt;
         std::vector<wt::Piece> pieces;
         std::vector<uint32_t> begin;
+        if (pass == 3) {
+          // tcgen05 launch: 128-row tiles, dealt round-robin; two tensor maps per matrix
+          L.umma = true;
+          uint32_t first = 0;
+          for (size_t k = 0; k < ms.size(); ++k) {
+            const uint32_t tiles = (ms[k].M + 127) / 128;
+            pieces.push_back({(uint32_t)k, first, tiles, 0});
+            first += tiles;
+          }
+          L.nmat = (uint32_t)ms.size();
+          L.ntiles = first;
+          L.grid = (int)std::max<uint32_t>(1, std::min<uint32_t>((uint32_t)wt::num_sms(), first));
+          L.mats = append(P->table, ms);
+          L.pieces = append(P->table, pieces);
+          L.begin = L.pieces;
+          L.maps = (P->table.size() + 127) & ~(size_t)127;
+          P->table.resize(L.maps + ms.size() * 2 * wt::kTensorMapBytes);
+          for (size_t k = 0; k < ms.size(); ++k) {
+            int rc = encode_umma_maps(ms[k], dt, P->table.data() + L.maps + k * 2 * wt::kTensorMapBytes);
+            if (rc) return rc;
+          }
+          g.cols.push_back(L);
+          continue;
+        }
         partition(ms, L.grid, pieces, begin, pass == 2 ? (uint32_t)wt::kColTileRows : 1u,
                   pass == 2 ? 1 : one_col_slices(dt));
         L.mats = append(P->table, ms);
@@ -1030,7 +1106,20 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
       gl.begin = reinterpret_cast<const uint32_t *>(P->dev + L.begin);
       gl.status = h->status;
       gl.maps = P->dev + L.maps;
-      CU(wt::launch_gemm_cols(gl, s));
+      if (L.umma) {
+        wt::UmmaLaunch ul;
+        ul.dtype = L.dtype;
+        ul.grid = L.grid;
+        ul.mats = gl.mats;
+        ul.pieces = gl.pieces;
+        ul.nmat = L.nmat;
+        ul.ntiles = L.ntiles;
+        ul.status = h->status;
+        ul.maps = gl.maps;
+        CU(wt::launch_gemm_cols_umma(ul, s));
+      } else {
+        CU(wt::launch_gemm_cols(gl, s));
+      }
       h->kernel_launches++;
     }
     for (const Plan::Generic &q : g.generic) {
