@@ -257,3 +257,44 @@ def test_checksum_many_buffers(torch):
         h.checksum([buf.data_ptr() + int(o) for o in offs], [int(s) for s in sizes], out.data_ptr(), 0)
         got = [int(v) & (2 ** 64 - 1) for v in out.cpu().tolist()]
     assert got == [oracle.fnv_tree(data[o:o + s]) for o, s in zip(offs, sizes)]
+
+
+def test_unaligned_operands_take_the_generic_kernel(torch):
+    """W and x 2 bytes past a 16-byte boundary (element-aligned only): the scalar fallback,
+    checked against the oracle; one and several columns."""
+    rng = np.random.default_rng(13)
+    M, K, T = 37, 1000, 3
+    Wb = synth.f32_to_bf16_bits((0.02 * rng.standard_normal(M * K)).astype(np.float32)).view(np.uint8)
+    X = synth.f32_to_bf16_bits(rng.standard_normal(T * K).astype(np.float32)).view(np.uint8)
+    Wd = torch.zeros(Wb.size + 16, dtype=torch.uint8, device="cuda")
+    Wd[2:2 + Wb.size] = torch.from_numpy(Wb.copy()).cuda()
+    Xd = torch.zeros(X.size + 16, dtype=torch.uint8, device="cuda")
+    Xd[2:2 + X.size] = torch.from_numpy(X.copy()).cuda()
+    y1 = torch.full((M,), float("nan"), dtype=torch.float32, device="cuda")
+    yT = torch.full((T * M,), float("nan"), dtype=torch.float32, device="cuda")
+    with wt.Handle([]) as h:
+        h.pass_([wt.gemv_desc(Wd.data_ptr() + 2, wt.WT_BF16, M, K, Xd.data_ptr() + 2, y1.data_ptr()),
+                 wt.gemv_desc(Wd.data_ptr() + 2, wt.WT_BF16, M, K, Xd.data_ptr() + 2, yT.data_ptr(), cols=T)], 0)
+        torch.cuda.synchronize()
+        assert h.device_status() == 0
+    Y, A = oracle.gemv_cols(Wb, wt.WT_BF16, M, K, X, T)
+    assert oracle.gemv_error(y1.cpu().numpy(), Y[0], A[0]) <= 2e-3
+    assert oracle.gemv_error(yT.cpu().numpy(), Y.reshape(-1), A.reshape(-1)) <= 2e-3
+
+
+def test_descriptor_bounds_are_refused_before_any_launch(torch):
+    x = torch.zeros(64, dtype=torch.bfloat16, device="cuda")
+    y = torch.zeros(64, dtype=torch.float32, device="cuda")
+    with wt.Handle([]) as h:
+        n0 = h.kernel_launches()
+        for M, K in ((2 ** 31, 16), (16, 2 ** 31)):
+            with pytest.raises(wt.WtError) as ei:
+                h.pass_([wt.gemv_desc(x.data_ptr(), wt.WT_BF16, M, K, x.data_ptr(), y.data_ptr())], 0)
+            assert ei.value.code == wt.WT_EINVAL
+        with pytest.raises(wt.WtError) as ei:                       # u8 weights have no GEMV
+            h.pass_([wt.gemv_desc(x.data_ptr(), wt.WT_U8, 4, 16, x.data_ptr(), y.data_ptr())], 0)
+        assert ei.value.code == wt.WT_ENOTSUP
+        with pytest.raises(wt.WtError) as ei:                       # null y with rows
+            h.pass_([wt.gemv_desc(x.data_ptr(), wt.WT_BF16, 4, 16, x.data_ptr(), 0)], 0)
+        assert ei.value.code == wt.WT_EINVAL
+        assert h.kernel_launches() == n0 and h.device_status() == 0
