@@ -36,7 +36,7 @@ namespace wt {
 
 namespace {
 
-constexpr int kColWarps = kConsumerWarps;
+constexpr int kColWarps = 8;  // consumer warps
 constexpr int kColConsumers = kColWarps * 32;
 constexpr int kColThreads = kColConsumers + 32;  // + one producer warp
 constexpr int kColRows = kColTileRows;           // rows of one stage (one MMA tile)
