@@ -744,11 +744,10 @@ bool cols_on_umma(int dtype, int cols) {
   return force == 1 || (force == 0 && cols > 8);
 }
 
-// The two tensor maps of a tcgen05 multi-column matrix (see wt::UmmaLaunch).
-int encode_umma_maps(const wt::MatDesc &m, int dtype, uint8_t *out) {
+// The two tensor maps of a tcgen05 multi-column matrix (2-byte weights; see wt::UmmaLaunch).
+int encode_umma_maps(const wt::MatDesc &m, uint8_t *out) {
   EncodeTiledFn fn = encode_tiled();
   if (!fn) return set_err(WT_ECUDA, "wt_pass: cuTensorMapEncodeTiled is not available from the driver");
-  (void)dtype;  // 2-byte weights only
   const uint64_t K = (uint64_t)m.V * 8;
   CUtensorMap mw, mx;
   {
@@ -977,7 +976,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
           L.maps = (P->table.size() + 127) & ~(size_t)127;
           P->table.resize(L.maps + ms.size() * 2 * wt::kTensorMapBytes);
           for (size_t k = 0; k < ms.size(); ++k) {
-            int rc = encode_umma_maps(ms[k], dt, P->table.data() + L.maps + k * 2 * wt::kTensorMapBytes);
+            int rc = encode_umma_maps(ms[k], P->table.data() + L.maps + k * 2 * wt::kTensorMapBytes);
             if (rc) return rc;
           }
           g.cols.push_back(L);

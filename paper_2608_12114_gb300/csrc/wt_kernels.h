@@ -121,11 +121,11 @@ cudaError_t gemm_cols_prepare();
 cudaError_t launch_gemm_cols(const GemvLaunch &L, cudaStream_t s);
 size_t gemm_cols_smem_bytes();
 
-// The same multi-column GEMV on tcgen05 (wt_umma.cu): row tiles of 128 rows, K in chunks of
-// 64 elements, accumulators in tensor memory.  pieces[m] = {m, first tile of matrix m, its
-// tiles, 0}; CTA b takes tiles b, b + grid, ...  maps holds two tensor maps per matrix: W
-// (bf16/f16: [M, K] 2-byte elements, box {64, 128}, 128-byte swizzle; int8: [M, K] bytes,
-// box {64, 128}, no swizzle) and X ([T, K] 2-byte elements, box {64, 16}, 128-byte swizzle).
+// The same multi-column GEMV on tcgen05 for 2-byte weights (wt_umma.cu): row tiles of 128
+// rows, K in chunks of 64 elements, accumulators in tensor memory.  pieces[m] = {m, first
+// tile of matrix m, its tiles, 0}; CTA b takes tiles b, b + grid, ...  maps holds two tensor
+// maps per matrix: W ([M, K] 2-byte elements, box {64, 128}, 128-byte swizzle) and X ([T, K]
+// 2-byte elements, box {64, 16}, 128-byte swizzle).
 struct UmmaLaunch {
   int dtype;
   int grid;

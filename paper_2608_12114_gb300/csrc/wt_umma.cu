@@ -20,8 +20,6 @@
 //
 // Every mbarrier wait is bounded; a timeout records WT_ETIMEDOUT and every role stops.  The
 // allocating warp frees the tensor memory after the whole CTA has synchronised.
-#include <cuda_fp16.h>
-
 #include "wt_device.cuh"
 #include "wt_kernels.h"
 
