@@ -707,8 +707,9 @@ def run_policy(args):
 
 def run_tsweep(args):
     """The T-sweep (Sec. 4.3): one multi-column pass over every matrix with T activation
-    columns, resident in HBM (CUDA events over `steps` passes) and per-use copy (wt_adopt +
-    the event-gated pass, wall time per rep)."""
+    columns, resident in HBM (CUDA events over `steps` passes), per-use copy (wt_adopt + the
+    event-gated pass, wall time per rep), and the map endpoint (W read in place from the
+    file mapping: the paper's adoption arm; CUDA events)."""
     if args.workload == "large":
         args.workload = "protocol_q8"
     ts = [int(v) for v in args.tsweep.split(",")]
@@ -769,6 +770,22 @@ def run_tsweep(args):
                 if rep:
                     copy_ms.append((time.perf_counter() - t0) * 1e3)
             cm = statistics.median(copy_ms)
+            # map endpoint: W read in place from the file mapping (prefaulted at plan build)
+            dm = dev.descs(xs, ys)
+            dm["cols"] = T
+            dm["W"] = [h.tensors[dev.mats[k].parts[0]].host_ptr for k in ks]
+            map_ms = None
+            if all(len(dev.mats[k].parts) == 1 for k in ks):
+                h.pass_(dm, s.cuda_stream)
+                s.synchronize()
+                em0, em1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                nmap = max(3, args.steps // 20)
+                em0.record(s)
+                for _ in range(nmap):
+                    h.pass_(dm, s.cuda_stream)
+                em1.record(s)
+                s.synchronize()
+                map_ms = em0.elapsed_time(em1) / nmap
             flops = 2.0 * sum(dev.mats[k].shape[0] * dev.mats[k].shape[1] for k in ks) * n
             two_byte = all(dev.mats[k].dtype in (wt.WT_BF16, wt.WT_F16) for k in ks)
             force = os.environ.get("WT_COLS_KERNEL")
@@ -779,9 +796,12 @@ def run_tsweep(args):
                          "ms": round(ms, 4), "weight_gbs": round(wbytes / ms / 1e6, 1),
                          "logical_gbs": round(n * wbytes / ms / 1e6, 1), "tflops": round(flops / ms / 1e9, 2),
                          "frac_of_hbm": round(wbytes / ms / 1e6 / peak, 4), "launches_per_pass": launches,
-                         "copy_ms": round(cm, 3), "resident_over_copy": round(cm / ms, 2)})
-            log("T=%d: %.4f ms, %.1f GB/s weights (%.1f%% of %s HBM), copy %.3f ms" % (
-                T, ms, wbytes / ms / 1e6, 100 * wbytes / ms / 1e6 / peak, peak_kind, cm))
+                         "copy_ms": round(cm, 3), "resident_over_copy": round(cm / ms, 2),
+                         "map_ms": round(map_ms, 3) if map_ms else None,
+                         "map_over_copy": round(cm / map_ms, 3) if map_ms else None})
+            log("T=%d: %.4f ms, %.1f GB/s weights (%.1f%% of %s HBM), copy %.3f ms, map %s ms" % (
+                T, ms, wbytes / ms / 1e6, 100 * wbytes / ms / 1e6 / peak, peak_kind, cm,
+                "%.3f" % map_ms if map_ms else "-"))
     h.close()
     out = {"metric": "multi-column T-sweep: resident pass time and weight GB/s per T", "unit": "GB/s",
            "config": {"workload": workload_desc(args), "weight_bytes": wbytes, "matrices": len(ks),

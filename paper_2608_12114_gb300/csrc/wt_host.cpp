@@ -192,6 +192,7 @@ struct Plan {
     size_t mats, pieces, begin;  // byte offsets in the table
     size_t maps = SIZE_MAX;      // multi-column launches: tensor maps (128-byte aligned)
     bool umma = false;           // multi-column launch on tcgen05 (wt_umma.cu)
+    bool mapped_cols = false;    // map endpoint with T columns
     uint32_t nmat = 0, ntiles = 0;
   };
   struct Generic {
@@ -883,7 +884,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
     while (j < n && d[j].wait_event == d[i].wait_event) ++j;
     Plan::Group g;
     g.first = i;
-    std::vector<wt::MatDesc> by_dt[4], mapped_dt[4], cols_dt[4], umma_dt[4];
+    std::vector<wt::MatDesc> by_dt[4], mapped_dt[4], cols_dt[4], umma_dt[4], mcols_dt[4];
     std::vector<int64_t> seg_ws[4];  // per by_dt entry: workspace float offset of its partials, or -1
     std::vector<wt::SegReduce> reds;
     std::vector<size_t> red_ws;      // per reds entry: workspace float offset
@@ -909,9 +910,16 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         if (!h->prefaulted && !f->populated) prefault(f->base + off, q.M * q.K * es);
         wt_gemv_desc qd = q;
         qd.W = f->dev + off;
-        if (fast && q.cols == 0) mapped_dt[q.dtype].push_back(make_mat(qd));
-        else g.generic.push_back({q.dtype, static_cast<const uint8_t *>(qd.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
-                                  static_cast<const uint8_t *>(q.scale), ncol});
+        if (fast && q.cols == 0) {
+          mapped_dt[q.dtype].push_back(make_mat(qd));
+        } else if (fast && q.dtype != WT_F32) {
+          wt::MatDesc m = make_mat(qd);
+          m.cols = (uint32_t)q.cols;
+          mcols_dt[q.dtype].push_back(m);
+        } else {
+          g.generic.push_back({q.dtype, static_cast<const uint8_t *>(qd.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
+                               static_cast<const uint8_t *>(q.scale), ncol});
+        }
       } else if (const int mc = memory_class(q.W, h->device); mc != 0) {
         if (mc < 0) return set_err(WT_ENOTSUP, "wt_pass: W of desc %zu is host memory this device cannot read", k);
         // host memory outside this handle (another mapping, a file-backed DLPack tensor, a
@@ -949,10 +957,13 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
                              static_cast<const uint8_t *>(q.scale), ncol});
       }
     }
-    for (int pass = 0; pass < 4; ++pass) {
+    for (int pass = 0; pass < 5; ++pass) {
       for (int dt = 0; dt < 4; ++dt) {
-        std::vector<wt::MatDesc> &ms =
-            pass == 0 ? by_dt[dt] : pass == 1 ? mapped_dt[dt] : pass == 2 ? cols_dt[dt] : umma_dt[dt];
+        std::vector<wt::MatDesc> &ms = pass == 0   ? by_dt[dt]
+                                       : pass == 1 ? mapped_dt[dt]
+                                       : pass == 2 ? cols_dt[dt]
+                                       : pass == 3 ? umma_dt[dt]
+                                                   : mcols_dt[dt];
         if (ms.empty()) continue;
         Plan::Launch L;
         L.dtype = dt;
@@ -983,7 +994,8 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
           continue;
         }
         partition(ms, L.grid, pieces, begin, pass == 2 ? (uint32_t)wt::kColTileRows : 1u,
-                  pass == 2 ? 1 : one_col_slices(dt));
+                  pass == 0 ? one_col_slices(dt) : 1);
+        L.mapped_cols = pass == 4;
         L.mats = append(P->table, ms);
         if (pass == 0)
           for (size_t k = 0; k < ms.size(); ++k)
@@ -999,7 +1011,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
             if (rc) return rc;
           }
         }
-        (pass == 0 ? g.launches : pass == 1 ? g.mapped : g.cols).push_back(L);
+        (pass == 0 ? g.launches : pass == 1 || pass == 4 ? g.mapped : g.cols).push_back(L);
       }
     }
     if (!reds.empty()) {
@@ -1093,7 +1105,7 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
       gl.pieces = reinterpret_cast<const wt::Piece *>(P->dev + L.pieces);
       gl.begin = reinterpret_cast<const uint32_t *>(P->dev + L.begin);
       gl.status = h->status;
-      CU(wt::launch_gemv_mapped(gl, s));
+      CU(L.mapped_cols ? wt::launch_gemv_mapped_cols(gl, s) : wt::launch_gemv_mapped(gl, s));
       h->kernel_launches++;
     }
     for (const Plan::Launch &L : g.cols) {

@@ -694,6 +694,96 @@ __global__ void __launch_bounds__(256) gemv_mapped_kernel(const MatDesc *__restr
   }
 }
 
+// Map endpoint with T activation columns: the one-column mapped kernel's loads of W, each
+// vector multiplied against every column's x (from L1/L2) into its own accumulators; the
+// link-bound W stream is read once for all T columns.
+template <int DT>
+__global__ void __launch_bounds__(256, 1) gemv_mapped_cols_kernel(const MatDesc *__restrict__ mats,
+                                                               const Piece *__restrict__ pieces,
+                                                               const uint32_t *__restrict__ begin) {
+  constexpr int NP = Pairs<DT>::N;
+  constexpr int kWarps = 8;
+  constexpr int kMaxT = 16;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (uint32_t pi = begin[blockIdx.x]; pi < begin[blockIdx.x + 1]; ++pi) {
+    const Piece pc = pieces[pi];
+    const MatDesc md = mats[pc.mat];
+    const uint32_t V = md.V, T = md.cols;
+    const uint64_t xstride = (uint64_t)V * (DT == 3 ? 32 : 16);  // bytes of one x column
+    const uint32_t G = V >= 32 ? 32u : (V <= 1 ? 1u : 1u << (32 - __clz(V - 1)));
+    const uint32_t gl = lane & (G - 1), sub = lane / G, rpw = 32 / G;
+    for (uint32_t base = pc.r0 + warp * rpw; base < pc.r1; base += kWarps * rpw) {
+      const uint32_t row = base + sub;
+      const bool valid = row < pc.r1;
+      const uint4 *w4 = reinterpret_cast<const uint4 *>(md.W + (uint64_t)(valid ? row : pc.r0) * V * 16);
+      Acc4 acc[kMaxT];
+      for (uint32_t v = gl; v < V; v += 4 * G) {
+        uint4 w[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const uint32_t vv = v + u * G;
+          w[u] = (valid && vv < V) ? w4[vv] : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const uint32_t vv = v + u * G;
+          // decode the vector once (int8: exact f16x2 words; else fp32 pairs), use it T times
+          uint32_t dh[8];
+          uint64_t dp[NP];
+          if constexpr (DT == 3) {
+            const uint32_t ws[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const uint32_t q = ws[i] ^ 0x80808080u;
+              dh[2 * i] = i8x2_to_f16x2(q, 0x4140u);
+              dh[2 * i + 1] = i8x2_to_f16x2(q, 0x4342u);
+            }
+          } else {
+#pragma unroll
+            for (int i = 0; i < NP; ++i) dp[i] = Pairs<DT>::get(w[u], i);
+          }
+#pragma unroll
+          for (int t = 0; t < kMaxT; ++t) {
+            if ((uint32_t)t < T) {
+              uint64_t xp[NP];
+              load_xpairs<DT>(md.x + t * xstride, vv, vv < V, xp);
+              if constexpr (DT == 3) {
+                uint32_t f[4];
+                asm("mov.b64 {%0, %1}, %2;" : "=r"(f[0]), "=r"(f[1]) : "l"(acc[t].a));
+                asm("mov.b64 {%0, %1}, %2;" : "=r"(f[2]), "=r"(f[3]) : "l"(acc[t].b));
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                  float c = __uint_as_float(f[i]);
+                  c = fma_h2(dh[2 * i], (uint32_t)xp[i], c);
+                  c = fma_h2(dh[2 * i + 1], (uint32_t)(xp[i] >> 32), c);
+                  f[i] = __float_as_uint(c);
+                }
+                acc[t].a = pack2(f[0], f[1]);
+                acc[t].b = pack2(f[2], f[3]);
+              } else {
+#pragma unroll
+                for (int i = 0; i < NP; ++i) {
+                  if (i & 1) acc[t].b = fma2(dp[i], xp[i], acc[t].b);
+                  else acc[t].a = fma2(dp[i], xp[i], acc[t].a);
+                }
+              }
+            }
+          }
+        }
+      }
+      const float sc = valid ? row_scale<DT>(md.s, row) : 0.f;
+#pragma unroll
+      for (int t = 0; t < kMaxT; ++t) {
+        if ((uint32_t)t < T) {
+          float r = acc[t].total();
+          for (uint32_t o = G >> 1; o > 0; o >>= 1) r += __shfl_xor_sync(0xffffffffu, r, o);
+          if (valid && gl == 0) md.y[(uint64_t)t * md.M + row] = r * sc;
+        }
+      }
+    }
+  }
+}
+
 // Fallback: one warp per row, byte-assembled scalar loads (any alignment).  Column c of a
 // multi-column call reads x + c * K elements and writes y + c * M.
 template <int DT>
@@ -896,6 +986,17 @@ cudaError_t launch_gemv_mapped(const GemvLaunch &L, cudaStream_t s) {
     case 1: gemv_mapped_kernel<1><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
     case 2: gemv_mapped_kernel<2><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
     case 3: gemv_mapped_kernel<3><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemv_mapped_cols(const GemvLaunch &L, cudaStream_t s) {
+  if (L.grid <= 0) return cudaSuccess;
+  switch (L.dtype) {
+    case 1: gemv_mapped_cols_kernel<1><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
+    case 2: gemv_mapped_cols_kernel<2><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
+    case 3: gemv_mapped_cols_kernel<3><<<L.grid, 256, 0, s>>>(L.mats, L.pieces, L.begin); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();

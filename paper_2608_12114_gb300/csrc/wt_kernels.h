@@ -60,7 +60,10 @@ struct alignas(16) MatDesc {
   uint16_t G;     // mode 0: lanes per row (power of two <= 32); kModeCols: columns T
   uint32_t rs;    // row pitch in 16-byte vectors: V, or the full row of a column segment
                   // (segments are split-K only); s == nullptr then means "no scale yet"
+  uint32_t cols;  // map endpoint with T activation columns: T (X [T, K], Y [T, M]); else 0
+  uint32_t pad;
 };
+static_assert(sizeof(MatDesc) == 64, "MatDesc is one 64-byte record");
 
 // Cross-CTA split-K: rows longer than seg_vectors(dtype) are cut into column segments of
 // that many vectors (the last one shorter).  Each segment is a matrix of its own (row pitch
@@ -110,6 +113,9 @@ size_t gemv_smem_bytes();
 // the device reaches over the host link, with 16-byte loads and no TMA; same tables as
 // launch_gemv (MatDesc.W holds the device-readable address of the mapped rows).
 cudaError_t launch_gemv_mapped(const GemvLaunch &L, cudaStream_t s);
+// The map endpoint with T <= 16 activation columns (MatDesc.cols = T): each mapped weight
+// vector is loaded once over the host link and used for every column.
+cudaError_t launch_gemv_mapped_cols(const GemvLaunch &L, cudaStream_t s);
 
 // Multi-column GEMV Y[t] = diag(s) W X[t] (t < T <= 16; X [T, K] and Y [T, M] row-major) on the
 // tensor cores (wt_cols.cu); dtype WT_BF16 / WT_F16 / WT_I8, tables as for launch_gemv with

@@ -210,3 +210,28 @@ def test_cols_full_size_matched_protocol(torch, tmp_path):
                     assert oracle.gemv_error(got.reshape(-1), Yhat.reshape(-1), A.reshape(-1)) <= TOL, (T, m.name)
     finally:
         co.close()
+
+
+def test_cols_map_endpoint_bf16_and_f16(torch, tmp_path):
+    """The map endpoint with T columns for 2-byte weights (mapped multi-column kernel)."""
+    for dtype, name in ((synth.DT_BF16, "mb"), (synth.DT_F16, "mh")):
+        shapes = [(70, 4096), (5, 40), (33, 1032)]
+        ck = synth.write_files(synth.custom(str(tmp_path / name), shapes, dtype=dtype, name=name))
+        co = oracle.CheckpointOracle(ck.paths)
+        T = 11
+        with wt.Handle(ck.paths) as h:
+            for i, (M, K) in enumerate(shapes):
+                t = h.tensors[i]
+                rng = np.random.default_rng(i)
+                if dtype == synth.DT_BF16:
+                    X = synth.f32_to_bf16_bits(rng.standard_normal((T, K)).astype(np.float32)).view(np.uint8)
+                else:
+                    X = rng.standard_normal((T, K)).astype(np.float16).view(np.uint8)
+                Xd = torch.from_numpy(X.reshape(-1).copy()).cuda()
+                Y = torch.full((T * M,), float("nan"), dtype=torch.float32, device="cuda")
+                h.pass_([wt.gemv_desc(t.host_ptr, dtype, M, K, Xd.data_ptr(), Y.data_ptr(), cols=T)], 0)
+                torch.cuda.synchronize()
+                Yhat, A = oracle.gemv_cols(co.blob_of(t.file, t.name), dtype, M, K, X.reshape(-1), T)
+                assert oracle.gemv_error(Y.cpu().numpy().astype(np.float64), Yhat.reshape(-1), A.reshape(-1)) <= TOL
+            assert h.device_status() == 0
+        co.close()
