@@ -924,9 +924,16 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         if (mc < 0) return set_err(WT_ENOTSUP, "wt_pass: W of desc %zu is host memory this device cannot read", k);
         // host memory outside this handle (another mapping, a file-backed DLPack tensor, a
         // pinned buffer): plain loads only, as for the map endpoint; TMA streams device memory
-        if (fast && q.cols == 0) mapped_dt[q.dtype].push_back(make_mat(q));
-        else g.generic.push_back({q.dtype, static_cast<const uint8_t *>(q.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
-                                  static_cast<const uint8_t *>(q.scale), ncol});
+        if (fast && q.cols == 0) {
+          mapped_dt[q.dtype].push_back(make_mat(q));
+        } else if (fast && q.dtype != WT_F32) {
+          wt::MatDesc m = make_mat(q);
+          m.cols = (uint32_t)q.cols;
+          mcols_dt[q.dtype].push_back(m);
+        } else {
+          g.generic.push_back({q.dtype, static_cast<const uint8_t *>(q.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
+                               static_cast<const uint8_t *>(q.scale), ncol});
+        }
       } else if (fast && q.cols > 0) {
         (cols_on_umma(q.dtype, q.cols) ? umma_dt : cols_dt)[q.dtype].push_back(make_cols_mat(q));
       } else if (fast && q.K * es / 16 > wt::seg_vectors(q.dtype)) {

@@ -57,6 +57,16 @@ def test_device_capsule_is_read_in_place(torch, tmp_path):
         assert h.device_status() == 0
     yhat, a = oracle.gemv(raw, wt.WT_BF16, M, K, synth.make_x(K, wt.WT_BF16))
     assert oracle.gemv_error(y.cpu().numpy(), yhat, a) <= 2e-3
+    T = 5                                                             # and with T columns
+    X = synth.f32_to_bf16_bits(np.random.default_rng(2).standard_normal((T, K)).astype(np.float32)).view(np.uint8)
+    Xd = torch.from_numpy(X.reshape(-1).copy()).cuda()
+    Y = torch.full((T * M,), float("nan"), dtype=torch.float32, device="cuda")
+    with wt.Handle([]) as h:
+        h.pass_([wt.gemv_desc(t.data_ptr(), wt.WT_BF16, M, K, Xd.data_ptr(), Y.data_ptr(), cols=T)], 0)
+        torch.cuda.synchronize()
+        assert h.device_status() == 0
+    Yh, A = oracle.gemv_cols(raw, wt.WT_BF16, M, K, X.reshape(-1), T)
+    assert oracle.gemv_error(Y.cpu().numpy(), Yh.reshape(-1), A.reshape(-1)) <= 2e-3
     fd = os.open(p, os.O_WRONLY)                                     # the file stays the storage
     os.pwrite(fd, b"\x80\x3f", 2 * (K + 1))                          # element (1, 1) = 1.0
     os.close(fd)
