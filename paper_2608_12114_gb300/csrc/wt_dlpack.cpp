@@ -87,10 +87,11 @@ int dlpack_map(const char *path, uint64_t off, uint64_t nbytes, int32_t dtype, i
   const uint64_t len = (off + nbytes + page - 1) / page * page - a0;
   const int fd = open(path, O_RDONLY | O_CLOEXEC);
   if (fd < 0) return err(WT_EIO, "dlpack: open %s: %s", path, strerror(errno));
-  void *p = mmap(nullptr, len, PROT_READ, MAP_SHARED, fd, (off_t)a0);
+  const bool injected = wt::fault_injected("mmap");
+  void *p = injected ? MAP_FAILED : mmap(nullptr, len, PROT_READ, MAP_SHARED, fd, (off_t)a0);
   const int e = errno;
   close(fd);  // the mapping keeps the file referenced
-  if (p == MAP_FAILED) return err(WT_EIO, "dlpack: mmap %s: %s", path, strerror(e));
+  if (p == MAP_FAILED) return err(WT_EIO, "dlpack: mmap %s: %s", path, injected ? "injected fault" : strerror(e));
   Ctx *c = new (std::nothrow) Ctx();
   if (!c) {
     munmap(p, len);

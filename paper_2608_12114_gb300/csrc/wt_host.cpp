@@ -282,6 +282,7 @@ int parse_file(File &f, int fd, uint64_t fsize) {
   const char *path = f.path.c_str();
   if (fsize < 16) return set_err(WT_EFORMAT, "%s: shorter than the 16-byte header", path);
   uint8_t hdr[16];
+  if (wt::fault_injected("pread")) return set_err(WT_EIO, "%s: pread header: injected fault", path);
   if (pread(fd, hdr, 16, 0) != 16) return set_err(WT_EIO, "%s: pread header: %s", path, strerror(errno));
   if (memcmp(hdr, "WTCKPT01", 8) != 0) return set_err(WT_EFORMAT, "%s: bad magic", path);
   Reader h{hdr, 16, 8};
@@ -353,6 +354,7 @@ void unmap_file(File &f) {
 
 // open, parse and map one file; closes the fd on every path.
 int open_one(File &f) {
+  if (wt::fault_injected("open")) return set_err(WT_EIO, "%s: open: injected fault", f.path.c_str());
   const int fd = open(f.path.c_str(), O_RDONLY | O_CLOEXEC);
   if (fd < 0) return set_err(WT_EIO, "%s: open: %s", f.path.c_str(), strerror(errno));
   struct stat st;
@@ -364,8 +366,9 @@ int open_one(File &f) {
   int rc = parse_file(f, fd, (uint64_t)st.st_size);
   if (rc == WT_OK) {
     f.size = (size_t)st.st_size;
-    void *p = mmap(nullptr, f.size, PROT_READ, MAP_SHARED, fd, 0);
-    if (p == MAP_FAILED) rc = set_err(WT_EIO, "%s: mmap: %s", f.path.c_str(), strerror(errno));
+    const bool injected = wt::fault_injected("mmap");
+    void *p = injected ? MAP_FAILED : mmap(nullptr, f.size, PROT_READ, MAP_SHARED, fd, 0);
+    if (p == MAP_FAILED) rc = set_err(WT_EIO, "%s: mmap: %s", f.path.c_str(), injected ? "injected fault" : strerror(errno));
     else f.base = static_cast<uint8_t *>(p);
   }
   close(fd);  // Algorithm 1: the mapping outlives the descriptor
@@ -1040,6 +1043,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
   const size_t bytes = std::max<size_t>(16, align16(P->table.size()));
   CU(cudaHostAlloc(reinterpret_cast<void **>(&P->host), bytes, cudaHostAllocDefault));
   memcpy(P->host, P->table.data(), P->table.size());
+  if (wt::fault_injected("alloc")) return set_err(WT_ENOMEM, "wt_pass: plan tables: injected allocation fault");
   CU(cudaMalloc(reinterpret_cast<void **>(&P->dev), bytes));
   CU(cudaEventCreateWithFlags(&P->uploaded, cudaEventDisableTiming));
   CU(cudaEventCreateWithFlags(&P->last, cudaEventDisableTiming));
@@ -1097,6 +1101,7 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
       gl.pieces = reinterpret_cast<const wt::Piece *>(P->dev + L.pieces);
       gl.begin = reinterpret_cast<const uint32_t *>(P->dev + L.begin);
       gl.status = h->status;
+      gl.stall = wt::fault_injected("stall") ? 1 : 0;
       CU(wt::launch_gemv(gl, s));
       h->kernel_launches++;
     }
@@ -1184,6 +1189,24 @@ int close_impl(wt_handle *h) {
 
 int wt::set_error(int code, const char *msg) { return set_err(code, "%s", msg); }
 
+bool wt::fault_injected(const char *site) {
+  const char *e = getenv("WT_FAULT");
+  if (!e || !*e) return false;
+  static std::mutex mu;
+  static std::string last;
+  static int count = 0;
+  std::lock_guard<std::mutex> g(mu);
+  if (last != e) {
+    last = e;
+    count = 0;
+  }
+  const char *colon = strchr(e, ':');
+  const size_t len = colon ? (size_t)(colon - e) : strlen(e);
+  if (len != strlen(site) || strncmp(e, site, len) != 0) return false;
+  const int n = colon ? atoi(colon + 1) : 1;
+  return ++count == n;
+}
+
 // ====================================================================== C ABI
 #pragma GCC visibility push(default)
 extern "C" {
@@ -1261,8 +1284,10 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
         f.route = WT_ROUTE_DIRECT;
         f.dev = f.base;
       } else if (want == WT_ROUTE_REGISTER) {
-        cudaError_t e = cudaHostRegister(f.base, f.size, cudaHostRegisterMapped | cudaHostRegisterReadOnly);
-        if (e != cudaSuccess) {
+        const bool injected = wt::fault_injected("register");
+        cudaError_t e = injected ? cudaErrorMemoryAllocation
+                                 : cudaHostRegister(f.base, f.size, cudaHostRegisterMapped | cudaHostRegisterReadOnly);
+        if (e != cudaSuccess && !injected) {
           cudaGetLastError();
           e = cudaHostRegister(f.base, f.size, cudaHostRegisterMapped);
         }

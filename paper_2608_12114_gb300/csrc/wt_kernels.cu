@@ -444,7 +444,7 @@ __device__ __forceinline__ bool block_rows_dispatch(uint32_t nj, uint32_t nr, ui
 template <int DT>
 __global__ void __launch_bounds__(kGemvThreads, 1)
     gemv_tma_kernel(const MatDesc *__restrict__ mats, const Piece *__restrict__ pieces,
-                    const uint32_t *__restrict__ begin, int *status) {
+                    const uint32_t *__restrict__ begin, int *status, int stall) {
   constexpr int NP = Pairs<DT>::N;
   extern __shared__ __align__(128) uint8_t smem[];
   const uint32_t stage0 = smem_u32(smem);
@@ -470,7 +470,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
 
   if (warp == kConsumerWarps) {
     // ---------------- producer: one thread issues every bulk copy of the CTA
-    if (lane == 0) {
+    if (lane == 0 && !stall) {
       const uint64_t pol = l2_evict_first_policy();
       uint32_t it = 0;
       bool live = true;
@@ -970,10 +970,10 @@ cudaError_t gemv_prepare() {
 cudaError_t launch_gemv(const GemvLaunch &L, cudaStream_t s) {
   if (L.grid <= 0) return cudaSuccess;
   switch (L.dtype) {
-    case 0: gemv_tma_kernel<0><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
-    case 1: gemv_tma_kernel<1><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
-    case 2: gemv_tma_kernel<2><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
-    case 3: gemv_tma_kernel<3><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status); break;
+    case 0: gemv_tma_kernel<0><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
+    case 1: gemv_tma_kernel<1><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
+    case 2: gemv_tma_kernel<2><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
+    case 3: gemv_tma_kernel<3><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();

@@ -103,6 +103,8 @@ struct GemvLaunch {
   int *status;             // device status word (bounded-wait failures)
   const uint8_t *maps = nullptr;  // multi-column kernel: one TMA tensor map per MatDesc
                                   // (kTensorMapBytes each, 128-byte aligned, device)
+  int stall = 0;  // failure test (host fault site "stall"): the producer issues no copy, so
+                  // every consumer wait runs out, reports WT_ETIMEDOUT and the CTA exits
 };
 
 cudaError_t gemv_prepare();  // one-time function attributes
@@ -172,6 +174,12 @@ int num_sms();  // of the current device (cached per device)
 
 // Records `msg` as this thread's wt_last_error() text and returns `code`.
 int set_error(int code, const char *msg);
+
+// Host-side fault injection (tests): true when WT_FAULT="<site>[:<n>]" names this site and
+// this is its n-th call (n = 1 by default) since the variable last changed.  Sites: open,
+// pread, mmap, register, alloc (the call fails as if the system or CUDA call had), and stall
+// (a resident GEMV launch whose producer issues nothing: its bounded waits run out).
+bool fault_injected(const char *site);
 
 }  // namespace wt
 
