@@ -168,8 +168,9 @@ int wt_file_route(const wt_handle *h, size_t f, unsigned *route);
  * stream, ready[i] also implies every earlier tensor of this call.  STAGED
  * mode blocks the calling thread until every byte has left the page cache
  * (the copy engine may still be draining the last slots).
- * Errors: WT_EINVAL (index, null, overlap with a mapping), WT_ENOTSUP (mode
- * needs a device route the file lacks), WT_ENOMEM, WT_ECUDA. */
+ * Errors: WT_EINVAL (index, null, overlap with a mapping, a dst that starts in a device
+ * allocation and runs past its end), WT_ENOTSUP (mode needs a device route the file
+ * lacks), WT_ENOMEM, WT_ECUDA. */
 int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsigned mode,
              void *stream, void **ready);
 
@@ -193,7 +194,8 @@ int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsign
  * kept until wt_close; every replay must complete before wt_close.
  *
  * Errors: WT_EINVAL (null pointer with M*K > 0, cols outside 0..16, dimension > 2^31-1, a
- * capture without the warm-up call), WT_ENOTSUP (dtype), WT_ENOMEM, WT_ECUDA. */
+ * capture without the warm-up call, an operand that starts in a device allocation and runs
+ * past its end), WT_ENOTSUP (dtype), WT_ENOMEM, WT_ECUDA. */
 int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream);
 
 /* Leaf-tree FNV-1a-64 digest of each device buffer ptr[i] (nbytes[i] bytes),

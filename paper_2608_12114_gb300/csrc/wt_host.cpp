@@ -854,6 +854,43 @@ int validate_desc(const wt_gemv_desc &d, size_t i) {
   return WT_OK;
 }
 
+// Bounds of device buffers, checked on the host before anything is enqueued: a range that
+// starts in a device allocation must end inside it (cuMemGetAddressRange, looked up once
+// through the runtime).  The last allocation seen is cached, so a slab of many tensors costs
+// one query.  Host memory (mappings, pinned buffers) cannot be asked and passes; mappings
+// have their own checks.
+struct RangeCache {
+  uintptr_t lo = 0, hi = 0;
+};
+
+using AddrRangeFn = CUresult (*)(CUdeviceptr *, size_t *, CUdeviceptr);
+
+AddrRangeFn addr_range_fn() {
+  static AddrRangeFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuMemGetAddressRange", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<AddrRangeFn>(p);
+  });
+  return fn;
+}
+
+// false only when [p, p + n) starts inside a device allocation and runs past its end
+bool device_range_ok(const void *p, uint64_t n, RangeCache &c) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+  if (n == 0 || (a >= c.lo && a + n <= c.hi && a + n >= a)) return true;
+  AddrRangeFn fn = addr_range_fn();
+  CUdeviceptr base = 0;
+  size_t size = 0;
+  if (!fn || fn(&base, &size, (CUdeviceptr)a) != CUDA_SUCCESS) return true;
+  c.lo = (uintptr_t)base;
+  c.hi = (uintptr_t)base + size;
+  return a + n <= c.hi && a + n >= a;
+}
+
 // Where W lives: 0 = device memory (cudaMalloc, a memory pool, managed): the TMA kernels
 // stream from there; 1 = host memory the device can load from (pinned or registered, or
 // pageable where the device reads through the host page tables); -1 = neither.
@@ -891,10 +928,19 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
     std::vector<int64_t> seg_ws[4];  // per by_dt entry: workspace float offset of its partials, or -1
     std::vector<wt::SegReduce> reds;
     std::vector<size_t> red_ws;      // per reds entry: workspace float offset
+    RangeCache rcw, rcx, rcy, rcs;
     for (size_t k = i; k < j; ++k) {
       const wt_gemv_desc &q = d[k];
       if (q.M == 0) continue;
       const int es = elem_bytes(q.dtype);
+      {
+        // every operand that starts in a device allocation must end inside it
+        const uint64_t T = q.cols > 0 ? (uint64_t)q.cols : 1;
+        const uint64_t xes = q.dtype == WT_I8 ? 2 : (uint64_t)es;
+        if (!device_range_ok(q.y, q.M * T * 4, rcy) || !device_range_ok(q.W, q.M * q.K * es, rcw) ||
+            !device_range_ok(q.x, q.K * T * xes, rcx) || (q.scale && !device_range_ok(q.scale, q.M * 2, rcs)))
+          return set_err(WT_EINVAL, "wt_pass: an operand of desc %zu runs past the end of its device allocation", k);
+      }
       const uint32_t ncol = q.cols > 0 ? (uint32_t)q.cols : 1;
       if (q.K == 0) {
         g.zero.push_back({q.y, q.M * ncol});
@@ -1398,6 +1444,7 @@ int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsign
     std::vector<Range> rs;
     rs.reserve(n);
     uint64_t total = 0;
+    RangeCache rc_dst;
     for (size_t k = 0; k < n; ++k) {
       if (idx[k] >= h->order.size()) return set_err(WT_EINVAL, "wt_adopt: tensor index %zu out of range", idx[k]);
       const File &f = h->files[h->order[idx[k]].first];
@@ -1405,6 +1452,9 @@ int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsign
       if (t.nbytes && !dst[k]) return set_err(WT_EINVAL, "wt_adopt: dst[%zu] is NULL", k);
       if (t.nbytes && inside_mapping(h, dst[k], t.nbytes))
         return set_err(WT_EINVAL, "wt_adopt: dst[%zu] lies inside a read-only mapping", k);
+      if (!device_range_ok(dst[k], t.nbytes, rc_dst))
+        return set_err(WT_EINVAL, "wt_adopt: dst[%zu] (%llu bytes) runs past the end of its device allocation", k,
+                       (unsigned long long)t.nbytes);
       if (mode != WT_ADOPT_STAGED && f.route == WT_ROUTE_NONE)
         return set_err(WT_ENOTSUP, "wt_adopt: %s has no device route; use WT_ADOPT_STAGED", f.path.c_str());
       ready[k] = nullptr;

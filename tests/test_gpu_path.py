@@ -298,3 +298,29 @@ def test_descriptor_bounds_are_refused_before_any_launch(torch):
             h.pass_([wt.gemv_desc(x.data_ptr(), wt.WT_BF16, 4, 16, x.data_ptr(), 0)], 0)
         assert ei.value.code == wt.WT_EINVAL
         assert h.kernel_launches() == n0 and h.device_status() == 0
+
+
+def test_device_overruns_are_refused_on_the_host(torch, tmp_path):
+    """A destination or operand that starts in a device allocation and runs past its end is
+    refused before anything is enqueued (no out-of-bounds GPU access is ever attempted)."""
+    ck = synth.write_files(synth.custom(str(tmp_path), [(1024, 8192)], name="big"))   # 16 MiB bf16
+    small = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")   # a 1 MiB block of a small segment
+    with wt.Handle(ck.paths) as h:
+        n0 = h.kernel_launches()
+        with pytest.raises(wt.WtError) as ei:
+            h.adopt([0], [small.data_ptr()], wt.WT_ADOPT_GATHER, 0)
+        assert ei.value.code == wt.WT_EINVAL and "past the end" in str(ei.value)
+        x = torch.zeros(8192, dtype=torch.bfloat16, device="cuda")
+        y = torch.zeros(16, dtype=torch.float32, device="cuda")
+        W = torch.zeros(1024 * 8192, dtype=torch.bfloat16, device="cuda")
+        for M, K, Wp, yp in ((1 << 20, 8192, W.data_ptr(), y.data_ptr()),     # y far too short
+                             (65536, 8192, small.data_ptr(), W.data_ptr())):  # W far too short
+            with pytest.raises(wt.WtError) as ei:
+                h.pass_([wt.gemv_desc(Wp, wt.WT_BF16, M, K, x.data_ptr(), yp)], 0)
+            assert ei.value.code == wt.WT_EINVAL and "past the end" in str(ei.value)
+        assert h.kernel_launches() == n0 and h.device_status() == 0
+        big = torch.empty(16 << 20, dtype=torch.uint8, device="cuda")     # right size: accepted
+        torch.cuda.synchronize()
+        h.adopt([0], [big.data_ptr()], wt.WT_ADOPT_GATHER, 0)
+        torch.cuda.synchronize()
+        assert h.device_status() == 0
