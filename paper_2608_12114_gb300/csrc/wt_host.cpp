@@ -629,9 +629,11 @@ wt::MatDesc make_mat(const wt_gemv_desc &d) {
     m.rt = std::min<uint32_t>(wt::kRowBlock, wt::kStageBytes / rowb);
     m.vc = m.V;
   } else {
-    m.mode = wt::kModeSplitK;
-    m.rt = wt::kRowBlock;
-    m.vc = wt::kStageBytes / (wt::kRowBlock * 16);
+    // the plain-load kernels read such rows directly; the TMA kernel gets them only as
+    // column segments of at most seg_vectors vectors (make_seg_mat)
+    m.mode = wt::kModeLongRows;
+    m.rt = 1;
+    m.vc = m.V;
   }
   return m;
 }
@@ -1049,6 +1051,10 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
           g.cols.push_back(L);
           continue;
         }
+        if (pass == 0)
+          for (const wt::MatDesc &m : ms)
+            if (m.mode != wt::kModeWarpRows && m.mode != wt::kModeBlockRows)
+              return set_err(WT_ENOTSUP, "wt_pass: internal: a %u-vector row reached the TMA kernel unsegmented", m.V);
         partition(ms, L.grid, pieces, begin, pass == 2 ? (uint32_t)wt::kColTileRows : 1u,
                   pass == 0 ? one_col_slices(dt) : 1);
         L.mapped_cols = pass == 4;

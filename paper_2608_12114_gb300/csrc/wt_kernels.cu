@@ -407,15 +407,6 @@ __device__ __forceinline__ void tile_block_rows(uint32_t tile, uint32_t V, int c
   if ((lane & ((32 >> L) - 1)) == 0 && q < NR) rb[q * kConsumerWarps + warp] = sum;
 }
 
-// Rows per tile for a piece of `rows` rows.  Split-K pieces use balanced row blocks of at
-// most kRowBlock rows (27 rows -> 7, 7, 7, 6), so no stage of the piece runs nearly empty.
-__device__ __forceinline__ uint32_t piece_rows_per_tile(const MatDesc &md, const Piece &pc) {
-  if (md.mode != kModeSplitK) return md.rt;
-  const uint32_t rows = pc.r1 - pc.r0;
-  const uint32_t nblk = (rows + kRowBlock - 1) / kRowBlock;
-  return nblk ? (rows + nblk - 1) / nblk : 1;
-}
-
 // Sum of the consumer warps' partials of one row, in warp order (deterministic).
 __device__ __forceinline__ float sum_warps(const float *p) {
   float t = 0.f;
@@ -477,38 +468,24 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
       for (uint32_t pi = p0; pi < p1 && live; ++pi) {
         const Piece pc = pieces[pi];
         const MatDesc md = mats[pc.mat];
-        const uint64_t rowb = (uint64_t)md.rs * 16;  // row pitch (== V * 16 outside split-K segments)
-        const uint32_t rt = piece_rows_per_tile(md, pc);
-        for (uint32_t r = pc.r0; r < pc.r1 && live; r += rt) {
-          const uint32_t nr = min(rt, pc.r1 - r);
-          const uint32_t nchunk = md.mode == kModeSplitK ? (md.V + md.vc - 1) / md.vc : 1;
-          for (uint32_t c = 0; c < nchunk; ++c) {
-            const uint32_t s = it % kStages;
-            if (it >= kStages &&
-                !bounded_wait(empty0 + 8 * s, ((it / kStages) - 1) & 1, abort_flag, status)) {
-              live = false;
-              break;
-            }
-            const uint32_t dst = stage0 + s * kStageBytes;
-            const uint32_t bar = full0 + 8 * s;
-            if (md.mode != kModeSplitK) {
-              const uint32_t vb = md.V * 16;  // tile rows sit at V * 16 pitch in shared memory
-              mbar_expect_tx(bar, nr * vb);
-              if (md.rs == md.V) {
-                bulk_g2s(dst, md.W + (uint64_t)r * rowb, nr * vb, bar, pol);
-              } else {
-                for (uint32_t q = 0; q < nr; ++q) bulk_g2s(dst + q * vb, md.W + (uint64_t)(r + q) * rowb, vb, bar, pol);
-              }
-            } else {
-              const uint32_t v0 = c * md.vc;
-              const uint32_t nv = min(md.vc, md.V - v0);
-              mbar_expect_tx(bar, nr * nv * 16);
-              for (uint32_t q = 0; q < nr; ++q)
-                bulk_g2s(dst + q * md.vc * 16, md.W + (uint64_t)(r + q) * rowb + (uint64_t)v0 * 16,
-                         nv * 16, bar, pol);
-            }
-            ++it;
+        const uint64_t rowb = (uint64_t)md.rs * 16;  // row pitch (the full row for a column segment)
+        const uint32_t vb = md.V * 16;                // tile rows sit at V * 16 pitch in shared memory
+        for (uint32_t r = pc.r0; r < pc.r1 && live; r += md.rt) {
+          const uint32_t nr = min(md.rt, pc.r1 - r);
+          const uint32_t s = it % kStages;
+          if (it >= kStages && !bounded_wait(empty0 + 8 * s, ((it / kStages) - 1) & 1, abort_flag, status)) {
+            live = false;
+            break;
           }
+          const uint32_t dst = stage0 + s * kStageBytes;
+          const uint32_t bar = full0 + 8 * s;
+          mbar_expect_tx(bar, nr * vb);
+          if (md.rs == md.V) {
+            bulk_g2s(dst, md.W + (uint64_t)r * rowb, nr * vb, bar, pol);  // contiguous rows: one copy
+          } else {
+            for (uint32_t q = 0; q < nr; ++q) bulk_g2s(dst + q * vb, md.W + (uint64_t)(r + q) * rowb, vb, bar, pol);
+          }
+          ++it;
         }
       }
       if (!live || *abort_flag) {
@@ -604,46 +581,6 @@ __global__ void __launch_bounds__(kGemvThreads, 1)
             g0 += gn;
             gn = 0;
           }
-        }
-      } else {
-        // split-K: row blocks of up to kRowBlock rows, streamed in column chunks of md.vc
-        // vectors; the x slice of the next chunk is fetched while the current one is used.
-        const uint32_t nchunk = (V + md.vc - 1) / md.vc;
-        const uint32_t rt = piece_rows_per_tile(md, pc);
-        load_xpairs<DT>(md.x, ct, (uint32_t)ct < min(md.vc, V), xp[0]);
-        for (uint32_t r = pc.r0; r < pc.r1; r += rt) {
-          const uint32_t nr = min(rt, pc.r1 - r);
-          Acc4 acc[kRowBlock];
-          for (uint32_t c = 0; c < nchunk; ++c) {
-            const uint32_t nv = min(md.vc, V - c * md.vc);
-            const uint32_t c1 = c + 1 < nchunk ? c + 1 : 0;  // next chunk (or chunk 0 of the next block)
-            const uint32_t nv1 = min(md.vc, V - c1 * md.vc);
-            load_xpairs<DT>(md.x, c1 * md.vc + ct, (uint32_t)ct < nv1, xp[1]);
-            const uint32_t s = it % kStages;
-            bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
-            const uint32_t tile = stage0 + s * kStageBytes;
-            uint4 w[kRowBlock];
-#pragma unroll
-            for (int q = 0; q < kRowBlock; ++q)
-              w[q] = lds_or_zero(tile + (q * md.vc + ct) * 16, q < (int)nr && (uint32_t)ct < nv);
-#pragma unroll
-            for (int q = 0; q < kRowBlock; ++q) dot16<DT>(w[q], xp[0], acc[q]);
-            __syncwarp();
-            if (lane == 0) mbar_arrive(empty0 + 8 * s);
-            ++it;
-#pragma unroll
-            for (int i = 0; i < NP; ++i) xp[0][i] = xp[1][i];
-          }
-          float t[kRowBlock];
-#pragma unroll
-          for (int q = 0; q < kRowBlock; ++q) t[q] = acc[q].total();
-          float *rb = red + par * (kConsumerWarps * kRedRows);
-          const float sum = transpose_reduce<kRowBlock>(t, lane);
-          const int q = lane >> 2;
-          if ((lane & 3) == 0 && q < (int)nr) rb[q * kConsumerWarps + warp] = sum;
-          named_bar(1, kConsumers);
-          if (ct < (int)nr) md.y[r + ct] = sum_warps(rb + ct * kConsumerWarps) * row_scale<DT>(md.s, r + ct);
-          par ^= 1;
         }
       }
     }

@@ -31,12 +31,12 @@ cudaError_t launch_gather(const GatherBatch &b, int grid, cudaStream_t s);
 constexpr int kStageBytes = 32768;
 constexpr int kStages = 6;
 constexpr int kConsumerWarps = 8;
-constexpr int kRowBlock = 8;  // rows of a block-mode tile / split-K row block
+constexpr int kRowBlock = 8;  // rows of a block-mode tile
 
 enum GemvMode : uint16_t {
   kModeWarpRows = 0,   // rows of <= 256 vectors: each warp owns whole rows
   kModeBlockRows = 1,  // 256 < vectors <= kStageBytes/16: whole CTA per row, full-row tiles
-  kModeSplitK = 2,     // longer rows: row blocks of kRowBlock rows x 4 KiB column chunks
+  kModeLongRows = 2,   // rows longer than one stage: split into column segments before any TMA launch
   kModeCols = 3,       // multi-column kernel (G = T columns): 16-row tiles x vc-vector chunks
 };
 
