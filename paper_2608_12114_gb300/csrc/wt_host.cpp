@@ -783,9 +783,10 @@ int encode_umma_maps(const wt::MatDesc &m, uint8_t *out) {
 
 // Split the rows of `mats` (in order) into grid * slices contiguous slices of nearly
 // equal bytes, cut at row boundaries; slice j goes to CTA j % grid, so every CTA streams
-// `slices` slices spread over the whole set and gets a similar mix of shapes.
+// `slices` slices spread over the whole set and gets a similar mix of shapes.  The grid is
+// at most ctas_per_sm CTAs per SM (all resident at once: the launch is persistent).
 void partition(const std::vector<wt::MatDesc> &mats, int &grid, std::vector<wt::Piece> &pieces,
-               std::vector<uint32_t> &begin, uint32_t row_align = 1, int slices = 1) {
+               std::vector<uint32_t> &begin, uint32_t row_align = 1, int slices = 1, int ctas_per_sm = 1) {
   uint64_t B = 0;
   std::vector<uint64_t> start(mats.size() + 1, 0);
   for (size_t i = 0; i < mats.size(); ++i) {
@@ -794,7 +795,8 @@ void partition(const std::vector<wt::MatDesc> &mats, int &grid, std::vector<wt::
   }
   start[mats.size()] = B;
   constexpr uint64_t kMinCtaBytes = 64 << 10;
-  grid = (int)std::max<uint64_t>(1, std::min<uint64_t>((uint64_t)wt::num_sms(), (B + kMinCtaBytes - 1) / kMinCtaBytes));
+  grid = (int)std::max<uint64_t>(
+      1, std::min<uint64_t>((uint64_t)wt::num_sms() * ctas_per_sm, (B + kMinCtaBytes - 1) / kMinCtaBytes));
   // slices of at least kMinSliceBytes: a slice costs the consumers a reload of x, and a
   // slice shorter than a tile makes its stages partial
   constexpr uint64_t kMinSliceBytes = 2ull << 20;
@@ -1056,7 +1058,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
             if (m.mode != wt::kModeWarpRows && m.mode != wt::kModeBlockRows)
               return set_err(WT_ENOTSUP, "wt_pass: internal: a %u-vector row reached the TMA kernel unsegmented", m.V);
         partition(ms, L.grid, pieces, begin, pass == 2 ? (uint32_t)wt::kColTileRows : 1u,
-                  pass == 0 ? one_col_slices(dt) : 1);
+                  pass == 0 ? one_col_slices(dt) : 1, pass == 0 ? wt::gemv_ctas_per_sm(dt) : 1);
         L.mapped_cols = pass == 4;
         L.mats = append(P->table, ms);
         if (pass == 0)

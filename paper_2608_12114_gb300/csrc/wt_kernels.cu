@@ -155,11 +155,22 @@ __global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ Gat
 // ------------------------------------------------------------------ GEMV
 constexpr int kConsumers = kConsumerWarps * 32;
 constexpr int kGemvThreads = kConsumers + 32;
-constexpr size_t kBarOff = (size_t)kStages * kStageBytes;
-constexpr size_t kRedOff = kBarOff + 2 * kStages * sizeof(uint64_t);
 constexpr int kRedRows = 64;  // rows whose warp partials are gathered before one cross-warp sum
-constexpr size_t kFlagOff = kRedOff + 2 * kConsumerWarps * kRedRows * sizeof(float);
-constexpr size_t kGemvSmem = kFlagOff + 16;
+
+// Shared-memory layout of one CTA: the stage ring, its full/empty barriers, the cross-warp
+// partials and the abort flag.  int8 weights run two CTAs per SM with half the ring each
+// (the same bytes in flight per SM, twice the warps: that path is latency-bound on its
+// decode, not on HBM).
+template <int DT>
+struct GemvGeo {
+  static constexpr int kCtasPerSm = DT == 3 ? 2 : 1;
+  static constexpr int kStages = DT == 3 ? 3 : 6;
+  static constexpr size_t kBarOff = (size_t)kStages * kStageBytes;
+  static constexpr size_t kRedOff = kBarOff + 2 * kStages * sizeof(uint64_t);
+  static constexpr size_t kFlagOff = kRedOff + 2 * kConsumerWarps * kRedRows * sizeof(float);
+  static constexpr size_t kSmem = kFlagOff + 16;
+};
+static_assert(GemvGeo<1>::kSmem <= 232448 && 2 * (GemvGeo<3>::kSmem + 1024) <= 233472, "GEMV shared memory");
 
 // Two fp32 values in one 64-bit register; fma.rn.f32x2 performs two independent
 // round-to-nearest FMAs (the same arithmetic as two fmaf calls) in one instruction.
@@ -433,16 +444,17 @@ __device__ __forceinline__ bool block_rows_dispatch(uint32_t nj, uint32_t nr, ui
 }
 
 template <int DT>
-__global__ void __launch_bounds__(kGemvThreads, 1)
+__global__ void __launch_bounds__(kGemvThreads, GemvGeo<DT>::kCtasPerSm)
     gemv_tma_kernel(const MatDesc *__restrict__ mats, const Piece *__restrict__ pieces,
                     const uint32_t *__restrict__ begin, int *status, int stall) {
   constexpr int NP = Pairs<DT>::N;
+  constexpr int kStages = GemvGeo<DT>::kStages;
   extern __shared__ __align__(128) uint8_t smem[];
   const uint32_t stage0 = smem_u32(smem);
-  const uint32_t full0 = smem_u32(smem + kBarOff);
+  const uint32_t full0 = smem_u32(smem + GemvGeo<DT>::kBarOff);
   const uint32_t empty0 = full0 + kStages * 8;
-  float *red = reinterpret_cast<float *>(smem + kRedOff);
-  volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + kFlagOff);
+  float *red = reinterpret_cast<float *>(smem + GemvGeo<DT>::kRedOff);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + GemvGeo<DT>::kFlagOff);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -894,23 +906,28 @@ cudaError_t launch_gather(const GatherBatch &b, int grid, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-size_t gemv_smem_bytes() { return kGemvSmem; }
+size_t gemv_smem_bytes(int dtype) { return dtype == 3 ? GemvGeo<3>::kSmem : GemvGeo<1>::kSmem; }
+int gemv_ctas_per_sm(int dtype) { return dtype == 3 ? GemvGeo<3>::kCtasPerSm : GemvGeo<1>::kCtasPerSm; }
+
+template <int DT>
+static cudaError_t gemv_attr() {
+  return cudaFuncSetAttribute(gemv_tma_kernel<DT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)GemvGeo<DT>::kSmem);
+}
 
 cudaError_t gemv_prepare() {
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(gemv_tma_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemvSmem)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(gemv_tma_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemvSmem)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(gemv_tma_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemvSmem)) != cudaSuccess) return e;
-  return cudaFuncSetAttribute(gemv_tma_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemvSmem);
+  if ((e = gemv_attr<0>()) != cudaSuccess || (e = gemv_attr<1>()) != cudaSuccess || (e = gemv_attr<2>()) != cudaSuccess)
+    return e;
+  return gemv_attr<3>();
 }
 
 cudaError_t launch_gemv(const GemvLaunch &L, cudaStream_t s) {
   if (L.grid <= 0) return cudaSuccess;
   switch (L.dtype) {
-    case 0: gemv_tma_kernel<0><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
-    case 1: gemv_tma_kernel<1><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
-    case 2: gemv_tma_kernel<2><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
-    case 3: gemv_tma_kernel<3><<<L.grid, kGemvThreads, kGemvSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
+    case 0: gemv_tma_kernel<0><<<L.grid, kGemvThreads, GemvGeo<0>::kSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
+    case 1: gemv_tma_kernel<1><<<L.grid, kGemvThreads, GemvGeo<1>::kSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
+    case 2: gemv_tma_kernel<2><<<L.grid, kGemvThreads, GemvGeo<2>::kSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
+    case 3: gemv_tma_kernel<3><<<L.grid, kGemvThreads, GemvGeo<3>::kSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();

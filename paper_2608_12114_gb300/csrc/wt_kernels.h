@@ -29,7 +29,6 @@ cudaError_t launch_gather(const GatherBatch &b, int grid, cudaStream_t s);
 // ---------------------------------------------------------------- GEMV
 // Tile geometry.  A stage is one TMA bulk transfer target in shared memory.
 constexpr int kStageBytes = 32768;
-constexpr int kStages = 6;
 constexpr int kConsumerWarps = 8;
 constexpr int kRowBlock = 8;  // rows of a block-mode tile
 
@@ -109,7 +108,8 @@ struct GemvLaunch {
 
 cudaError_t gemv_prepare();  // one-time function attributes
 cudaError_t launch_gemv(const GemvLaunch &L, cudaStream_t s);
-size_t gemv_smem_bytes();
+size_t gemv_smem_bytes(int dtype);
+int gemv_ctas_per_sm(int dtype);  // resident CTAs per SM the one-column launch is sized for
 
 // Map endpoint (the paper's adoption, contract C1): W is read in place from a file mapping
 // the device reaches over the host link, with 16-byte loads and no TMA; same tables as
