@@ -616,9 +616,9 @@ wt::MatDesc make_mat(const wt_gemv_desc &d) {
   m.V = (uint32_t)(d.K * es / 16);
   m.rs = m.V;
   const uint32_t rowb = m.V * 16;
-  // a consumer thread keeps at most 8 (bf16/f16/f32) or 4 (int8: 16 f16 activations per
-  // weight vector) x vectors in registers; the mode limits follow from that
-  const uint32_t xj = d.dtype == WT_I8 ? 4 : 8;
+  // a consumer thread keeps at most 8 (bf16/f16/f32) or 2 (int8: 16 f16 activations per
+  // weight vector, two CTAs per SM) x vectors in registers; the mode limits follow from that
+  const uint32_t xj = d.dtype == WT_I8 ? 2 : 8;
   if (m.V <= 32 * xj) {
     m.mode = wt::kModeWarpRows;
     m.G = (uint16_t)(m.V <= 32 ? pow2ceil(m.V) : 32);

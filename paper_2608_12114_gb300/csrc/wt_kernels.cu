@@ -93,10 +93,12 @@ struct XElem {
   static constexpr int value = DT == 3 ? 2 : DT;
 };
 
-// x vectors a consumer thread keeps in registers (16-byte weight vectors it covers).
+// x vectors a consumer thread keeps in registers (16-byte weight vectors it covers).  An
+// int8 vector needs 32 bytes of f16 x, and the int8 kernel runs two CTAs per SM under a
+// 96-register cap, so it keeps two (rows of up to 512 vectors; longer ones are segmented).
 template <int DT>
 struct XJ {
-  static constexpr int value = DT == 3 ? 4 : 8;
+  static constexpr int value = DT == 3 ? 2 : 8;
 };
 
 // Vector counts above XJ never reach a kernel of that type (the planner keeps them out);

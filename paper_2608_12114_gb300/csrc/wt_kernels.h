@@ -72,7 +72,7 @@ static_assert(sizeof(MatDesc) == 64, "MatDesc is one 64-byte record");
 // depend only on the matrix, so a row's result never depends on how rows and segments were
 // spread over CTAs.
 constexpr uint32_t kSegVec = 2048;  // bf16 / f16 / f32: 32 KB per segment row
-constexpr uint32_t seg_vectors(int dtype) { return dtype == 3 ? kSegVec / 2 : kSegVec; }
+constexpr uint32_t seg_vectors(int dtype) { return dtype == 3 ? kSegVec / 4 : kSegVec; }  // int8: 8 KB
 
 struct alignas(16) SegReduce {
   const float *ws;   // nseg x M partial sums (segment-major)

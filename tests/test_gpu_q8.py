@@ -10,9 +10,10 @@ from paper_2608_12114_gb300 import build, pipeline, synth, wt
 pytestmark = pytest.mark.gpu
 TOL = 2e-3
 
-# vectors per row V = K / 16: warp rows (V <= 128, lane groups of 1..16 and 32), block rows
-# (128 < V <= 1024, 1..4 vectors per thread), split-K (V > 1024), and K % 16 != 0 (fallback)
-SHAPES = [(9, 16), (33, 48), (100, 512), (40, 2048), (17, 2064), (11, 4096), (7, 7168), (5, 12288),
+# vectors per row V = K / 16: warp rows (V <= 64, lane groups of 1..16 and 32, 1..2 vectors
+# per lane), block rows (64 < V <= 512, 1..2 vectors per thread), split-K (V > 512), and
+# K % 16 != 0 (fallback)
+SHAPES = [(9, 16), (33, 48), (100, 512), (13, 960), (40, 2048), (17, 2064), (11, 4096), (7, 7168), (5, 12288),
           (3, 16384), (6, 16400), (2, 65536), (4, 24), (0, 32), (3, 0)]
 
 

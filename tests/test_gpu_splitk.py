@@ -10,11 +10,11 @@ pytestmark = pytest.mark.gpu
 TOL = 2e-3
 F32, BF16, F16, I8 = wt.WT_F32, wt.WT_BF16, wt.WT_F16, wt.WT_I8
 
-# (dtype, M, K): V = K * es / 16 vectors per row, cut into ceil(V / 2048) (int8: 1024)
+# (dtype, M, K): V = K * es / 16 vectors per row, cut into ceil(V / 2048) (int8: 512)
 # segments of nearly equal length
 SHAPES = [(BF16, 1, 8 * 1024 * 1024),      # V = 1,048,576: 512 one-row segments
           (BF16, 5, 65544),                 # V = 8193: 5 segments, the last shorter
-          (I8, 3, 600000),                  # V = 37500: 37 segments
+          (I8, 3, 600000),                  # V = 37500: 74 segments
           (F32, 2, 1048580),                # V = 262145: 129 segments
           (F16, 9, 40000),                  # V = 5000: 3 segments
           (BF16, 17, 32768),                # V = 4096: 2 segments
