@@ -73,6 +73,8 @@ def parse_args():
     p.add_argument("--tsweep", default=None, metavar="T,T,...",
                    help="multi-column T-sweep (e.g. 0,1,2,4,8,16; 0 = the one-column kernel) on the "
                         "int8 matched protocol by default (one JSON line)")
+    p.add_argument("--checksum", action="store_true",
+                   help="time wt_checksum (leaf-tree FNV-1a-64) over every resident tensor of the workload")
     p.add_argument("--policy", action="store_true",
                    help="measure the map / resident / per-use-copy endpoints and apply Algorithm 2 (one JSON line)")
     return p.parse_args()
@@ -810,6 +812,73 @@ def run_tsweep(args):
     print(json.dumps(out), flush=True)
 
 
+# Issue peak of the SMs: 152 SMs x 4 schedulers x one warp instruction (32 lanes) per clock.
+# FNV-1a-64 is integer ALU work, so its ceiling is this rate divided by the instructions the
+# kernel spends per byte (ncu's smsp__inst_executed x 32 / bytes), or HBM, whichever is lower.
+def issue_peak_lane_ops(sm_mhz, sms=152):
+    return sms * 4 * 32 * sm_mhz * 1e6
+
+
+def run_checksum(args):
+    """Step 9 measured: wt_checksum (per-tensor FNV-1a-64 leaf digests plus the combine pass)
+    over every tensor of the workload, resident in HBM, CUDA events over `steps` calls on the
+    launching stream.  Digests are verification: this is their throughput, outside the
+    first-use and resident-pass figures."""
+    ck, gen_s = make_files(args, 0, 1)
+    import torch
+    from paper_2608_12114_gb300 import build, pipeline, wt
+    build.build()
+    torch.cuda.set_device(0)
+    h = wt.Handle(ck.paths)
+    mats = pipeline.matrices(h)
+    dev = pipeline.DeviceCheckpoint.allocate(h, mats)
+    s = torch.cuda.Stream()
+    dev.adopt(h, wt.WT_ADOPT_GATHER, s.cuda_stream)
+    s.synchronize()
+    idx = sorted(dev.dst)
+    ptrs = [dev.dst[i] for i in idx]
+    nb = [h.tensors[i].nbytes for i in idx]
+    total = sum(nb)
+    out = torch.zeros(len(idx), dtype=torch.int64, device="cuda")
+    base = out.data_ptr()
+    outs = [base + 8 * j for j in range(len(idx))]
+
+    def call():
+        h.checksum(ptrs, nb, base, s.cuda_stream)
+
+    for _ in range(max(3, args.warmup)):
+        call()
+    s.synchronize()
+    first = out.clone()
+    steps = max(1, min(args.steps, 50))
+    n0 = h.kernel_launches()
+    with Clocks(bus_id()) as clk:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(s)
+        for _ in range(steps):
+            call()
+        e1.record(s)
+        s.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    launches = (h.kernel_launches() - n0) / steps
+    stable = bool(torch.equal(first, out))
+    h.close()
+    peak, peak_kind = measured_peaks()
+    gbs = total / ms / 1e6
+    csum = clk.summary()
+    row = {"metric": "per-tensor FNV-1a-64 digest throughput (wt_checksum, leaf tree)", "value": round(gbs, 1),
+           "unit": "GB/s", "ms_per_call": round(ms, 4), "bytes_per_call": total, "tensors": len(idx),
+           "launches_per_call": launches, "digests_repeat": stable, "frac_of_hbm": round(gbs / peak, 4),
+           "peak_hbm_gbs": peak, "peak_kind": peak_kind,
+           "issue_peak_lane_ops_per_s": issue_peak_lane_ops(csum.get("sm_mhz") or 2070.0),
+           "config": {"workload": workload_desc(args), "steps": steps, "l2": "inputs larger than L2 (no flush)"
+                      if total > L2_BYTES else "inputs smaller than L2"},
+           "clocks": csum}
+    log("checksum: %.4f ms per call, %.1f GB/s (%.1f%% of %s HBM), %d launches, digests repeat: %s" % (
+        ms, gbs, 100 * gbs / peak, peak_kind, launches, stable))
+    print(json.dumps(row), flush=True)
+
+
 def main():
     args = parse_args()
     rank = int(os.environ.get("RANK", "0"))
@@ -825,6 +894,9 @@ def main():
         return
     if args.cube:
         run_cube(args)
+        return
+    if args.checksum:
+        run_checksum(args)
         return
     run_wt(args, rank, world)
 
