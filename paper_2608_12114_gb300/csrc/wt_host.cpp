@@ -30,6 +30,7 @@
 #include <string>
 #include <thread>
 #include <unordered_set>
+#include <memory>
 #include <vector>
 
 #include <cuda.h>  // CUtensorMap and its encoder's signature (resolved through the runtime)
@@ -1556,29 +1557,22 @@ static int checksum_impl(wt_handle *h, const void *const *ptr, const uint64_t *n
   }
   const cudaStream_t s = static_cast<cudaStream_t>(stream);
   std::lock_guard<std::mutex> g(h->mu);
+  std::vector<uint64_t *> outs(n);
+  for (size_t i = 0; i < n; ++i) outs[i] = out_dev + i;
   for (size_t i0 = 0; i0 < n; i0 += wt::kMaxFnv) {
     const size_t m = std::min<size_t>(wt::kMaxFnv, n - i0);
-    wt::FnvBatch b;
-    memset(&b, 0, sizeof b);
-    b.n = (uint32_t)m;
-    uint64_t leaves = 0;
-    for (size_t k = 0; k < m; ++k) {
-      b.leaf_prefix[k] = leaves;
-      b.ptr[k] = static_cast<const uint8_t *>(ptr[i0 + k]);
-      b.nbytes[k] = nbytes[i0 + k];
-      b.out[k] = out_dev + i0 + k;
-      leaves += (nbytes[i0 + k] + wt::kLeafBytes - 1) / wt::kLeafBytes;
-    }
-    b.leaf_prefix[m] = leaves;
+    std::unique_ptr<wt::FnvBatch> b(new wt::FnvBatch);
+    const size_t scratch = wt::fnv_fill_batch(*b, ptr + i0, nbytes + i0, outs.data() + i0, m);
     if (plain) {
-      CU(wt::launch_fnv_plain(b, s));
+      CU(wt::launch_fnv_plain(*b, s));
       h->kernel_launches++;
     } else {
-      uint64_t *lv = nullptr;
-      if (leaves) CU(cudaMallocAsync(reinterpret_cast<void **>(&lv), leaves * 8, s));
-      CU(wt::launch_fnv_tree(b, lv, s));
-      h->kernel_launches += leaves ? 2 : 1;
-      if (lv) CU(cudaFreeAsync(lv, s));
+      void *sc = nullptr;
+      CU(cudaMallocAsync(&sc, scratch, s));
+      const cudaError_t e = wt::launch_fnv_tree(*b, sc, s);
+      cudaFreeAsync(sc, s);
+      CU(e);
+      h->kernel_launches += wt::fnv_tree_launches(*b);
     }
   }
   return WT_OK;

@@ -10,7 +10,7 @@
 // uses a fixed array compiled into the library instead.
 //
 // The array below is a file-scope __device__ object: every GPU that loads this
-// library holds its 8 MiB until the process exits.  Host code cannot use its
+// library holds its ~11 MiB until the process exits.  Host code cannot use its
 // name as a device address, so the first call on each device (with that device
 // current) asks the runtime for the address with cudaGetSymbolAddress and
 // caches it; that first call should come before any stream capture.  All calls
@@ -26,7 +26,11 @@
 namespace {
 
 constexpr uint64_t kNoAllocMaxLeaves = 1ull << 20;  // 4096-byte leaves: 4 GiB of input per call
-__device__ __align__(256) uint64_t g_noalloc_leaves[kNoAllocMaxLeaves];
+// leaf digests plus the chunk tables of the parallel second level (at most one chunk per
+// kChunkWords leaves and one partial chunk per buffer of a batch)
+constexpr uint64_t kNoAllocWords =
+    kNoAllocMaxLeaves + ((kNoAllocMaxLeaves / wt::kChunkWords + wt::kMaxFnv) * 1288 + wt::kMaxFnv * 8 + 2048) / 8;
+__device__ __align__(256) uint64_t g_noalloc_leaves[kNoAllocWords];
 
 std::mutex g_mu;
 uint64_t *g_leaves_addr[64] = {nullptr};
@@ -67,20 +71,13 @@ extern "C" __attribute__((visibility("default"))) int wt_checksum_noalloc(
   }
   // Batches run in order on one stream, so each reuses the array from slot 0.
   const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  static thread_local wt::FnvBatch b;  // 18 KB: kept off the stack
+  uint64_t *outs[wt::kMaxFnv];
   for (size_t i0 = 0; i0 < n; i0 += wt::kMaxFnv) {
     const size_t m = n - i0 < (size_t)wt::kMaxFnv ? n - i0 : (size_t)wt::kMaxFnv;
-    wt::FnvBatch b;
-    memset(&b, 0, sizeof b);
-    b.n = (uint32_t)m;
-    uint64_t l = 0;
-    for (size_t k = 0; k < m; ++k) {
-      b.leaf_prefix[k] = l;
-      b.ptr[k] = static_cast<const uint8_t *>(ptr[i0 + k]);
-      b.nbytes[k] = nbytes[i0 + k];
-      b.out[k] = out_dev + i0 + k;
-      l += (nbytes[i0 + k] + wt::kLeafBytes - 1) / wt::kLeafBytes;
-    }
-    b.leaf_prefix[m] = l;
+    for (size_t k = 0; k < m; ++k) outs[k] = out_dev + i0 + k;
+    const size_t need = wt::fnv_fill_batch(b, ptr + i0, nbytes + i0, outs, m);
+    if (need > sizeof(g_noalloc_leaves)) return fail(WT_EINVAL, "wt_checksum_noalloc: batch scratch exceeds the fixed array");
     e = wt::launch_fnv_tree(b, scratch, s);
     if (e != cudaSuccess) {
       cudaGetLastError();

@@ -231,9 +231,12 @@ def test_first_use_pipeline_mid(torch, tmp_path):
 
 def test_checksum_edges(torch):
     rng = np.random.default_rng(7)
-    data = rng.integers(0, 256, 3 * 4096 + 100, dtype=np.uint8)
+    data = rng.integers(0, 256, 40 * 4096 + 100, dtype=np.uint8)
     buf = torch.from_numpy(data).cuda()
-    cases = [(0, 0), (0, 1), (1, 15), (3, 4095), (0, 4096), (0, 4097), (5, 8192 + 17), (16, 3 * 4096 + 84)]
+    # empty, sub-vector, unaligned starts (bytewise staging), ragged last leaves, and
+    # buffers of more leaves than the combine kernel loads ahead (16)
+    cases = [(0, 0), (0, 1), (1, 15), (3, 4095), (0, 4096), (0, 4097), (5, 8192 + 17), (16, 3 * 4096 + 84),
+             (0, 37 * 4096 + 5), (7, 20 * 4096), (32, 17 * 4096)]
     base = buf.data_ptr()
     for plain in (False, True):
         with wt.Handle([]) as h:
@@ -257,6 +260,30 @@ def test_checksum_many_buffers(torch):
         h.checksum([buf.data_ptr() + int(o) for o in offs], [int(s) for s in sizes], out.data_ptr(), 0)
         got = [int(v) & (2 ** 64 - 1) for v in out.cpu().tolist()]
     assert got == [oracle.fnv_tree(data[o:o + s]) for o, s in zip(offs, sizes)]
+
+
+def test_checksum_chunked_second_level(torch):
+    """Buffers above 4096 leaves combine their leaf digests in parallel chunks of 512; the
+    digest must equal the oracle's serial chain: 4096 leaves (serial), 4097 (eight full
+    chunks and one of one digest), a ragged unaligned 40 MiB buffer, and zero-chunk buffers
+    between chunked ones in one batch; through wt_checksum and wt_checksum_noalloc."""
+    rng = np.random.default_rng(9)
+    data = rng.integers(0, 256, 100 << 20, dtype=np.uint8)
+    buf = torch.from_numpy(data).cuda()
+    cases = [(0, 4096 * 4096), (64, 4096 * 4096 + 1), (3, (40 << 20) + 777), (5, 100),
+             (4096, 4096 * (4096 + 512) - 5), (0, 0), (17, 9000), (1 << 20, 4096 * 8192)]
+    want = [oracle.fnv_tree(data[o:o + n]) for o, n in cases]
+    base = buf.data_ptr()
+    for noalloc in (False, True):
+        out = torch.zeros(len(cases), dtype=torch.int64, device="cuda")
+        if noalloc:
+            wt.checksum_noalloc([base + o for o, n in cases], [n for o, n in cases], out.data_ptr(), 0)
+        else:
+            with wt.Handle([]) as h:
+                h.checksum([base + o for o, n in cases], [n for o, n in cases], out.data_ptr(), 0)
+        torch.cuda.synchronize()
+        got = [int(v) & (2 ** 64 - 1) for v in out.cpu().tolist()]
+        assert got == want, noalloc
 
 
 def test_unaligned_operands_take_the_generic_kernel(torch):
