@@ -978,7 +978,7 @@ __global__ void __launch_bounds__(256) fnv_table_kernel(const __grid_constant__ 
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
       const uint32_t u = l ^ (uint32_t)((v >> (8 * k)) & 0xffu);
-      B = B * kFnvP + (u - l) * kFnvP;
+      B = (B + u - l) * kFnvP;
       l = (u * kFnvP) & 0xffu;
     }
   }
@@ -1005,30 +1005,56 @@ __device__ __forceinline__ void fnv_leaf_run(Fnv &h, const uint64_t *leaves, uin
   }
 }
 
-// One thread per buffer.  Small buffers: the whole chain.  Chunked buffers: pass 2 (the
-// lo walk over the chunk tables).
-__global__ void fnv_combine_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
-  const uint32_t t = blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= b.n) return;
-  Fnv h;
-  h.le64(b.nbytes[t]);
+// One warp per buffer.  Small buffers: lane 0 runs the whole chain.  Chunked buffers: pass 2,
+// the lo walk, in lane 0, over table rows the warp copies into a shared-memory ring
+// kWalkAhead chunks ahead (one lookup per chunk instead of one L2 round trip).
+constexpr int kWalkAhead = 8;
+
+__global__ void __launch_bounds__(32) fnv_combine_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
+  __shared__ __align__(16) uint32_t rows[kWalkAhead][256];
+  const uint32_t t = blockIdx.x;
+  const int lane = threadIdx.x;
   const uint64_t l0 = b.leaf_prefix[t], l1 = b.leaf_prefix[t + 1];
   const uint32_t c0 = b.chunk_prefix[t], c1 = b.chunk_prefix[t + 1];
   if (c0 == c1) {
-    fnv_leaf_run(h, sc.leaves, l0, l1);
-    *b.out[t] = h.value();
+    if (lane == 0) {
+      Fnv h;
+      h.le64(b.nbytes[t]);
+      fnv_leaf_run(h, sc.leaves, l0, l1);
+      *b.out[t] = h.value();
+    }
     return;
   }
+  const uint32_t nc = c1 - c0;
+  // row of chunk c0 + j into slot j % kWalkAhead; one commit group per call, empty past the end
+  auto fetch = [&](uint32_t j) {
+    if (j < nc) {
+      const uint32_t *src = sc.btab + (size_t)(c0 + j) * 256 + lane * 4;
+      uint32_t *dst = rows[j % kWalkAhead] + lane * 4;
+      cp_async16(smem_u32(dst), src);
+      cp_async16(smem_u32(dst + 128), src + 128);
+    }
+    cp_async_commit();
+  };
+  for (uint32_t j = 0; j < (uint32_t)kWalkAhead; ++j) fetch(j);
+  Fnv h;
+  h.le64(b.nbytes[t]);
   const uint32_t pfull = fnv_pow(8 * kChunkWords);
   uint32_t lo = h.lo;
-  for (uint32_t c = c0; c < c1; ++c) {
-    sc.lo_start[c] = lo;
-    const uint64_t first = l0 + (uint64_t)(c - c0) * kChunkWords;
-    const uint32_t w = (uint32_t)min((uint64_t)kChunkWords, l1 - first);
-    const uint32_t pm = w == kChunkWords ? pfull : fnv_pow(8 * w);
-    lo = pm * lo + sc.btab[(size_t)c * 256 + (lo & 0xffu)];
+  for (uint32_t j = 0; j < nc; ++j) {
+    cp_async_wait<kWalkAhead - 1>();  // this lane's copies of row j have landed
+    __syncwarp();                     // and every lane's
+    if (lane == 0) {
+      sc.lo_start[c0 + j] = lo;
+      const uint64_t first = l0 + (uint64_t)j * kChunkWords;
+      const uint32_t w = (uint32_t)min((uint64_t)kChunkWords, l1 - first);
+      lo = (w == kChunkWords ? pfull : fnv_pow(8 * w)) * lo + rows[j % kWalkAhead][lo & 0xffu];
+    }
+    __syncwarp();  // lane 0 is done with slot j % kWalkAhead before it is refilled
+    fetch(j + kWalkAhead);
   }
-  sc.head[t] = ((uint64_t)h.hi << 32) | lo;
+  cp_async_wait<0>();
+  if (lane == 0) sc.head[t] = ((uint64_t)h.hi << 32) | lo;
 }
 
 // Pass 3: one thread per chunk, the exact chain from (lo_start, 0).
@@ -1242,7 +1268,7 @@ cudaError_t launch_fnv_tree(const FnvBatch &b, void *scratch, cudaStream_t s) {
     fnv_table_kernel<<<chunks, 256, 0, s>>>(b, sc);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
-  fnv_combine_kernel<<<(b.n + 127) / 128, 128, 0, s>>>(b, sc);
+  fnv_combine_kernel<<<b.n, 32, 0, s>>>(b, sc);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (chunks) {
     fnv_exact_kernel<<<(chunks + 127) / 128, 128, 0, s>>>(b, sc);
