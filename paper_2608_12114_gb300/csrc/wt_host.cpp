@@ -38,6 +38,7 @@
 
 #include "../../include/wt.h"
 #include "../../include/wt_dlpack.h"
+#include "wt_fnv.h"
 #include "wt_kernels.h"
 
 #ifndef MADV_POPULATE_READ

@@ -9,15 +9,13 @@
 //                      matrix).  W streams HBM -> shared memory through 1-D TMA
 //                      bulk copies on an mbarrier ring; warps reduce with
 //                      shuffles.  No tensor cores: ~1 flop per weight byte.
-//   fnv_*              per-buffer FNV-1a-64 digests (plain and 4 KiB leaf tree)
-//                      that prove ingested bytes equal the file's.
+//
+// The FNV-1a-64 digest kernels are in wt_fnv.cu.
 //
 // Every wait on an mbarrier is bounded (clock64 budget); a wait that runs out
 // records WT_ETIMEDOUT in the caller's status word, makes every later wait of
 // the CTA return at once, and the producer drains its own copies in flight
 // before the CTA exits.
-#include <cstring>
-
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -769,343 +767,6 @@ __global__ void seg_reduce_kernel(const SegReduce *__restrict__ tab) {
   r.y[row] = r.s ? sum * __half2float(reinterpret_cast<const __half *>(r.s)[row]) : sum;
 }
 
-// ------------------------------------------------------------------ FNV-1a-64
-// The 64-bit state is held as two 32-bit words.  With p = 2^40 + 0x1b3 and x = lo ^ b,
-//   (hi 2^32 + x) p mod 2^64 = (hi 0x1b3 + (x << 8) + high32(x 0x1b3)) 2^32 + low32(x 0x1b3),
-// since hi 2^72 vanishes and x 2^40 keeps only (x << 8) in the high word.  The serial chain
-// through a byte is then an xor and one 32 x 32 multiply on the low word; the high word is a
-// multiply-add beside it.  The constants are FNV-1a-64's offset basis and prime.
-constexpr uint32_t kFnvOffLo = 0x84222325u, kFnvOffHi = 0xcbf29ce4u;
-constexpr uint32_t kFnvP = 0x1b3u;
-
-struct Fnv {
-  uint32_t lo = kFnvOffLo, hi = kFnvOffHi;
-  __device__ __forceinline__ void byte(uint32_t b) {
-    const uint32_t x = lo ^ b;
-    const uint64_t w = (uint64_t)x * kFnvP;
-    lo = (uint32_t)w;
-    hi = hi * kFnvP + ((uint32_t)(w >> 32) + (x << 8));
-  }
-  __device__ __forceinline__ void word(uint32_t v) {
-    byte(v & 0xffu);
-    byte((v >> 8) & 0xffu);
-    byte((v >> 16) & 0xffu);
-    byte(v >> 24);
-  }
-  __device__ __forceinline__ void vec(const uint4 &v) {
-    word(v.x);
-    word(v.y);
-    word(v.z);
-    word(v.w);
-  }
-  __device__ __forceinline__ void le64(uint64_t v) {
-    word((uint32_t)v);
-    word((uint32_t)(v >> 32));
-  }
-  __device__ __forceinline__ uint64_t value() const { return ((uint64_t)hi << 32) | lo; }
-};
-
-__device__ __forceinline__ uint32_t find_buf(const FnvBatch &b, uint64_t leaf) {
-  uint32_t lo = 0, hi = b.n - 1;
-  while (lo < hi) {
-    uint32_t mid = (lo + hi + 1) >> 1;
-    if (b.leaf_prefix[mid] <= leaf) lo = mid; else hi = mid - 1;
-  }
-  return lo;
-}
-
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
-// One thread per 4 KiB leaf.  A warp stages 128-byte slices of its 32 leaves in shared
-// memory with coalesced asynchronous 16-byte copies (eight lanes per leaf slice, four
-// leaves per warp instruction), double-buffered: slice s + 1 is in flight while each lane
-// hashes its own row of slice s.  Rows are padded to 144 bytes, so the eight lanes of a
-// quarter-warp read distinct banks.  A warp whose 32 leaves are whole, 16-byte aligned and
-// from one buffer (every warp inside a large tensor) computes the copy addresses directly;
-// other warps fetch each leaf's pointer and length from its lane.
-constexpr int kFnvWarps = 4;
-constexpr int kSlice = 128;
-constexpr int kSliceStride = kSlice + 16;
-constexpr int kLanesPerLeaf = kSlice / 16;
-constexpr int kLeavesPerRound = 32 / kLanesPerLeaf;
-constexpr uint32_t kSlices = (uint32_t)(kLeafBytes / kSlice);
-
-__device__ __forceinline__ void fnv_stage_fast(uint8_t (*dst)[kSliceStride], const uint8_t *wbase, uint32_t s0,
-                                               int lane) {
-  const int sub = lane / kLanesPerLeaf, q = lane % kLanesPerLeaf;
-  const uint8_t *src = wbase + (size_t)sub * kLeafBytes + s0 + q * 16;
-#pragma unroll
-  for (int r = 0; r < 32; r += kLeavesPerRound)
-    cp_async16(smem_u32(&dst[r + sub][q * 16]), src + (size_t)r * kLeafBytes);
-  cp_async_commit();
-}
-
-__device__ __forceinline__ void fnv_stage(uint8_t (*dst)[kSliceStride], const uint8_t *lp, uint32_t llen,
-                                          uint32_t s0, int lane) {
-  const int sub = lane / kLanesPerLeaf, q = lane % kLanesPerLeaf;
-#pragma unroll 2
-  for (int r = 0; r < 32; r += kLeavesPerRound) {
-    const int src = r + sub;
-    const uint8_t *p = reinterpret_cast<const uint8_t *>(__shfl_sync(0xffffffffu, (unsigned long long)lp, src));
-    const uint32_t n = __shfl_sync(0xffffffffu, llen, src);
-    const uint32_t o = s0 + q * 16;
-    uint8_t *d = &dst[src][q * 16];
-    if (p != nullptr && o < n) {
-      if (o + 16 <= n && ((reinterpret_cast<uintptr_t>(p) + o) & 15) == 0) {
-        cp_async16(smem_u32(d), p + o);
-      } else {
-        for (uint32_t k = 0; k < 16 && o + k < n; ++k) d[k] = p[o + k];
-      }
-    }
-  }
-  cp_async_commit();
-}
-
-__global__ void __launch_bounds__(kFnvWarps * 32) fnv_leaf_kernel(const __grid_constant__ FnvBatch b,
-                                                                   uint64_t *leaves) {
-  __shared__ __align__(16) uint8_t buf[kFnvWarps][2][32][kSliceStride];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint64_t total = b.leaf_prefix[b.n];
-  const uint64_t nwarps = (uint64_t)gridDim.x * kFnvWarps;
-  for (uint64_t base = ((uint64_t)blockIdx.x * kFnvWarps + warp) * 32; base < total; base += nwarps * 32) {
-    const uint64_t leaf = base + lane;
-    const bool mine = leaf < total;
-    const uint8_t *lp = nullptr;
-    uint32_t llen = 0, t = 0xffffffffu;
-    if (mine) {
-      t = find_buf(b, leaf);
-      const uint64_t off = (leaf - b.leaf_prefix[t]) * kLeafBytes;
-      lp = b.ptr[t] + off;
-      llen = (uint32_t)min(kLeafBytes, b.nbytes[t] - off);
-    }
-    const uint32_t t0 = __shfl_sync(0xffffffffu, t, 0);
-    const bool fast = __all_sync(0xffffffffu, mine && t == t0 && llen == kLeafBytes &&
-                                                   (reinterpret_cast<uintptr_t>(lp) & 15) == 0);
-    const uint8_t *wbase = reinterpret_cast<const uint8_t *>(__shfl_sync(0xffffffffu, (unsigned long long)lp, 0));
-    // slices the longest leaf of the warp needs (warp-uniform)
-    const uint32_t nsl = (__reduce_max_sync(0xffffffffu, llen) + kSlice - 1) / kSlice;
-    Fnv h;
-    if (nsl) {
-      if (fast) fnv_stage_fast(buf[warp][0], wbase, 0, lane);
-      else fnv_stage(buf[warp][0], lp, llen, 0, lane);
-    }
-    for (uint32_t si = 0; si < nsl; ++si) {
-      if (si + 1 < nsl) {
-        if (fast) fnv_stage_fast(buf[warp][(si + 1) & 1], wbase, (si + 1) * kSlice, lane);
-        else fnv_stage(buf[warp][(si + 1) & 1], lp, llen, (si + 1) * kSlice, lane);
-        cp_async_wait<1>();
-      } else {
-        cp_async_wait<0>();
-      }
-      __syncwarp();
-      const uint32_t s0 = si * kSlice;
-      if (mine && s0 < llen) {
-        const uint32_t m = min((uint32_t)kSlice, llen - s0);
-        const uint8_t *row = buf[warp][si & 1][lane];
-        uint32_t k = 0;
-        for (; k + 16 <= m; k += 16) h.vec(*reinterpret_cast<const uint4 *>(row + k));
-        for (; k < m; ++k) h.byte(row[k]);
-      }
-      __syncwarp();  // every lane is done with this buffer before it is refilled
-    }
-    if (mine) leaves[leaf] = h.value();
-  }
-}
-
-// ---- second level: FNV-1a over LE64(nbytes), then the LE64 of each leaf digest
-//
-// The chain costs one dependent xor and 32 x 32 multiply per byte.  For a buffer of L
-// leaves that is 8 L bytes in one thread (a 1 GB tensor: 2 MB of chain).  Larger buffers
-// split the leaf stream into chunks of kChunkWords digests and combine them exactly in
-// parallel, from three facts about one FNV step (all arithmetic mod 2^32):
-//  1. the low byte of lo evolves on its own: l' = ((l ^ b) p) & 0xff;
-//  2. lo ^ b = lo + d with d = (l ^ b) - l, so lo' = (lo + d) p, and over a chunk of m bytes
-//     lo_end = p^m lo_start + B, where B depends only on the chunk's bytes and the low
-//     byte of lo_start;
-//  3. hi' = hi p + t with t a function of lo and b alone, so hi_end = p^m hi_start + H,
-//     where H is the chunk's hi run from 0 along the true lo sequence.
-// Pass 1 tabulates (l_end, B) for all 256 starting low bytes of every chunk; pass 2 walks
-// the chunks of a buffer serially with one table lookup each, giving every chunk's lo_start;
-// pass 3 runs every chunk exactly from its lo_start with hi = 0, giving H; pass 4 folds the
-// H values into hi.  The result equals the serial chain bit for bit.
-
-// p^e mod 2^32 by square and multiply
-__device__ __forceinline__ uint32_t fnv_pow(uint32_t e) {
-  uint32_t r = 1, q = kFnvP;
-  for (; e; e >>= 1, q *= q)
-    if (e & 1) r *= q;
-  return r;
-}
-
-struct FnvScratch {
-  uint64_t *leaves;   // [total leaves]
-  uint32_t *btab;     // [chunks][256]
-  uint8_t *ltab;      // [chunks][256]
-  uint32_t *lo_start; // [chunks]
-  uint32_t *hpart;    // [chunks]
-  uint64_t *head;     // [n]: (hi after LE64(nbytes)) << 32 | lo at the end of the leaf stream
-};
-
-__device__ __forceinline__ uint32_t find_chunk_buf(const FnvBatch &b, uint32_t c) {
-  uint32_t lo = 0, hi = b.n - 1;
-  while (lo < hi) {
-    uint32_t mid = (lo + hi + 1) >> 1;
-    if (b.chunk_prefix[mid] <= c) lo = mid; else hi = mid - 1;
-  }
-  return lo;
-}
-
-// Pass 1: one block per chunk, one thread per starting low byte; the chunk's digests are
-// staged in shared memory and read as broadcasts.
-__global__ void __launch_bounds__(256) fnv_table_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
-  __shared__ uint64_t words[kChunkWords];
-  const uint32_t c = blockIdx.x;
-  const uint32_t t = find_chunk_buf(b, c);
-  const uint64_t first = b.leaf_prefix[t] + (uint64_t)(c - b.chunk_prefix[t]) * kChunkWords;
-  const uint32_t w = (uint32_t)min((uint64_t)kChunkWords, b.leaf_prefix[t + 1] - first);
-  for (uint32_t i = threadIdx.x; i < w; i += blockDim.x) words[i] = sc.leaves[first + i];
-  __syncthreads();
-  uint32_t l = threadIdx.x, B = 0;
-  for (uint32_t i = 0; i < w; ++i) {
-    const uint64_t v = words[i];
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      const uint32_t u = l ^ (uint32_t)((v >> (8 * k)) & 0xffu);
-      B = (B + u - l) * kFnvP;
-      l = (u * kFnvP) & 0xffu;
-    }
-  }
-  sc.btab[(size_t)c * 256 + threadIdx.x] = B;
-  sc.ltab[(size_t)c * 256 + threadIdx.x] = (uint8_t)l;
-}
-
-// Serial chain over leaves [l0, l1) from state h; kCombineAhead digests are loaded ahead.
-constexpr int kCombineAhead = 16;
-__device__ __forceinline__ void fnv_leaf_run(Fnv &h, const uint64_t *leaves, uint64_t l0, uint64_t l1) {
-  uint64_t r[kCombineAhead];
-#pragma unroll
-  for (int j = 0; j < kCombineAhead; ++j) r[j] = l0 + j < l1 ? leaves[l0 + j] : 0;
-  for (uint64_t l = l0; l < l1; l += kCombineAhead) {
-#pragma unroll
-    for (int j = 0; j < kCombineAhead; ++j) {
-      if (l + j < l1) {
-        const uint64_t v = r[j];
-        const uint64_t ln = l + j + kCombineAhead;
-        if (ln < l1) r[j] = leaves[ln];
-        h.le64(v);
-      }
-    }
-  }
-}
-
-// One warp per buffer.  Small buffers: lane 0 runs the whole chain.  Chunked buffers: pass 2,
-// the lo walk, in lane 0, over table rows the warp copies into a shared-memory ring
-// kWalkAhead chunks ahead (one lookup per chunk instead of one L2 round trip).
-constexpr int kWalkAhead = 8;
-
-__global__ void __launch_bounds__(32) fnv_combine_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
-  __shared__ __align__(16) uint32_t rows[kWalkAhead][256];
-  const uint32_t t = blockIdx.x;
-  const int lane = threadIdx.x;
-  const uint64_t l0 = b.leaf_prefix[t], l1 = b.leaf_prefix[t + 1];
-  const uint32_t c0 = b.chunk_prefix[t], c1 = b.chunk_prefix[t + 1];
-  if (c0 == c1) {
-    if (lane == 0) {
-      Fnv h;
-      h.le64(b.nbytes[t]);
-      fnv_leaf_run(h, sc.leaves, l0, l1);
-      *b.out[t] = h.value();
-    }
-    return;
-  }
-  const uint32_t nc = c1 - c0;
-  // row of chunk c0 + j into slot j % kWalkAhead; one commit group per call, empty past the end
-  auto fetch = [&](uint32_t j) {
-    if (j < nc) {
-      const uint32_t *src = sc.btab + (size_t)(c0 + j) * 256 + lane * 4;
-      uint32_t *dst = rows[j % kWalkAhead] + lane * 4;
-      cp_async16(smem_u32(dst), src);
-      cp_async16(smem_u32(dst + 128), src + 128);
-    }
-    cp_async_commit();
-  };
-  for (uint32_t j = 0; j < (uint32_t)kWalkAhead; ++j) fetch(j);
-  Fnv h;
-  h.le64(b.nbytes[t]);
-  const uint32_t pfull = fnv_pow(8 * kChunkWords);
-  uint32_t lo = h.lo;
-  for (uint32_t j = 0; j < nc; ++j) {
-    cp_async_wait<kWalkAhead - 1>();  // this lane's copies of row j have landed
-    __syncwarp();                     // and every lane's
-    if (lane == 0) {
-      sc.lo_start[c0 + j] = lo;
-      const uint64_t first = l0 + (uint64_t)j * kChunkWords;
-      const uint32_t w = (uint32_t)min((uint64_t)kChunkWords, l1 - first);
-      lo = (w == kChunkWords ? pfull : fnv_pow(8 * w)) * lo + rows[j % kWalkAhead][lo & 0xffu];
-    }
-    __syncwarp();  // lane 0 is done with slot j % kWalkAhead before it is refilled
-    fetch(j + kWalkAhead);
-  }
-  cp_async_wait<0>();
-  if (lane == 0) sc.head[t] = ((uint64_t)h.hi << 32) | lo;
-}
-
-// Pass 3: one thread per chunk, the exact chain from (lo_start, 0).
-__global__ void fnv_exact_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
-  const uint32_t c = blockIdx.x * blockDim.x + threadIdx.x;
-  if (c >= b.chunk_prefix[b.n]) return;
-  const uint32_t t = find_chunk_buf(b, c);
-  const uint64_t first = b.leaf_prefix[t] + (uint64_t)(c - b.chunk_prefix[t]) * kChunkWords;
-  const uint64_t last = min(first + kChunkWords, b.leaf_prefix[t + 1]);
-  Fnv h;
-  h.lo = sc.lo_start[c];
-  h.hi = 0;
-  fnv_leaf_run(h, sc.leaves, first, last);
-  sc.hpart[c] = h.hi;
-}
-
-// Pass 4: one thread per chunked buffer, hi folded over its chunks.
-__global__ void fnv_finish_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
-  const uint32_t t = blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= b.n) return;
-  const uint32_t c0 = b.chunk_prefix[t], c1 = b.chunk_prefix[t + 1];
-  if (c0 == c1) return;
-  const uint64_t l0 = b.leaf_prefix[t], l1 = b.leaf_prefix[t + 1];
-  const uint32_t pfull = fnv_pow(8 * kChunkWords);
-  const uint64_t head = sc.head[t];
-  uint32_t hi = (uint32_t)(head >> 32);
-  for (uint32_t c = c0; c < c1; ++c) {
-    const uint64_t first = l0 + (uint64_t)(c - c0) * kChunkWords;
-    const uint32_t w = (uint32_t)min((uint64_t)kChunkWords, l1 - first);
-    hi = (w == kChunkWords ? pfull : fnv_pow(8 * w)) * hi + sc.hpart[c];
-  }
-  *b.out[t] = ((uint64_t)hi << 32) | (uint32_t)head;
-}
-
-// One thread per buffer: the literal serial FNV-1a-64.
-__global__ void fnv_plain_kernel(const __grid_constant__ FnvBatch b) {
-  const uint32_t t = blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= b.n) return;
-  const uint8_t *p = b.ptr[t];
-  const uint64_t n = b.nbytes[t];
-  Fnv h;
-  uint64_t i = 0;
-  // bytes up to the first 16-byte boundary, then vectors, then the tail
-  while (i < n && ((reinterpret_cast<uintptr_t>(p) + i) & 15) != 0) h.byte(p[i++]);
-  const uint4 *v = reinterpret_cast<const uint4 *>(p + i);
-  const uint64_t nv = (n - i) >> 4;
-  for (uint64_t k = 0; k < nv; ++k) h.vec(v[k]);
-  for (i += nv << 4; i < n; ++i) h.byte(p[i]);
-  *b.out[t] = h.value();
-}
-
 }  // namespace
 
 // ------------------------------------------------------------------ launchers
@@ -1196,92 +857,6 @@ cudaError_t launch_seg_reduce(const SegReduce *tab, int n, uint32_t max_rows, cu
   if (n == 0 || max_rows == 0) return cudaSuccess;
   const dim3 grid((max_rows + 255) / 256, (unsigned)n);
   seg_reduce_kernel<<<grid, 256, 0, s>>>(tab);
-  return cudaGetLastError();
-}
-
-static size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
-
-// Scratch layout of one batch: leaves, btab, ltab, lo_start, hpart, head (256-byte aligned).
-static FnvScratch fnv_layout(const FnvBatch &b, void *base, size_t *bytes) {
-  const uint64_t L = b.leaf_prefix[b.n];
-  const uint64_t C = b.chunk_prefix[b.n];
-  size_t off[6];
-  size_t o = 0;
-  const size_t len[6] = {L * 8, C * 256 * 4, C * 256, C * 4, C * 4, (size_t)b.n * 8};
-  for (int i = 0; i < 6; ++i) {
-    off[i] = o;
-    o = align256(o + len[i]);
-  }
-  if (bytes) *bytes = o;
-  FnvScratch sc;
-  const uintptr_t p = reinterpret_cast<uintptr_t>(base);
-  sc.leaves = reinterpret_cast<uint64_t *>(p + off[0]);
-  sc.btab = reinterpret_cast<uint32_t *>(p + off[1]);
-  sc.ltab = reinterpret_cast<uint8_t *>(p + off[2]);
-  sc.lo_start = reinterpret_cast<uint32_t *>(p + off[3]);
-  sc.hpart = reinterpret_cast<uint32_t *>(p + off[4]);
-  sc.head = reinterpret_cast<uint64_t *>(p + off[5]);
-  return sc;
-}
-
-size_t fnv_fill_batch(FnvBatch &b, const void *const *ptr, const uint64_t *nbytes, uint64_t *const *out, size_t n) {
-  memset(&b, 0, sizeof b);
-  b.n = (uint32_t)n;
-  uint64_t leaves = 0;
-  uint32_t chunks = 0;
-  for (size_t k = 0; k < n; ++k) {
-    b.leaf_prefix[k] = leaves;
-    b.chunk_prefix[k] = chunks;
-    b.ptr[k] = static_cast<const uint8_t *>(ptr[k]);
-    b.nbytes[k] = nbytes[k];
-    b.out[k] = out[k];
-    const uint64_t l = (nbytes[k] + kLeafBytes - 1) / kLeafBytes;
-    leaves += l;
-    if (l > kParallelLeaves) chunks += (uint32_t)((l + kChunkWords - 1) / kChunkWords);
-  }
-  b.leaf_prefix[n] = leaves;
-  b.chunk_prefix[n] = chunks;
-  size_t bytes = 0;
-  fnv_layout(b, nullptr, &bytes);
-  return bytes;
-}
-
-int fnv_tree_launches(const FnvBatch &b) {
-  if (b.n == 0) return 0;
-  return (b.leaf_prefix[b.n] ? 1 : 0) + 1 + (b.chunk_prefix[b.n] ? 3 : 0);
-}
-
-cudaError_t launch_fnv_tree(const FnvBatch &b, void *scratch, cudaStream_t s) {
-  if (b.n == 0) return cudaSuccess;
-  const FnvScratch sc = fnv_layout(b, scratch, nullptr);
-  const uint64_t total = b.leaf_prefix[b.n];
-  const uint32_t chunks = b.chunk_prefix[b.n];
-  cudaError_t e;
-  if (total > 0) {
-    const uint64_t warps = (total + 31) / 32;
-    const uint64_t blocks = (warps + kFnvWarps - 1) / kFnvWarps;
-    const uint64_t cap = (uint64_t)num_sms() * 24;
-    fnv_leaf_kernel<<<(int)(blocks < cap ? blocks : cap), kFnvWarps * 32, 0, s>>>(b, sc.leaves);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  }
-  if (chunks) {
-    fnv_table_kernel<<<chunks, 256, 0, s>>>(b, sc);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  }
-  fnv_combine_kernel<<<b.n, 32, 0, s>>>(b, sc);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  if (chunks) {
-    fnv_exact_kernel<<<(chunks + 127) / 128, 128, 0, s>>>(b, sc);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    fnv_finish_kernel<<<(b.n + 127) / 128, 128, 0, s>>>(b, sc);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  }
-  return cudaSuccess;
-}
-
-cudaError_t launch_fnv_plain(const FnvBatch &b, cudaStream_t s) {
-  if (b.n == 0) return cudaSuccess;
-  fnv_plain_kernel<<<(b.n + 63) / 64, 64, 0, s>>>(b);
   return cudaGetLastError();
 }
 

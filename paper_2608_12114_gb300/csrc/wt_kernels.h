@@ -154,36 +154,6 @@ cudaError_t launch_gemv_generic(int dtype, const uint8_t *W, const uint8_t *x, f
                                 uint64_t M, uint64_t K, const uint8_t *scale, uint32_t cols,
                                 cudaStream_t s);
 
-// ---------------------------------------------------------------- FNV-1a-64
-constexpr int kMaxFnv = 512;  // buffers per launch: the batch is an 18 KB kernel parameter
-constexpr uint64_t kLeafBytes = 4096;
-
-// The tree digest's second level is a serial FNV chain over 8 bytes per leaf.  Buffers of
-// more than kParallelLeaves leaves split that chain into chunks of kChunkWords leaf digests
-// and combine the chunks in parallel (exact; see the kernels), others run it in one thread.
-constexpr uint64_t kParallelLeaves = 4096;
-constexpr uint32_t kChunkWords = 512;
-
-struct FnvBatch {
-  uint32_t n;
-  uint32_t pad;
-  uint64_t leaf_prefix[kMaxFnv + 1];   // first global leaf of buffer i; [n] = total leaves
-  uint32_t chunk_prefix[kMaxFnv + 1];  // first global chunk of buffer i; [n] = total chunks
-  const uint8_t *ptr[kMaxFnv];
-  uint64_t nbytes[kMaxFnv];
-  uint64_t *out[kMaxFnv];  // device address of the digest of buffer i
-};
-
-// Fills n, ptr, nbytes, out and both prefixes from the buffers; returns the device scratch
-// bytes launch_fnv_tree needs for the batch (leaf digests, then the chunk tables).
-size_t fnv_fill_batch(FnvBatch &b, const void *const *ptr, const uint64_t *nbytes, uint64_t *const *out, size_t n);
-
-// Kernel launches of launch_fnv_tree for the batch: leaves, combine, and the three chunk passes.
-int fnv_tree_launches(const FnvBatch &b);
-
-cudaError_t launch_fnv_tree(const FnvBatch &b, void *scratch, cudaStream_t s);
-cudaError_t launch_fnv_plain(const FnvBatch &b, cudaStream_t s);
-
 int num_sms();  // of the current device (cached per device)
 
 // Records `msg` as this thread's wt_last_error() text and returns `code`.

@@ -21,6 +21,7 @@
 #include <mutex>
 
 #include "../../include/wt.h"
+#include "wt_fnv.h"
 #include "wt_kernels.h"
 
 namespace {
