@@ -43,16 +43,27 @@ constexpr int kColRows = kColTileRows;           // rows of one stage (one MMA t
 constexpr int kColBlocks = 4;                    // tiles per super block
 constexpr int kColSuper = kColRows * kColBlocks;
 constexpr int kColGroups = (kColVecMax / 4 + kColWarps - 1) / kColWarps;  // 4-vector groups per warp
-constexpr int kColStages = 6;
 constexpr uint32_t kColStageBytes = kColRows * kColVecMax * 16;
-constexpr size_t kColRedOff = (size_t)kColStages * kColStageBytes;
-constexpr size_t kColRedFloats = (size_t)kColBlocks * kColWarps * 256;  // one of two halves
-constexpr size_t kColBarOff = kColRedOff + 2 * kColRedFloats * sizeof(float);
-constexpr size_t kColFlagOff = kColBarOff + 2 * kColStages * sizeof(uint64_t);
-constexpr size_t kColSmem = kColFlagOff + 16;
 static_assert(kColVecMax % 8 == 4, "row pitch 64 bytes past a multiple of 128");
 static_assert(kColStageBytes % 128 == 0, "stages stay 128-byte aligned for the tensor copies");
-static_assert(kColSmem <= 232448, "shared memory of one CTA");
+
+// Per-launch geometry: NT = 8-column MMA tiles (T <= 8: 1, else 2).  int8 weights with
+// T <= 8 run two CTAs per SM with half the ring each (the same bytes in flight per SM,
+// twice the warps; that case is latency-bound on its decode).  The cross-warp partials of
+// one 16-row tile take 16 x 8 NT floats per warp, in two alternating halves.
+template <int DT, int NT>
+struct ColGeo {
+  static constexpr int kCtasPerSm = DT == 3 && NT == 1 ? 2 : 1;
+  static constexpr int kStages = kCtasPerSm == 2 ? 3 : 6;
+  static constexpr uint32_t kRedStride = 128 * NT;  // floats per (tile, warp)
+  static constexpr size_t kRedFloats = (size_t)kColBlocks * kColWarps * kRedStride;  // one half
+  static constexpr size_t kRedOff = (size_t)kStages * kColStageBytes;
+  static constexpr size_t kBarOff = kRedOff + 2 * kRedFloats * sizeof(float);
+  static constexpr size_t kFlagOff = kBarOff + 2 * kStages * sizeof(uint64_t);
+  static constexpr size_t kSmem = kFlagOff + 16;
+};
+static_assert(ColGeo<1, 2>::kSmem <= 232448 && 2 * (ColGeo<3, 1>::kSmem + 1024) <= 233472,
+              "multi-column shared memory");
 
 // 32-bit words of X per weight vector: 16 fp16 activations for an int8 vector, else 8.
 template <int DT>
@@ -192,8 +203,8 @@ __device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, c
 #pragma unroll
       for (int b = 0; b < kColBlocks; ++b) {
         if ((uint32_t)b < nrb) {
-          const uint32_t s = it % kColStages;
-          bounded_wait(R.full0 + 8 * s, (it / kColStages) & 1, R.abort_flag, R.status);
+          const uint32_t s = it % ColGeo<DT, NT>::kStages;
+          bounded_wait(R.full0 + 8 * s, (it / ColGeo<DT, NT>::kStages) & 1, R.abort_flag, R.status);
           cols_stage<DT, NT>(R.stage0 + s * kColStageBytes, vc, warp, g, t, xr, acc[b]);
           __syncwarp();
           if (lane == 0) mbar_arrive(R.empty0 + 8 * s);
@@ -204,12 +215,13 @@ __device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, c
     // warp partials -> red[b][warp][col][row]; C fragment: (g, 2t), (g, 2t+1), (g+8, 2t), (g+8, 2t+1).
     // Two halves alternate, so one barrier per super block suffices: a half is rewritten
     // only after every thread has passed the next super block's barrier.
-    float *red = red_base + par * kColRedFloats;
+    constexpr uint32_t kStride = ColGeo<DT, NT>::kRedStride;
+    float *red = red_base + par * ColGeo<DT, NT>::kRedFloats;
     par ^= 1;
 #pragma unroll
     for (int b = 0; b < kColBlocks; ++b) {
       if ((uint32_t)b < nrb) {
-        float *r = red + (b * kColWarps + warp) * 256;
+        float *r = red + (b * kColWarps + warp) * kStride;
 #pragma unroll
         for (int n = 0; n < NT; ++n) {
           const uint32_t c0 = 2 * t + 8 * n;
@@ -221,31 +233,33 @@ __device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, c
       }
     }
     named_bar(1, kColConsumers);
-    for (uint32_t o = ct; o < nrb * 256; o += kColConsumers) {
-      const uint32_t b = o >> 8, e = o & 255, col = e >> 4, row = b * kColRows + (e & 15);
+    for (uint32_t o = ct; o < nrb * kStride; o += kColConsumers) {
+      const uint32_t b = o / kStride, e = o % kStride, col = e >> 4, row = b * kColRows + (e & 15);
       if (col < T && row < rows) {
-        const float *r = red + b * kColWarps * 256 + e;
+        const float *r = red + b * kColWarps * kStride + e;
         float sum = 0.f;
 #pragma unroll
-        for (int w = 0; w < kColWarps; ++w) sum += r[w * 256];
+        for (int w = 0; w < kColWarps; ++w) sum += r[w * kStride];
         md.y[(uint64_t)col * md.M + sb + row] = sum * col_scale<DT>(md.s, sb + row);
       }
     }
   }
 }
 
-template <int DT>
-__global__ void __launch_bounds__(kColThreads, 1)
+template <int DT, int NT>
+__global__ void __launch_bounds__(kColThreads, (ColGeo<DT, NT>::kCtasPerSm))
     gemm_cols_kernel(const MatDesc *__restrict__ mats, const Piece *__restrict__ pieces,
                      const uint32_t *__restrict__ begin, int *status, const uint8_t *__restrict__ maps) {
+  using Geo = ColGeo<DT, NT>;
+  constexpr int kColStages = Geo::kStages;
   extern __shared__ __align__(128) uint8_t smem[];
   Ring R;
   R.stage0 = smem_u32(smem);
-  R.full0 = smem_u32(smem + kColBarOff);
+  R.full0 = smem_u32(smem + Geo::kBarOff);
   R.empty0 = R.full0 + kColStages * 8;
-  R.abort_flag = reinterpret_cast<volatile int *>(smem + kColFlagOff);
+  R.abort_flag = reinterpret_cast<volatile int *>(smem + Geo::kFlagOff);
   R.status = status;
-  float *red = reinterpret_cast<float *>(smem + kColRedOff);
+  float *red = reinterpret_cast<float *>(smem + Geo::kRedOff);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const uint32_t p0 = begin[blockIdx.x];
@@ -305,13 +319,12 @@ __global__ void __launch_bounds__(kColThreads, 1)
     }
     __syncwarp();
   } else {
-    // ---------------- consumers: 8 warps
+    // ---------------- consumers: 8 warps (every matrix of the launch has T <= 8 NT)
     uint32_t it = 0, par = 0;
     for (uint32_t pi = p0; pi < p1; ++pi) {
       const Piece pc = pieces[pi];
       const MatDesc md = mats[pc.mat];
-      if (md.G > 8) cols_piece<DT, 2>(md, pc, R, red, it, par, warp, lane);
-      else cols_piece<DT, 1>(md, pc, R, red, it, par, warp, lane);
+      cols_piece<DT, NT>(md, pc, R, red, it, par, warp, lane);
     }
   }
   __syncthreads();
@@ -319,25 +332,38 @@ __global__ void __launch_bounds__(kColThreads, 1)
 
 }  // namespace
 
-size_t gemm_cols_smem_bytes() { return kColSmem; }
+int gemm_cols_ctas_per_sm(int dtype, int nt) { return dtype == 3 && nt == 1 ? 2 : 1; }
+
+template <int DT, int NT>
+static cudaError_t cols_attr() {
+  return cudaFuncSetAttribute(gemm_cols_kernel<DT, NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)ColGeo<DT, NT>::kSmem);
+}
 
 cudaError_t gemm_cols_prepare() {
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(gemm_cols_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kColSmem)) !=
-      cudaSuccess)
+  if ((e = cols_attr<1, 1>()) != cudaSuccess || (e = cols_attr<1, 2>()) != cudaSuccess ||
+      (e = cols_attr<2, 1>()) != cudaSuccess || (e = cols_attr<2, 2>()) != cudaSuccess ||
+      (e = cols_attr<3, 1>()) != cudaSuccess)
     return e;
-  if ((e = cudaFuncSetAttribute(gemm_cols_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kColSmem)) !=
-      cudaSuccess)
-    return e;
-  return cudaFuncSetAttribute(gemm_cols_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kColSmem);
+  return cols_attr<3, 2>();
+}
+
+template <int DT, int NT>
+static void cols_launch(const GemvLaunch &L, cudaStream_t s) {
+  gemm_cols_kernel<DT, NT><<<L.grid, kColThreads, ColGeo<DT, NT>::kSmem, s>>>(L.mats, L.pieces, L.begin, L.status,
+                                                                             L.maps);
 }
 
 cudaError_t launch_gemm_cols(const GemvLaunch &L, cudaStream_t s) {
-  if (L.maps == nullptr) return cudaErrorInvalidValue;
-  switch (L.dtype) {
-    case 1: gemm_cols_kernel<1><<<L.grid, kColThreads, kColSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.maps); break;
-    case 2: gemm_cols_kernel<2><<<L.grid, kColThreads, kColSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.maps); break;
-    case 3: gemm_cols_kernel<3><<<L.grid, kColThreads, kColSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.maps); break;
+  if (L.maps == nullptr || (L.nt != 1 && L.nt != 2)) return cudaErrorInvalidValue;
+  switch (L.dtype * 4 + L.nt) {
+    case 1 * 4 + 1: cols_launch<1, 1>(L, s); break;
+    case 1 * 4 + 2: cols_launch<1, 2>(L, s); break;
+    case 2 * 4 + 1: cols_launch<2, 1>(L, s); break;
+    case 2 * 4 + 2: cols_launch<2, 2>(L, s); break;
+    case 3 * 4 + 1: cols_launch<3, 1>(L, s); break;
+    case 3 * 4 + 2: cols_launch<3, 2>(L, s); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();

@@ -195,6 +195,7 @@ struct Plan {
     size_t maps = SIZE_MAX;      // multi-column launches: tensor maps (128-byte aligned)
     bool umma = false;           // multi-column launch on tcgen05 (wt_umma.cu)
     bool mapped_cols = false;    // map endpoint with T columns
+    int nt = 0;                  // warp-MMA multi-column launches: 8-column tiles (1 or 2)
     uint32_t nmat = 0, ntiles = 0;
   };
   struct Generic {
@@ -930,7 +931,8 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
     while (j < n && d[j].wait_event == d[i].wait_event) ++j;
     Plan::Group g;
     g.first = i;
-    std::vector<wt::MatDesc> by_dt[4], mapped_dt[4], cols_dt[4], umma_dt[4], mcols_dt[4];
+    // cols_dt: warp-MMA multi-column with T <= 8, colsw_dt: with 8 < T <= 16
+    std::vector<wt::MatDesc> by_dt[4], mapped_dt[4], cols_dt[4], umma_dt[4], mcols_dt[4], colsw_dt[4];
     std::vector<int64_t> seg_ws[4];  // per by_dt entry: workspace float offset of its partials, or -1
     std::vector<wt::SegReduce> reds;
     std::vector<size_t> red_ws;      // per reds entry: workspace float offset
@@ -990,7 +992,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
                                static_cast<const uint8_t *>(q.scale), ncol});
         }
       } else if (fast && q.cols > 0) {
-        (cols_on_umma(q.dtype, q.cols) ? umma_dt : cols_dt)[q.dtype].push_back(make_cols_mat(q));
+        (cols_on_umma(q.dtype, q.cols) ? umma_dt : q.cols > 8 ? colsw_dt : cols_dt)[q.dtype].push_back(make_cols_mat(q));
       } else if (fast && q.K * es / 16 > wt::seg_vectors(q.dtype)) {
         // long rows: column segments spread over CTAs, summed by the second pass
         const uint32_t V = (uint32_t)(q.K * es / 16);
@@ -1019,13 +1021,15 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
                              static_cast<const uint8_t *>(q.scale), ncol});
       }
     }
-    for (int pass = 0; pass < 5; ++pass) {
+    for (int pass = 0; pass < 6; ++pass) {
       for (int dt = 0; dt < 4; ++dt) {
         std::vector<wt::MatDesc> &ms = pass == 0   ? by_dt[dt]
                                        : pass == 1 ? mapped_dt[dt]
                                        : pass == 2 ? cols_dt[dt]
                                        : pass == 3 ? umma_dt[dt]
-                                                   : mcols_dt[dt];
+                                       : pass == 4 ? mcols_dt[dt]
+                                                   : colsw_dt[dt];
+        const bool warp_mma = pass == 2 || pass == 5;
         if (ms.empty()) continue;
         Plan::Launch L;
         L.dtype = dt;
@@ -1059,8 +1063,10 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
           for (const wt::MatDesc &m : ms)
             if (m.mode != wt::kModeWarpRows && m.mode != wt::kModeBlockRows)
               return set_err(WT_ENOTSUP, "wt_pass: internal: a %u-vector row reached the TMA kernel unsegmented", m.V);
-        partition(ms, L.grid, pieces, begin, pass == 2 ? (uint32_t)wt::kColTileRows : 1u,
-                  pass == 0 ? one_col_slices(dt) : 1, pass == 0 ? wt::gemv_ctas_per_sm(dt) : 1);
+        L.nt = pass == 2 ? 1 : pass == 5 ? 2 : 0;
+        partition(ms, L.grid, pieces, begin, warp_mma ? (uint32_t)wt::kColTileRows : 1u,
+                  pass == 0 ? one_col_slices(dt) : 1,
+                  pass == 0 ? wt::gemv_ctas_per_sm(dt) : warp_mma ? wt::gemm_cols_ctas_per_sm(dt, L.nt) : 1);
         L.mapped_cols = pass == 4;
         L.mats = append(P->table, ms);
         if (pass == 0)
@@ -1069,7 +1075,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
               P->ws_patches.push_back({L.mats + k * sizeof(wt::MatDesc) + offsetof(wt::MatDesc, y), (size_t)seg_ws[dt][k]});
         L.pieces = append(P->table, pieces);
         L.begin = append(P->table, begin);
-        if (pass == 2) {
+        if (warp_mma) {
           L.maps = (P->table.size() + 127) & ~(size_t)127;
           P->table.resize(L.maps + ms.size() * wt::kTensorMapBytes);
           for (size_t k = 0; k < ms.size(); ++k) {
@@ -1185,6 +1191,7 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
       gl.begin = reinterpret_cast<const uint32_t *>(P->dev + L.begin);
       gl.status = h->status;
       gl.maps = P->dev + L.maps;
+      gl.nt = L.nt;
       if (L.umma) {
         wt::UmmaLaunch ul;
         ul.dtype = L.dtype;

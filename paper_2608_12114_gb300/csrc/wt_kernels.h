@@ -104,6 +104,7 @@ struct GemvLaunch {
                                   // (kTensorMapBytes each, 128-byte aligned, device)
   int stall = 0;  // failure test (host fault site "stall"): the producer issues no copy, so
                   // every consumer wait runs out, reports WT_ETIMEDOUT and the CTA exits
+  int nt = 0;     // multi-column kernel: 8-column MMA tiles of every matrix (T <= 8 nt)
 };
 
 cudaError_t gemv_prepare();  // one-time function attributes
@@ -125,9 +126,11 @@ cudaError_t launch_gemv_mapped_cols(const GemvLaunch &L, cudaStream_t s);
 // vc = 4 mod 8), plus GemvLaunch.maps: per matrix a 2-D tensor map of W viewed as
 // [M, 2V] 8-byte elements with box {2 vc, kColTileRows} (rows and columns past the end
 // arrive as zeros).
+// One launch holds matrices of one dtype and one nt (GemvLaunch.nt: 1 for T <= 8, 2 for
+// 8 < T <= 16); int8 with nt = 1 runs two CTAs per SM (gemm_cols_ctas_per_sm).
 cudaError_t gemm_cols_prepare();
 cudaError_t launch_gemm_cols(const GemvLaunch &L, cudaStream_t s);
-size_t gemm_cols_smem_bytes();
+int gemm_cols_ctas_per_sm(int dtype, int nt);
 
 // The same multi-column GEMV on tcgen05 for 2-byte weights (wt_umma.cu): row tiles of 128
 // rows, K in chunks of 64 elements, accumulators in tensor memory.  pieces[m] = {m, first
