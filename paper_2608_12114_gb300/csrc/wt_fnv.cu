@@ -78,7 +78,6 @@ constexpr int kSlice = 128;
 constexpr int kSliceStride = kSlice + 16;
 constexpr int kLanesPerLeaf = kSlice / 16;
 constexpr int kLeavesPerRound = 32 / kLanesPerLeaf;
-constexpr uint32_t kSlices = (uint32_t)(kLeafBytes / kSlice);
 
 __device__ __forceinline__ void fnv_stage_fast(uint8_t (*dst)[kSliceStride], const uint8_t *wbase, uint32_t s0,
                                                int lane) {
