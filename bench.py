@@ -66,6 +66,8 @@ def parse_args():
                    help="also time N file -> first-use runs with the files evicted from the page cache")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=15.0, help="CPU budget of the oracle sample")
+    p.add_argument("--ref-seconds", type=float, default=150.0,
+                   help="total CPU budget of the reference arm (--impl reference), split over its steps")
     p.add_argument("--data-dir", default=None)
     p.add_argument("--workers", type=int, default=0)
     p.add_argument("--cube", action="store_true",
@@ -648,7 +650,7 @@ def run_reference(args, rank, world):
         return
     ck, gen_s = make_files(args, 0, 1)
     steps, warm = max(1, args.steps), max(0, args.warmup)
-    budget = min(10.0, max(0.05, 150.0 / (steps + warm)))
+    budget = min(10.0, max(0.05, args.ref_seconds / (steps + warm)))
     o = OracleSample(ck)
     rates, tot_b, tot_s = [], 0, 0.0
     for i in range(warm + steps):
