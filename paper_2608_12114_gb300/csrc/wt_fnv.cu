@@ -170,13 +170,14 @@ __global__ void __launch_bounds__(kFnvWarps * 32) fnv_leaf_kernel(const __grid_c
 //  1. the low byte of lo evolves on its own: l' = ((l ^ b) p) & 0xff;
 //  2. lo ^ b = lo + d with d = (l ^ b) - l, so lo' = (lo + d) p, and over a chunk of m bytes
 //     lo_end = p^m lo_start + B, where B depends only on the chunk's bytes and the low
-//     byte of lo_start;
+//     byte of lo_start (so the chain run from lo = that low byte alone gives B);
 //  3. hi' = hi p + t with t a function of lo and b alone, so hi_end = p^m hi_start + H,
 //     where H is the chunk's hi run from 0 along the true lo sequence.
-// Pass 1 tabulates (l_end, B) for all 256 starting low bytes of every chunk; pass 2 walks
-// the chunks of a buffer serially with one table lookup each, giving every chunk's lo_start;
-// pass 3 runs every chunk exactly from its lo_start with hi = 0, giving H; pass 4 folds the
-// H values into hi.  The result equals the serial chain bit for bit.
+// Passes: (1) l_end for all 256 starting low bytes of every chunk; (2) per buffer, walk the
+// chunks' low bytes through those tables; (3) per chunk, B from its starting low byte;
+// (4) per buffer, lo at every chunk start (lo' = p^m lo + B); (5) per chunk, H from the true
+// lo start; (6) per buffer, fold the H values into hi.  The result equals the serial chain
+// bit for bit.
 
 // p^e mod 2^32 by square and multiply
 __device__ __forceinline__ uint32_t fnv_pow(uint32_t e) {
@@ -188,11 +189,12 @@ __device__ __forceinline__ uint32_t fnv_pow(uint32_t e) {
 
 struct FnvScratch {
   uint64_t *leaves;   // [total leaves]
-  uint32_t *btab;     // [chunks][256]
-  uint8_t *ltab;      // [chunks][256]
+  uint8_t *ltab;      // [chunks][256]: low byte at the chunk's end per starting low byte
+  uint32_t *lstart;   // [chunks]: low byte of lo at the chunk's start
+  uint32_t *bpart;    // [chunks]: B
   uint32_t *lo_start; // [chunks]
-  uint32_t *hpart;    // [chunks]
-  uint64_t *head;     // [n]: (hi after LE64(nbytes)) << 32 | lo at the end of the leaf stream
+  uint32_t *hpart;    // [chunks]: H
+  uint64_t *head;     // [n]: hi << 32 | lo after LE64(nbytes); lo replaced by the final lo
 };
 
 __device__ __forceinline__ uint32_t find_chunk_buf(const FnvBatch &b, uint32_t c) {
@@ -204,33 +206,49 @@ __device__ __forceinline__ uint32_t find_chunk_buf(const FnvBatch &b, uint32_t c
   return lo;
 }
 
-// Pass 1: one block per chunk, one thread per starting low byte; the chunk's digests are
-// staged in shared memory and read as broadcasts.
-__global__ void __launch_bounds__(256) fnv_table_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
-  __shared__ uint64_t words[kChunkWords];
-  const uint32_t c = blockIdx.x;
+// Leaf digests [first, last) of chunk c.
+__device__ __forceinline__ void chunk_range(const FnvBatch &b, uint32_t c, uint64_t &first, uint64_t &last) {
   const uint32_t t = find_chunk_buf(b, c);
-  const uint64_t first = b.leaf_prefix[t] + (uint64_t)(c - b.chunk_prefix[t]) * kChunkWords;
-  const uint32_t w = (uint32_t)min((uint64_t)kChunkWords, b.leaf_prefix[t + 1] - first);
-  for (uint32_t i = threadIdx.x; i < w; i += blockDim.x) words[i] = sc.leaves[first + i];
+  first = b.leaf_prefix[t] + (uint64_t)(c - b.chunk_prefix[t]) * kChunkWords;
+  last = min(first + kChunkWords, b.leaf_prefix[t + 1]);
+}
+
+// Pass 1: one block of 64 threads per chunk, four starting low bytes per thread, two per
+// register in 16-bit lanes: (u 0xb3) < 2^16 for u < 256 and 0xb3 = p mod 256, so one
+// multiply advances two starts and the lanes never carry into each other.  The mask of one
+// byte step merges with the xor of the next (one three-input logic op).  The chunk's
+// digests are staged in shared memory and read as broadcasts.
+__global__ void __launch_bounds__(64) fnv_table_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
+  __shared__ uint64_t words[kChunkWords];
+  const uint32_t c = blockIdx.x, tid = threadIdx.x;
+  uint64_t first, last;
+  chunk_range(b, c, first, last);
+  const uint32_t w = (uint32_t)(last - first);
+  for (uint32_t i = tid; i < w; i += blockDim.x) words[i] = sc.leaves[first + i];
   __syncthreads();
-  uint32_t l = threadIdx.x, B = 0;
+  constexpr uint32_t kMask = 0x00ff00ffu;
+  uint32_t r0 = tid | (tid + 64) << 16, r1 = (tid + 128) | (tid + 192) << 16;
   for (uint32_t i = 0; i < w; ++i) {
     const uint64_t v = words[i];
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
-      const uint32_t u = l ^ (uint32_t)((v >> (8 * k)) & 0xffu);
-      B = (B + u - l) * kFnvP;
-      l = (u * kFnvP) & 0xffu;
+      const uint32_t half = k < 4 ? (uint32_t)v : (uint32_t)(v >> 32);
+      const uint32_t bb = __byte_perm(half, 0, 0x4040u | (k & 3) | (k & 3) << 8);  // b in both lanes
+      r0 = ((r0 & kMask) ^ bb) * 0xb3u;
+      r1 = ((r1 & kMask) ^ bb) * 0xb3u;
     }
   }
-  sc.btab[(size_t)c * 256 + threadIdx.x] = B;
-  sc.ltab[(size_t)c * 256 + threadIdx.x] = (uint8_t)l;
+  uint8_t *lt = sc.ltab + (size_t)c * 256;
+  lt[tid] = (uint8_t)r0;
+  lt[tid + 64] = (uint8_t)(r0 >> 16);
+  lt[tid + 128] = (uint8_t)r1;
+  lt[tid + 192] = (uint8_t)(r1 >> 16);
 }
 
 // Serial chain over leaves [l0, l1) from state h; kCombineAhead digests are loaded ahead.
 constexpr int kCombineAhead = 16;
-__device__ __forceinline__ void fnv_leaf_run(Fnv &h, const uint64_t *leaves, uint64_t l0, uint64_t l1) {
+template <class H>
+__device__ __forceinline__ void fnv_leaf_run(H &h, const uint64_t *leaves, uint64_t l0, uint64_t l1) {
   uint64_t r[kCombineAhead];
 #pragma unroll
   for (int j = 0; j < kCombineAhead; ++j) r[j] = l0 + j < l1 ? leaves[l0 + j] : 0;
@@ -247,21 +265,30 @@ __device__ __forceinline__ void fnv_leaf_run(Fnv &h, const uint64_t *leaves, uin
   }
 }
 
+// The low word alone (fact 2): what pass 3 needs.
+struct FnvLo {
+  uint32_t lo;
+  __device__ __forceinline__ void le64(uint64_t v) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) lo = (lo ^ (uint32_t)((v >> (8 * k)) & 0xffu)) * kFnvP;
+  }
+};
+
 // One warp per buffer.  Small buffers: lane 0 runs the whole chain.  Chunked buffers: pass 2,
-// the lo walk, in lane 0, over table rows the warp copies into a shared-memory ring
+// the low-byte walk, in lane 0, over table rows the warp copies into a shared-memory ring
 // kWalkAhead chunks ahead (one lookup per chunk instead of one L2 round trip).
 constexpr int kWalkAhead = 8;
 
 __global__ void __launch_bounds__(32) fnv_combine_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
-  __shared__ __align__(16) uint32_t rows[kWalkAhead][256];
+  __shared__ __align__(16) uint8_t rows[kWalkAhead][256];
   const uint32_t t = blockIdx.x;
   const int lane = threadIdx.x;
   const uint64_t l0 = b.leaf_prefix[t], l1 = b.leaf_prefix[t + 1];
   const uint32_t c0 = b.chunk_prefix[t], c1 = b.chunk_prefix[t + 1];
+  Fnv h;
+  h.le64(b.nbytes[t]);
   if (c0 == c1) {
     if (lane == 0) {
-      Fnv h;
-      h.le64(b.nbytes[t]);
       fnv_leaf_run(h, sc.leaves, l0, l1);
       *b.out[t] = h.value();
     }
@@ -270,42 +297,63 @@ __global__ void __launch_bounds__(32) fnv_combine_kernel(const __grid_constant__
   const uint32_t nc = c1 - c0;
   // row of chunk c0 + j into slot j % kWalkAhead; one commit group per call, empty past the end
   auto fetch = [&](uint32_t j) {
-    if (j < nc) {
-      const uint32_t *src = sc.btab + (size_t)(c0 + j) * 256 + lane * 4;
-      uint32_t *dst = rows[j % kWalkAhead] + lane * 4;
-      cp_async16(smem_u32(dst), src);
-      cp_async16(smem_u32(dst + 128), src + 128);
-    }
+    if (j < nc && lane < 16)
+      cp_async16(smem_u32(rows[j % kWalkAhead] + lane * 16), sc.ltab + (size_t)(c0 + j) * 256 + lane * 16);
     cp_async_commit();
   };
   for (uint32_t j = 0; j < (uint32_t)kWalkAhead; ++j) fetch(j);
-  Fnv h;
-  h.le64(b.nbytes[t]);
-  const uint32_t pfull = fnv_pow(8 * kChunkWords);
-  uint32_t lo = h.lo;
+  uint32_t l = h.lo & 0xffu;
   for (uint32_t j = 0; j < nc; ++j) {
-    cp_async_wait<kWalkAhead - 1>();  // this lane's copies of row j have landed
+    cp_async_wait<kWalkAhead - 1>();  // this lane's copy of row j has landed
     __syncwarp();                     // and every lane's
     if (lane == 0) {
-      sc.lo_start[c0 + j] = lo;
-      const uint64_t first = l0 + (uint64_t)j * kChunkWords;
-      const uint32_t w = (uint32_t)min((uint64_t)kChunkWords, l1 - first);
-      lo = (w == kChunkWords ? pfull : fnv_pow(8 * w)) * lo + rows[j % kWalkAhead][lo & 0xffu];
+      sc.lstart[c0 + j] = l;
+      l = rows[j % kWalkAhead][l];
     }
     __syncwarp();  // lane 0 is done with slot j % kWalkAhead before it is refilled
     fetch(j + kWalkAhead);
   }
   cp_async_wait<0>();
-  if (lane == 0) sc.head[t] = ((uint64_t)h.hi << 32) | lo;
+  if (lane == 0) sc.head[t] = h.value();
 }
 
-// Pass 3: one thread per chunk, the exact chain from (lo_start, 0).
+// Pass 3: one thread per chunk, the low word from its starting low byte: B = lo_end - p^m l.
+__global__ void fnv_bpart_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
+  const uint32_t c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= b.chunk_prefix[b.n]) return;
+  uint64_t first, last;
+  chunk_range(b, c, first, last);
+  const uint32_t l = sc.lstart[c];
+  FnvLo h{l};
+  fnv_leaf_run(h, sc.leaves, first, last);
+  sc.bpart[c] = h.lo - fnv_pow(8 * (uint32_t)(last - first)) * l;
+}
+
+// Pass 4: one thread per chunked buffer, lo at every chunk start.
+__global__ void fnv_scan_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
+  const uint32_t t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= b.n) return;
+  const uint32_t c0 = b.chunk_prefix[t], c1 = b.chunk_prefix[t + 1];
+  if (c0 == c1) return;
+  const uint64_t l0 = b.leaf_prefix[t], l1 = b.leaf_prefix[t + 1];
+  const uint32_t pfull = fnv_pow(8 * kChunkWords);
+  const uint64_t head = sc.head[t];
+  uint32_t lo = (uint32_t)head;
+  for (uint32_t c = c0; c < c1; ++c) {
+    sc.lo_start[c] = lo;
+    const uint64_t first = l0 + (uint64_t)(c - c0) * kChunkWords;
+    const uint32_t w = (uint32_t)min((uint64_t)kChunkWords, l1 - first);
+    lo = (w == kChunkWords ? pfull : fnv_pow(8 * w)) * lo + sc.bpart[c];
+  }
+  sc.head[t] = (head & 0xffffffff00000000ull) | lo;
+}
+
+// Pass 5: one thread per chunk, the exact chain from (lo_start, 0).
 __global__ void fnv_exact_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
   const uint32_t c = blockIdx.x * blockDim.x + threadIdx.x;
   if (c >= b.chunk_prefix[b.n]) return;
-  const uint32_t t = find_chunk_buf(b, c);
-  const uint64_t first = b.leaf_prefix[t] + (uint64_t)(c - b.chunk_prefix[t]) * kChunkWords;
-  const uint64_t last = min(first + kChunkWords, b.leaf_prefix[t + 1]);
+  uint64_t first, last;
+  chunk_range(b, c, first, last);
   Fnv h;
   h.lo = sc.lo_start[c];
   h.hi = 0;
@@ -313,7 +361,7 @@ __global__ void fnv_exact_kernel(const __grid_constant__ FnvBatch b, FnvScratch 
   sc.hpart[c] = h.hi;
 }
 
-// Pass 4: one thread per chunked buffer, hi folded over its chunks.
+// Pass 6: one thread per chunked buffer, hi folded over its chunks.
 __global__ void fnv_finish_kernel(const __grid_constant__ FnvBatch b, FnvScratch sc) {
   const uint32_t t = blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= b.n) return;
@@ -352,14 +400,16 @@ __global__ void fnv_plain_kernel(const __grid_constant__ FnvBatch b) {
 
 static size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
 
-// Scratch layout of one batch: leaves, btab, ltab, lo_start, hpart, head (256-byte aligned).
+// Scratch layout of one batch: leaves, ltab, lstart, bpart, lo_start, hpart, head
+// (256-byte aligned).
 static FnvScratch fnv_layout(const FnvBatch &b, void *base, size_t *bytes) {
   const uint64_t L = b.leaf_prefix[b.n];
   const uint64_t C = b.chunk_prefix[b.n];
-  size_t off[6];
+  constexpr int kParts = 7;
+  const size_t len[kParts] = {L * 8, C * 256, C * 4, C * 4, C * 4, C * 4, (size_t)b.n * 8};
+  size_t off[kParts];
   size_t o = 0;
-  const size_t len[6] = {L * 8, C * 256 * 4, C * 256, C * 4, C * 4, (size_t)b.n * 8};
-  for (int i = 0; i < 6; ++i) {
+  for (int i = 0; i < kParts; ++i) {
     off[i] = o;
     o = align256(o + len[i]);
   }
@@ -367,11 +417,12 @@ static FnvScratch fnv_layout(const FnvBatch &b, void *base, size_t *bytes) {
   FnvScratch sc;
   const uintptr_t p = reinterpret_cast<uintptr_t>(base);
   sc.leaves = reinterpret_cast<uint64_t *>(p + off[0]);
-  sc.btab = reinterpret_cast<uint32_t *>(p + off[1]);
-  sc.ltab = reinterpret_cast<uint8_t *>(p + off[2]);
-  sc.lo_start = reinterpret_cast<uint32_t *>(p + off[3]);
-  sc.hpart = reinterpret_cast<uint32_t *>(p + off[4]);
-  sc.head = reinterpret_cast<uint64_t *>(p + off[5]);
+  sc.ltab = reinterpret_cast<uint8_t *>(p + off[1]);
+  sc.lstart = reinterpret_cast<uint32_t *>(p + off[2]);
+  sc.bpart = reinterpret_cast<uint32_t *>(p + off[3]);
+  sc.lo_start = reinterpret_cast<uint32_t *>(p + off[4]);
+  sc.hpart = reinterpret_cast<uint32_t *>(p + off[5]);
+  sc.head = reinterpret_cast<uint64_t *>(p + off[6]);
   return sc;
 }
 
@@ -399,7 +450,7 @@ size_t fnv_fill_batch(FnvBatch &b, const void *const *ptr, const uint64_t *nbyte
 
 int fnv_tree_launches(const FnvBatch &b) {
   if (b.n == 0) return 0;
-  return (b.leaf_prefix[b.n] ? 1 : 0) + 1 + (b.chunk_prefix[b.n] ? 3 : 0);
+  return (b.leaf_prefix[b.n] ? 1 : 0) + 1 + (b.chunk_prefix[b.n] ? 5 : 0);
 }
 
 cudaError_t launch_fnv_tree(const FnvBatch &b, void *scratch, cudaStream_t s) {
@@ -416,12 +467,16 @@ cudaError_t launch_fnv_tree(const FnvBatch &b, void *scratch, cudaStream_t s) {
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (chunks) {
-    fnv_table_kernel<<<chunks, 256, 0, s>>>(b, sc);
+    fnv_table_kernel<<<chunks, 64, 0, s>>>(b, sc);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   fnv_combine_kernel<<<b.n, 32, 0, s>>>(b, sc);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (chunks) {
+    fnv_bpart_kernel<<<(chunks + 127) / 128, 128, 0, s>>>(b, sc);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    fnv_scan_kernel<<<(b.n + 127) / 128, 128, 0, s>>>(b, sc);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
     fnv_exact_kernel<<<(chunks + 127) / 128, 128, 0, s>>>(b, sc);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     fnv_finish_kernel<<<(b.n + 127) / 128, 128, 0, s>>>(b, sc);

@@ -33,7 +33,11 @@ struct FnvBatch {
 // bytes launch_fnv_tree needs for the batch (leaf digests, then the chunk tables).
 size_t fnv_fill_batch(FnvBatch &b, const void *const *ptr, const uint64_t *nbytes, uint64_t *const *out, size_t n);
 
-// Kernel launches of launch_fnv_tree for the batch: leaves, combine, and the three chunk passes.
+// Device scratch per chunk of the parallel second level: a 256-entry low-byte table and four
+// 32-bit words (starting low byte, B, starting lo, H).
+constexpr size_t kChunkScratchBytes = 256 + 4 * 4;
+
+// Kernel launches of launch_fnv_tree for the batch: leaves, combine, and five chunk passes.
 int fnv_tree_launches(const FnvBatch &b);
 
 cudaError_t launch_fnv_tree(const FnvBatch &b, void *scratch, cudaStream_t s);

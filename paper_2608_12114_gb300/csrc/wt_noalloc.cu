@@ -10,7 +10,7 @@
 // uses a fixed array compiled into the library instead.
 //
 // The array below is a file-scope __device__ object: every GPU that loads this
-// library holds its ~11 MiB until the process exits.  Host code cannot use its
+// library holds its ~9 MiB until the process exits.  Host code cannot use its
 // name as a device address, so the first call on each device (with that device
 // current) asks the runtime for the address with cudaGetSymbolAddress and
 // caches it; that first call should come before any stream capture.  All calls
@@ -30,7 +30,8 @@ constexpr uint64_t kNoAllocMaxLeaves = 1ull << 20;  // 4096-byte leaves: 4 GiB o
 // leaf digests plus the chunk tables of the parallel second level (at most one chunk per
 // kChunkWords leaves and one partial chunk per buffer of a batch)
 constexpr uint64_t kNoAllocWords =
-    kNoAllocMaxLeaves + ((kNoAllocMaxLeaves / wt::kChunkWords + wt::kMaxFnv) * 1288 + wt::kMaxFnv * 8 + 2048) / 8;
+    kNoAllocMaxLeaves +
+    ((kNoAllocMaxLeaves / wt::kChunkWords + wt::kMaxFnv) * wt::kChunkScratchBytes + wt::kMaxFnv * 8 + 2048) / 8;
 __device__ __align__(256) uint64_t g_noalloc_leaves[kNoAllocWords];
 
 std::mutex g_mu;
