@@ -216,8 +216,9 @@ int wt_checksum_plain(wt_handle *h, const void *const *ptr, const uint64_t *nbyt
  * the allocator it serves), programs whose device memory is all handed to
  * their own pool, and loops that cannot take the device-wide synchronisation
  * of cudaFree.  The paper has no counterpart; this is a library convenience.
- * No handle is needed.  The leaf digests live in an 8 MiB array compiled into
- * the library (every GPU that loads the library keeps it until exit); a call
+ * No handle is needed.  The leaf digests and the chunk tables of the parallel
+ * second level live in an array of about 8.7 MiB compiled into the library
+ * (every GPU that loads the library keeps it until exit); a call
  * whose buffers need more than 1,048,576 leaves of 4096 bytes (4 GiB of input
  * in total) is rejected with WT_EINVAL.  The first call on each device looks
  * up that array's device address (cudaGetSymbolAddress) with the device
