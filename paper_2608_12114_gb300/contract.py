@@ -18,11 +18,10 @@ from __future__ import annotations
 import itertools
 import statistics
 import time
-from typing import Dict, List, Optional, Tuple
 
 import numpy as np
 
-from . import pipeline, synth, wt
+from . import synth, wt
 
 CELLS = [c for c in itertools.product((1, 0), repeat=3)]  # (C1, C2, C3)
 ORDERINGS = ("stream", "event", "host_event", "drain")

@@ -1,7 +1,6 @@
 """The map endpoint (Sec. 8.1, contract C1): the GEMV reads W in place from the file mapping
 over the host link.  Parity against the oracle, determinism, mixing with resident matrices
 in one pass, refusals, and Algorithm 2 measured on this GPU."""
-import numpy as np
 import pytest
 
 import oracle

@@ -1,7 +1,6 @@
 """The N > 1 host logic of bench.py (replicas, one per GPU, no data-path collective) on
 CPU: two gloo ranks on 127.0.0.1, each with its own timings."""
 import multiprocessing as mp
-import os
 import socket
 
 import pytest

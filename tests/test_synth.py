@@ -1,5 +1,4 @@
 """The seeded workloads have the shapes, sizes and structure they are meant to have."""
-import os
 
 import numpy as np
 
