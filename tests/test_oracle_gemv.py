@@ -181,11 +181,13 @@ def test_q8_one_hot_gives_scaled_column_and_matches_numpy():
 
 # ----------------------------------------------------------------------------- T activation columns
 
-def test_cols_integer_exact_and_orientation():
+@pytest.mark.parametrize("T", [1, 5, 8, 9, 16])
+def test_cols_integer_exact_and_orientation(T):
     """X is [T, K] row-major: column t of the result uses row t of X.  Distinct integer
-    columns make a transposed or shared X fail."""
-    rng = np.random.default_rng(31)
-    M, K, T = 6, 40, 5
+    columns make a transposed or shared X fail.  T spans one column, both sides of the
+    8-column tile boundary and the largest T."""
+    rng = np.random.default_rng(31 + T)
+    M, K = 6, 40
     W = rng.integers(-8, 9, (M, K))
     X = rng.integers(-4, 5, (T, K))
     Y, A = oracle.gemv_cols(enc(W, BF16), BF16, M, K, enc(X, BF16), T)
