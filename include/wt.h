@@ -73,6 +73,10 @@ extern "C" {
  * PREFAULT     populate every mapping's page-table entries at open
  *              (MADV_POPULATE_READ); otherwise wt_adopt populates each batch's
  *              source range just before it enqueues that batch.
+ * TIMELINE     record a timing event before and after every ingest batch of
+ *              wt_adopt and every GEMV group of wt_pass (outside stream capture),
+ *              for wt_trace: the per-tensor overlap timeline of the first use.
+ *              The ready events wt_adopt returns then carry timing too.
  */
 #define WT_ROUTE_AUTO 0u
 #define WT_ROUTE_REGISTER 1u
@@ -81,6 +85,7 @@ extern "C" {
 #define WT_ROUTE_MASK 3u
 #define WT_OPEN_HOST_ONLY (1u << 4)
 #define WT_OPEN_PREFAULT (1u << 5)
+#define WT_OPEN_TIMELINE (1u << 6)  /* timing events around every ingest batch and GEMV group (wt_trace) */
 
 /* ---- wt_adopt modes ---------------------------------------------------------
  *   GATHER   SM gather kernel: 16-byte vector loads from the device-readable
@@ -158,6 +163,14 @@ int wt_tensor_info(const wt_handle *h, size_t i, wt_tensor_meta *out);
 int wt_find(const wt_handle *h, const char *name, size_t *i);
 /* Route actually taken for file f (WT_ROUTE_REGISTER / DIRECT / NONE). */
 int wt_file_route(const wt_handle *h, size_t f, unsigned *route);
+/* The cudaHostRegister flags file f's registration holds: cudaHostRegisterMapped (0x02),
+ * with cudaHostRegisterReadOnly (0x08) when the driver accepted read-only registration of
+ * the file-backed pages, or 0 when the file is not registered (routes DIRECT and NONE).
+ * The REGISTER route asks for read-only first and, when the driver refuses it, registers
+ * the PROT_READ mapping without the flag; this call tells the two apart (Sec. 5.1: the
+ * read-only intent is then enforced by the mapping's protection and the host-side checks,
+ * not by the registration).  Errors: WT_EINVAL. */
+int wt_file_registration(const wt_handle *h, size_t f, unsigned *flags);
 
 /* Copy tensors idx[0..n) into device memory dst[0..n) (each at least nbytes of
  * that tensor, 16-byte aligned for the vector path) on `stream`, in order.
@@ -220,14 +233,46 @@ int wt_checksum_plain(wt_handle *h, const void *const *ptr, const uint64_t *nbyt
  * second level live in an array of about 8.7 MiB compiled into the library
  * (every GPU that loads the library keeps it until exit); a call
  * whose buffers need more than 1,048,576 leaves of 4096 bytes (4 GiB of input
- * in total) is rejected with WT_EINVAL.  The first call on each device looks
- * up that array's device address (cudaGetSymbolAddress) with the device
- * current; make that first call before any stream capture.  Calls share the
+ * in total) is rejected with WT_EINVAL, before any CUDA call.  The first call on each device
+ * looks up that array's device address (cudaGetSymbolAddress) with the device
+ * current and remembers it with the CUDA context that was current; make that first call
+ * before any stream capture.  Under another context (after cudaDeviceReset, or a context
+ * created through the driver API) the array is a different one and the address is looked
+ * up again, so such a first call, too, belongs outside a capture.  Calls share the
  * array, so two calls whose kernels overlap on the GPU race; calls ordered on
  * one stream do not.  Nothing in the array needs clearing between calls.
  * Errors: WT_EINVAL (NULL array or buffer, too large), WT_ECUDA. */
 int wt_checksum_noalloc(const void *const *ptr, const uint64_t *nbytes, size_t n, uint64_t *out_dev,
                         void *stream);
+
+/* One record of the first-use timeline (handles opened with WT_OPEN_TIMELINE).  An ingest
+ * record is one batch of wt_adopt: begin when its stream reached the batch, end when its
+ * bytes had landed (the ready event of its tensors).  A GEMV record is one group of wt_pass:
+ * begin when its stream had waited for the group's event and reached its first launch, end
+ * when its last launch had finished.  Contract C3 (Table "tab:contract"; Sec. 4.3) holds
+ * when each group begins right after its batch ends, not after the last batch. */
+#define WT_TRACE_INGEST 0
+#define WT_TRACE_GEMV 1
+typedef struct {
+  int32_t kind;      /* WT_TRACE_INGEST or WT_TRACE_GEMV */
+  int32_t pad;
+  uint64_t index;    /* ordinal of the batch (or group) within the handle, in enqueue order */
+  uint64_t bytes;    /* bytes the batch moved, or weight bytes the group's GEMVs stream */
+  void *event;       /* ingest: the batch's ready event, as wt_adopt returned it for the
+                        tensors whose last byte the batch holds; GEMV: the wait_event of the
+                        group's descriptors (NULL: none) */
+  double begin_ms;   /* milliseconds from the origin event */
+  double end_ms;
+} wt_trace_rec;
+
+/* Read the handle's timeline: waits for every recorded event, writes the first min(cap, *n)
+ * records (in enqueue order, ingest batches and GEMV groups interleaved as they were
+ * enqueued) with times relative to `origin` (a cudaEvent_t created with timing and recorded
+ * before the traced work, e.g. on the ingest stream just before wt_adopt), sets *n to the
+ * number recorded, then releases them (a second call returns only later records).  Blocks
+ * the calling thread.  Errors: WT_EINVAL (NULL argument, handle without WT_OPEN_TIMELINE),
+ * WT_ECUDA (e.g. origin without timing, or not recorded). */
+int wt_trace(wt_handle *h, void *origin, wt_trace_rec *out, size_t cap, size_t *n);
 
 /* Device-side status word of the handle: 0, or the first WT_ETIMEDOUT-class
  * code a bounded wait inside a kernel recorded (reads it synchronously). */
@@ -242,6 +287,21 @@ int wt_residency(const wt_handle *h, uint64_t *resident, uint64_t *total);
 
 /* Kernels this handle has launched so far (gather, GEMV, checksum launches). */
 int wt_kernel_launches(const wt_handle *h, uint64_t *n);
+
+/* Objects the library holds right now, over all handles of the process: open handles,
+ * cached launch plans, CUDA events it created, and the device and pinned host bytes it
+ * allocated itself (status words, plan tables, split-K workspaces, the staged ring).  Buffers
+ * the caller owns are not counted.  After wt_close of every handle all five return to their
+ * earlier values (Sec. 5.1: a producer's lifetime leaves nothing behind; the 200-cycle checks
+ * read these).  Errors: WT_EINVAL. */
+typedef struct {
+  int64_t handles;
+  int64_t plans;
+  int64_t events;
+  int64_t device_bytes;
+  int64_t pinned_bytes;
+} wt_live_counts;
+int wt_live(wt_live_counts *out);
 
 /* Wait for the library's own enqueued work that reads the mappings, then
  * cudaHostUnregister, munmap, destroy events, free library allocations.

@@ -12,6 +12,9 @@ namespace wt {
 // ---------------------------------------------------------------- FNV-1a-64
 constexpr int kMaxFnv = 512;  // buffers per launch: the batch is an 18 KB kernel parameter
 constexpr uint64_t kLeafBytes = 4096;
+// Largest buffer a digest call accepts (1 TiB, above any device's memory): bounds the leaf and
+// chunk counts so that no size the caller passes can wrap them.
+constexpr uint64_t kMaxFnvBufferBytes = 1ull << 40;
 
 // The tree digest's second level is a serial FNV chain over 8 bytes per leaf.  Buffers of
 // more than kParallelLeaves leaves split that chain into chunks of kChunkWords leaf digests

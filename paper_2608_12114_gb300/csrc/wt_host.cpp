@@ -22,6 +22,7 @@
 #include <condition_variable>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <functional>
 #include <list>
@@ -69,6 +70,41 @@ int cuda_err(cudaError_t e, const char *what) {
     cudaError_t e_ = (call);                            \
     if (e_ != cudaSuccess) return cuda_err(e_, #call);  \
   } while (0)
+
+// Live objects of the library (wt_live): handles, launch plans, CUDA events, and the device
+// and pinned host bytes the library itself allocated.  Every create/allocate below goes
+// through these helpers so that a leak shows up as a count that does not return.
+std::atomic<int64_t> g_live_handles{0}, g_live_plans{0}, g_live_events{0}, g_dev_bytes{0}, g_pinned_bytes{0};
+
+cudaError_t ev_create(cudaEvent_t *ev, unsigned flags) {
+  const cudaError_t e = cudaEventCreateWithFlags(ev, flags);
+  if (e == cudaSuccess) g_live_events++;
+  return e;
+}
+
+void ev_destroy(cudaEvent_t ev) {
+  if (ev && cudaEventDestroy(ev) == cudaSuccess) g_live_events--;
+}
+
+cudaError_t dev_alloc(void **p, size_t n) {
+  const cudaError_t e = cudaMalloc(p, n);
+  if (e == cudaSuccess) g_dev_bytes += (int64_t)n;
+  return e;
+}
+
+void dev_free(void *p, size_t n) {
+  if (p && cudaFree(p) == cudaSuccess) g_dev_bytes -= (int64_t)n;
+}
+
+cudaError_t pinned_alloc(void **p, size_t n) {
+  const cudaError_t e = cudaHostAlloc(p, n, cudaHostAllocDefault);
+  if (e == cudaSuccess) g_pinned_bytes += (int64_t)n;
+  return e;
+}
+
+void pinned_free(void *p, size_t n) {
+  if (p && cudaFreeHost(p) == cudaSuccess) g_pinned_bytes -= (int64_t)n;
+}
 
 constexpr uint64_t kAlign = 64;
 constexpr int kMaxDims = 4;
@@ -181,6 +217,7 @@ struct File {
   size_t size = 0;
   unsigned route = WT_ROUTE_NONE;
   bool registered = false;
+  unsigned reg_flags = 0;        // cudaHostRegister flags the registration holds (0: none)
   bool populated = false;        // page-table entries already filled (registered files)
   const uint8_t *dev = nullptr;  // device-readable address of base
   std::vector<Tensor> tensors;
@@ -220,6 +257,7 @@ struct Plan {
     uint32_t reduce_rows = 0;
     std::vector<Generic> generic;
     std::vector<Zero> zero;
+    uint64_t wbytes = 0;         // weight bytes the group streams (timeline records)
   };
   std::vector<Group> groups;
   std::vector<uint8_t> table;
@@ -230,6 +268,7 @@ struct Plan {
   bool sent = false;
   cudaStream_t sent_on = nullptr;
   bool pinned = false;  // used inside a captured CUDA graph: kept until wt_close
+  size_t table_bytes = 0;  // size of `host` and `dev`
   float *ws = nullptr;  // split-K segment partials (device), ws_floats floats
   size_t ws_floats = 0;
   std::vector<std::pair<size_t, size_t>> ws_patches;  // (table byte offset of a pointer, ws float offset)
@@ -252,6 +291,18 @@ struct wt_handle {
   std::vector<std::pair<uint32_t, uint32_t>> order;  // global tensor index -> (file, entry)
   bool host_only = false;
   bool prefaulted = false;
+  // WT_OPEN_TIMELINE: timing events around every ingest batch and every GEMV group, read
+  // back (and released) by wt_trace
+  struct TraceEv {
+    int kind;
+    uint64_t index, bytes;
+    cudaEvent_t begin, end;
+    bool own_end;       // an ingest batch's end event is its ready event, owned by `events`
+    cudaEvent_t event;  // ingest: the batch's ready event; GEMV: the event the group waited on
+  };
+  bool timeline = false;
+  std::vector<TraceEv> trace;
+  uint64_t n_batches = 0, n_groups = 0;
   int device = -1;
   int *status = nullptr;
   std::vector<cudaEvent_t> events;
@@ -418,8 +469,20 @@ bool inside_mapping(const wt_handle *h, const void *p, uint64_t n) {
 }
 
 int new_event(wt_handle *h, cudaEvent_t *ev) {
-  CU(cudaEventCreateWithFlags(ev, cudaEventDisableTiming));
+  CU(ev_create(ev, h->timeline ? cudaEventDefault : cudaEventDisableTiming));
   h->events.push_back(*ev);
+  return WT_OK;
+}
+
+// A timing event recorded on s now, kept for wt_trace (WT_OPEN_TIMELINE handles only).
+int trace_mark(cudaStream_t s, cudaEvent_t *ev) {
+  CU(ev_create(ev, cudaEventDefault));
+  const cudaError_t e = cudaEventRecord(*ev, s);
+  if (e != cudaSuccess) {
+    ev_destroy(*ev);
+    *ev = nullptr;
+    return cuda_err(e, "cudaEventRecord (timeline)");
+  }
   return WT_OK;
 }
 
@@ -504,6 +567,11 @@ int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cuda
       cv.wait(lk, [&] { return populated > b; });
     }
     const size_t i = batches[b].first, j = batches[b].second;
+    cudaEvent_t tb = nullptr;
+    if (h->timeline) {
+      int rc = trace_mark(s, &tb);
+      if (rc) return rc;
+    }
     if (mode == WT_ADOPT_GATHER) {
       wt::GatherBatch gb;
       memset(&gb, 0, sizeof gb);
@@ -527,9 +595,18 @@ int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cuda
     }
     cudaEvent_t ev;
     int rc = new_event(h, &ev);
-    if (rc) return rc;
+    if (rc) {
+      if (tb) ev_destroy(tb);
+      return rc;
+    }
     CU(cudaEventRecord(ev, s));
     for (size_t k = i; k < j; ++k) ready[ps[k].tensor] = ev;
+    if (tb) {
+      uint64_t bytes = 0;
+      for (size_t k = i; k < j; ++k) bytes += ps[k].n;
+      h->trace.push_back({WT_TRACE_INGEST, h->n_batches, bytes, tb, ev, false, ev});
+    }
+    h->n_batches++;
   }
   return WT_OK;
 }
@@ -537,8 +614,8 @@ int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cuda
 int ring_setup(wt_handle *h) {
   if (h->ring_ready) return WT_OK;
   for (int k = 0; k < Ring::kSlots; ++k) {
-    CU(cudaHostAlloc(reinterpret_cast<void **>(&h->ring.slot[k]), Ring::kSlotBytes, cudaHostAllocDefault));
-    CU(cudaEventCreateWithFlags(&h->ring.done[k], cudaEventDisableTiming));
+    CU(pinned_alloc(reinterpret_cast<void **>(&h->ring.slot[k]), Ring::kSlotBytes));
+    CU(ev_create(&h->ring.done[k], cudaEventDisableTiming));
   }
   h->ring_ready = true;
   return WT_OK;
@@ -800,10 +877,15 @@ void partition(const std::vector<wt::MatDesc> &mats, int &grid, std::vector<wt::
   constexpr uint64_t kMinCtaBytes = 64 << 10;
   grid = (int)std::max<uint64_t>(
       1, std::min<uint64_t>((uint64_t)wt::num_sms() * ctas_per_sm, (B + kMinCtaBytes - 1) / kMinCtaBytes));
-  // slices of at least kMinSliceBytes: a slice costs the consumers a reload of x, and a
-  // slice shorter than a tile makes its stages partial
-  constexpr uint64_t kMinSliceBytes = 2ull << 20;
-  slices = (int)std::max<uint64_t>(1, std::min<uint64_t>((uint64_t)slices, B / ((uint64_t)grid * kMinSliceBytes)));
+  // slices of at least 2 MiB: a slice costs the consumers a reload of x, and a slice shorter
+  // than a tile makes its stages partial.  WT_MIN_SLICE_BYTES (>= 4096) lowers the floor so
+  // that tests reach the many-slices-per-CTA partition on sets far smaller than a decoder.
+  uint64_t min_slice = 2ull << 20;
+  if (const char *e = getenv("WT_MIN_SLICE_BYTES")) {
+    const uint64_t v = strtoull(e, nullptr, 10);
+    if (v >= 4096) min_slice = v;
+  }
+  slices = (int)std::max<uint64_t>(1, std::min<uint64_t>((uint64_t)slices, B / ((uint64_t)grid * min_slice)));
   const int nslice = grid * slices;
   // cut c (1..nslice-1) at the row boundary nearest byte B*c/nslice
   std::vector<std::pair<uint32_t, uint32_t>> cuts;  // (mat, row)
@@ -950,6 +1032,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
           return set_err(WT_EINVAL, "wt_pass: an operand of desc %zu runs past the end of its device allocation", k);
       }
       const uint32_t ncol = q.cols > 0 ? (uint32_t)q.cols : 1;
+      g.wbytes += q.M * q.K * (uint64_t)es;
       if (q.K == 0) {
         g.zero.push_back({q.y, q.M * ncol});
         continue;
@@ -1096,30 +1179,32 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
     i = j;
   }
   if (P->ws_floats) {
-    CU(cudaMalloc(reinterpret_cast<void **>(&P->ws), P->ws_floats * sizeof(float)));
+    CU(dev_alloc(reinterpret_cast<void **>(&P->ws), P->ws_floats * sizeof(float)));
     for (const auto &pt : P->ws_patches) {
       const float *p = P->ws + pt.second;
       memcpy(P->table.data() + pt.first, &p, sizeof p);
     }
   }
   const size_t bytes = std::max<size_t>(16, align16(P->table.size()));
-  CU(cudaHostAlloc(reinterpret_cast<void **>(&P->host), bytes, cudaHostAllocDefault));
+  CU(pinned_alloc(reinterpret_cast<void **>(&P->host), bytes));
+  P->table_bytes = bytes;
   memcpy(P->host, P->table.data(), P->table.size());
   if (wt::fault_injected("alloc")) return set_err(WT_ENOMEM, "wt_pass: plan tables: injected allocation fault");
-  CU(cudaMalloc(reinterpret_cast<void **>(&P->dev), bytes));
-  CU(cudaEventCreateWithFlags(&P->uploaded, cudaEventDisableTiming));
-  CU(cudaEventCreateWithFlags(&P->last, cudaEventDisableTiming));
+  CU(dev_alloc(reinterpret_cast<void **>(&P->dev), bytes));
+  CU(ev_create(&P->uploaded, cudaEventDisableTiming));
+  CU(ev_create(&P->last, cudaEventDisableTiming));
   return WT_OK;
 }
 
 void destroy_plan(Plan *P) {
   if (P->last) cudaEventSynchronize(P->last);
-  if (P->dev) cudaFree(P->dev);
-  if (P->ws) cudaFree(P->ws);
-  if (P->host) cudaFreeHost(P->host);
-  if (P->uploaded) cudaEventDestroy(P->uploaded);
-  if (P->last) cudaEventDestroy(P->last);
+  dev_free(P->dev, P->table_bytes);
+  dev_free(P->ws, P->ws_floats * sizeof(float));
+  pinned_free(P->host, P->table_bytes);
+  ev_destroy(P->uploaded);
+  ev_destroy(P->last);
   delete P;
+  g_live_plans--;
 }
 
 // True if the tables of P are in device memory: the stream-ordered upload of its first use
@@ -1154,6 +1239,25 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
   for (const Plan::Group &g : P->groups) {
     cudaEvent_t wait = static_cast<cudaEvent_t>(d[g.first].wait_event);
     if (wait) CU(cudaStreamWaitEvent(s, wait, 0));
+    cudaEvent_t tb = nullptr;
+    if (h->timeline && !capturing) {
+      int rc = trace_mark(s, &tb);
+      if (rc) return rc;
+    }
+    struct TraceEnd {  // closes the group's timeline record on every path out of this scope
+      wt_handle *h;
+      cudaStream_t s;
+      cudaEvent_t tb;
+      uint64_t bytes;
+      cudaEvent_t wait;
+      ~TraceEnd() {
+        if (!tb) return;
+        cudaEvent_t te = nullptr;
+        if (trace_mark(s, &te) == WT_OK) h->trace.push_back({WT_TRACE_GEMV, h->n_groups, bytes, tb, te, true, wait});
+        else ev_destroy(tb);
+      }
+    } trace_end{h, s, tb, g.wbytes, wait};
+    if (!capturing) h->n_groups++;
     for (const Plan::Zero &z : g.zero) CU(cudaMemsetAsync(z.y, 0, z.M * sizeof(float), s));
     for (const Plan::Launch &L : g.launches) {
       wt::GemvLaunch gl;
@@ -1224,20 +1328,28 @@ int close_impl(wt_handle *h) {
     cudaGetDevice(&cur);
     if (cur != h->device) cudaSetDevice(h->device);
     for (cudaEvent_t e : h->events) cudaEventSynchronize(e);
+    for (auto &t : h->trace) {
+      ev_destroy(t.begin);
+      if (t.own_end && t.end) {
+        cudaEventSynchronize(t.end);
+        ev_destroy(t.end);
+      }
+    }
+    h->trace.clear();
     for (Plan *P : h->plans) destroy_plan(P);
     h->plans.clear();
     if (h->ring_ready) {
       for (int k = 0; k < Ring::kSlots; ++k) {
         if (h->ring.done[k]) {
           cudaEventSynchronize(h->ring.done[k]);
-          cudaEventDestroy(h->ring.done[k]);
+          ev_destroy(h->ring.done[k]);
         }
-        if (h->ring.slot[k]) cudaFreeHost(h->ring.slot[k]);
+        pinned_free(h->ring.slot[k], Ring::kSlotBytes);
       }
     }
-    for (cudaEvent_t e : h->events) cudaEventDestroy(e);
+    for (cudaEvent_t e : h->events) ev_destroy(e);
     h->events.clear();
-    if (h->status) cudaFree(h->status);
+    dev_free(h->status, 256);
     h->status = nullptr;
     for (File &f : h->files) unmap_file(f);
     if (cur >= 0 && cur != h->device) cudaSetDevice(cur);
@@ -1245,6 +1357,7 @@ int close_impl(wt_handle *h) {
     for (File &f : h->files) unmap_file(f);
   }
   delete h;
+  g_live_handles--;
   return rc;
 }
 
@@ -1283,16 +1396,19 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
   *out = nullptr;
   if (n_paths < 0 || (n_paths > 0 && !paths)) return set_err(WT_EINVAL, "wt_open: bad path list");
   const unsigned route_req = flags & WT_ROUTE_MASK;
-  if (flags & ~(WT_ROUTE_MASK | WT_OPEN_HOST_ONLY | WT_OPEN_PREFAULT))
+  if (flags & ~(WT_ROUTE_MASK | WT_OPEN_HOST_ONLY | WT_OPEN_PREFAULT | WT_OPEN_TIMELINE))
     return set_err(WT_EINVAL, "wt_open: unknown flag bits 0x%x", flags);
   wt_handle *h = nullptr;
   try {
     h = new wt_handle();
+    g_live_handles++;
     h->host_only = (flags & WT_OPEN_HOST_ONLY) != 0;
+    h->timeline = (flags & WT_OPEN_TIMELINE) != 0 && !h->host_only;
     h->files.resize(n_paths);
     for (int i = 0; i < n_paths; ++i) {
       if (!paths[i]) {
         delete h;
+        g_live_handles--;
         return set_err(WT_EINVAL, "wt_open: path %d is NULL", i);
       }
       h->files[i].path = paths[i];
@@ -1347,15 +1463,20 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
         f.route = WT_ROUTE_DIRECT;
         f.dev = f.base;
       } else if (want == WT_ROUTE_REGISTER) {
+        // Read-only registration first (the mapping is PROT_READ); a driver that refuses the
+        // flag for file-backed pages gets a plain mapped registration, and wt_file_registration
+        // reports which one the file holds.
         const bool injected = wt::fault_injected("register");
-        cudaError_t e = injected ? cudaErrorMemoryAllocation
-                                 : cudaHostRegister(f.base, f.size, cudaHostRegisterMapped | cudaHostRegisterReadOnly);
+        unsigned rf = cudaHostRegisterMapped | cudaHostRegisterReadOnly;
+        cudaError_t e = injected ? cudaErrorMemoryAllocation : cudaHostRegister(f.base, f.size, rf);
         if (e != cudaSuccess && !injected) {
           cudaGetLastError();
-          e = cudaHostRegister(f.base, f.size, cudaHostRegisterMapped);
+          rf = cudaHostRegisterMapped;
+          e = cudaHostRegister(f.base, f.size, rf);
         }
         if (e == cudaSuccess) {
           f.registered = true;
+          f.reg_flags = rf;
           f.populated = true;  // registration pins (and so maps) every page
           void *dp = nullptr;
           e = cudaHostGetDevicePointer(&dp, f.base, 0);
@@ -1376,7 +1497,7 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
         f.route = WT_ROUTE_NONE;
       }
     }
-    ce = cudaMalloc(reinterpret_cast<void **>(&h->status), 256);
+    ce = dev_alloc(reinterpret_cast<void **>(&h->status), 256);
     if (ce == cudaSuccess) ce = cudaMemset(h->status, 0, 256);
     if (ce != cudaSuccess) {
       close_impl(h);
@@ -1446,6 +1567,13 @@ int wt_file_route(const wt_handle *h, size_t f, unsigned *route) {
   if (!h || !route) return set_err(WT_EINVAL, "wt_file_route: NULL argument");
   if (f >= h->files.size()) return set_err(WT_EINVAL, "wt_file_route: file %zu out of range", f);
   *route = h->files[f].route;
+  return WT_OK;
+}
+
+int wt_file_registration(const wt_handle *h, size_t f, unsigned *flags) {
+  if (!h || !flags) return set_err(WT_EINVAL, "wt_file_registration: NULL argument");
+  if (f >= h->files.size()) return set_err(WT_EINVAL, "wt_file_registration: file %zu out of range", f);
+  *flags = h->files[f].registered ? h->files[f].reg_flags : 0u;
   return WT_OK;
 }
 
@@ -1530,6 +1658,7 @@ int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream) {
                      "with that stream synchronised, before the capture begins");
     if (!P) {
       P = new Plan();
+      g_live_plans++;
       P->key = std::move(key);
       int rc = build_plan(h, d, n, P);
       if (rc) {
@@ -1561,6 +1690,9 @@ static int checksum_impl(wt_handle *h, const void *const *ptr, const uint64_t *n
   if (!ptr || !nbytes || !out_dev) return set_err(WT_EINVAL, "wt_checksum: NULL array");
   for (size_t i = 0; i < n; ++i) {
     if (nbytes[i] && !ptr[i]) return set_err(WT_EINVAL, "wt_checksum: ptr[%zu] is NULL", i);
+    if (nbytes[i] > wt::kMaxFnvBufferBytes)
+      return set_err(WT_EINVAL, "wt_checksum: buffer %zu: %llu bytes is not a device buffer size", i,
+                     (unsigned long long)nbytes[i]);
     if (plain && nbytes[i] > (256ull << 20)) return set_err(WT_EINVAL, "wt_checksum_plain: buffer %zu above 256 MiB", i);
   }
   const cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -1628,6 +1760,46 @@ int wt_residency(const wt_handle *h, uint64_t *resident, uint64_t *total) {
 int wt_kernel_launches(const wt_handle *h, uint64_t *n) {
   if (!h || !n) return set_err(WT_EINVAL, "wt_kernel_launches: NULL argument");
   *n = h->kernel_launches;
+  return WT_OK;
+}
+
+int wt_trace(wt_handle *h, void *origin, wt_trace_rec *out, size_t cap, size_t *n) {
+  if (!h || !n || (cap && !out)) return set_err(WT_EINVAL, "wt_trace: NULL argument");
+  if (!h->timeline) return set_err(WT_EINVAL, "wt_trace: the handle was not opened with WT_OPEN_TIMELINE");
+  if (!origin) return set_err(WT_EINVAL, "wt_trace: NULL origin event");
+  std::lock_guard<std::mutex> g(h->mu);
+  const cudaEvent_t o = static_cast<cudaEvent_t>(origin);
+  CU(cudaEventSynchronize(o));
+  *n = h->trace.size();
+  for (size_t k = 0; k < h->trace.size() && k < cap; ++k) {
+    const auto &t = h->trace[k];
+    CU(cudaEventSynchronize(t.end));
+    float b = 0.f, e = 0.f;
+    CU(cudaEventElapsedTime(&b, o, t.begin));
+    CU(cudaEventElapsedTime(&e, o, t.end));
+    out[k].kind = t.kind;
+    out[k].pad = 0;
+    out[k].index = t.index;
+    out[k].bytes = t.bytes;
+    out[k].event = t.event;
+    out[k].begin_ms = b;
+    out[k].end_ms = e;
+  }
+  for (auto &t : h->trace) {
+    ev_destroy(t.begin);
+    if (t.own_end) ev_destroy(t.end);
+  }
+  h->trace.clear();
+  return WT_OK;
+}
+
+int wt_live(wt_live_counts *out) {
+  if (!out) return set_err(WT_EINVAL, "wt_live: NULL argument");
+  out->handles = g_live_handles.load();
+  out->plans = g_live_plans.load();
+  out->events = g_live_events.load();
+  out->device_bytes = g_dev_bytes.load();
+  out->pinned_bytes = g_pinned_bytes.load();
   return WT_OK;
 }
 

@@ -21,16 +21,17 @@ LIB_PATH = os.path.join(HERE, "libwt.so")
 WT_OK, WT_EINVAL, WT_EIO, WT_EFORMAT, WT_ENOMEM, WT_ECUDA, WT_ENOTSUP, WT_ETIMEDOUT = 0, -1, -2, -3, -4, -5, -6, -7
 WT_F32, WT_BF16, WT_F16, WT_I8, WT_U8 = 0, 1, 2, 3, 4
 WT_ROUTE_AUTO, WT_ROUTE_REGISTER, WT_ROUTE_DIRECT, WT_ROUTE_NONE = 0, 1, 2, 3
-WT_OPEN_HOST_ONLY, WT_OPEN_PREFAULT = 1 << 4, 1 << 5
+WT_OPEN_HOST_ONLY, WT_OPEN_PREFAULT, WT_OPEN_TIMELINE = 1 << 4, 1 << 5, 1 << 6
+WT_TRACE_INGEST, WT_TRACE_GEMV = 0, 1
 WT_ADOPT_GATHER, WT_ADOPT_CE, WT_ADOPT_STAGED = 0, 1, 2
 ROUTE_NAMES = {WT_ROUTE_REGISTER: "register", WT_ROUTE_DIRECT: "direct", WT_ROUTE_NONE: "none"}
 MODE_NAMES = {WT_ADOPT_GATHER: "gather", WT_ADOPT_CE: "ce", WT_ADOPT_STAGED: "staged"}
 
 # every entry point declared in include/wt.h
 SYMBOLS = ("wt_last_error", "wt_abi_version", "wt_open", "wt_num_tensors", "wt_num_files",
-           "wt_tensor_info", "wt_find", "wt_file_route", "wt_adopt", "wt_pass", "wt_checksum",
+           "wt_tensor_info", "wt_find", "wt_file_route", "wt_file_registration", "wt_adopt", "wt_pass", "wt_checksum",
            "wt_checksum_plain", "wt_checksum_noalloc", "wt_device_status", "wt_residency",
-           "wt_kernel_launches", "wt_close",
+           "wt_kernel_launches", "wt_trace", "wt_live", "wt_close",
            # include/wt_dlpack.h
            "wt_dlpack_file", "wt_dlpack_tensor", "wt_dlpack_release", "wt_dlpack_live")
 WT_DLPACK_DEVICE, WT_DLPACK_HOST = 0, 1
@@ -53,6 +54,16 @@ class GemvDesc(C.Structure):
     _fields_ = [("W", C.c_void_p), ("dtype", C.c_int32), ("cols", C.c_int32),
                 ("M", C.c_uint64), ("K", C.c_uint64), ("x", C.c_void_p), ("y", C.c_void_p),
                 ("wait_event", C.c_void_p), ("scale", C.c_void_p)]
+
+
+class LiveCounts(C.Structure):
+    _fields_ = [("handles", C.c_int64), ("plans", C.c_int64), ("events", C.c_int64),
+                ("device_bytes", C.c_int64), ("pinned_bytes", C.c_int64)]
+
+
+class TraceRec(C.Structure):
+    _fields_ = [("kind", C.c_int32), ("pad", C.c_int32), ("index", C.c_uint64), ("bytes", C.c_uint64),
+                ("event", C.c_void_p), ("begin_ms", C.c_double), ("end_ms", C.c_double)]
 
 
 # The same 64-byte layout as a numpy record, for building many descriptors at once.
@@ -81,6 +92,7 @@ def lib(path: str = LIB_PATH):
     L.wt_tensor_info.argtypes = [vp, sz, C.POINTER(TensorMeta)]
     L.wt_find.argtypes = [vp, C.c_char_p, C.POINTER(sz)]
     L.wt_file_route.argtypes = [vp, sz, C.POINTER(C.c_uint)]
+    L.wt_file_registration.argtypes = [vp, sz, C.POINTER(C.c_uint)]
     L.wt_adopt.argtypes = [vp, C.POINTER(sz), C.POINTER(vp), sz, C.c_uint, vp, C.POINTER(vp)]
     L.wt_pass.argtypes = [vp, C.POINTER(GemvDesc), sz, vp]
     L.wt_checksum.argtypes = [vp, C.POINTER(vp), u64p, sz, vp, vp]
@@ -89,6 +101,8 @@ def lib(path: str = LIB_PATH):
     L.wt_device_status.argtypes = [vp, C.POINTER(C.c_int)]
     L.wt_kernel_launches.argtypes = [vp, u64p]
     L.wt_residency.argtypes = [vp, u64p, u64p]
+    L.wt_trace.argtypes = [vp, vp, C.POINTER(TraceRec), sz, C.POINTER(sz)]
+    L.wt_live.argtypes = [C.POINTER(LiveCounts)]
     L.wt_close.argtypes = [vp]
     L.wt_dlpack_file.argtypes = [C.c_char_p, C.c_int32, C.c_uint64, C.c_uint64, C.c_uint, C.POINTER(vp)]
     L.wt_dlpack_tensor.argtypes = [vp, sz, C.c_uint, C.POINTER(vp)]
@@ -156,6 +170,12 @@ class Handle:
         _check(lib().wt_file_route(self.ptr, f, C.byref(r)))
         return r.value
 
+    def registration(self, f: int) -> int:
+        """wt_file_registration: cudaHostRegister flags of file f (0 when not registered)."""
+        r = C.c_uint()
+        _check(lib().wt_file_registration(self.ptr, f, C.byref(r)))
+        return r.value
+
     def adopt(self, idx: Sequence[int], dst: Sequence[int], mode: int = WT_ADOPT_GATHER,
               stream: int = 0) -> List[int]:
         """wt_adopt: returns the ready event (cudaEvent_t as int) of each tensor."""
@@ -202,6 +222,19 @@ class Handle:
         _check(lib().wt_kernel_launches(self.ptr, C.byref(v)))
         return v.value
 
+    def trace(self, origin_event: int) -> List[dict]:
+        """wt_trace (WT_OPEN_TIMELINE handles): the ingest-batch and GEMV-group records, in
+        enqueue order, with times in ms from `origin_event` (a cudaEvent_t with timing, e.g.
+        ``torch.cuda.Event(enable_timing=True).cuda_event``).  Consumes the records."""
+        n = C.c_size_t()
+        cap = 1 << 16
+        buf = (TraceRec * cap)()
+        _check(lib().wt_trace(self.ptr, C.c_void_p(origin_event), buf, cap, C.byref(n)))
+        kinds = {WT_TRACE_INGEST: "ingest", WT_TRACE_GEMV: "gemv"}
+        return [dict(kind=kinds.get(buf[i].kind, "?"), index=buf[i].index, bytes=buf[i].bytes,
+                     event=buf[i].event or 0, begin_ms=buf[i].begin_ms, end_ms=buf[i].end_ms)
+                for i in range(min(n.value, cap))]
+
     def close(self):
         if self._h is not None:
             h, self._h = self._h, None
@@ -218,6 +251,13 @@ class Handle:
             self.close()
         except Exception:
             pass
+
+
+def live() -> dict:
+    """wt_live: handles, plans, events, device and pinned bytes the library holds now."""
+    c = LiveCounts()
+    _check(lib().wt_live(C.byref(c)))
+    return {f: getattr(c, f) for f, _ in LiveCounts._fields_}
 
 
 def checksum_noalloc(ptrs: Sequence[int], nbytes: Sequence[int], out_dev: int, stream: int = 0):

@@ -134,3 +134,31 @@ def test_device_calls_refused_on_host_only_handle(L, tmp_path):
             h.pass_([wt.gemv_desc(16, wt.WT_F32, 1, 4, 16, 16)])
         assert ei.value.code == wt.WT_ENOTSUP
         assert h.device_status() == 0
+
+
+def test_live_counts_follow_handles(L, tmp_path):
+    ck = synth.build("many", str(tmp_path / "lv"), n_matrices=4)
+    base = wt.live()
+    hs = [wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY) for _ in range(3)]
+    assert wt.live()["handles"] == base["handles"] + 3
+    for h in hs:
+        h.close()
+    assert wt.live() == base
+    # a failed open leaves no handle behind
+    with pytest.raises(wt.WtError):
+        wt.Handle(ck.paths + [str(tmp_path / "missing.wt")], wt.WT_OPEN_HOST_ONLY)
+    assert wt.live() == base
+
+
+def test_registration_and_trace_queries_on_host_only_handle(L, tmp_path):
+    ck = synth.build("tiny", str(tmp_path))
+    with wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY) as h:
+        assert h.registration(0) == 0  # nothing is registered without a device route
+        with pytest.raises(wt.WtError) as ei:
+            h.registration(1)
+        assert ei.value.code == wt.WT_EINVAL
+        with pytest.raises(wt.WtError) as ei:  # no timeline: the handle was not opened with one
+            h.trace(1)
+        assert ei.value.code == wt.WT_EINVAL
+    # TIMELINE is a known flag (a host-only handle ignores it)
+    wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY | wt.WT_OPEN_TIMELINE).close()
