@@ -830,6 +830,19 @@ bool cols_on_umma(int dtype, int cols) {
   return force == 1 || (force == 0 && cols > 8);
 }
 
+// int8 weights with one activation column: the warp-level MMA kernel at T = 1 (wt_cols.cu)
+// streams the matched protocol at 6662 GB/s against 6386 for the CUDA-core kernel, which is
+// issue-bound (ncu: 66.5 % issue active, not_selected on top) while the MMA path decodes a
+// 16-byte vector straight into an MMA operand with 1.6x fewer instructions.  It takes rows up
+// to seg_vectors(int8) vectors (K <= 8192); longer rows keep the CUDA-core kernel's cross-CTA
+// split-K, since the MMA kernel gives a whole row to one CTA.  WT_I8_ONECOL=cuda keeps every
+// int8 one-column matrix on the CUDA-core kernel (its parity tests run both ways).
+bool i8_onecol_on_mma(uint32_t V) {
+  const char *e = getenv("WT_I8_ONECOL");
+  if (e && strcmp(e, "cuda") == 0) return false;
+  return V <= wt::seg_vectors(WT_I8);
+}
+
 // The two tensor maps of a tcgen05 multi-column matrix (2-byte weights; see wt::UmmaLaunch).
 int encode_umma_maps(const wt::MatDesc &m, uint8_t *out) {
   EncodeTiledFn fn = encode_tiled();
@@ -1076,6 +1089,11 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         }
       } else if (fast && q.cols > 0) {
         (cols_on_umma(q.dtype, q.cols) ? umma_dt : q.cols > 8 ? colsw_dt : cols_dt)[q.dtype].push_back(make_cols_mat(q));
+      } else if (fast && q.dtype == WT_I8 && i8_onecol_on_mma((uint32_t)(q.K / 16))) {
+        // y[M] is Y[1, M] and x[K] is X[1, K]: the one-column GEMV as the T = 1 MMA kernel
+        wt_gemv_desc q1 = q;
+        q1.cols = 1;
+        cols_dt[WT_I8].push_back(make_cols_mat(q1));
       } else if (fast && q.K * es / 16 > wt::seg_vectors(q.dtype)) {
         // long rows: column segments spread over CTAs, summed by the second pass
         const uint32_t V = (uint32_t)(q.K * es / 16);

@@ -111,6 +111,51 @@ class DeviceCheckpoint:
                 off += h.tensors[i].nbytes
         return dc
 
+    @staticmethod
+    def stream_in(h: wt.Handle, mats: Sequence[MatrixRef], mode: int = wt.WT_ADOPT_GATHER, stream: int = 0,
+                  first_bytes: int = 256 << 20, segments: int = 8, device="cuda"):
+        """Allocation (step 4) interleaved with ingest (step 5): the logical tensors are cut, at
+        tensor boundaries and in order, into a small first segment (about `first_bytes`) and
+        then `segments` segments of nearly equal bytes; each segment gets its own device slab
+        right before its wt_adopt call, so the link starts after the first small allocation
+        and every later allocation runs while earlier bytes are in flight.  Returns
+        (DeviceCheckpoint, tensor -> ready event, host seconds spent allocating)."""
+        import time
+        import torch
+        sizes = [sum(h.tensors[i].nbytes for i in m.parts) for m in mats]
+        total = sum(sizes)
+        cuts, acc, limit = [], 0, min(first_bytes, total)
+        step = max(1, -(-(total - limit) // max(1, segments)))
+        for k, n in enumerate(sizes):
+            acc += n
+            if acc >= limit and k + 1 < len(sizes):
+                cuts.append(k + 1)
+                limit = acc + step
+        bounds = [0] + cuts + [len(mats)]
+        dc = DeviceCheckpoint(list(mats), [None] * len(mats))
+        events: Dict[int, int] = {}
+        alloc_s = 0.0
+        for a, b in zip(bounds, bounds[1:]):
+            t0 = time.perf_counter()
+            offs, pos = [], 0
+            for k in range(a, b):
+                offs.append(pos)
+                pos += -(-sizes[k] // _ALIGN) * _ALIGN
+            big = torch.empty(max(pos, 1), dtype=torch.uint8, device=device)
+            alloc_s += time.perf_counter() - t0
+            idx = []
+            for k, o in zip(range(a, b), offs):
+                dc.bufs[k] = big[o:o + sizes[k]]
+                off = 0
+                for i in mats[k].parts:
+                    dc.dst[i] = dc.bufs[k].data_ptr() + off
+                    off += h.tensors[i].nbytes
+                    idx.append(i)
+            idx.sort()
+            if idx:
+                events.update(zip(idx, h.adopt(idx, [dc.dst[i] for i in idx], mode, stream)))
+        return dc, events, alloc_s
+
     def adopt(self, h: wt.Handle, mode: int = wt.WT_ADOPT_GATHER, stream: int = 0,
               order: Optional[Sequence[int]] = None) -> Dict[int, int]:
         """wt_adopt every tensor (file/index order unless `order`); returns tensor -> event."""

@@ -26,6 +26,18 @@ def torch():
     return torch
 
 
+@pytest.fixture(params=["default", "cuda"], autouse=True)
+def onecol_kernel(request, monkeypatch):
+    """Every test runs twice: with the default routing (rows up to K = 8192 on the warp-MMA
+    kernel at T = 1, longer rows on the CUDA-core kernel's split-K) and with every int8 row on
+    the CUDA-core kernel (WT_I8_ONECOL=cuda), so both kernels' tile modes stay covered."""
+    if request.param == "cuda":
+        monkeypatch.setenv("WT_I8_ONECOL", "cuda")
+    else:
+        monkeypatch.delenv("WT_I8_ONECOL", raising=False)
+    return request.param
+
+
 def check(h, dev, co, ys, ks):
     for k in ks:
         m = dev.mats[k]
