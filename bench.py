@@ -57,6 +57,8 @@ def parse_args():
     p.add_argument("--workload", default="large")
     p.add_argument("--layers", type=int, default=None, help="override decoder layer count (small profiling cases)")
     p.add_argument("--mode", default="gather", choices=["gather", "ce", "staged"])
+    p.add_argument("--open", default="map", choices=["map", "nomap"],
+                   help="nomap: wt_open maps nothing (WT_OPEN_NOMAP) and --mode staged preads into the pinned ring")
     p.add_argument("--e2e-reps", type=int, default=5)
     p.add_argument("--skip-e2e", action="store_true", help="resident passes only (profiling runs)")
     p.add_argument("--arms", action="store_true", help="also time the ce/staged/stock-torch ingest arms")
@@ -464,6 +466,7 @@ def run_wt(args, rank, world):
         dist.barrier()
     build.build()  # no-op when fresh; loads the same in-tree library on every rank
     mode = {"gather": wt.WT_ADOPT_GATHER, "ce": wt.WT_ADOPT_CE, "staged": wt.WT_ADOPT_STAGED}[args.mode]
+    oflags = wt.WT_OPEN_NOMAP if args.open == "nomap" else 0
 
     probe = h2d_probe(torch)
     h2d = max(probe.values())
@@ -494,7 +497,7 @@ def run_wt(args, rank, world):
             if dist:
                 dist.barrier()
             dt, nl, st, nm = first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host,
-                                       None if fresh else slab, ph if rep > 0 else None)
+                                       None if fresh else slab, ph if rep > 0 else None, flags=oflags)
             if st != 0:
                 raise SystemExit("device status %d after first-use run" % st)
             if rep > 0:
@@ -549,7 +552,7 @@ def run_wt(args, rank, world):
     h0.close()
 
     # ---------------- resident pass: the steady-state consumer
-    h = wt.Handle(ck.paths)
+    h = wt.Handle(ck.paths, oflags)
     ev = dev.adopt(h, mode, ingest_s.cuda_stream)
     ingest_s.synchronize()
     descs = dev.descs(xs, ys)
@@ -621,6 +624,7 @@ def run_wt(args, rank, world):
         "data": DATA_DESC.get(wdt, "synthetic"),
         "config": {"workload": workload_desc(args), "weight_bytes": weight_bytes, "data_bytes": data_bytes,
                    "files": len(ck.paths), "matrices": len(dev.gemv_mats()), "ingest_mode": args.mode,
+                   "open": "WT_OPEN_NOMAP (pread)" if oflags else "mapped",
                    "l2": ("inputs larger than L2 (no flush)" if weight_bytes > L2_BYTES else
                           "inputs smaller than L2, no flush: passes may hit L2 (a dispatch-overhead point)"),
                    "parallelism": "replicas" if world > 1 else "1 GPU",
@@ -847,18 +851,19 @@ def run_timeline(args):
     build.build()
     torch.cuda.set_device(0)
     mode = {"gather": wt.WT_ADOPT_GATHER, "ce": wt.WT_ADOPT_CE, "staged": wt.WT_ADOPT_STAGED}[args.mode]
-    h0 = wt.Handle(ck.paths)
+    oflags = wt.WT_OPEN_NOMAP if args.open == "nomap" else 0
+    h0 = wt.Handle(ck.paths, oflags)
     mats = pipeline.matrices(h0)
     slab = make_slab(torch, pipeline, h0, mats)
     rows = sum(mats[k].shape[0] for k in slab["dev"].gemv_mats())
     y_host = torch.empty(rows, dtype=torch.float32, pin_memory=True)
     ingest_s, consume_s = torch.cuda.Stream(), torch.cuda.Stream()
     for _ in range(2):  # warm-up, untraced
-        first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab)
+        first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, flags=oflags)
     runs = []
     for _ in range(max(1, min(args.e2e_reps, 5))):
         tr = []
-        first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, trace=tr)
+        first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, flags=oflags, trace=tr)
         runs.append(tr[0])
     h0.close()
     sums = [overlap_summary(r["records"]) for r in runs]

@@ -73,6 +73,14 @@ extern "C" {
  * PREFAULT     populate every mapping's page-table entries at open
  *              (MADV_POPULATE_READ); otherwise wt_adopt populates each batch's
  *              source range just before it enqueues that batch.
+ * NOMAP        parse and validate each file (open, fstat, pread of the index, close)
+ *              but map nothing: the route of every file is NONE, tensor host_ptr is
+ *              NULL, and only WT_ADOPT_STAGED adopts, reading the bytes with pread
+ *              into the pinned ring (after checking that each path still names the
+ *              file that was parsed: device, inode, size, mtime; WT_EIO otherwise).
+ *              For checkpoints of many small files, where mapping every file costs
+ *              more host time than their bytes take on the link (Sec. 5.3: the
+ *              2506-file spine's map cost).  Not with REGISTER, DIRECT or PREFAULT.
  * TIMELINE     record a timing event before and after every ingest batch of
  *              wt_adopt and every GEMV group of wt_pass (outside stream capture),
  *              for wt_trace: the per-tensor overlap timeline of the first use.
@@ -86,14 +94,19 @@ extern "C" {
 #define WT_OPEN_HOST_ONLY (1u << 4)
 #define WT_OPEN_PREFAULT (1u << 5)
 #define WT_OPEN_TIMELINE (1u << 6)  /* timing events around every ingest batch and GEMV group (wt_trace) */
+#define WT_OPEN_NOMAP (1u << 7)     /* parse only; no mapping; staged adopt reads with pread */
 
 /* ---- wt_adopt modes ---------------------------------------------------------
  *   GATHER   SM gather kernel: 16-byte vector loads from the device-readable
  *            mapping, coalesced stores to HBM (the default).
  *   CE       copy engine: cudaMemcpyAsync from the device-readable mapping.
- *   STAGED   host threads copy page-cache bytes into a pinned ring, the copy
- *            engine moves each slot (the paper's staged/overlapped copy arm,
- *            Table "tab:tax" and Table "tab:gh-endpoints").
+ *   STAGED   host threads copy page-cache bytes into a pinned ring (memcpy from
+ *            the mapping, or pread for WT_OPEN_NOMAP files) and the gather kernel
+ *            moves each slot to its destinations over the host link (the paper's
+ *            staged/overlapped copy arm, Table "tab:tax" and Table
+ *            "tab:gh-endpoints").  The ring (4 x 64 MiB of pinned memory per
+ *            device) is allocated by the first staged adopt on a device and kept
+ *            until the process exits; staged adopts on one device take turns on it.
  */
 #define WT_ADOPT_GATHER 0u
 #define WT_ADOPT_CE 1u
@@ -109,7 +122,7 @@ typedef struct {
   uint64_t nbytes;      /* prod(shape) * sizeof(dtype) */
   uint32_t file;        /* index into the wt_open path list */
   uint64_t offset;      /* absolute file offset, multiple of 64 */
-  const void *host_ptr; /* address of the blob in the read-only mapping */
+  const void *host_ptr; /* address of the blob in the read-only mapping (NULL: WT_OPEN_NOMAP) */
 } wt_tensor_meta;
 
 /* One GEMV of wt_pass: y[M] = W[M,K] . x[K], fp32 accumulate (Sec. 3.1 protocol:
@@ -279,7 +292,8 @@ int wt_trace(wt_handle *h, void *origin, wt_trace_rec *out, size_t cap, size_t *
 int wt_device_status(wt_handle *h, int *status);
 
 /* Bytes of the handle's file mappings that are resident in the page cache right now
- * (mincore over every mapping, page granular, clipped to the file sizes) and their total.
+ * (mincore over every mapping, page granular, clipped to the file sizes) and their total
+ * (WT_ENOTSUP for a WT_OPEN_NOMAP handle, which maps nothing).
  * Algorithm 2 stops with "storage-bound" when the mapped set is not resident (Sec. 8.1);
  * Table "controls" queries residency before and after a measurement.  Host-only handles
  * work too.  Errors: WT_EINVAL, WT_EIO. */
@@ -293,7 +307,8 @@ int wt_kernel_launches(const wt_handle *h, uint64_t *n);
  * allocated itself (status words, plan tables, split-K workspaces, the staged ring).  Buffers
  * the caller owns are not counted.  After wt_close of every handle all five return to their
  * earlier values (Sec. 5.1: a producer's lifetime leaves nothing behind; the 200-cycle checks
- * read these).  Errors: WT_EINVAL. */
+ * read these), except that the first staged adopt on a device adds its ring for good: 4
+ * events and 268,435,456 pinned bytes.  Errors: WT_EINVAL. */
 typedef struct {
   int64_t handles;
   int64_t plans;

@@ -213,8 +213,12 @@ struct Tensor {
 
 struct File {
   std::string path;
-  uint8_t *base = nullptr;  // mapping
+  uint8_t *base = nullptr;  // mapping (nullptr: opened with WT_OPEN_NOMAP)
   size_t size = 0;
+  // identity at wt_open: a WT_OPEN_NOMAP file is opened again by a staged adopt, which checks
+  // that the path still names the file whose index was validated
+  uint64_t st_dev = 0, st_ino = 0;
+  int64_t mtime_ns = 0;
   unsigned route = WT_ROUTE_NONE;
   bool registered = false;
   unsigned reg_flags = 0;        // cudaHostRegister flags the registration holds (0: none)
@@ -275,13 +279,22 @@ struct Plan {
   uint64_t launches = 0;
 };
 
+// The staged arm's pinned ring: one per device for the whole process (pinning host memory
+// costs far more than a first use of a small checkpoint, so it is paid once), allocated by
+// the first staged adopt on the device and kept until the process exits.  Staged adopts on
+// one device take turns on it (its mutex); a slot is refilled once the device has read it.
 struct Ring {
   static constexpr int kSlots = 4;
   static constexpr size_t kSlotBytes = 64ull << 20;
+  std::mutex mu;
+  bool ready = false;
   uint8_t *slot[kSlots] = {nullptr, nullptr, nullptr, nullptr};
   cudaEvent_t done[kSlots] = {nullptr, nullptr, nullptr, nullptr};
   bool used[kSlots] = {false, false, false, false};
+  int next = 0;
 };
+
+Ring g_ring[64];
 
 }  // namespace
 
@@ -307,8 +320,6 @@ struct wt_handle {
   int *status = nullptr;
   std::vector<cudaEvent_t> events;
   std::list<Plan *> plans;
-  Ring ring;
-  bool ring_ready = false;
   uint64_t kernel_launches = 0;
   std::mutex mu;
 
@@ -406,8 +417,8 @@ void unmap_file(File &f) {
   }
 }
 
-// open, parse and map one file; closes the fd on every path.
-int open_one(File &f) {
+// open, parse and map one file (not with `nomap`); closes the fd on every path.
+int open_one(File &f, bool nomap) {
   if (wt::fault_injected("open")) return set_err(WT_EIO, "%s: open: injected fault", f.path.c_str());
   const int fd = open(f.path.c_str(), O_RDONLY | O_CLOEXEC);
   if (fd < 0) return set_err(WT_EIO, "%s: open: %s", f.path.c_str(), strerror(errno));
@@ -418,7 +429,11 @@ int open_one(File &f) {
     return set_err(WT_EIO, "%s: fstat: %s", f.path.c_str(), strerror(e));
   }
   int rc = parse_file(f, fd, (uint64_t)st.st_size);
-  if (rc == WT_OK) {
+  f.st_dev = (uint64_t)st.st_dev;
+  f.st_ino = (uint64_t)st.st_ino;
+  f.mtime_ns = (int64_t)st.st_mtim.tv_sec * 1000000000ll + st.st_mtim.tv_nsec;
+  if (rc == WT_OK && nomap) f.size = (size_t)st.st_size;
+  if (rc == WT_OK && !nomap) {
     f.size = (size_t)st.st_size;
     const bool injected = wt::fault_injected("mmap");
     void *p = injected ? MAP_FAILED : mmap(nullptr, f.size, PROT_READ, MAP_SHARED, fd, 0);
@@ -489,7 +504,9 @@ int trace_mark(cudaStream_t s, cudaEvent_t *ev) {
 // ------------------------------------------------------------------ adopt
 struct Range {
   size_t tensor;  // position in the caller's list
-  const uint8_t *src_host;
+  uint32_t file;  // file index and byte offset of the source (pread of WT_OPEN_NOMAP files)
+  uint64_t foff;
+  const uint8_t *src_host;  // nullptr for a WT_OPEN_NOMAP file
   const uint8_t *src_dev;
   uint8_t *dst;
   uint64_t n;
@@ -499,7 +516,10 @@ struct Range {
 int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cudaStream_t s,
                  void **ready, uint64_t total) {
   const uint64_t target = std::min<uint64_t>(128ull << 20, std::max<uint64_t>(2ull << 20, total / 64));
-  const int grid_cap = 2 * wt::num_sms();
+  // One gather CTA per SM saturates the link (210 GB/s either way) and leaves each SM room
+  // for a resident GEMV CTA beside it (registers: 256 x 48 + 288 x 168 of 65536), so the
+  // event-gated consumer of a batch runs while the next batch is in flight.
+  const int grid_cap = wt::num_sms();
   // Tensors larger than a batch are cut into pieces (multiples of 64 KiB, so each piece keeps
   // its range's alignment): page-table population and transfer then pipeline inside a tensor.
   // A tensor's event is the event of the batch holding its last piece.
@@ -512,8 +532,8 @@ int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cuda
       continue;
     }
     for (uint64_t o = 0; o < r.n; o += piece)
-      ps.push_back({r.tensor, r.src_host + o, r.src_dev ? r.src_dev + o : nullptr, r.dst + o, std::min(piece, r.n - o),
-                    r.populated});
+      ps.push_back({r.tensor, r.file, r.foff + o, r.src_host + o, r.src_dev ? r.src_dev + o : nullptr, r.dst + o,
+                    std::min(piece, r.n - o), r.populated});
   }
   std::vector<std::pair<size_t, size_t>> batches;
   for (size_t i = 0; i < ps.size();) {
@@ -611,40 +631,101 @@ int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cuda
   return WT_OK;
 }
 
-int ring_setup(wt_handle *h) {
-  if (h->ring_ready) return WT_OK;
+int ring_setup(Ring &R) {
+  if (R.ready) return WT_OK;
   for (int k = 0; k < Ring::kSlots; ++k) {
-    CU(pinned_alloc(reinterpret_cast<void **>(&h->ring.slot[k]), Ring::kSlotBytes));
-    CU(ev_create(&h->ring.done[k], cudaEventDisableTiming));
+    if (!R.slot[k]) CU(pinned_alloc(reinterpret_cast<void **>(&R.slot[k]), Ring::kSlotBytes));
+    if (!R.done[k]) CU(ev_create(&R.done[k], cudaEventDisableTiming));
   }
-  h->ring_ready = true;
+  R.ready = true;
   return WT_OK;
 }
 
-// Staged: page cache -> pinned slot (host threads) -> HBM (copy engine).
+// Opens a WT_OPEN_NOMAP file again for a staged adopt and checks it is the file wt_open
+// parsed (same device, inode, size and modification time).  Returns the fd or -1.
+int reopen_checked(const File &f) {
+  if (wt::fault_injected("open")) {
+    set_err(WT_EIO, "%s: open: injected fault", f.path.c_str());
+    return -1;
+  }
+  const int fd = open(f.path.c_str(), O_RDONLY | O_CLOEXEC);
+  if (fd < 0) {
+    set_err(WT_EIO, "%s: open: %s", f.path.c_str(), strerror(errno));
+    return -1;
+  }
+  struct stat st;
+  if (fstat(fd, &st) != 0 || (uint64_t)st.st_dev != f.st_dev || (uint64_t)st.st_ino != f.st_ino ||
+      (size_t)st.st_size != f.size ||
+      (int64_t)st.st_mtim.tv_sec * 1000000000ll + st.st_mtim.tv_nsec != f.mtime_ns) {
+    close(fd);
+    set_err(WT_EIO, "%s: the file changed since wt_open", f.path.c_str());
+    return -1;
+  }
+  return fd;
+}
+
+// Staged: page cache -> pinned slot (host threads: memcpy from the mapping, or pread for a
+// WT_OPEN_NOMAP file, which then needs no mapping at all) -> HBM (the gather kernel reading
+// the pinned slot over the host link: one launch per up to kMaxGather pieces, so a slot of many
+// small tensors costs one or two launches instead of one copy call per tensor).
 int adopt_staged(wt_handle *h, const std::vector<Range> &rs, cudaStream_t s, void **ready) {
-  int rc = ring_setup(h);
+  Ring &R = g_ring[h->device];
+  std::lock_guard<std::mutex> ring_lock(R.mu);
+  int rc = ring_setup(R);
   if (rc) return rc;
+  // descriptors of the unmapped files this call reads, opened in parallel and closed on return
+  std::vector<int> fds(h->files.size(), -1);
+  std::vector<uint32_t> need;
+  {
+    std::vector<char> seen(h->files.size(), 0);
+    for (const Range &r : rs)
+      if (!r.src_host && r.n && !seen[r.file]) {
+        seen[r.file] = 1;
+        need.push_back(r.file);
+      }
+  }
+  struct Closer {
+    std::vector<int> &fds;
+    ~Closer() {
+      for (int fd : fds)
+        if (fd >= 0) close(fd);
+    }
+  } closer{fds};
+  Pool &pool = host_pool();
+  if (!need.empty()) {
+    std::vector<std::string> errs(need.size());
+    std::atomic<bool> bad{false};
+    pool.parallel_for(need.size(), [&](size_t k) {
+      fds[need[k]] = reopen_checked(h->files[need[k]]);
+      if (fds[need[k]] < 0) {
+        errs[k] = t_err;
+        bad = true;
+      }
+    });
+    if (bad)
+      for (const std::string &e : errs)
+        if (!e.empty()) return set_err(WT_EIO, "wt_adopt: %s", e.c_str());
+  }
   struct PieceCopy {
-    const uint8_t *src;
-    size_t off;  // in slot
-    uint8_t *dst;
+    const Range *r;
+    uint64_t roff;  // offset in the range
+    size_t off;     // in slot (16-byte aligned)
     size_t n;
   };
-  int slot = 0;
   size_t r = 0;
   uint64_t roff = 0;
-  Pool &pool = host_pool();
   while (r < rs.size()) {
-    if (h->ring.used[slot]) CU(cudaEventSynchronize(h->ring.done[slot]));
-    uint8_t *buf = h->ring.slot[slot];
+    const int slot = R.next;
+    R.next = (R.next + 1) % Ring::kSlots;
+    if (R.used[slot]) CU(cudaEventSynchronize(R.done[slot]));
+    uint8_t *buf = R.slot[slot];
     std::vector<PieceCopy> pcs;
     std::vector<size_t> finished;  // tensors whose last byte is in this slot
     size_t fill = 0;
     while (r < rs.size() && fill < Ring::kSlotBytes) {
       const uint64_t take = std::min<uint64_t>(rs[r].n - roff, Ring::kSlotBytes - fill);
-      if (take) pcs.push_back({rs[r].src_host + roff, fill, rs[r].dst + roff, (size_t)take});
-      fill += take;
+      if (take) pcs.push_back({&rs[r], roff, fill, (size_t)take});
+      fill = (fill + take + 63) & ~(size_t)63;  // next piece 64-byte aligned in the slot
       roff += take;
       if (roff == rs[r].n) {
         finished.push_back(rs[r].tensor);
@@ -652,27 +733,86 @@ int adopt_staged(wt_handle *h, const std::vector<Range> &rs, cudaStream_t s, voi
         roff = 0;
       }
     }
-    // host copy in 4 MiB pieces across the pool
+    // host copy in pieces of at most 4 MiB across the pool
     std::vector<std::pair<size_t, size_t>> work;  // (piece, sub-offset)
     constexpr size_t kSub = 4u << 20;
     for (size_t p = 0; p < pcs.size(); ++p)
       for (size_t o = 0; o < pcs[p].n; o += kSub) work.push_back({p, o});
+    std::atomic<int> io_err{0};
+    std::vector<std::string> io_msg(1);
+    std::mutex io_mu;
     pool.parallel_for(work.size(), [&](size_t w) {
       const PieceCopy &pc = pcs[work[w].first];
-      const size_t o = work[w].second;
-      memcpy(buf + pc.off + o, pc.src + o, std::min(kSub, pc.n - o));
+      const size_t o = work[w].second, len = std::min(kSub, pc.n - o);
+      uint8_t *dst = buf + pc.off + o;
+      if (pc.r->src_host) {
+        memcpy(dst, pc.r->src_host + pc.roff + o, len);
+        return;
+      }
+      const int fd = fds[pc.r->file];
+      size_t got = 0;
+      const bool injected = wt::fault_injected("pread");
+      while (!injected && got < len) {
+        const ssize_t k = pread(fd, dst + got, len - got, (off_t)(pc.r->foff + pc.roff + o + got));
+        if (k <= 0) {
+          if (k < 0 && errno == EINTR) continue;
+          break;
+        }
+        got += (size_t)k;
+      }
+      if (got != len && io_err.exchange(1) == 0) {
+        std::lock_guard<std::mutex> g(io_mu);
+        io_msg[0] = h->files[pc.r->file].path + (injected ? ": pread: injected fault" : ": pread: short read");
+      }
     });
-    for (const PieceCopy &pc : pcs) CU(cudaMemcpyAsync(pc.dst, buf + pc.off, pc.n, cudaMemcpyHostToDevice, s));
-    CU(cudaEventRecord(h->ring.done[slot], s));
-    h->ring.used[slot] = true;
-    if (!finished.empty()) {
-      cudaEvent_t ev;
-      rc = new_event(h, &ev);
+    if (io_err) return set_err(WT_EIO, "wt_adopt: %s", io_msg[0].c_str());
+    cudaEvent_t tb = nullptr;
+    if (h->timeline) {
+      rc = trace_mark(s, &tb);
       if (rc) return rc;
+    }
+    for (size_t i = 0; i < pcs.size();) {
+      wt::GatherBatch gb;
+      memset(&gb, 0, sizeof gb);
+      uint64_t chunks = 0;
+      for (; i < pcs.size() && gb.n < (uint32_t)wt::kMaxGather; ++i) {
+        const uint32_t q = gb.n++;
+        gb.chunk_prefix[q] = chunks;
+        gb.src[q] = buf + pcs[i].off;
+        gb.dst[q] = pcs[i].r->dst + pcs[i].roff;
+        gb.nbytes[q] = pcs[i].n;
+        chunks += (pcs[i].n + (1ull << wt::kGatherChunkLog2) - 1) >> wt::kGatherChunkLog2;
+      }
+      gb.chunk_prefix[gb.n] = chunks;
+      if (chunks) {
+        CU(wt::launch_gather(gb, (int)std::min<uint64_t>(chunks, (uint64_t)wt::num_sms()), s));
+        h->kernel_launches++;
+      }
+    }
+    CU(cudaEventRecord(R.done[slot], s));
+    R.used[slot] = true;
+    cudaEvent_t ev = nullptr;
+    if (!finished.empty()) {
+      rc = new_event(h, &ev);
+      if (rc) {
+        if (tb) ev_destroy(tb);
+        return rc;
+      }
       CU(cudaEventRecord(ev, s));
       for (size_t t : finished) ready[t] = ev;
     }
-    slot = (slot + 1) % Ring::kSlots;
+    if (tb) {
+      cudaEvent_t te = nullptr;
+      rc = trace_mark(s, &te);
+      if (rc) {
+        ev_destroy(tb);
+        return rc;
+      }
+      uint64_t bytes = 0;
+      for (const PieceCopy &pc : pcs) bytes += pc.n;
+      h->trace.push_back({WT_TRACE_INGEST, h->n_batches, bytes, tb, te, true, ev});
+    }
+    h->n_batches++;
   }
   return WT_OK;
 }
@@ -1356,15 +1496,6 @@ int close_impl(wt_handle *h) {
     h->trace.clear();
     for (Plan *P : h->plans) destroy_plan(P);
     h->plans.clear();
-    if (h->ring_ready) {
-      for (int k = 0; k < Ring::kSlots; ++k) {
-        if (h->ring.done[k]) {
-          cudaEventSynchronize(h->ring.done[k]);
-          ev_destroy(h->ring.done[k]);
-        }
-        pinned_free(h->ring.slot[k], Ring::kSlotBytes);
-      }
-    }
     for (cudaEvent_t e : h->events) ev_destroy(e);
     h->events.clear();
     dev_free(h->status, 256);
@@ -1414,8 +1545,11 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
   *out = nullptr;
   if (n_paths < 0 || (n_paths > 0 && !paths)) return set_err(WT_EINVAL, "wt_open: bad path list");
   const unsigned route_req = flags & WT_ROUTE_MASK;
-  if (flags & ~(WT_ROUTE_MASK | WT_OPEN_HOST_ONLY | WT_OPEN_PREFAULT | WT_OPEN_TIMELINE))
+  if (flags & ~(WT_ROUTE_MASK | WT_OPEN_HOST_ONLY | WT_OPEN_PREFAULT | WT_OPEN_TIMELINE | WT_OPEN_NOMAP))
     return set_err(WT_EINVAL, "wt_open: unknown flag bits 0x%x", flags);
+  const bool nomap = (flags & WT_OPEN_NOMAP) != 0;
+  if (nomap && (route_req == WT_ROUTE_REGISTER || route_req == WT_ROUTE_DIRECT || (flags & WT_OPEN_PREFAULT)))
+    return set_err(WT_EINVAL, "wt_open: WT_OPEN_NOMAP maps nothing: no REGISTER or DIRECT route, no PREFAULT");
   wt_handle *h = nullptr;
   try {
     h = new wt_handle();
@@ -1435,7 +1569,7 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
     std::vector<int> rcs(n_paths, WT_OK);
     std::vector<std::string> errs(n_paths);
     host_pool().parallel_for((size_t)n_paths, [&](size_t i) {
-      rcs[i] = open_one(h->files[i]);
+      rcs[i] = open_one(h->files[i], nomap);
       if (rcs[i]) errs[i] = t_err;
     });
     for (int i = 0; i < n_paths; ++i) {
@@ -1447,7 +1581,8 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
     }
     for (int f = 0; f < n_paths; ++f)
       for (uint32_t e = 0; e < h->files[f].tensors.size(); ++e) h->order.push_back({(uint32_t)f, e});
-    for (int f = 0; f < n_paths; ++f) h->by_base.push_back({reinterpret_cast<uintptr_t>(h->files[f].base), (uint32_t)f});
+    for (int f = 0; f < n_paths; ++f)
+      if (h->files[f].base) h->by_base.push_back({reinterpret_cast<uintptr_t>(h->files[f].base), (uint32_t)f});
     std::sort(h->by_base.begin(), h->by_base.end());
     if (flags & WT_OPEN_PREFAULT) {
       host_pool().parallel_for((size_t)n_paths, [&](size_t i) { prefault(h->files[i].base, h->files[i].size); });
@@ -1471,7 +1606,7 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
     int ats = 0;
     cudaDeviceGetAttribute(&ats, cudaDevAttrPageableMemoryAccessUsesHostPageTables, h->device);
     for (File &f : h->files) {
-      unsigned want = route_req;
+      unsigned want = nomap ? WT_ROUTE_NONE : route_req;
       if (want == WT_ROUTE_AUTO) want = ats ? WT_ROUTE_DIRECT : WT_ROUTE_REGISTER;
       if (want == WT_ROUTE_DIRECT) {
         if (!ats) {
@@ -1567,7 +1702,7 @@ int wt_tensor_info(const wt_handle *h, size_t i, wt_tensor_meta *out) {
   out->nbytes = t.nbytes;
   out->file = h->order[i].first;
   out->offset = t.offset;
-  out->host_ptr = h->files[out->file].base + t.offset;
+  out->host_ptr = h->files[out->file].base ? h->files[out->file].base + t.offset : nullptr;
   return WT_OK;
 }
 
@@ -1621,7 +1756,8 @@ int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsign
       if (mode != WT_ADOPT_STAGED && f.route == WT_ROUTE_NONE)
         return set_err(WT_ENOTSUP, "wt_adopt: %s has no device route; use WT_ADOPT_STAGED", f.path.c_str());
       ready[k] = nullptr;
-      rs.push_back({k, f.base + t.offset, f.dev ? f.dev + t.offset : nullptr, static_cast<uint8_t *>(dst[k]), t.nbytes,
+      rs.push_back({k, h->order[idx[k]].first, t.offset, f.base ? f.base + t.offset : nullptr,
+                    f.dev ? f.dev + t.offset : nullptr, static_cast<uint8_t *>(dst[k]), t.nbytes,
                     f.populated || h->prefaulted});
       total += t.nbytes;
     }
@@ -1762,6 +1898,7 @@ int wt_residency(const wt_handle *h, uint64_t *resident, uint64_t *total) {
   uint64_t res = 0, tot = 0;
   std::vector<unsigned char> vec;
   for (const File &f : h->files) {
+    if (!f.base) return set_err(WT_ENOTSUP, "wt_residency: %s is not mapped (WT_OPEN_NOMAP)", f.path.c_str());
     const size_t pages = (f.size + pg - 1) / pg;
     vec.assign(pages, 0);
     if (pages && mincore(f.base, f.size, vec.data()) != 0)

@@ -21,7 +21,7 @@ LIB_PATH = os.path.join(HERE, "libwt.so")
 WT_OK, WT_EINVAL, WT_EIO, WT_EFORMAT, WT_ENOMEM, WT_ECUDA, WT_ENOTSUP, WT_ETIMEDOUT = 0, -1, -2, -3, -4, -5, -6, -7
 WT_F32, WT_BF16, WT_F16, WT_I8, WT_U8 = 0, 1, 2, 3, 4
 WT_ROUTE_AUTO, WT_ROUTE_REGISTER, WT_ROUTE_DIRECT, WT_ROUTE_NONE = 0, 1, 2, 3
-WT_OPEN_HOST_ONLY, WT_OPEN_PREFAULT, WT_OPEN_TIMELINE = 1 << 4, 1 << 5, 1 << 6
+WT_OPEN_HOST_ONLY, WT_OPEN_PREFAULT, WT_OPEN_TIMELINE, WT_OPEN_NOMAP = 1 << 4, 1 << 5, 1 << 6, 1 << 7
 WT_TRACE_INGEST, WT_TRACE_GEMV = 0, 1
 WT_ADOPT_GATHER, WT_ADOPT_CE, WT_ADOPT_STAGED = 0, 1, 2
 ROUTE_NAMES = {WT_ROUTE_REGISTER: "register", WT_ROUTE_DIRECT: "direct", WT_ROUTE_NONE: "none"}

@@ -162,3 +162,20 @@ def test_registration_and_trace_queries_on_host_only_handle(L, tmp_path):
         assert ei.value.code == wt.WT_EINVAL
     # TIMELINE is a known flag (a host-only handle ignores it)
     wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY | wt.WT_OPEN_TIMELINE).close()
+
+
+def test_nomap_open_parses_without_mapping(L, tmp_path):
+    ck = synth.build("many", str(tmp_path / "nm"), n_matrices=5)
+    with wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY) as hm:
+        want = [(t.name, t.dtype, t.shape, t.nbytes, t.file, t.offset) for t in hm.tensors]
+    with wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY | wt.WT_OPEN_NOMAP) as h:
+        assert [(t.name, t.dtype, t.shape, t.nbytes, t.file, t.offset) for t in h.tensors] == want
+        assert all(t.host_ptr == 0 for t in h.tensors)
+        assert not [l for l in open("/proc/self/maps") if str(tmp_path) in l]  # nothing mapped
+        with pytest.raises(wt.WtError) as ei:
+            h.residency()
+        assert ei.value.code == wt.WT_ENOTSUP
+    for bad in (wt.WT_ROUTE_REGISTER, wt.WT_ROUTE_DIRECT, wt.WT_OPEN_PREFAULT):
+        with pytest.raises(wt.WtError) as ei:
+            wt.Handle(ck.paths, wt.WT_OPEN_NOMAP | bad)
+        assert ei.value.code == wt.WT_EINVAL

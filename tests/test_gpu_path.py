@@ -351,3 +351,57 @@ def test_device_overruns_are_refused_on_the_host(torch, tmp_path):
         h.adopt([0], [big.data_ptr()], wt.WT_ADOPT_GATHER, 0)
         torch.cuda.synchronize()
         assert h.device_status() == 0
+
+
+# ----------------------------------------------------------------------------- unmapped (pread) route
+
+@pytest.mark.parametrize("workload,kw", [("many", dict(n_matrices=300)), ("mid", dict(layers=1, vocab=40000))],
+                         ids=["many-300", "mid-1-layer"])
+def test_nomap_staged_ingest_matches_oracle(torch, tmp_path, workload, kw):
+    """WT_OPEN_NOMAP + STAGED: no file is mapped; host threads pread into the pinned ring and the
+    gather kernel moves each slot.  Row blocks land contiguously, tensors larger than a 64 MiB
+    slot (the 40000 x 2560 embedding, 205 MB) span slots; bytes and canaries bit-exact, digests
+    and every GEMV row against the oracle, with the event-gated pass."""
+    ck = synth.build(workload, str(tmp_path), workers=4, **kw)
+    co = oracle.CheckpointOracle(ck.paths)
+    h, dev, ev, s = ingest(torch, ck, wt.WT_ADOPT_STAGED, wt.WT_OPEN_NOMAP)
+    assert not [l for l in open("/proc/self/maps") if str(tmp_path) in l]
+    xs, ys = dev.inputs(), dev.outputs()
+    for y in ys.values():
+        y.fill_(float("nan"))
+    c = torch.cuda.Stream()
+    h.pass_(dev.descs(xs, ys, ev), c.cuda_stream)
+    c.synchronize()
+    s.synchronize()
+    check_bytes(torch, h, dev, co)
+    od = oracle_digests(h, co)
+    tree = device_digests(torch, h, dev)
+    assert all(tree[i] == od[i][1] for i in od)
+    check_gemv(h, dev, co, ys)
+    assert h.device_status() == 0
+    h.close()
+
+
+def test_nomap_refuses_device_routes_and_changed_files(torch, tmp_path):
+    ck = synth.build("tiny", str(tmp_path))
+    with pytest.raises(wt.WtError) as ei:  # no mapping, so no gather or copy-engine route
+        ingest(torch, ck, wt.WT_ADOPT_GATHER, wt.WT_OPEN_NOMAP)
+    assert ei.value.code == wt.WT_ENOTSUP
+    h = wt.Handle(ck.paths, wt.WT_OPEN_NOMAP)
+    dev = pipeline.DeviceCheckpoint.allocate(h, pipeline.matrices(h))
+    # the path now names another file of the same size: the staged adopt refuses it
+    p = ck.paths[0]
+    data = open(p, "rb").read()
+    open(p + ".new", "wb").write(data)
+    import os
+    os.replace(p + ".new", p)
+    with pytest.raises(wt.WtError) as ei:
+        dev.adopt(h, wt.WT_ADOPT_STAGED, 0)
+    assert ei.value.code == wt.WT_EIO and "changed" in str(ei.value)
+    h.close()
+    # a fresh handle on the new file adopts it
+    co = oracle.CheckpointOracle(ck.paths)
+    h, dev, ev, s = ingest(torch, ck, wt.WT_ADOPT_STAGED, wt.WT_OPEN_NOMAP)
+    s.synchronize()
+    check_bytes(torch, h, dev, co)
+    h.close()
