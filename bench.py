@@ -57,8 +57,9 @@ def parse_args():
     p.add_argument("--workload", default="large")
     p.add_argument("--layers", type=int, default=None, help="override decoder layer count (small profiling cases)")
     p.add_argument("--mode", default="gather", choices=["gather", "ce", "staged"])
-    p.add_argument("--open", default="map", choices=["map", "nomap"],
-                   help="nomap: wt_open maps nothing (WT_OPEN_NOMAP) and --mode staged preads into the pinned ring")
+    p.add_argument("--open", default="map", choices=["map", "nomap", "prefault"],
+                   help="nomap: wt_open maps nothing (WT_OPEN_NOMAP) and --mode staged preads into the pinned ring; "
+                        "prefault: wt_open populates every mapping (WT_OPEN_PREFAULT)")
     p.add_argument("--e2e-reps", type=int, default=5)
     p.add_argument("--skip-e2e", action="store_true", help="resident passes only (profiling runs)")
     p.add_argument("--arms", action="store_true", help="also time the ce/staged/stock-torch ingest arms")
@@ -466,7 +467,7 @@ def run_wt(args, rank, world):
         dist.barrier()
     build.build()  # no-op when fresh; loads the same in-tree library on every rank
     mode = {"gather": wt.WT_ADOPT_GATHER, "ce": wt.WT_ADOPT_CE, "staged": wt.WT_ADOPT_STAGED}[args.mode]
-    oflags = wt.WT_OPEN_NOMAP if args.open == "nomap" else 0
+    oflags = {"map": 0, "nomap": wt.WT_OPEN_NOMAP, "prefault": wt.WT_OPEN_PREFAULT}[args.open]
 
     probe = h2d_probe(torch)
     h2d = max(probe.values())
@@ -624,7 +625,7 @@ def run_wt(args, rank, world):
         "data": DATA_DESC.get(wdt, "synthetic"),
         "config": {"workload": workload_desc(args), "weight_bytes": weight_bytes, "data_bytes": data_bytes,
                    "files": len(ck.paths), "matrices": len(dev.gemv_mats()), "ingest_mode": args.mode,
-                   "open": "WT_OPEN_NOMAP (pread)" if oflags else "mapped",
+                   "open": {"map": "mapped", "nomap": "WT_OPEN_NOMAP (pread)", "prefault": "mapped, WT_OPEN_PREFAULT"}[args.open],
                    "l2": ("inputs larger than L2 (no flush)" if weight_bytes > L2_BYTES else
                           "inputs smaller than L2, no flush: passes may hit L2 (a dispatch-overhead point)"),
                    "parallelism": "replicas" if world > 1 else "1 GPU",
@@ -851,7 +852,7 @@ def run_timeline(args):
     build.build()
     torch.cuda.set_device(0)
     mode = {"gather": wt.WT_ADOPT_GATHER, "ce": wt.WT_ADOPT_CE, "staged": wt.WT_ADOPT_STAGED}[args.mode]
-    oflags = wt.WT_OPEN_NOMAP if args.open == "nomap" else 0
+    oflags = {"map": 0, "nomap": wt.WT_OPEN_NOMAP, "prefault": wt.WT_OPEN_PREFAULT}[args.open]
     h0 = wt.Handle(ck.paths, oflags)
     mats = pipeline.matrices(h0)
     slab = make_slab(torch, pipeline, h0, mats)

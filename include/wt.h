@@ -172,6 +172,13 @@ int wt_num_tensors(const wt_handle *h, size_t *n);
 int wt_num_files(const wt_handle *h, size_t *n);
 /* Tensor i in (file, index) order. */
 int wt_tensor_info(const wt_handle *h, size_t i, wt_tensor_meta *out);
+/* wt_tensor_info of tensors [first, first + n) into out[0..n), in one call (a checkpoint of
+ * thousands of files has thousands of entries).  Errors: WT_EINVAL (range, NULL). */
+int wt_tensor_table(const wt_handle *h, size_t first, size_t n, wt_tensor_meta *out);
+/* Every tensor name, in tensor order, each followed by a NUL byte, into buf.  *needed receives
+ * the bytes required; with cap == 0 only *needed is set.  Errors: WT_EINVAL (NULL, cap too
+ * small). */
+int wt_tensor_names(const wt_handle *h, char *buf, size_t cap, size_t *needed);
 /* First tensor whose name equals `name`; WT_EINVAL if none. */
 int wt_find(const wt_handle *h, const char *name, size_t *i);
 /* Route actually taken for file f (WT_ROUTE_REGISTER / DIRECT / NONE). */

@@ -545,8 +545,9 @@ int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cuda
   }
   // A helper thread populates the page-table entries of batch after batch; batch b is
   // enqueued once its sources are populated, so this host work (about 1 TB/s for large
-  // ranges, a few microseconds per small one) overlaps the transfer of earlier batches.
-  // Concurrent populate calls on one address space contend, so one thread does them all.
+  // ranges, about 5 us per small mapping) overlaps the transfer of earlier batches.  A batch
+  // of many ranges (many small files) is populated by the host pool in parallel: every
+  // mapping exists by now, so the populate calls share the address-space lock as readers.
   std::vector<std::vector<std::pair<const uint8_t *, size_t>>> work(batches.size());
   bool any = false;
   for (size_t b = 0; b < batches.size(); ++b)
@@ -564,7 +565,10 @@ int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cuda
   if (any) {
     helper = std::thread([&] {
       for (size_t b = 0; b < batches.size() && !stop.load(); ++b) {
-        for (const auto &w : work[b]) prefault(w.first, w.second);
+        if (work[b].size() >= 8)
+          host_pool().parallel_for(work[b].size(), [&](size_t k) { prefault(work[b][k].first, work[b][k].second); });
+        else
+          for (const auto &w : work[b]) prefault(w.first, w.second);
         {
           std::lock_guard<std::mutex> g(mu);
           populated = b + 1;
@@ -1703,6 +1707,29 @@ int wt_tensor_info(const wt_handle *h, size_t i, wt_tensor_meta *out) {
   out->file = h->order[i].first;
   out->offset = t.offset;
   out->host_ptr = h->files[out->file].base ? h->files[out->file].base + t.offset : nullptr;
+  return WT_OK;
+}
+
+int wt_tensor_table(const wt_handle *h, size_t first, size_t n, wt_tensor_meta *out) {
+  if (!h || (n && !out)) return set_err(WT_EINVAL, "wt_tensor_table: NULL argument");
+  if (first > h->order.size() || n > h->order.size() - first)
+    return set_err(WT_EINVAL, "wt_tensor_table: tensors [%zu, %zu) out of range", first, first + n);
+  for (size_t k = 0; k < n; ++k) wt_tensor_info(h, first + k, out + k);
+  return WT_OK;
+}
+
+int wt_tensor_names(const wt_handle *h, char *buf, size_t cap, size_t *needed) {
+  if (!h || !needed || (cap && !buf)) return set_err(WT_EINVAL, "wt_tensor_names: NULL argument");
+  size_t total = 0;
+  for (size_t i = 0; i < h->order.size(); ++i) total += h->tensor(i).name.size() + 1;
+  *needed = total;
+  if (cap < total) return cap ? set_err(WT_EINVAL, "wt_tensor_names: buffer of %zu bytes, %zu needed", cap, total) : WT_OK;
+  size_t pos = 0;
+  for (size_t i = 0; i < h->order.size(); ++i) {
+    const std::string &nm = h->tensor(i).name;
+    memcpy(buf + pos, nm.c_str(), nm.size() + 1);
+    pos += nm.size() + 1;
+  }
   return WT_OK;
 }
 

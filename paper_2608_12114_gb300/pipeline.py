@@ -28,7 +28,7 @@ _ESZ = {wt.WT_F32: 4, wt.WT_BF16: 2, wt.WT_F16: 2, wt.WT_I8: 1, wt.WT_U8: 1}
 _ALIGN = 256
 
 
-@dataclass
+@dataclass(slots=True)
 class MatrixRef:
     name: str
     dtype: int
@@ -43,36 +43,48 @@ def matrices(h: wt.Handle) -> List[MatrixRef]:
     out: List[MatrixRef] = []
     by_name: Dict[str, MatrixRef] = {}
     blocks: Dict[str, Dict[int, int]] = {}
+    gemv_dt = (wt.WT_F32, wt.WT_BF16, wt.WT_F16)
+    match = _BLOCK.match
     for i, t in enumerate(h.tensors):
-        m = _BLOCK.match(t.name)
-        if not m:
-            ref = MatrixRef(t.name, t.dtype, t.shape, [i],
-                            len(t.shape) == 2 and t.dtype in (wt.WT_F32, wt.WT_BF16, wt.WT_F16))
+        nm = t.name
+        m = match(nm) if "#r" in nm else None
+        if m is None:
+            ref = MatrixRef(nm, t.dtype, t.shape, [i], len(t.shape) == 2 and t.dtype in gemv_dt)
             out.append(ref)
-            by_name[t.name] = ref
+            by_name[nm] = ref
             continue
-        base, k = m.group(1), int(m.group(2))
-        blocks.setdefault(base, {})[k] = i
-        if base not in by_name:
-            ref = MatrixRef(base, t.dtype, (), [], False)
-            out.append(ref)
-            by_name[base] = ref
+        base = m.group(1)
+        bl = blocks.get(base)
+        if bl is None:
+            bl = blocks[base] = {}
+            if base not in by_name:
+                ref = MatrixRef(base, t.dtype, (), [], False)
+                out.append(ref)
+                by_name[base] = ref
+        bl[int(m.group(2))] = i
+    tensors = h.tensors
     for base, parts in blocks.items():
         ref = by_name[base]
         idx = [parts[k] for k in sorted(parts)]
-        ts = [h.tensors[i] for i in idx]
-        K = ts[0].shape[1] if len(ts[0].shape) == 2 else None
-        if K is None or any(len(t.shape) != 2 or t.shape[1] != K or t.dtype != ts[0].dtype for t in ts):
-            raise ValueError("row blocks of %s do not stack" % base)
+        t0 = tensors[idx[0]]
+        K = t0.shape[1] if len(t0.shape) == 2 else None
+        rows = 0
+        for i in idx:
+            t = tensors[i]
+            if K is None or len(t.shape) != 2 or t.shape[1] != K or t.dtype != t0.dtype:
+                raise ValueError("row blocks of %s do not stack" % base)
+            rows += t.shape[0]
         ref.parts = idx
-        ref.shape = (sum(t.shape[0] for t in ts), K)
-        ref.gemv = ts[0].dtype in (wt.WT_F32, wt.WT_BF16, wt.WT_F16)
+        ref.shape = (rows, K)
+        ref.gemv = t0.dtype in gemv_dt
     # int8 matrices are GEMV matrices when their fp16 row scales "<name>.scale" are present
-    names = {t.name: i for i, t in enumerate(h.tensors)}
+    names = None
     for ref in out:
         if ref.dtype == wt.WT_I8 and len(ref.shape) == 2 and len(ref.parts) == 1:
+            if names is None:
+                names = {t.name: i for i, t in enumerate(tensors)}
             si = names.get(ref.name + ".scale")
-            if si is not None and h.tensors[si].dtype == wt.WT_F16 and h.tensors[si].shape == (ref.shape[0],):
+            if si is not None and tensors[si].dtype == wt.WT_F16 and tensors[si].shape == (ref.shape[0],):
                 ref.scale, ref.gemv = si, True
     return out
 

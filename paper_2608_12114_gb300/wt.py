@@ -29,7 +29,7 @@ MODE_NAMES = {WT_ADOPT_GATHER: "gather", WT_ADOPT_CE: "ce", WT_ADOPT_STAGED: "st
 
 # every entry point declared in include/wt.h
 SYMBOLS = ("wt_last_error", "wt_abi_version", "wt_open", "wt_num_tensors", "wt_num_files",
-           "wt_tensor_info", "wt_find", "wt_file_route", "wt_file_registration", "wt_adopt", "wt_pass", "wt_checksum",
+           "wt_tensor_info", "wt_tensor_table", "wt_tensor_names", "wt_find", "wt_file_route", "wt_file_registration", "wt_adopt", "wt_pass", "wt_checksum",
            "wt_checksum_plain", "wt_checksum_noalloc", "wt_device_status", "wt_residency",
            "wt_kernel_launches", "wt_trace", "wt_live", "wt_close",
            # include/wt_dlpack.h
@@ -66,6 +66,12 @@ class TraceRec(C.Structure):
                 ("event", C.c_void_p), ("begin_ms", C.c_double), ("end_ms", C.c_double)]
 
 
+# wt_tensor_meta as a numpy record (wt_tensor_table fills an array of them in one call).
+META_DTYPE = np.dtype([("name", "<u8"), ("dtype", "<i4"), ("ndim", "<i4"), ("shape", "<u8", (4,)),
+                       ("nbytes", "<u8"), ("file", "<u4"), ("pad", "<u4"), ("offset", "<u8"), ("host_ptr", "<u8")])
+assert META_DTYPE.itemsize == C.sizeof(TensorMeta)
+
+
 # The same 64-byte layout as a numpy record, for building many descriptors at once.
 DESC_DTYPE = np.dtype([("W", "<u8"), ("dtype", "<i4"), ("cols", "<i4"), ("M", "<u8"), ("K", "<u8"),
                        ("x", "<u8"), ("y", "<u8"), ("wait_event", "<u8"), ("scale", "<u8")])
@@ -90,6 +96,8 @@ def lib(path: str = LIB_PATH):
     L.wt_num_tensors.argtypes = [vp, C.POINTER(sz)]
     L.wt_num_files.argtypes = [vp, C.POINTER(sz)]
     L.wt_tensor_info.argtypes = [vp, sz, C.POINTER(TensorMeta)]
+    L.wt_tensor_table.argtypes = [vp, sz, sz, vp]
+    L.wt_tensor_names.argtypes = [vp, C.c_char_p, sz, C.POINTER(sz)]
     L.wt_find.argtypes = [vp, C.c_char_p, C.POINTER(sz)]
     L.wt_file_route.argtypes = [vp, sz, C.POINTER(C.c_uint)]
     L.wt_file_registration.argtypes = [vp, sz, C.POINTER(C.c_uint)]
@@ -122,7 +130,7 @@ def _check(rc: int):
         raise WtError(rc, lib().wt_last_error().decode(errors="replace"))
 
 
-@dataclass
+@dataclass(slots=True)
 class TensorInfo:
     name: str
     dtype: int
@@ -138,18 +146,32 @@ class Handle:
 
     def __init__(self, paths: Sequence[str], flags: int = 0):
         L = lib()
-        arr = (C.c_char_p * max(1, len(paths)))(*[p.encode() for p in paths])
+        # every path in one NUL-separated buffer, pointers computed from the NUL positions
+        blob = ("\0".join(os.fspath(p) for p in paths) + "\0").encode() if len(paths) else b"\0"
+        cbuf = C.create_string_buffer(blob, len(blob))
+        ends = np.flatnonzero(np.frombuffer(blob, np.uint8) == 0)
+        starts = np.concatenate(([0], ends[:-1] + 1)).astype(np.uint64) + np.uint64(C.addressof(cbuf))
+        arr = np.ascontiguousarray(starts[:len(paths)] if len(paths) else np.zeros(1, np.uint64))
         h = C.c_void_p()
-        _check(L.wt_open(arr, len(paths), flags, C.byref(h)))
+        _check(L.wt_open(C.cast(arr.ctypes.data, C.POINTER(C.c_char_p)), len(paths), flags, C.byref(h)))
+        del cbuf, arr
         self._h = h
         n = C.c_size_t()
         _check(L.wt_num_tensors(h, C.byref(n)))
-        self.tensors: List[TensorInfo] = []
-        for i in range(n.value):
-            m = TensorMeta()
-            _check(L.wt_tensor_info(h, i, C.byref(m)))
-            self.tensors.append(TensorInfo(m.name.decode(), m.dtype, tuple(m.shape[:m.ndim]), m.nbytes,
-                                           m.file, m.offset, m.host_ptr or 0))
+        # two calls for the whole index (metadata table, then every name), not one per tensor
+        meta = np.zeros(n.value, META_DTYPE)
+        if n.value:
+            _check(L.wt_tensor_table(h, 0, n.value, meta.ctypes.data))
+        need = C.c_size_t()
+        _check(L.wt_tensor_names(h, None, 0, C.byref(need)))
+        buf = C.create_string_buffer(max(1, need.value))
+        _check(L.wt_tensor_names(h, buf, need.value, C.byref(need)))
+        names = buf.raw[:need.value].split(b"\0")[:-1] if need.value else []
+        cols = [meta[f].tolist() for f in ("dtype", "ndim", "nbytes", "file", "offset", "host_ptr")]
+        shapes = meta["shape"].tolist()
+        self.tensors: List[TensorInfo] = [
+            TensorInfo(nm.decode(), dt, tuple(sh[:nd]), nb, fi, off, hp)
+            for nm, dt, nd, nb, fi, off, hp, sh in zip(names, *cols, shapes)]
         nf = C.c_size_t()
         _check(L.wt_num_files(h, C.byref(nf)))
         self.n_files = nf.value
