@@ -80,6 +80,8 @@ def parse_args():
                         "int8 matched protocol by default (one JSON line)")
     p.add_argument("--checksum", action="store_true",
                    help="time wt_checksum (leaf-tree FNV-1a-64) over every resident tensor of the workload")
+    p.add_argument("--consumer-priority", default="high", choices=["high", "normal"],
+                   help="priority of the stream the event-gated first-use GEMVs run on")
     p.add_argument("--timeline", action="store_true",
                    help="one traced file -> first-use run (WT_OPEN_TIMELINE): per ingest batch and GEMV group, "
                         "device begin/end times (one JSON line)")
@@ -353,6 +355,14 @@ def aggregate_gbs(bytes_per_rank, world, seconds):
 
 # ----------------------------------------------------------------------------- the wt arm
 
+def consumer_stream(torch, args):
+    """The stream of the event-gated GEMVs.  At high priority the block scheduler places a
+    GEMV group's CTAs before those of the gather batch that becomes ready at the same moment."""
+    if args.consumer_priority == "high":
+        return torch.cuda.Stream(priority=-1)
+    return torch.cuda.Stream()
+
+
 def make_slab(torch, pipeline, h, mats, dev=None):
     """Step 4, device allocation: one torch slab for the checkpoint (256-byte aligned views;
     or `dev`, already allocated), the x of every inner size and one fp32 buffer for every
@@ -488,7 +498,7 @@ def run_wt(args, rank, world):
     wdt = DT_NAME[gdt.pop()] if len(gdt) == 1 else "mixed"
     torch.cuda.synchronize()
 
-    ingest_s, consume_s = torch.cuda.Stream(), torch.cuda.Stream()
+    ingest_s, consume_s = torch.cuda.Stream(), consumer_stream(torch, args)
 
     # ---------------- e2e: file -> first use (1 warm-up, then timed repetitions), with the
     # device buffers allocated inside each run (fresh), and with buffers allocated once (reused)
@@ -625,6 +635,7 @@ def run_wt(args, rank, world):
         "data": DATA_DESC.get(wdt, "synthetic"),
         "config": {"workload": workload_desc(args), "weight_bytes": weight_bytes, "data_bytes": data_bytes,
                    "files": len(ck.paths), "matrices": len(dev.gemv_mats()), "ingest_mode": args.mode,
+                   "consumer_stream_priority": args.consumer_priority,
                    "open": {"map": "mapped", "nomap": "WT_OPEN_NOMAP (pread)", "prefault": "mapped, WT_OPEN_PREFAULT"}[args.open],
                    "l2": ("inputs larger than L2 (no flush)" if weight_bytes > L2_BYTES else
                           "inputs smaller than L2, no flush: passes may hit L2 (a dispatch-overhead point)"),
@@ -858,7 +869,7 @@ def run_timeline(args):
     slab = make_slab(torch, pipeline, h0, mats)
     rows = sum(mats[k].shape[0] for k in slab["dev"].gemv_mats())
     y_host = torch.empty(rows, dtype=torch.float32, pin_memory=True)
-    ingest_s, consume_s = torch.cuda.Stream(), torch.cuda.Stream()
+    ingest_s, consume_s = torch.cuda.Stream(), consumer_stream(torch, args)
     for _ in range(2):  # warm-up, untraced
         first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, flags=oflags)
     runs = []

@@ -18,7 +18,8 @@
 // same four k of X: A and B fragments come straight from whole vector loads, and an int8
 // word decodes into exactly the two f16x2 registers a fragment needs.
 //
-// Four 16-row tiles form a super block whose X registers are loaded once per K chunk.  At
+// Four 16-row tiles (two for int8 with T > 8) form a super block whose X registers are loaded
+// once per K chunk.  At
 // the end of a super block the warps' partial tiles meet in shared memory and are summed in
 // warp order (deterministic; rows never depend on the partition across CTAs).
 //
@@ -40,29 +41,36 @@ constexpr int kColWarps = 8;  // consumer warps
 constexpr int kColConsumers = kColWarps * 32;
 constexpr int kColThreads = kColConsumers + 32;  // + one producer warp
 constexpr int kColRows = kColTileRows;           // rows of one stage (one MMA tile)
-constexpr int kColBlocks = 4;                    // tiles per super block
-constexpr int kColSuper = kColRows * kColBlocks;
 constexpr int kColGroups = (kColVecMax / 4 + kColWarps - 1) / kColWarps;  // 4-vector groups per warp
 constexpr uint32_t kColStageBytes = kColRows * kColVecMax * 16;
 static_assert(kColVecMax % 8 == 4, "row pitch 64 bytes past a multiple of 128");
 static_assert(kColStageBytes % 128 == 0, "stages stay 128-byte aligned for the tensor copies");
 
-// Per-launch geometry: NT = 8-column MMA tiles (T <= 8: 1, else 2).  int8 weights with
-// T <= 8 run two CTAs per SM with half the ring each (the same bytes in flight per SM,
-// twice the warps; that case is latency-bound on its decode).  The cross-warp partials of
-// one 16-row tile take 16 x 8 NT floats per warp, in two alternating halves.
+// Per-launch geometry: NT = 8-column MMA tiles (T <= 8: 1, else 2).  int8 weights run two
+// CTAs per SM with half the ring each (the same bytes in flight per SM, twice the warps; the
+// int8 path is latency-bound on its decode).  The cross-warp partials of one 16-row tile take
+// 16 x 8 NT floats per warp, in two alternating halves.
 template <int DT, int NT>
 struct ColGeo {
-  static constexpr int kCtasPerSm = DT == 3 && NT == 1 ? 2 : 1;
+  static constexpr int kCtasPerSm = DT == 3 ? 2 : 1;
   static constexpr int kStages = kCtasPerSm == 2 ? 3 : 6;
+  // 16-row tiles per super block (X registers are loaded once per super block and chunk):
+  // four, or two for int8 with 16 columns, which then fits two CTAs per SM (registers and
+  // partial buffers halve; X is reloaded every 32 rows instead of 64)
+  static constexpr int kBlocks = DT == 3 && NT == 2 ? 2 : 4;
+  // accumulator sets per tile (even / odd k16 steps: shorter MMA chains); int8 with 16
+  // columns keeps one, its two column tiles already give two independent chains per A
+  static constexpr int kAcc = DT == 3 && NT == 2 ? 1 : 2;
+  static constexpr int kSuper = kColRows * kBlocks;
   static constexpr uint32_t kRedStride = 128 * NT;  // floats per (tile, warp)
-  static constexpr size_t kRedFloats = (size_t)kColBlocks * kColWarps * kRedStride;  // one half
+  static constexpr size_t kRedFloats = (size_t)kBlocks * kColWarps * kRedStride;  // one half
   static constexpr size_t kRedOff = (size_t)kStages * kColStageBytes;
   static constexpr size_t kBarOff = kRedOff + 2 * kRedFloats * sizeof(float);
   static constexpr size_t kFlagOff = kBarOff + 2 * kStages * sizeof(uint64_t);
   static constexpr size_t kSmem = kFlagOff + 16;
 };
-static_assert(ColGeo<1, 2>::kSmem <= 232448 && 2 * (ColGeo<3, 1>::kSmem + 1024) <= 233472,
+static_assert(ColGeo<1, 2>::kSmem <= 232448 && 2 * (ColGeo<3, 1>::kSmem + 1024) <= 233472 &&
+                  2 * (ColGeo<3, 2>::kSmem + 1024) <= 233472,
               "multi-column shared memory");
 
 // 32-bit words of X per weight vector: 16 fp16 activations for an int8 vector, else 8.
@@ -127,9 +135,9 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *tmap, int3
 // Thread (g, t) takes vector (q * warps + warp) * 4 + t of group q.
 // The box holds vc vectors per row at pitch vc * 16; rows and vectors past the matrix are
 // zeros, so only whole groups past vc are skipped.
-template <int DT, int NT>
+template <int DT, int NT, int H>
 __device__ __forceinline__ void cols_stage(uint32_t tile, uint32_t vc, int warp, uint32_t g, uint32_t t,
-                                           const uint32_t (&xr)[kColGroups][NT][ColX<DT>::W], float (&acc)[2][NT][4]) {
+                                           const uint32_t (&xr)[kColGroups][NT][ColX<DT>::W], float (&acc)[H][NT][4]) {
   const uint32_t pitch = vc * 16;
 #pragma unroll
   for (int q = 0; q < kColGroups; ++q) {
@@ -149,7 +157,7 @@ __device__ __forceinline__ void cols_stage(uint32_t tile, uint32_t vc, int warp,
         const uint32_t a1 = i8x2_to_f16x2(u1, 0x4140u), a3 = i8x2_to_f16x2(u1, 0x4342u);
 #pragma unroll
         for (int n = 0; n < NT; ++n)
-          mma16816<2>(acc[j & 1][n], a0, a1, a2, a3, xr[q][n][2 * j], xr[q][n][2 * j + 1]);
+          mma16816<2>(acc[(j & 1) % H][n], a0, a1, a2, a3, xr[q][n][2 * j], xr[q][n][2 * j + 1]);
       }
     } else {
       // words 2s, 2s+1 = elements 4s..4s+3 of the vector
@@ -157,7 +165,7 @@ __device__ __forceinline__ void cols_stage(uint32_t tile, uint32_t vc, int warp,
       for (int s = 0; s < 2; ++s) {
 #pragma unroll
         for (int n = 0; n < NT; ++n)
-          mma16816<DT>(acc[s][n], ra[2 * s], rb[2 * s], ra[2 * s + 1], rb[2 * s + 1], xr[q][n][2 * s],
+          mma16816<DT>(acc[s % H][n], ra[2 * s], rb[2 * s], ra[2 * s + 1], rb[2 * s + 1], xr[q][n][2 * s],
                        xr[q][n][2 * s + 1]);
       }
     }
@@ -178,14 +186,17 @@ __device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, c
   const uint32_t nchunk = (V + vc - 1) / vc;
   const uint32_t g = lane >> 2, t = lane & 3;
   const int ct = threadIdx.x;
+  constexpr int kColBlocks = ColGeo<DT, NT>::kBlocks;
+  constexpr int kColSuper = ColGeo<DT, NT>::kSuper;
   for (uint32_t sb = pc.r0; sb < pc.r1; sb += kColSuper) {
     const uint32_t rows = min((uint32_t)kColSuper, pc.r1 - sb);
     const uint32_t nrb = (rows + kColRows - 1) / kColRows;
-    float acc[kColBlocks][2][NT][4];  // two accumulator sets (even / odd k16 steps): shorter MMA chains
+    constexpr int H = ColGeo<DT, NT>::kAcc;
+    float acc[kColBlocks][H][NT][4];
 #pragma unroll
     for (int b = 0; b < kColBlocks; ++b)
 #pragma unroll
-      for (int h = 0; h < 2; ++h)
+      for (int h = 0; h < H; ++h)
 #pragma unroll
         for (int n = 0; n < NT; ++n) acc[b][h][n][0] = acc[b][h][n][1] = acc[b][h][n][2] = acc[b][h][n][3] = 0.f;
     for (uint32_t c = 0; c < nchunk; ++c) {
@@ -205,7 +216,7 @@ __device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, c
         if ((uint32_t)b < nrb) {
           const uint32_t s = it % ColGeo<DT, NT>::kStages;
           bounded_wait(R.full0 + 8 * s, (it / ColGeo<DT, NT>::kStages) & 1, R.abort_flag, R.status);
-          cols_stage<DT, NT>(R.stage0 + s * kColStageBytes, vc, warp, g, t, xr, acc[b]);
+          cols_stage<DT, NT, H>(R.stage0 + s * kColStageBytes, vc, warp, g, t, xr, acc[b]);
           __syncwarp();
           if (lane == 0) mbar_arrive(R.empty0 + 8 * s);
           ++it;
@@ -225,10 +236,10 @@ __device__ __forceinline__ void cols_piece(const MatDesc &md, const Piece &pc, c
 #pragma unroll
         for (int n = 0; n < NT; ++n) {
           const uint32_t c0 = 2 * t + 8 * n;
-          r[c0 * 16 + g] = acc[b][0][n][0] + acc[b][1][n][0];
-          r[(c0 + 1) * 16 + g] = acc[b][0][n][1] + acc[b][1][n][1];
-          r[c0 * 16 + g + 8] = acc[b][0][n][2] + acc[b][1][n][2];
-          r[(c0 + 1) * 16 + g + 8] = acc[b][0][n][3] + acc[b][1][n][3];
+          r[c0 * 16 + g] = acc[b][0][n][0] + (H == 2 ? acc[b][H - 1][n][0] : 0.f);
+          r[(c0 + 1) * 16 + g] = acc[b][0][n][1] + (H == 2 ? acc[b][H - 1][n][1] : 0.f);
+          r[c0 * 16 + g + 8] = acc[b][0][n][2] + (H == 2 ? acc[b][H - 1][n][2] : 0.f);
+          r[(c0 + 1) * 16 + g + 8] = acc[b][0][n][3] + (H == 2 ? acc[b][H - 1][n][3] : 0.f);
         }
       }
     }
@@ -286,8 +297,8 @@ __global__ void __launch_bounds__(kColThreads, (ColGeo<DT, NT>::kCtasPerSm))
         const MatDesc md = mats[pc.mat];
         const uint8_t *tmap = maps + (size_t)pc.mat * kTensorMapBytes;
         const uint32_t nchunk = (md.V + md.vc - 1) / md.vc;
-        for (uint32_t sb = pc.r0; sb < pc.r1 && live; sb += kColSuper) {
-          const uint32_t rows = min((uint32_t)kColSuper, pc.r1 - sb);
+        for (uint32_t sb = pc.r0; sb < pc.r1 && live; sb += Geo::kSuper) {
+          const uint32_t rows = min((uint32_t)Geo::kSuper, pc.r1 - sb);
           const uint32_t nrb = (rows + kColRows - 1) / kColRows;
           for (uint32_t c = 0; c < nchunk && live; ++c) {
             for (uint32_t b = 0; b < nrb; ++b) {
@@ -332,7 +343,7 @@ __global__ void __launch_bounds__(kColThreads, (ColGeo<DT, NT>::kCtasPerSm))
 
 }  // namespace
 
-int gemm_cols_ctas_per_sm(int dtype, int nt) { return dtype == 3 && nt == 1 ? 2 : 1; }
+int gemm_cols_ctas_per_sm(int dtype, int nt) { return dtype == 3 ? 2 : 1; }
 
 template <int DT, int NT>
 static cudaError_t cols_attr() {

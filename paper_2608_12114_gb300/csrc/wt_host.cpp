@@ -1428,9 +1428,6 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
       gl.begin = reinterpret_cast<const uint32_t *>(P->dev + L.begin);
       gl.status = h->status;
       gl.stall = wt::fault_injected("stall") ? 1 : 0;
-      // overlap with the previous kernel only when no event gates the group: a gated group
-      // keeps the plain stream order behind its cudaStreamWaitEvent
-      gl.pdl = wait ? 0 : 1;
       CU(wt::launch_gemv(gl, s));
       h->kernel_launches++;
     }
