@@ -57,7 +57,7 @@ def parse_args():
     p.add_argument("--workload", default="large")
     p.add_argument("--layers", type=int, default=None, help="override decoder layer count (small profiling cases)")
     p.add_argument("--mode", default="gather", choices=["gather", "ce", "staged"])
-    p.add_argument("--open", default="map", choices=["map", "nomap", "prefault"],
+    p.add_argument("--open", default="map", choices=["map", "nomap", "prefault", "register"],
                    help="nomap: wt_open maps nothing (WT_OPEN_NOMAP) and --mode staged preads into the pinned ring; "
                         "prefault: wt_open populates every mapping (WT_OPEN_PREFAULT)")
     p.add_argument("--e2e-reps", type=int, default=5)
@@ -477,7 +477,8 @@ def run_wt(args, rank, world):
         dist.barrier()
     build.build()  # no-op when fresh; loads the same in-tree library on every rank
     mode = {"gather": wt.WT_ADOPT_GATHER, "ce": wt.WT_ADOPT_CE, "staged": wt.WT_ADOPT_STAGED}[args.mode]
-    oflags = {"map": 0, "nomap": wt.WT_OPEN_NOMAP, "prefault": wt.WT_OPEN_PREFAULT}[args.open]
+    oflags = {"map": 0, "nomap": wt.WT_OPEN_NOMAP, "prefault": wt.WT_OPEN_PREFAULT,
+              "register": wt.WT_ROUTE_REGISTER}[args.open]
 
     probe = h2d_probe(torch)
     h2d = max(probe.values())
@@ -636,7 +637,8 @@ def run_wt(args, rank, world):
         "config": {"workload": workload_desc(args), "weight_bytes": weight_bytes, "data_bytes": data_bytes,
                    "files": len(ck.paths), "matrices": len(dev.gemv_mats()), "ingest_mode": args.mode,
                    "consumer_stream_priority": args.consumer_priority,
-                   "open": {"map": "mapped", "nomap": "WT_OPEN_NOMAP (pread)", "prefault": "mapped, WT_OPEN_PREFAULT"}[args.open],
+                   "open": {"map": "mapped", "nomap": "WT_OPEN_NOMAP (pread)", "prefault": "mapped, WT_OPEN_PREFAULT",
+                            "register": "mapped, WT_ROUTE_REGISTER"}[args.open],
                    "l2": ("inputs larger than L2 (no flush)" if weight_bytes > L2_BYTES else
                           "inputs smaller than L2, no flush: passes may hit L2 (a dispatch-overhead point)"),
                    "parallelism": "replicas" if world > 1 else "1 GPU",
@@ -863,7 +865,8 @@ def run_timeline(args):
     build.build()
     torch.cuda.set_device(0)
     mode = {"gather": wt.WT_ADOPT_GATHER, "ce": wt.WT_ADOPT_CE, "staged": wt.WT_ADOPT_STAGED}[args.mode]
-    oflags = {"map": 0, "nomap": wt.WT_OPEN_NOMAP, "prefault": wt.WT_OPEN_PREFAULT}[args.open]
+    oflags = {"map": 0, "nomap": wt.WT_OPEN_NOMAP, "prefault": wt.WT_OPEN_PREFAULT,
+              "register": wt.WT_ROUTE_REGISTER}[args.open]
     h0 = wt.Handle(ck.paths, oflags)
     mats = pipeline.matrices(h0)
     slab = make_slab(torch, pipeline, h0, mats)

@@ -516,9 +516,11 @@ struct Range {
 int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cudaStream_t s,
                  void **ready, uint64_t total) {
   const uint64_t target = std::min<uint64_t>(128ull << 20, std::max<uint64_t>(2ull << 20, total / 64));
-  // One gather CTA per SM saturates the link (210 GB/s either way) and leaves each SM room
-  // for a resident GEMV CTA beside it (registers: 256 x 48 + 288 x 168 of 65536), so the
-  // event-gated consumer of a batch runs while the next batch is in flight.
+  // One gather CTA per SM: the link runs at 207 GB/s with 2, 1 or a third of a CTA per SM.
+  // An event-gated GEMV group shares the SMs with the next batch's gather and advances at
+  // about the gather's pace (a 200 MB group in ~1 ms instead of ~30 us alone); 48 or 64
+  // gather CTAs leave it almost untouched, but file -> first use measured 86-97 ms with
+  // them against 78 ms here, so the link-bound whole keeps the wide grid.
   const int grid_cap = wt::num_sms();
   // Tensors larger than a batch are cut into pieces (multiples of 64 KiB, so each piece keeps
   // its range's alignment): page-table population and transfer then pipeline inside a tensor.

@@ -797,14 +797,9 @@ static cudaError_t gemv_attr() {
 
 cudaError_t gemv_prepare() {
   cudaError_t e;
-  if ((e = gemv_attr<0>()) != cudaSuccess || (e = gemv_attr<1>()) != cudaSuccess || (e = gemv_attr<2>()) != cudaSuccess ||
-      (e = gemv_attr<3>()) != cudaSuccess)
+  if ((e = gemv_attr<0>()) != cudaSuccess || (e = gemv_attr<1>()) != cudaSuccess || (e = gemv_attr<2>()) != cudaSuccess)
     return e;
-  // The gather uses no shared memory, but an SM running it keeps the largest shared-memory
-  // carveout: an SM configured for less cannot take a GEMV CTA (197 KB) until it drains, so
-  // the event-gated GEMV of batch i would wait for the gather of batch i + 1 to finish.
-  return cudaFuncSetAttribute(gather_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                              (int)cudaSharedmemCarveoutMaxShared);
+  return gemv_attr<3>();
 }
 
 cudaError_t launch_gemv(const GemvLaunch &L, cudaStream_t s) {
