@@ -370,13 +370,8 @@ def make_slab(torch, pipeline, h, mats, dev=None):
     if dev is None:
         dev = pipeline.DeviceCheckpoint.allocate(h, mats)
     xs = dev.inputs()
-    rows = [mats[k].shape[0] for k in dev.gemv_mats()]
-    yflat = torch.empty(sum(rows), dtype=torch.float32, device="cuda")
-    ys, o = {}, 0
-    for k, r in zip(dev.gemv_mats(), rows):
-        ys[k] = yflat[o:o + r]
-        o += r
-    return {"dev": dev, "xs": xs, "ys": ys, "yflat": yflat}
+    ys = dev.outputs_flat()
+    return {"dev": dev, "xs": xs, "ys": ys, "yflat": ys.buf}
 
 
 def first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, phases=None, flags=0,

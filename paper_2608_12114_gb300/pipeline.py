@@ -89,6 +89,23 @@ def matrices(h: wt.Handle) -> List[MatrixRef]:
     return out
 
 
+class FlatOutputs:
+    """Every GEMV matrix's fp32 y in one device buffer (one D2H copy reads them all); y of
+    matrix k starts `offset[k]` floats into it.  descs() takes the addresses from here without
+    building a tensor per matrix."""
+
+    def __init__(self, buf, offset: Dict[int, int]):
+        self.buf = buf
+        self.offset = offset
+
+    def __getitem__(self, k):
+        return self.buf[self.offset[k]:self.offset[k] + self._rows[k]]
+
+    def ptrs(self, ks) -> np.ndarray:
+        base = self.buf.data_ptr()
+        return base + 4 * np.fromiter((self.offset[k] for k in ks), np.uint64, len(ks))
+
+
 @dataclass
 class DeviceCheckpoint:
     mats: List[MatrixRef]
@@ -125,17 +142,23 @@ class DeviceCheckpoint:
 
     @staticmethod
     def stream_in(h: wt.Handle, mats: Sequence[MatrixRef], mode: int = wt.WT_ADOPT_GATHER, stream: int = 0,
-                  first_bytes: int = 256 << 20, segments: int = 8, device="cuda"):
+                  first_bytes: int = 256 << 20, segments: Optional[int] = None, device="cuda"):
         """Allocation (step 4) interleaved with ingest (step 5): the logical tensors are cut, at
         tensor boundaries and in order, into a small first segment (about `first_bytes`) and
         then `segments` segments of nearly equal bytes; each segment gets its own device slab
         right before its wt_adopt call, so the link starts after the first small allocation
-        and every later allocation runs while earlier bytes are in flight.  Returns
+        and every later allocation runs while earlier bytes are in flight.  By default one
+        segment per 2 GB, at most 8: below that, allocating costs less than a wt_adopt call
+        (under 0.2 ms per GB), and a checkpoint is one slab and one call.  Returns
         (DeviceCheckpoint, tensor -> ready event, host seconds spent allocating)."""
         import time
         import torch
         sizes = [sum(h.tensors[i].nbytes for i in m.parts) for m in mats]
         total = sum(sizes)
+        if segments is None:
+            segments = min(8, total // (2 << 30))
+        if segments == 0:
+            first_bytes = total
         cuts, acc, limit = [], 0, min(first_bytes, total)
         step = max(1, -(-(total - limit) // max(1, segments)))
         for k, n in enumerate(sizes):
@@ -189,6 +212,16 @@ class DeviceCheckpoint:
                 xs[key] = torch.from_numpy(synth.make_x(m.shape[1], m.dtype)).to(device)
         return xs
 
+    def outputs_flat(self, device="cuda") -> FlatOutputs:
+        """One fp32 buffer holding every GEMV matrix's y, in gemv_mats() order."""
+        import torch
+        ks = self.gemv_mats()
+        rows = [self.mats[k].shape[0] for k in ks]
+        offs = np.concatenate(([0], np.cumsum(rows)[:-1])).astype(np.int64).tolist() if ks else []
+        fo = FlatOutputs(torch.empty(max(1, sum(rows)), dtype=torch.float32, device=device), dict(zip(ks, offs)))
+        fo._rows = dict(zip(ks, rows))
+        return fo
+
     def outputs(self, device="cuda") -> Dict[int, object]:
         import torch
         return {k: torch.empty(self.mats[k].shape[0], dtype=torch.float32, device=device)
@@ -213,7 +246,7 @@ class DeviceCheckpoint:
             self._tables[key] = base
         out = base.copy()
         out["x"] = [xs[(self.mats[k].shape[1], self.mats[k].dtype)].data_ptr() for k in ks]
-        out["y"] = [ys[k].data_ptr() for k in ks]
+        out["y"] = ys.ptrs(ks) if isinstance(ys, FlatOutputs) else [ys[k].data_ptr() for k in ks]
         if events:
             pos = {i: n for n, i in enumerate(events)}
             out["wait_event"] = [events[max(self.mats[k].parts + ([self.mats[k].scale] if self.mats[k].scale is not None else []),
