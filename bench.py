@@ -303,11 +303,22 @@ def h2d_probe(torch, nbytes=1 << 30, reps=10, streams=(1, 2, 4), sm_loads=True):
     return out
 
 
-def onecol_kernel_name(wdt, ks):
+def int8_tc_kernel(ms, T):
+    """The tensor-core kernel an int8 launch of matrices ms ([(M, K)]) with T columns runs:
+    the row-owner kernel when its 128-row blocks number at least two per CTA slot (or when
+    WT_COLS_KERNEL=q8rows), else the warp-MMA kernel (as the library decides)."""
+    force = os.environ.get("WT_COLS_KERNEL")
+    blocks = sum(-(-M // 128) for M, _ in ms)
+    if force == "q8rows" or (force != "mma" and blocks >= 2 * 152):
+        return "gemm_q8_rows_kernel<NT=%d> (mma.sync m16n8k16, row-owner warps)" % (2 if T > 8 else 1)
+    return "gemm_cols_kernel<int8, NT=%d> (mma.sync m16n8k16)" % (2 if T > 8 else 1)
+
+
+def onecol_kernel_name(wdt, ms):
     """The kernel a one-column resident pass runs: the TMA GEMV, or for int8 rows up to
-    K = 8192 the warp-MMA kernel at T = 1 (unless WT_I8_ONECOL=cuda)."""
-    if wdt == "int8" and os.environ.get("WT_I8_ONECOL") != "cuda" and max(ks) <= 8192:
-        return "gemm_cols_kernel<int8, T=1> (mma.sync m16n8k16)"
+    K = 8192 a tensor-core kernel at T = 1 (unless WT_I8_ONECOL=cuda)."""
+    if wdt == "int8" and os.environ.get("WT_I8_ONECOL") != "cuda" and max(K for _, K in ms) <= 8192:
+        return int8_tc_kernel(ms, 1)
     return "gemv_tma_kernel<%s>" % wdt
 
 
@@ -621,7 +632,7 @@ def run_wt(args, rank, world):
                 "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
                 "traffic": (tr["dram_bytes_per_launch_full"] if tr else None),
                 "algorithmic_bytes_per_launch": alg_bytes,
-                "kernel": onecol_kernel_name(wdt, [dev.mats[k].shape[1] for k in dev.gemv_mats()]),
+                "kernel": onecol_kernel_name(wdt, [dev.mats[k].shape for k in dev.gemv_mats()]),
                 "frac_of_nominal_8TBps": round(achieved / NOMINAL_HBM_GBS, 4)}
     clocks = clk.summary()
     out = {
@@ -1005,8 +1016,11 @@ def run_tsweep(args):
             two_byte = all(dev.mats[k].dtype in (wt.WT_BF16, wt.WT_F16) for k in ks)
             force = os.environ.get("WT_COLS_KERNEL")
             on_umma = two_byte and (force == "umma" or (force != "mma" and T > 8))
-            kname = ("gemv_tma (one column)" if T == 0 else
-                     "gemm_cols_umma (tcgen05, M128 N16 K16)" if on_umma else "gemm_cols (mma.sync m16n8k16)")
+            shapes = [dev.mats[k].shape for k in ks]
+            int8 = all(dev.mats[k].dtype == wt.WT_I8 for k in ks)
+            kname = (onecol_kernel_name(DT_NAME[dev.mats[ks[0]].dtype], shapes) if T == 0 else
+                     "gemm_cols_umma (tcgen05, M128 N16 K16)" if on_umma else
+                     int8_tc_kernel(shapes, T) if int8 else "gemm_cols (mma.sync m16n8k16)")
             rows.append({"T": T, "kernel": kname,
                          "ms": round(ms, 4), "weight_gbs": round(wbytes / ms / 1e6, 1),
                          "logical_gbs": round(n * wbytes / ms / 1e6, 1), "tflops": round(flops / ms / 1e9, 2),

@@ -8,8 +8,9 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 LIB = os.path.join(HERE, "libwt.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["wt_kernels.cu", "wt_fnv.cu", "wt_cols.cu", "wt_umma.cu", "wt_host.cpp", "wt_dlpack.cpp", "wt_noalloc.cu"]
-HEADERS = ["wt_kernels.h", "wt_fnv.h", "wt_device.cuh", os.path.join("..", "..", "include", "wt.h"),
+SOURCES = ["wt_kernels.cu", "wt_fnv.cu", "wt_cols.cu", "wt_umma.cu", "wt_q8rows.cu", "wt_host.cpp", "wt_dlpack.cpp",
+           "wt_noalloc.cu"]
+HEADERS = ["wt_kernels.h", "wt_fnv.h", "wt_q8rows.h", "wt_device.cuh", os.path.join("..", "..", "include", "wt.h"),
            os.path.join("..", "..", "include", "wt_dlpack.h")]
 
 

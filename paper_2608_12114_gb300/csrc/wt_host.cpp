@@ -41,6 +41,7 @@
 #include "../../include/wt_dlpack.h"
 #include "wt_fnv.h"
 #include "wt_kernels.h"
+#include "wt_q8rows.h"
 
 #ifndef MADV_POPULATE_READ
 #define MADV_POPULATE_READ 22
@@ -235,6 +236,7 @@ struct Plan {
     size_t mats, pieces, begin;  // byte offsets in the table
     size_t maps = SIZE_MAX;      // multi-column launches: tensor maps (128-byte aligned)
     bool umma = false;           // multi-column launch on tcgen05 (wt_umma.cu)
+    bool q8rows = false;         // int8 multi-column launch on the row-owner kernel (wt_q8rows.cu)
     bool mapped_cols = false;    // map endpoint with T columns
     int nt = 0;                  // warp-MMA multi-column launches: 8-column tiles (1 or 2)
     uint32_t nmat = 0, ntiles = 0;
@@ -467,6 +469,7 @@ int prepare_device(int dev) {
     CU(wt::gemv_prepare());
     CU(wt::gemm_cols_prepare());
     CU(wt::gemm_cols_umma_prepare());
+    CU(wt::gemm_q8_rows_prepare());
     g_prepared[dev] = true;
   }
   return WT_OK;
@@ -964,23 +967,65 @@ int one_col_slices(int dtype) { return dtype == WT_I8 ? 1 : 16; }
 // 6580; int8 decodes in registers there).  WT_COLS_KERNEL=mma or =umma forces one kernel
 // (umma still only for 2-byte weights).
 bool cols_on_umma(int dtype, int cols) {
-  static const int force = [] {
-    const char *e = getenv("WT_COLS_KERNEL");
-    if (e && strcmp(e, "umma") == 0) return 1;
-    if (e && strcmp(e, "mma") == 0) return 2;
-    return 0;
-  }();
+  const char *e = getenv("WT_COLS_KERNEL");
+  const int force = e && strcmp(e, "umma") == 0 ? 1 : e && strcmp(e, "mma") == 0 ? 2 : 0;
   if (dtype != WT_BF16 && dtype != WT_F16) return false;
   return force == 1 || (force == 0 && cols > 8);
 }
 
-// int8 weights with one activation column: the warp-level MMA kernel at T = 1 (wt_cols.cu)
-// streams the matched protocol at 6662 GB/s against 6386 for the CUDA-core kernel, which is
-// issue-bound (ncu: 66.5 % issue active, not_selected on top) while the MMA path decodes a
-// 16-byte vector straight into an MMA operand with 1.6x fewer instructions.  It takes rows up
-// to seg_vectors(int8) vectors (K <= 8192); longer rows keep the CUDA-core kernel's cross-CTA
-// split-K, since the MMA kernel gives a whole row to one CTA.  WT_I8_ONECOL=cuda keeps every
-// int8 one-column matrix on the CUDA-core kernel (its parity tests run both ways).
+// int8 weights on the tensor cores (T columns, and one column with rows up to K = 8192) run
+// the row-owner kernel (wt_q8rows.cu) when its 128-row blocks fill the GPU (at least two per
+// CTA slot over the launch): its warps keep no activation registers and meet in no reduction.
+// The matched protocol: T = 1 / 8 / 16 at 6663 / 6581 / 6502 GB/s against 6565 / 6250 / 5004
+// on the warp-MMA kernel.  Launches of fewer rows keep the warp-MMA kernel's 16-row tiles,
+// which spread over 8 times as many CTAs.  WT_COLS_KERNEL=mma or =q8rows forces one kernel
+// for every int8 matrix (the parity tests run each routing).
+bool i8_on_q8rows(uint64_t blocks) {
+  const char *e = getenv("WT_COLS_KERNEL");
+  if (e && strcmp(e, "mma") == 0) return false;
+  if (e && strcmp(e, "q8rows") == 0) return true;
+  return blocks >= 2ull * wt::num_sms();
+}
+
+// The two tensor maps of a row-owner int8 matrix (see wt::launch_gemm_q8_rows).
+int encode_q8rows_maps(const wt::MatDesc &m, uint8_t *out) {
+  EncodeTiledFn fn = encode_tiled();
+  if (!fn) return set_err(WT_ECUDA, "wt_pass: cuTensorMapEncodeTiled is not available from the driver");
+  const uint64_t K = (uint64_t)m.V * 16;
+  CUtensorMap mw, mx;
+  {
+    const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)m.M};
+    const cuuint64_t strides[1] = {(cuuint64_t)K};
+    const cuuint32_t box[2] = {192, (cuuint32_t)wt::kQ8RowsBlock};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = fn(&mw, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(m.W), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return set_err(WT_ECUDA, "wt_pass: tensor map of int8 W failed (%d)", (int)r);
+  }
+  {
+    const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)m.G};
+    const cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+    const cuuint32_t box[2] = {64, 16};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = fn(&mx, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<uint8_t *>(m.x), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return set_err(WT_ECUDA, "wt_pass: tensor map of fp16 X failed (%d)", (int)r);
+  }
+  memcpy(out, &mw, sizeof mw);
+  memcpy(out + wt::kTensorMapBytes, &mx, sizeof mx);
+  return WT_OK;
+}
+
+// int8 weights with one activation column go to the tensor-core kernels at T = 1: the CUDA-core
+// kernel is issue-bound (ncu: 66.5 % issue active, not_selected on top), while the MMA paths
+// decode a 16-byte vector straight into an MMA operand with 1.6x fewer instructions (matched
+// protocol: 6386 GB/s on CUDA cores, 6565 on the warp-MMA kernel, 6663 on the row-owner
+// kernel).  They take rows up to seg_vectors(int8) vectors (K <= 8192); longer rows keep the
+// CUDA-core kernel's cross-CTA split-K, since the MMA kernels give a whole row to one CTA.
+// WT_I8_ONECOL=cuda keeps every int8 one-column matrix on the CUDA-core kernel (its parity
+// tests run both ways).
 bool i8_onecol_on_mma(uint32_t V) {
   const char *e = getenv("WT_I8_ONECOL");
   if (e && strcmp(e, "cuda") == 0) return false;
@@ -1171,7 +1216,10 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
     Plan::Group g;
     g.first = i;
     // cols_dt: warp-MMA multi-column with T <= 8, colsw_dt: with 8 < T <= 16
-    std::vector<wt::MatDesc> by_dt[4], mapped_dt[4], cols_dt[4], umma_dt[4], mcols_dt[4], colsw_dt[4];
+    std::vector<wt::MatDesc> by_dt[4], mapped_dt[4], cols_dt[4], umma_dt[4], mcols_dt[4], colsw_dt[4], q8r_dt[4],
+        q8r1_dt[4];  // row-owner int8 launches with two 8-column tiles (T > 8) and with one
+    std::vector<wt::MatDesc> i8c[2];  // int8 on the tensor cores, T <= 8 and T > 8: kernel chosen below
+    uint64_t i8_blocks = 0;           // their 128-row blocks
     std::vector<int64_t> seg_ws[4];  // per by_dt entry: workspace float offset of its partials, or -1
     std::vector<wt::SegReduce> reds;
     std::vector<size_t> red_ws;      // per reds entry: workspace float offset
@@ -1231,13 +1279,17 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
           g.generic.push_back({q.dtype, static_cast<const uint8_t *>(q.W), static_cast<const uint8_t *>(q.x), q.y, q.M, q.K,
                                static_cast<const uint8_t *>(q.scale), ncol});
         }
+      } else if (fast && q.cols > 0 && q.dtype == WT_I8) {
+        i8c[q.cols > 8 ? 1 : 0].push_back(make_cols_mat(q));
+        i8_blocks += (q.M + wt::kQ8RowsBlock - 1) / wt::kQ8RowsBlock;
       } else if (fast && q.cols > 0) {
         (cols_on_umma(q.dtype, q.cols) ? umma_dt : q.cols > 8 ? colsw_dt : cols_dt)[q.dtype].push_back(make_cols_mat(q));
       } else if (fast && q.dtype == WT_I8 && i8_onecol_on_mma((uint32_t)(q.K / 16))) {
-        // y[M] is Y[1, M] and x[K] is X[1, K]: the one-column GEMV as the T = 1 MMA kernel
+        // y[M] is Y[1, M] and x[K] is X[1, K]: the one-column GEMV as a T = 1 tensor-core GEMV
         wt_gemv_desc q1 = q;
         q1.cols = 1;
-        cols_dt[WT_I8].push_back(make_cols_mat(q1));
+        i8c[0].push_back(make_cols_mat(q1));
+        i8_blocks += (q.M + wt::kQ8RowsBlock - 1) / wt::kQ8RowsBlock;
       } else if (fast && q.K * es / 16 > wt::seg_vectors(q.dtype)) {
         // long rows: column segments spread over CTAs, summed by the second pass
         const uint32_t V = (uint32_t)(q.K * es / 16);
@@ -1266,14 +1318,23 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
                              static_cast<const uint8_t *>(q.scale), ncol});
       }
     }
-    for (int pass = 0; pass < 6; ++pass) {
+    if (!i8c[0].empty() || !i8c[1].empty()) {
+      const bool rows = i8_on_q8rows(i8_blocks);
+      auto &lo = rows ? q8r1_dt[WT_I8] : cols_dt[WT_I8];
+      auto &hi = rows ? q8r_dt[WT_I8] : colsw_dt[WT_I8];
+      lo.insert(lo.end(), i8c[0].begin(), i8c[0].end());
+      hi.insert(hi.end(), i8c[1].begin(), i8c[1].end());
+    }
+    for (int pass = 0; pass < 8; ++pass) {
       for (int dt = 0; dt < 4; ++dt) {
         std::vector<wt::MatDesc> &ms = pass == 0   ? by_dt[dt]
                                        : pass == 1 ? mapped_dt[dt]
                                        : pass == 2 ? cols_dt[dt]
                                        : pass == 3 ? umma_dt[dt]
                                        : pass == 4 ? mcols_dt[dt]
-                                                   : colsw_dt[dt];
+                                       : pass == 5 ? colsw_dt[dt]
+                                       : pass == 6 ? q8r_dt[dt]
+                                                   : q8r1_dt[dt];
         const bool warp_mma = pass == 2 || pass == 5;
         if (ms.empty()) continue;
         Plan::Launch L;
@@ -1299,6 +1360,23 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
           P->table.resize(L.maps + ms.size() * 2 * wt::kTensorMapBytes);
           for (size_t k = 0; k < ms.size(); ++k) {
             int rc = encode_umma_maps(ms[k], P->table.data() + L.maps + k * 2 * wt::kTensorMapBytes);
+            if (rc) return rc;
+          }
+          g.cols.push_back(L);
+          continue;
+        }
+        if (pass >= 6) {
+          // row-owner int8 launch: pieces cut at 128-row blocks, two tensor maps per matrix
+          L.q8rows = true;
+          L.nt = pass == 6 ? 2 : 1;
+          partition(ms, L.grid, pieces, begin, (uint32_t)wt::kQ8RowsBlock, 1, 2);
+          L.mats = append(P->table, ms);
+          L.pieces = append(P->table, pieces);
+          L.begin = append(P->table, begin);
+          L.maps = (P->table.size() + 127) & ~(size_t)127;
+          P->table.resize(L.maps + ms.size() * 2 * wt::kTensorMapBytes);
+          for (size_t k = 0; k < ms.size(); ++k) {
+            int rc = encode_q8rows_maps(ms[k], P->table.data() + L.maps + k * 2 * wt::kTensorMapBytes);
             if (rc) return rc;
           }
           g.cols.push_back(L);
@@ -1458,7 +1536,9 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
       gl.status = h->status;
       gl.maps = P->dev + L.maps;
       gl.nt = L.nt;
-      if (L.umma) {
+      if (L.q8rows) {
+        CU(wt::launch_gemm_q8_rows(gl, s));
+      } else if (L.umma) {
         wt::UmmaLaunch ul;
         ul.dtype = L.dtype;
         ul.grid = L.grid;

@@ -28,6 +28,19 @@ def torch():
     return torch
 
 
+@pytest.fixture(params=["default", "mma", "umma", "q8rows"], autouse=True)
+def cols_kernel(request, monkeypatch):
+    """Every test runs under each routing of the multi-column kernels: the default (int8 with
+    T > 8 on the row-owner kernel, 2-byte weights with T > 8 on tcgen05, the rest on the
+    warp-MMA kernel), everything on the warp-MMA kernel (WT_COLS_KERNEL=mma), 2-byte weights
+    on tcgen05 at every T (=umma), and int8 on the row-owner kernel at every T (=q8rows)."""
+    if request.param == "default":
+        monkeypatch.delenv("WT_COLS_KERNEL", raising=False)
+    else:
+        monkeypatch.setenv("WT_COLS_KERNEL", request.param)
+    return request.param
+
+
 def make(torch, rng, dtype, M, K, T):
     """Host bytes and device copies of W, X (and s for int8)."""
     if dtype == I8:
@@ -178,10 +191,15 @@ def test_cols_mixed_column_counts_and_dtypes_in_one_pass(torch):
         check(c, c["Y"])
 
 
-def test_cols_full_size_matched_protocol(torch, tmp_path):
+def test_cols_full_size_matched_protocol(torch, tmp_path, cols_kernel):
     """The T-sweep's launch configuration at full size: 12 matrices of 12288 x 7168 int8 with
-    fp16 row scales in one pass, T = 8 and 16; first, last and 16 seeded rows per matrix."""
+    fp16 row scales in one pass, T = 8 and 16; every output against the oracle (its functions
+    run unchanged on blocks of rows, in threads), Y NaN-filled first."""
+    from concurrent.futures import ThreadPoolExecutor
     from paper_2608_12114_gb300 import pipeline
+    if cols_kernel != "default":
+        pytest.skip("full size runs the default routing; the small cases cover the forced ones")
+    pool = ThreadPoolExecutor(16)
     ck = synth.build("protocol_q8", str(tmp_path), workers=16)
     co = oracle.CheckpointOracle(ck.paths)
     try:
@@ -203,10 +221,14 @@ def test_cols_full_size_matched_protocol(torch, tmp_path):
                 for k in ks:
                     m = dev.mats[k]
                     t, sc = h.tensors[m.parts[0]], h.tensors[m.scale]
-                    r = sorted({0, 12287} | {int(v) for v in np.random.default_rng(k).integers(0, 12288, 16)})
-                    Yhat, A = oracle.gemv_cols(co.blob_of(t.file, t.name), 3, 12288, 7168, X.view(np.uint8), T,
-                                               scale=co.blob_of(sc.file, sc.name), rows=r)
-                    got = ys[k].cpu().numpy().reshape(T, 12288)[:, r]
+                    W, S = co.blob_of(t.file, t.name), co.blob_of(sc.file, sc.name)
+                    blocks = [(r, min(12288, r + 1024)) for r in range(0, 12288, 1024)]
+                    parts = list(pool.map(lambda b: oracle.gemv_cols(W[b[0] * 7168:b[1] * 7168], 3, b[1] - b[0], 7168,
+                                                                     X.view(np.uint8), T, scale=S[2 * b[0]:2 * b[1]]),
+                                          blocks))
+                    Yhat = np.concatenate([p[0] for p in parts], axis=1)
+                    A = np.concatenate([p[1] for p in parts], axis=1)
+                    got = ys[k].cpu().numpy().reshape(T, 12288)
                     assert oracle.gemv_error(got.reshape(-1), Yhat.reshape(-1), A.reshape(-1)) <= TOL, (T, m.name)
     finally:
         co.close()

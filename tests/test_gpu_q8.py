@@ -26,15 +26,20 @@ def torch():
     return torch
 
 
-@pytest.fixture(params=["default", "cuda"], autouse=True)
+@pytest.fixture(params=["default", "cuda", "q8rows"], autouse=True)
 def onecol_kernel(request, monkeypatch):
-    """Every test runs twice: with the default routing (rows up to K = 8192 on the warp-MMA
-    kernel at T = 1, longer rows on the CUDA-core kernel's split-K) and with every int8 row on
-    the CUDA-core kernel (WT_I8_ONECOL=cuda), so both kernels' tile modes stay covered."""
+    """Every test runs three times: with the default routing (rows up to K = 8192 on a
+    tensor-core kernel at T = 1: the warp-MMA kernel for launches this small, longer rows on the
+    CUDA-core kernel's split-K), with every int8 row on the CUDA-core kernel
+    (WT_I8_ONECOL=cuda), and with the tensor-core rows on the row-owner kernel
+    (WT_COLS_KERNEL=q8rows, the kernel full-size launches take), so every kernel's tile
+    modes stay covered."""
+    monkeypatch.delenv("WT_I8_ONECOL", raising=False)
+    monkeypatch.delenv("WT_COLS_KERNEL", raising=False)
     if request.param == "cuda":
         monkeypatch.setenv("WT_I8_ONECOL", "cuda")
-    else:
-        monkeypatch.delenv("WT_I8_ONECOL", raising=False)
+    elif request.param == "q8rows":
+        monkeypatch.setenv("WT_COLS_KERNEL", "q8rows")
     return request.param
 
 
