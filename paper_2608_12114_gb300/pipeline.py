@@ -89,6 +89,29 @@ def matrices(h: wt.Handle) -> List[MatrixRef]:
     return out
 
 
+class SlabViews:
+    """Per logical tensor, a uint8 view of the slab that holds it, made on first access: a
+    checkpoint of thousands of tensors needs their addresses (DeviceCheckpoint.ptrs) at once,
+    but a torch view of each only when a caller reads one."""
+
+    def __init__(self, spans):
+        self._spans = spans  # (slab tensor, byte offset, bytes) per logical tensor
+        self._views = {}
+
+    def __len__(self):
+        return len(self._spans)
+
+    def __getitem__(self, k):
+        v = self._views.get(k)
+        if v is None:
+            t, o, n = self._spans[k]
+            v = self._views[k] = t[o:o + n]
+        return v
+
+    def __iter__(self):
+        return (self[k] for k in range(len(self._spans)))
+
+
 class FlatOutputs:
     """Every GEMV matrix's fp32 y in one device buffer (one D2H copy reads them all); y of
     matrix k starts `offset[k]` floats into it.  descs() takes the addresses from here without
@@ -109,10 +132,11 @@ class FlatOutputs:
 @dataclass
 class DeviceCheckpoint:
     mats: List[MatrixRef]
-    bufs: List[object]                   # torch uint8 tensors, one per MatrixRef
+    bufs: object                         # per MatrixRef a torch uint8 view (SlabViews or a list)
     dst: Dict[int, int] = field(default_factory=dict)  # tensor index -> device address
     canary: int = 0
     _tables: Dict[tuple, object] = field(default_factory=dict)
+    ptrs: List[int] = field(default_factory=list)  # device address of each MatrixRef's buffer
 
     @staticmethod
     def allocate(h: wt.Handle, mats: Sequence[MatrixRef], device="cuda", canary: int = 0,
@@ -122,22 +146,25 @@ class DeviceCheckpoint:
         slab=True carves every buffer out of one allocation (256-byte aligned offsets)."""
         import torch
         sizes = [sum(h.tensors[i].nbytes for i in m.parts) for m in mats]
-        bufs = []
         if slab:
             offs, pos = [], 0
             for n in sizes:
                 offs.append(pos)
                 pos += -(-(n + canary) // _ALIGN) * _ALIGN
             big = torch.empty(max(pos, 1), dtype=torch.uint8, device=device)
-            bufs = [big[o:o + n + canary] for o, n in zip(offs, sizes)]
+            bufs = SlabViews([(big, o, n + canary) for o, n in zip(offs, sizes)])
+            base = big.data_ptr()
+            ptrs = [base + o for o in offs]
         else:
             bufs = [torch.empty(n + canary, dtype=torch.uint8, device=device) for n in sizes]
-        dc = DeviceCheckpoint(list(mats), bufs, canary=canary)
-        for m, b in zip(mats, bufs):
+            ptrs = [b.data_ptr() for b in bufs]
+        dc = DeviceCheckpoint(list(mats), bufs, canary=canary, ptrs=ptrs)
+        tensors = h.tensors
+        for m, p in zip(mats, ptrs):
             off = 0
             for i in m.parts:
-                dc.dst[i] = b.data_ptr() + off
-                off += h.tensors[i].nbytes
+                dc.dst[i] = p + off
+                off += tensors[i].nbytes
         return dc
 
     @staticmethod
@@ -167,7 +194,9 @@ class DeviceCheckpoint:
                 cuts.append(k + 1)
                 limit = acc + step
         bounds = [0] + cuts + [len(mats)]
-        dc = DeviceCheckpoint(list(mats), [None] * len(mats))
+        spans = [None] * len(mats)
+        dc = DeviceCheckpoint(list(mats), SlabViews(spans), ptrs=[0] * len(mats))
+        tensors = h.tensors
         events: Dict[int, int] = {}
         alloc_s = 0.0
         for a, b in zip(bounds, bounds[1:]):
@@ -178,13 +207,15 @@ class DeviceCheckpoint:
                 pos += -(-sizes[k] // _ALIGN) * _ALIGN
             big = torch.empty(max(pos, 1), dtype=torch.uint8, device=device)
             alloc_s += time.perf_counter() - t0
+            base = big.data_ptr()
             idx = []
             for k, o in zip(range(a, b), offs):
-                dc.bufs[k] = big[o:o + sizes[k]]
+                spans[k] = (big, o, sizes[k])
+                dc.ptrs[k] = p = base + o
                 off = 0
                 for i in mats[k].parts:
-                    dc.dst[i] = dc.bufs[k].data_ptr() + off
-                    off += h.tensors[i].nbytes
+                    dc.dst[i] = p + off
+                    off += tensors[i].nbytes
                     idx.append(i)
             idx.sort()
             if idx:
@@ -238,7 +269,7 @@ class DeviceCheckpoint:
         if base is None:  # the parts that depend only on this checkpoint's buffers
             base = np.zeros(len(ks), wt.DESC_DTYPE)
             mats = [self.mats[k] for k in ks]
-            base["W"] = [self.bufs[k].data_ptr() for k in ks]
+            base["W"] = [self.ptrs[k] for k in ks]
             base["dtype"] = [m.dtype for m in mats]
             base["M"] = [m.shape[0] for m in mats]
             base["K"] = [m.shape[1] for m in mats]
@@ -262,4 +293,4 @@ class DeviceCheckpoint:
 
     @property
     def data_bytes(self) -> int:
-        return sum(int(b.numel()) - self.canary for b in self.bufs)
+        return sum(int(np.prod(m.shape)) * _ESZ[m.dtype] for m in self.mats)
