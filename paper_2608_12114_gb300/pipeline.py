@@ -169,30 +169,27 @@ class DeviceCheckpoint:
 
     @staticmethod
     def stream_in(h: wt.Handle, mats: Sequence[MatrixRef], mode: int = wt.WT_ADOPT_GATHER, stream: int = 0,
-                  first_bytes: int = 256 << 20, segments: Optional[int] = None, device="cuda"):
+                  first_bytes: int = 256 << 20, growth: float = 2.0, device="cuda"):
         """Allocation (step 4) interleaved with ingest (step 5): the logical tensors are cut, at
-        tensor boundaries and in order, into a small first segment (about `first_bytes`) and
-        then `segments` segments of nearly equal bytes; each segment gets its own device slab
-        right before its wt_adopt call, so the link starts after the first small allocation
-        and every later allocation runs while earlier bytes are in flight.  By default one
-        segment per 2 GB, at most 8: below that, allocating costs less than a wt_adopt call
-        (under 0.2 ms per GB), and a checkpoint is one slab and one call.  Returns
-        (DeviceCheckpoint, tensor -> ready event, host seconds spent allocating)."""
+        tensor boundaries and in order, into segments that start at about `first_bytes` and grow
+        by `growth` each time; each segment gets its own device slab right before its wt_adopt
+        call.  The link starts after the first small allocation, every later allocation (under
+        0.2 ms per GB) runs while the previous, half as large segment crosses the link (about
+        4.8 ms per GB), and the few, mostly large calls keep wt_adopt's batches large.  A
+        checkpoint under 2 GB is one slab and one call.  Returns (DeviceCheckpoint,
+        tensor -> ready event, host seconds spent allocating)."""
         import time
         import torch
         sizes = [sum(h.tensors[i].nbytes for i in m.parts) for m in mats]
         total = sum(sizes)
-        if segments is None:
-            segments = min(8, total // (2 << 30))
-        if segments == 0:
-            first_bytes = total
-        cuts, acc, limit = [], 0, min(first_bytes, total)
-        step = max(1, -(-(total - limit) // max(1, segments)))
+        seg = total if total < (2 << 30) else min(first_bytes, total)
+        cuts, acc, limit = [], 0, seg
         for k, n in enumerate(sizes):
             acc += n
             if acc >= limit and k + 1 < len(sizes):
                 cuts.append(k + 1)
-                limit = acc + step
+                seg = int(seg * growth)
+                limit = acc + seg
         bounds = [0] + cuts + [len(mats)]
         spans = [None] * len(mats)
         dc = DeviceCheckpoint(list(mats), SlabViews(spans), ptrs=[0] * len(mats))
