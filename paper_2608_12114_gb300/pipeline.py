@@ -15,7 +15,6 @@ order, so that event implies the earlier blocks).
 """
 from __future__ import annotations
 
-import re
 from dataclasses import dataclass, field
 from typing import Dict, List, Optional, Sequence
 
@@ -23,7 +22,6 @@ import numpy as np
 
 from . import synth, wt
 
-_BLOCK = re.compile(r"^(.*)#r(\d+)$")
 _ESZ = {wt.WT_F32: 4, wt.WT_BF16: 2, wt.WT_F16: 2, wt.WT_I8: 1, wt.WT_U8: 1}
 _ALIGN = 256
 
@@ -44,47 +42,46 @@ def matrices(h: wt.Handle) -> List[MatrixRef]:
     by_name: Dict[str, MatrixRef] = {}
     blocks: Dict[str, Dict[int, int]] = {}
     gemv_dt = (wt.WT_F32, wt.WT_BF16, wt.WT_F16)
-    match = _BLOCK.match
-    for i, t in enumerate(h.tensors):
-        nm = t.name
-        m = match(nm) if "#r" in nm else None
-        if m is None:
-            ref = MatrixRef(nm, t.dtype, t.shape, [i], len(t.shape) == 2 and t.dtype in gemv_dt)
+    T = h.tensors
+    tnames, tdt, tshape = T.names, T.dtypes, T.shapes
+    for i, nm in enumerate(tnames):
+        base, sep, k = nm.rpartition("#r")
+        if not sep or not k.isdigit() or not k.isascii():
+            sh = tshape[i]
+            ref = MatrixRef(nm, tdt[i], sh, [i], len(sh) == 2 and tdt[i] in gemv_dt)
             out.append(ref)
             by_name[nm] = ref
             continue
-        base = m.group(1)
         bl = blocks.get(base)
         if bl is None:
             bl = blocks[base] = {}
             if base not in by_name:
-                ref = MatrixRef(base, t.dtype, (), [], False)
+                ref = MatrixRef(base, tdt[i], (), [], False)
                 out.append(ref)
                 by_name[base] = ref
-        bl[int(m.group(2))] = i
-    tensors = h.tensors
+        bl[int(k)] = i
     for base, parts in blocks.items():
         ref = by_name[base]
         idx = [parts[k] for k in sorted(parts)]
-        t0 = tensors[idx[0]]
-        K = t0.shape[1] if len(t0.shape) == 2 else None
+        sh0, dt0 = tshape[idx[0]], tdt[idx[0]]
+        K = sh0[1] if len(sh0) == 2 else None
         rows = 0
         for i in idx:
-            t = tensors[i]
-            if K is None or len(t.shape) != 2 or t.shape[1] != K or t.dtype != t0.dtype:
+            sh = tshape[i]
+            if K is None or len(sh) != 2 or sh[1] != K or tdt[i] != dt0:
                 raise ValueError("row blocks of %s do not stack" % base)
-            rows += t.shape[0]
+            rows += sh[0]
         ref.parts = idx
         ref.shape = (rows, K)
-        ref.gemv = t0.dtype in gemv_dt
+        ref.gemv = dt0 in gemv_dt
     # int8 matrices are GEMV matrices when their fp16 row scales "<name>.scale" are present
     names = None
     for ref in out:
         if ref.dtype == wt.WT_I8 and len(ref.shape) == 2 and len(ref.parts) == 1:
             if names is None:
-                names = {t.name: i for i, t in enumerate(tensors)}
+                names = {nm: i for i, nm in enumerate(tnames)}
             si = names.get(ref.name + ".scale")
-            if si is not None and tensors[si].dtype == wt.WT_F16 and tensors[si].shape == (ref.shape[0],):
+            if si is not None and tdt[si] == wt.WT_F16 and tshape[si] == (ref.shape[0],):
                 ref.scale, ref.gemv = si, True
     return out
 
@@ -145,7 +142,8 @@ class DeviceCheckpoint:
 
         slab=True carves every buffer out of one allocation (256-byte aligned offsets)."""
         import torch
-        sizes = [sum(h.tensors[i].nbytes for i in m.parts) for m in mats]
+        tnb = h.tensors.nbytes
+        sizes = [sum(tnb[i] for i in m.parts) for m in mats]
         if slab:
             offs, pos = [], 0
             for n in sizes:
@@ -159,12 +157,11 @@ class DeviceCheckpoint:
             bufs = [torch.empty(n + canary, dtype=torch.uint8, device=device) for n in sizes]
             ptrs = [b.data_ptr() for b in bufs]
         dc = DeviceCheckpoint(list(mats), bufs, canary=canary, ptrs=ptrs)
-        tensors = h.tensors
         for m, p in zip(mats, ptrs):
             off = 0
             for i in m.parts:
                 dc.dst[i] = p + off
-                off += tensors[i].nbytes
+                off += tnb[i]
         return dc
 
     @staticmethod
@@ -180,7 +177,8 @@ class DeviceCheckpoint:
         tensor -> ready event, host seconds spent allocating)."""
         import time
         import torch
-        sizes = [sum(h.tensors[i].nbytes for i in m.parts) for m in mats]
+        tnb = h.tensors.nbytes
+        sizes = [sum(tnb[i] for i in m.parts) for m in mats]
         total = sum(sizes)
         seg = total if total < (2 << 30) else min(first_bytes, total)
         cuts, acc, limit = [], 0, seg
@@ -193,7 +191,6 @@ class DeviceCheckpoint:
         bounds = [0] + cuts + [len(mats)]
         spans = [None] * len(mats)
         dc = DeviceCheckpoint(list(mats), SlabViews(spans), ptrs=[0] * len(mats))
-        tensors = h.tensors
         events: Dict[int, int] = {}
         alloc_s = 0.0
         for a, b in zip(bounds, bounds[1:]):
@@ -212,7 +209,7 @@ class DeviceCheckpoint:
                 off = 0
                 for i in mats[k].parts:
                     dc.dst[i] = p + off
-                    off += tensors[i].nbytes
+                    off += tnb[i]
                     idx.append(i)
             idx.sort()
             if idx:

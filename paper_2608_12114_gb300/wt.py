@@ -141,6 +141,38 @@ class TensorInfo:
     host_ptr: int
 
 
+class TensorTable:
+    """The index of an open checkpoint: TensorInfo per tensor, made on first access, and the
+    columns as plain lists (`names`, `dtypes`, `shapes`, `nbytes`, `files`, `offsets`) for
+    code that walks thousands of entries."""
+
+    def __init__(self, meta: np.ndarray, names: List[str]):
+        self.names = names
+        self.dtypes = meta["dtype"].tolist()
+        nds = meta["ndim"].tolist()
+        self.shapes = [tuple(sh[:nd]) for sh, nd in zip(meta["shape"].tolist(), nds)]
+        self.nbytes = meta["nbytes"].tolist()
+        self.files = meta["file"].tolist()
+        self.offsets = meta["offset"].tolist()
+        self.host_ptrs = meta["host_ptr"].tolist()
+        self._items: List[object] = [None] * len(names)
+
+    def __len__(self) -> int:
+        return len(self.names)
+
+    def __getitem__(self, i):
+        if isinstance(i, slice):
+            return [self[k] for k in range(*i.indices(len(self)))]
+        t = self._items[i]
+        if t is None:
+            t = self._items[i] = TensorInfo(self.names[i], self.dtypes[i], self.shapes[i], self.nbytes[i],
+                                            self.files[i], self.offsets[i], self.host_ptrs[i])
+        return t
+
+    def __iter__(self):
+        return (self[i] for i in range(len(self)))
+
+
 class Handle:
     """An open checkpoint (wt_open ... wt_close)."""
 
@@ -166,12 +198,8 @@ class Handle:
         _check(L.wt_tensor_names(h, None, 0, C.byref(need)))
         buf = C.create_string_buffer(max(1, need.value))
         _check(L.wt_tensor_names(h, buf, need.value, C.byref(need)))
-        names = buf.raw[:need.value].split(b"\0")[:-1] if need.value else []
-        cols = [meta[f].tolist() for f in ("dtype", "ndim", "nbytes", "file", "offset", "host_ptr")]
-        shapes = meta["shape"].tolist()
-        self.tensors: List[TensorInfo] = [
-            TensorInfo(nm.decode(), dt, tuple(sh[:nd]), nb, fi, off, hp)
-            for nm, dt, nd, nb, fi, off, hp, sh in zip(names, *cols, shapes)]
+        names = buf.raw[:need.value].decode().split("\0")[:-1] if need.value else []
+        self.tensors = TensorTable(meta, names)
         nf = C.c_size_t()
         _check(L.wt_num_files(h, C.byref(nf)))
         self.n_files = nf.value
