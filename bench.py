@@ -65,6 +65,8 @@ def parse_args():
     p.add_argument("--arms", action="store_true", help="also time the ce/staged/stock-torch ingest arms")
     p.add_argument("--graph", action="store_true",
                    help="time the resident pass as replays of one captured CUDA graph")
+    p.add_argument("--graph-passes", type=int, default=1,
+                   help="with --graph: resident passes captured in the graph (steps rounds up to a multiple)")
     p.add_argument("--cold-reps", type=int, default=0,
                    help="also time N file -> first-use runs with the files evicted from the page cache")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -579,19 +581,25 @@ def run_wt(args, rank, world):
         h.pass_(descs, s.cuda_stream)
     s.synchronize()
     graph, graph_launches = None, 0
+    gp = max(1, args.graph_passes) if args.graph else 1
+    if gp > 1:
+        args.steps = -(-args.steps // gp) * gp
     if args.graph:
-        # one resident pass captured into a CUDA graph; each step replays it (no host work)
+        # gp resident passes captured into one CUDA graph; each replay runs gp steps with no
+        # host work between them (the replay's own launch is paid once per gp passes)
         n_cap = h.kernel_launches()
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph, stream=s):
-            h.pass_(descs, torch.cuda.current_stream().cuda_stream)
-        graph_launches = h.kernel_launches() - n_cap
+            for _ in range(gp):
+                h.pass_(descs, torch.cuda.current_stream().cuda_stream)
+        graph_launches = (h.kernel_launches() - n_cap) / gp
         with torch.cuda.stream(s):
             for _ in range(args.warmup):
                 graph.replay()
         s.synchronize()
     n0 = h.kernel_launches()
-    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    nrec = args.steps // gp
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(nrec + 1)]
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
@@ -599,7 +607,7 @@ def run_wt(args, rank, world):
         evs[0].record(s)
         if graph is not None:
             with torch.cuda.stream(s):
-                for i in range(args.steps):
+                for i in range(nrec):
                     graph.replay()
                     evs[i + 1].record(s)
         else:
@@ -610,8 +618,8 @@ def run_wt(args, rank, world):
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
-    launches = h.kernel_launches() - n0 + graph_launches * args.steps
-    per = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
+    launches = int(round(h.kernel_launches() - n0 + graph_launches * args.steps))
+    per = [evs[i].elapsed_time(evs[i + 1]) / gp for i in range(nrec)]
     total_ms = evs[0].elapsed_time(evs[-1])
     status = h.device_status()
     h.close()
@@ -648,7 +656,7 @@ def run_wt(args, rank, world):
                    "l2": ("inputs larger than L2 (no flush)" if weight_bytes > L2_BYTES else
                           "inputs smaller than L2, no flush: passes may hit L2 (a dispatch-overhead point)"),
                    "parallelism": "replicas" if world > 1 else "1 GPU",
-                   "cuda_graph": bool(args.graph)},
+                   "cuda_graph": bool(args.graph), "passes_per_graph": gp if args.graph else None},
         "resident_frac_of_hbm": {"measured": round(value / world / peak, 4), "nominal_8TBps": round(value / world / NOMINAL_HBM_GBS, 4)},
         "clocks": clocks,
         "e2e": {"value": round(aggregate_gbs(data_bytes, world, e2e_s_max), 1), "unit": "GB/s",

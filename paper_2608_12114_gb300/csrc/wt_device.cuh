@@ -82,6 +82,13 @@ __device__ __forceinline__ bool bounded_wait(uint32_t bar, uint32_t parity, vola
   return true;
 }
 
+// Programmatic dependent launch (launch attribute cudaLaunchAttributeProgrammaticStreamSerialization):
+// griddep_wait blocks until the grid this one depends on in its stream has completed and its
+// memory is visible (a no-op when the launch had no such dependency); griddep_launch lets the
+// next grid of the stream be launched, its CTAs taking SMs as this grid's CTAs leave them.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 __device__ __forceinline__ uint4 lds128(uint32_t addr) {
   uint4 v;
   asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"

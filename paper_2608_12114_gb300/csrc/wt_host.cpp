@@ -1508,6 +1508,11 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
       gl.begin = reinterpret_cast<const uint32_t *>(P->dev + L.begin);
       gl.status = h->status;
       gl.stall = wt::fault_injected("stall") ? 1 : 0;
+      // Inside a captured graph of consecutive passes, each pass may start its launch and
+      // prologue while the previous one finishes (a programmatic edge); a group gated on an
+      // event, and every pass issued from the host, keep the plain stream order (measured:
+      // programmatic launches issued one by one from the host made small passes slower).
+      gl.pdl = capturing && !wait ? 1 : 0;
       CU(wt::launch_gemv(gl, s));
       h->kernel_launches++;
     }

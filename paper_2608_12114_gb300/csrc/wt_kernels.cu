@@ -472,6 +472,13 @@ __global__ void __launch_bounds__(kGemvThreads, GemvGeo<DT>::kCtasPerSm)
     mbar_fence_init();
   }
   __syncthreads();
+  // Up to here only the plan tables (written once, by the upload before the first launch) and
+  // shared memory are touched, so under a programmatic launch this prologue may overlap the
+  // previous kernel of the stream; W, x, y and the scales are read or written only after that
+  // kernel has completed.  The next pass may then be launched at once: its CTAs take an SM
+  // only as this grid leaves it.  Without a programmatic launch both are no-ops.
+  griddep_wait();
+  griddep_launch();
 
   if (warp == kConsumerWarps) {
     // ---------------- producer: one thread issues every bulk copy of the CTA
@@ -802,16 +809,33 @@ cudaError_t gemv_prepare() {
   return gemv_attr<3>();
 }
 
+// With L.pdl the launch carries programmatic stream serialization: inside a captured graph of
+// consecutive passes, the next pass's launch and prologue overlap the tail of the one before;
+// the kernel waits for that one's completion before it touches any operand.
+template <int DT>
+static cudaError_t gemv_launch(const GemvLaunch &L, cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)L.grid);
+  cfg.blockDim = dim3(kGemvThreads);
+  cfg.dynamicSmemBytes = GemvGeo<DT>::kSmem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = L.pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, gemv_tma_kernel<DT>, L.mats, L.pieces, L.begin, L.status, L.stall);
+}
+
 cudaError_t launch_gemv(const GemvLaunch &L, cudaStream_t s) {
   if (L.grid <= 0) return cudaSuccess;
   switch (L.dtype) {
-    case 0: gemv_tma_kernel<0><<<L.grid, kGemvThreads, GemvGeo<0>::kSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
-    case 1: gemv_tma_kernel<1><<<L.grid, kGemvThreads, GemvGeo<1>::kSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
-    case 2: gemv_tma_kernel<2><<<L.grid, kGemvThreads, GemvGeo<2>::kSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
-    case 3: gemv_tma_kernel<3><<<L.grid, kGemvThreads, GemvGeo<3>::kSmem, s>>>(L.mats, L.pieces, L.begin, L.status, L.stall); break;
+    case 0: return gemv_launch<0>(L, s);
+    case 1: return gemv_launch<1>(L, s);
+    case 2: return gemv_launch<2>(L, s);
+    case 3: return gemv_launch<3>(L, s);
     default: return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 cudaError_t launch_gemv_mapped(const GemvLaunch &L, cudaStream_t s) {

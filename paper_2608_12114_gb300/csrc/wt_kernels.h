@@ -105,6 +105,8 @@ struct GemvLaunch {
   int stall = 0;  // failure test (host fault site "stall"): the producer issues no copy, so
                   // every consumer wait runs out, reports WT_ETIMEDOUT and the CTA exits
   int nt = 0;     // multi-column kernel: 8-column MMA tiles of every matrix (T <= 8 nt)
+  int pdl = 0;    // one-column kernel: launch with programmatic stream serialization (the
+                  // launch and prologue may overlap the previous kernel of the stream)
 };
 
 cudaError_t gemv_prepare();  // one-time function attributes
