@@ -65,6 +65,9 @@ def parse_args():
     p.add_argument("--arms", action="store_true", help="also time the ce/staged/stock-torch ingest arms")
     p.add_argument("--graph", action="store_true",
                    help="time the resident pass as replays of one captured CUDA graph")
+    p.add_argument("--stamps", action="store_true",
+                   help="after the timed region, per-CTA stamps of the resident pass (WT_OPEN_STAMPS): "
+                        "prologue, plan-table reads, first copy, streaming, tail")
     p.add_argument("--graph-passes", type=int, default=1,
                    help="with --graph: resident passes captured in the graph (steps rounds up to a multiple)")
     p.add_argument("--cold-reps", type=int, default=0,
@@ -368,6 +371,51 @@ def aggregate_gbs(bytes_per_rank, world, seconds):
 
 # ----------------------------------------------------------------------------- the wt arm
 
+def stamp_summary(wt, st):
+    """Medians over the CTAs with rows of each stamp, in us from the CTA's own entry, plus the
+    launch's span (first entry to last exit) and the spread of the CTAs' entries."""
+    import numpy as np
+    F = {f: i for i, f in enumerate(wt.STAMP_FIELDS)}
+    t = st.astype(np.int64)
+    busy = t[t[:, F["first_copy"]] > 0]
+    rel = lambda f: round(float(np.median(busy[:, F[f]] - busy[:, F["entry"]])) / 1e3, 3)
+    return {"ctas": int(t.shape[0]), "ctas_with_rows": int(busy.shape[0]),
+            "median_us_from_entry": {f: rel(f) for f in wt.STAMP_FIELDS[1:-1]},
+            "span_us": round(float(t[:, F["exit"]].max() - t[:, F["entry"]].min()) / 1e3, 3),
+            "entry_spread_us": round(float(t[:, F["entry"]].max() - t[:, F["entry"]].min()) / 1e3, 3),
+            "first_copy_to_last_full_us_median": round(float(np.median(busy[:, F["last_full"]] - busy[:, F["first_copy"]])) / 1e3, 3)}
+
+
+def run_stamps(torch, wt, descs, s, args, gp):
+    """The resident pass on a WT_OPEN_STAMPS handle (outside the timed region): the stamps of
+    the last of `warmup` + 20 host-issued passes and, with --graph, of the last pass of the last
+    replay of a graph of gp passes."""
+    out = {"what": "per-CTA %globaltimer stamps of the stamping instantiation of the resident kernel, "
+                   "medians over the CTAs with rows, us from each CTA's entry (prologue: mbarriers ready; "
+                   "operands: past the wait for the previous grid; first_copy: first bulk copy issued, after "
+                   "the plan-table reads; first_full / last_full: first / last stage landed; exit)"}
+    with wt.Handle([], wt.WT_OPEN_STAMPS) as hs:
+        for _ in range(args.warmup + 20):
+            hs.pass_(descs, s.cuda_stream)
+        s.synchronize()
+        out["host_issued"] = stamp_summary(wt, hs.pass_stamps())
+        if args.graph:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=s):
+                for _ in range(gp):
+                    hs.pass_(descs, torch.cuda.current_stream().cuda_stream)
+            with torch.cuda.stream(s):
+                for _ in range(args.warmup + 5):
+                    g.replay()
+            s.synchronize()
+            out["graph"] = stamp_summary(wt, hs.pass_stamps())
+            out["graph"]["passes_per_graph"] = gp
+            del g
+        if hs.device_status() != 0:
+            raise SystemExit("device status %d after stamped passes" % hs.device_status())
+    return out
+
+
 def consumer_stream(torch, args):
     """The stream of the event-gated GEMVs.  At high priority the block scheduler places a
     GEMV group's CTAs before those of the gather batch that becomes ready at the same moment."""
@@ -623,6 +671,7 @@ def run_wt(args, rank, world):
     total_ms = evs[0].elapsed_time(evs[-1])
     status = h.device_status()
     h.close()
+    stamps = run_stamps(torch, wt, descs, s, args, gp) if args.stamps and status == 0 else None
     if status != 0:
         raise SystemExit("device status %d after resident passes" % status)
 
@@ -681,6 +730,8 @@ def run_wt(args, rank, world):
         "gpu_launches": int(launches),
         "roofline": roof,
     }
+    if stamps:
+        out["stamps"] = stamps
     if arms:
         out["ingest_arms_gbs"] = arms
     if cold:

@@ -85,6 +85,11 @@ extern "C" {
  *              wt_adopt and every GEMV group of wt_pass (outside stream capture),
  *              for wt_trace: the per-tensor overlap timeline of the first use.
  *              The ready events wt_adopt returns then carry timing too.
+ * STAMPS       every one-column resident GEMV launch of wt_pass on the handle runs the
+ *              stamping instantiation of its kernel, which also writes per-CTA
+ *              %globaltimer stamps (the WT_STAMP_* record below) for wt_pass_stamps:
+ *              where a small pass spends its time (prologue, plan-table reads, first
+ *              copy, streaming, tail).  Same results; a diagnostic, not for timing runs.
  */
 #define WT_ROUTE_AUTO 0u
 #define WT_ROUTE_REGISTER 1u
@@ -95,6 +100,7 @@ extern "C" {
 #define WT_OPEN_PREFAULT (1u << 5)
 #define WT_OPEN_TIMELINE (1u << 6)  /* timing events around every ingest batch and GEMV group (wt_trace) */
 #define WT_OPEN_NOMAP (1u << 7)     /* parse only; no mapping; staged adopt reads with pread */
+#define WT_OPEN_STAMPS (1u << 8)    /* per-CTA stamps of each one-column GEMV launch (wt_pass_stamps) */
 
 /* ---- wt_adopt modes ---------------------------------------------------------
  *   GATHER   SM gather kernel: 16-byte vector loads from the device-readable
@@ -293,6 +299,28 @@ typedef struct {
  * the calling thread.  Errors: WT_EINVAL (NULL argument, handle without WT_OPEN_TIMELINE),
  * WT_ECUDA (e.g. origin without timing, or not recorded). */
 int wt_trace(wt_handle *h, void *origin, wt_trace_rec *out, size_t cap, size_t *n);
+
+/* Per-CTA stamps of the latest one-column resident GEMV launch that wt_pass issued on a
+ * handle opened with WT_OPEN_STAMPS (the persistent TMA kernel of Sec. 4.2's resident
+ * consumer; the multi-column, map-endpoint and split-K reduction kernels are not stamped).
+ * Each CTA has WT_STAMP_FIELDS words, CTA b at out[b * WT_STAMP_FIELDS]; every field but
+ * WT_STAMP_SM is the GPU's global nanosecond timer (comparable across SMs), and a field
+ * the CTA never reached (a CTA with no rows) is 0.  "Latest" is in host issue order: for a
+ * pass captured in a CUDA graph, the stamps of its latest replay.  Waits until the device
+ * is idle, copies min(cap, *n) CTAs' records to out (host memory) and sets *n to the
+ * launch's grid (0: no stamped launch yet).  Errors: WT_EINVAL (NULL argument, handle
+ * without WT_OPEN_STAMPS), WT_ECUDA. */
+#define WT_STAMP_ENTRY 0       /* CTA entry */
+#define WT_STAMP_PROLOGUE 1    /* mbarriers initialised (shared-memory set-up done) */
+#define WT_STAMP_OPERANDS 2    /* past the wait for the previous grid of the stream (a
+                                  programmatic launch in a captured graph); operands readable */
+#define WT_STAMP_FIRST_COPY 3  /* first bulk copy issued (after the plan-table reads) */
+#define WT_STAMP_FIRST_FULL 4  /* first stage landed, as the first consumer warp saw it */
+#define WT_STAMP_LAST_FULL 5   /* last stage landed, as the first consumer warp saw it */
+#define WT_STAMP_EXIT 6        /* every warp of the CTA done */
+#define WT_STAMP_SM 7          /* the SM the CTA ran on (not a time) */
+#define WT_STAMP_FIELDS 8
+int wt_pass_stamps(wt_handle *h, uint64_t *out, size_t cap, size_t *n);
 
 /* Device-side status word of the handle: 0, or the first WT_ETIMEDOUT-class
  * code a bounded wait inside a kernel recorded (reads it synchronously). */

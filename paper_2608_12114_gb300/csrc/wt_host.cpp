@@ -318,6 +318,12 @@ struct wt_handle {
   bool timeline = false;
   std::vector<TraceEv> trace;
   uint64_t n_batches = 0, n_groups = 0;
+  // WT_OPEN_STAMPS: one-column GEMV launches run the stamping kernel into stamp_dev
+  // (stamp_cap CTAs of wt::kStampFields words); stamp_ctas is the grid of the latest one
+  bool stamping = false;
+  uint64_t *stamp_dev = nullptr;
+  size_t stamp_cap = 0;
+  int stamp_ctas = 0;
   int device = -1;
   int *status = nullptr;
   std::vector<cudaEvent_t> events;
@@ -1513,6 +1519,23 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
       // event, and every pass issued from the host, keep the plain stream order (measured:
       // programmatic launches issued one by one from the host made small passes slower).
       gl.pdl = capturing && !wait ? 1 : 0;
+      if (h->stamping) {
+        if ((size_t)L.grid > h->stamp_cap) {
+          if (capturing)
+            return set_err(WT_EINVAL, "wt_pass: a stamped pass needs the same descriptors run once outside the capture");
+          const size_t cap = std::max<size_t>((size_t)L.grid, 2u * (size_t)wt::num_sms());
+          uint64_t *buf = nullptr;
+          CU(dev_alloc(reinterpret_cast<void **>(&buf), cap * wt::kStampFields * sizeof(uint64_t)));
+          if (h->stamp_dev) {
+            cudaDeviceSynchronize();  // earlier stamped launches may still write the old buffer
+            dev_free(h->stamp_dev, h->stamp_cap * wt::kStampFields * sizeof(uint64_t));
+          }
+          h->stamp_dev = buf;
+          h->stamp_cap = cap;
+        }
+        gl.stamps = h->stamp_dev;
+        h->stamp_ctas = L.grid;
+      }
       CU(wt::launch_gemv(gl, s));
       h->kernel_launches++;
     }
@@ -1589,6 +1612,10 @@ int close_impl(wt_handle *h) {
     h->events.clear();
     dev_free(h->status, 256);
     h->status = nullptr;
+    if (h->stamp_dev) {
+      dev_free(h->stamp_dev, h->stamp_cap * wt::kStampFields * sizeof(uint64_t));
+      h->stamp_dev = nullptr;
+    }
     for (File &f : h->files) unmap_file(f);
     if (cur >= 0 && cur != h->device) cudaSetDevice(cur);
   } else {
@@ -1634,7 +1661,7 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
   *out = nullptr;
   if (n_paths < 0 || (n_paths > 0 && !paths)) return set_err(WT_EINVAL, "wt_open: bad path list");
   const unsigned route_req = flags & WT_ROUTE_MASK;
-  if (flags & ~(WT_ROUTE_MASK | WT_OPEN_HOST_ONLY | WT_OPEN_PREFAULT | WT_OPEN_TIMELINE | WT_OPEN_NOMAP))
+  if (flags & ~(WT_ROUTE_MASK | WT_OPEN_HOST_ONLY | WT_OPEN_PREFAULT | WT_OPEN_TIMELINE | WT_OPEN_NOMAP | WT_OPEN_STAMPS))
     return set_err(WT_EINVAL, "wt_open: unknown flag bits 0x%x", flags);
   const bool nomap = (flags & WT_OPEN_NOMAP) != 0;
   if (nomap && (route_req == WT_ROUTE_REGISTER || route_req == WT_ROUTE_DIRECT || (flags & WT_OPEN_PREFAULT)))
@@ -1645,6 +1672,7 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
     g_live_handles++;
     h->host_only = (flags & WT_OPEN_HOST_ONLY) != 0;
     h->timeline = (flags & WT_OPEN_TIMELINE) != 0 && !h->host_only;
+    h->stamping = (flags & WT_OPEN_STAMPS) != 0 && !h->host_only;
     h->files.resize(n_paths);
     for (int i = 0; i < n_paths; ++i) {
       if (!paths[i]) {
@@ -2057,6 +2085,30 @@ int wt_trace(wt_handle *h, void *origin, wt_trace_rec *out, size_t cap, size_t *
     if (t.own_end) ev_destroy(t.end);
   }
   h->trace.clear();
+  return WT_OK;
+}
+
+static_assert(WT_STAMP_ENTRY == wt::kStEntry && WT_STAMP_PROLOGUE == wt::kStPrologue &&
+                  WT_STAMP_OPERANDS == wt::kStOperands && WT_STAMP_FIRST_COPY == wt::kStFirstCopy &&
+                  WT_STAMP_FIRST_FULL == wt::kStFirstFull && WT_STAMP_LAST_FULL == wt::kStLastFull &&
+                  WT_STAMP_EXIT == wt::kStExit && WT_STAMP_SM == wt::kStSm && WT_STAMP_FIELDS == wt::kStampFields,
+              "the stamp record of include/wt.h is the kernel's");
+
+int wt_pass_stamps(wt_handle *h, uint64_t *out, size_t cap, size_t *n) {
+  if (!h || !n || (cap && !out)) return set_err(WT_EINVAL, "wt_pass_stamps: NULL argument");
+  if (!h->stamping) return set_err(WT_EINVAL, "wt_pass_stamps: the handle was not opened with WT_OPEN_STAMPS");
+  std::lock_guard<std::mutex> g(h->mu);
+  *n = (size_t)h->stamp_ctas;
+  if (!h->stamp_ctas) return WT_OK;
+  // the handle's device, whichever device is current: every stamped launch has finished first
+  int cur = -1;
+  CU(cudaGetDevice(&cur));
+  if (cur != h->device) CU(cudaSetDevice(h->device));
+  cudaError_t e = cudaDeviceSynchronize();
+  const size_t k = std::min(cap, (size_t)h->stamp_ctas);
+  if (e == cudaSuccess && k) e = cudaMemcpy(out, h->stamp_dev, k * wt::kStampFields * sizeof(uint64_t), cudaMemcpyDeviceToHost);
+  if (cur != h->device) cudaSetDevice(cur);
+  if (e != cudaSuccess) return cuda_err(e, "wt_pass_stamps");
   return WT_OK;
 }
 

@@ -445,12 +445,28 @@ __device__ __forceinline__ bool block_rows_dispatch(uint32_t nj, uint32_t nr, ui
 #undef WT_BR
 }
 
-template <int DT>
+// Consumer warp 0 records when it saw its first and its latest stage land.
+__device__ __forceinline__ void stamp_full(uint64_t *st, uint32_t it, int warp, int lane) {
+  if (warp == 0 && lane == 0) {
+    const uint64_t t = globaltimer_ns();
+    if (it == 0) st[kStFirstFull] = t;
+    st[kStLastFull] = t;
+  }
+}
+
+// ST: the stamping instantiation, which also writes the per-CTA times of StampField to
+// stamps[blockIdx.x * kStampFields ...]; otherwise identical.
+template <int DT, bool ST>
 __global__ void __launch_bounds__(kGemvThreads, GemvGeo<DT>::kCtasPerSm)
     gemv_tma_kernel(const MatDesc *__restrict__ mats, const Piece *__restrict__ pieces,
-                    const uint32_t *__restrict__ begin, int *status, int stall) {
+                    const uint32_t *__restrict__ begin, int *status, int stall, uint64_t *stamps) {
   constexpr int NP = Pairs<DT>::N;
   constexpr int kStages = GemvGeo<DT>::kStages;
+  uint64_t *const st = ST ? stamps + (uint64_t)blockIdx.x * kStampFields : nullptr;
+  if (ST && threadIdx.x == 0) {
+    st[kStEntry] = globaltimer_ns();
+    st[kStFirstCopy] = st[kStFirstFull] = st[kStLastFull] = 0;
+  }
   extern __shared__ __align__(128) uint8_t smem[];
   const uint32_t stage0 = smem_u32(smem);
   const uint32_t full0 = smem_u32(smem + GemvGeo<DT>::kBarOff);
@@ -472,6 +488,7 @@ __global__ void __launch_bounds__(kGemvThreads, GemvGeo<DT>::kCtasPerSm)
     mbar_fence_init();
   }
   __syncthreads();
+  if (ST && threadIdx.x == 0) st[kStPrologue] = globaltimer_ns();
   // Up to here only the plan tables (written once, by the upload before the first launch) and
   // shared memory are touched, so under a programmatic launch this prologue may overlap the
   // previous kernel of the stream; W, x, y and the scales are read or written only after that
@@ -479,6 +496,7 @@ __global__ void __launch_bounds__(kGemvThreads, GemvGeo<DT>::kCtasPerSm)
   // only as this grid leaves it.  Without a programmatic launch both are no-ops.
   griddep_wait();
   griddep_launch();
+  if (ST && threadIdx.x == 0) st[kStOperands] = globaltimer_ns();
 
   if (warp == kConsumerWarps) {
     // ---------------- producer: one thread issues every bulk copy of the CTA
@@ -500,6 +518,7 @@ __global__ void __launch_bounds__(kGemvThreads, GemvGeo<DT>::kCtasPerSm)
           }
           const uint32_t dst = stage0 + s * kStageBytes;
           const uint32_t bar = full0 + 8 * s;
+          if (ST && it == 0) st[kStFirstCopy] = globaltimer_ns();
           mbar_expect_tx(bar, nr * vb);
           if (md.rs == md.V) {
             bulk_g2s(dst, md.W + (uint64_t)r * rowb, nr * vb, bar, pol);  // contiguous rows: one copy
@@ -546,6 +565,7 @@ __global__ void __launch_bounds__(kGemvThreads, GemvGeo<DT>::kCtasPerSm)
           const uint32_t nr = min(md.rt, pc.r1 - r);
           const uint32_t s = it % kStages;
           bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
+          if (ST) stamp_full(st, it, warp, lane);
           const uint32_t tile = stage0 + s * kStageBytes;
           float *y = md.y + r;
           const uint8_t *sr = md.s ? md.s + 2ull * r : nullptr;  // f16 row scales (int8 weights)
@@ -586,6 +606,7 @@ __global__ void __launch_bounds__(kGemvThreads, GemvGeo<DT>::kCtasPerSm)
           const uint32_t nr = min(md.rt, pc.r1 - r);
           const uint32_t s = it % kStages;
           bounded_wait(full0 + 8 * s, (it / kStages) & 1, abort_flag, status);
+          if (ST) stamp_full(st, it, warp, lane);
           const uint32_t tile = stage0 + s * kStageBytes;
           float *rb = red + par * (kConsumerWarps * kRedRows) + gn * kConsumerWarps;
           if (!block_rows_dispatch<DT>(nj, nr, tile, V, ct, warp, lane, xp, rb) && ct == 0)
@@ -607,6 +628,10 @@ __global__ void __launch_bounds__(kGemvThreads, GemvGeo<DT>::kCtasPerSm)
     }
   }
   __syncthreads();
+  if (ST && threadIdx.x == 0) {
+    st[kStExit] = globaltimer_ns();
+    st[kStSm] = sm_id();
+  }
 }
 
 // Map endpoint: one lane group per row (G = pow2ceil(V) lanes for rows shorter than 32
@@ -799,7 +824,10 @@ int gemv_ctas_per_sm(int dtype) { return dtype == 3 ? GemvGeo<3>::kCtasPerSm : G
 
 template <int DT>
 static cudaError_t gemv_attr() {
-  return cudaFuncSetAttribute(gemv_tma_kernel<DT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)GemvGeo<DT>::kSmem);
+  const cudaError_t e =
+      cudaFuncSetAttribute(gemv_tma_kernel<DT, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)GemvGeo<DT>::kSmem);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(gemv_tma_kernel<DT, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)GemvGeo<DT>::kSmem);
 }
 
 cudaError_t gemv_prepare() {
@@ -824,7 +852,10 @@ static cudaError_t gemv_launch(const GemvLaunch &L, cudaStream_t s) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = L.pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, gemv_tma_kernel<DT>, L.mats, L.pieces, L.begin, L.status, L.stall);
+  if (L.stamps)
+    return cudaLaunchKernelEx(&cfg, gemv_tma_kernel<DT, true>, L.mats, L.pieces, L.begin, L.status, L.stall, L.stamps);
+  return cudaLaunchKernelEx(&cfg, gemv_tma_kernel<DT, false>, L.mats, L.pieces, L.begin, L.status, L.stall,
+                            (uint64_t *)nullptr);
 }
 
 cudaError_t launch_gemv(const GemvLaunch &L, cudaStream_t s) {

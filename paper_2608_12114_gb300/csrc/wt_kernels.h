@@ -107,6 +107,22 @@ struct GemvLaunch {
   int nt = 0;     // multi-column kernel: 8-column MMA tiles of every matrix (T <= 8 nt)
   int pdl = 0;    // one-column kernel: launch with programmatic stream serialization (the
                   // launch and prologue may overlap the previous kernel of the stream)
+  uint64_t *stamps = nullptr;  // one-column kernel: non-null runs the stamping instantiation,
+                               // kStampFields words per CTA (grid x kStampFields, device)
+};
+
+// Per-CTA stamps of the one-column kernel (%globaltimer nanoseconds, but kStSm): the record
+// layout of wt_pass_stamps.  A time the CTA never reached (no rows: no copy, no stage) is 0.
+enum StampField : int {
+  kStEntry = 0,      // CTA entry
+  kStPrologue = 1,   // barriers initialised (shared-memory set-up done)
+  kStOperands = 2,   // past the wait for the previous grid: operands may be read
+  kStFirstCopy = 3,  // first bulk copy issued (after the plan-table reads)
+  kStFirstFull = 4,  // first stage landed, as consumer warp 0 saw it
+  kStLastFull = 5,   // last stage landed, as consumer warp 0 saw it
+  kStExit = 6,       // every warp done
+  kStSm = 7,         // %smid of the CTA (not a time)
+  kStampFields = 8
 };
 
 cudaError_t gemv_prepare();  // one-time function attributes

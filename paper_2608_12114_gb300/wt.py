@@ -22,6 +22,9 @@ WT_OK, WT_EINVAL, WT_EIO, WT_EFORMAT, WT_ENOMEM, WT_ECUDA, WT_ENOTSUP, WT_ETIMED
 WT_F32, WT_BF16, WT_F16, WT_I8, WT_U8 = 0, 1, 2, 3, 4
 WT_ROUTE_AUTO, WT_ROUTE_REGISTER, WT_ROUTE_DIRECT, WT_ROUTE_NONE = 0, 1, 2, 3
 WT_OPEN_HOST_ONLY, WT_OPEN_PREFAULT, WT_OPEN_TIMELINE, WT_OPEN_NOMAP = 1 << 4, 1 << 5, 1 << 6, 1 << 7
+WT_OPEN_STAMPS = 1 << 8
+# the per-CTA record of wt_pass_stamps, in field order
+STAMP_FIELDS = ("entry", "prologue", "operands", "first_copy", "first_full", "last_full", "exit", "sm")
 WT_TRACE_INGEST, WT_TRACE_GEMV = 0, 1
 WT_ADOPT_GATHER, WT_ADOPT_CE, WT_ADOPT_STAGED = 0, 1, 2
 ROUTE_NAMES = {WT_ROUTE_REGISTER: "register", WT_ROUTE_DIRECT: "direct", WT_ROUTE_NONE: "none"}
@@ -31,7 +34,7 @@ MODE_NAMES = {WT_ADOPT_GATHER: "gather", WT_ADOPT_CE: "ce", WT_ADOPT_STAGED: "st
 SYMBOLS = ("wt_last_error", "wt_abi_version", "wt_open", "wt_num_tensors", "wt_num_files",
            "wt_tensor_info", "wt_tensor_table", "wt_tensor_names", "wt_find", "wt_file_route", "wt_file_registration", "wt_adopt", "wt_pass", "wt_checksum",
            "wt_checksum_plain", "wt_checksum_noalloc", "wt_device_status", "wt_residency",
-           "wt_kernel_launches", "wt_trace", "wt_live", "wt_close",
+           "wt_kernel_launches", "wt_trace", "wt_pass_stamps", "wt_live", "wt_close",
            # include/wt_dlpack.h
            "wt_dlpack_file", "wt_dlpack_tensor", "wt_dlpack_release", "wt_dlpack_live")
 WT_DLPACK_DEVICE, WT_DLPACK_HOST = 0, 1
@@ -110,6 +113,7 @@ def lib(path: str = LIB_PATH):
     L.wt_kernel_launches.argtypes = [vp, u64p]
     L.wt_residency.argtypes = [vp, u64p, u64p]
     L.wt_trace.argtypes = [vp, vp, C.POINTER(TraceRec), sz, C.POINTER(sz)]
+    L.wt_pass_stamps.argtypes = [vp, vp, sz, C.POINTER(sz)]
     L.wt_live.argtypes = [C.POINTER(LiveCounts)]
     L.wt_close.argtypes = [vp]
     L.wt_dlpack_file.argtypes = [C.c_char_p, C.c_int32, C.c_uint64, C.c_uint64, C.c_uint, C.POINTER(vp)]
@@ -284,6 +288,18 @@ class Handle:
         return [dict(kind=kinds.get(buf[i].kind, "?"), index=buf[i].index, bytes=buf[i].bytes,
                      event=buf[i].event or 0, begin_ms=buf[i].begin_ms, end_ms=buf[i].end_ms)
                 for i in range(min(n.value, cap))]
+
+    def pass_stamps(self):
+        """wt_pass_stamps (WT_OPEN_STAMPS handles): the per-CTA stamps of the latest one-column
+        GEMV launch, a uint64 array [grid, len(STAMP_FIELDS)] (nanoseconds but the "sm" column);
+        empty before the first stamped launch.  Waits for the device."""
+        import numpy as np
+        n = C.c_size_t()
+        _check(lib().wt_pass_stamps(self.ptr, None, 0, C.byref(n)))
+        out = np.zeros((n.value, len(STAMP_FIELDS)), np.uint64)
+        if n.value:
+            _check(lib().wt_pass_stamps(self.ptr, C.c_void_p(out.ctypes.data), n.value, C.byref(n)))
+        return out
 
     def close(self):
         if self._h is not None:

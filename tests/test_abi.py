@@ -164,6 +164,36 @@ def test_registration_and_trace_queries_on_host_only_handle(L, tmp_path):
     wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY | wt.WT_OPEN_TIMELINE).close()
 
 
+def header_defines():
+    """Every integer #define of include/wt.h: name -> value."""
+    src = open(os.path.join(ROOT, "include", "wt.h")).read()
+    return {m.group(1): int(m.group(2)) << int(m.group(3) or 0)
+            for m in re.finditer(r"#define\s+(WT_[A-Z0-9_]+)\s+\(?([0-9]+)u?(?:\s*<<\s*([0-9]+))?\)?", src)}
+
+
+def test_binding_constants_match_the_header():
+    d = header_defines()
+    for name in ("WT_OPEN_HOST_ONLY", "WT_OPEN_PREFAULT", "WT_OPEN_TIMELINE", "WT_OPEN_NOMAP", "WT_OPEN_STAMPS",
+                 "WT_TRACE_INGEST", "WT_TRACE_GEMV", "WT_ADOPT_GATHER", "WT_ADOPT_CE", "WT_ADOPT_STAGED"):
+        assert d[name] == getattr(wt, name), name
+    # the stamp record: field order and width
+    assert d["WT_STAMP_FIELDS"] == len(wt.STAMP_FIELDS)
+    for i, f in enumerate(wt.STAMP_FIELDS):
+        assert d["WT_STAMP_" + f.upper()] == i, f
+
+
+def test_stamps_query_on_host_only_handle(L, tmp_path):
+    ck = synth.build("tiny", str(tmp_path))
+    # STAMPS is a known flag; a host-only handle launches nothing, so it records no stamps
+    with wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY | wt.WT_OPEN_STAMPS) as h:
+        with pytest.raises(wt.WtError) as ei:
+            h.pass_stamps()
+        assert ei.value.code == wt.WT_EINVAL
+    with pytest.raises(wt.WtError) as ei:
+        wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY | (1 << 9))  # unknown flag bit
+    assert ei.value.code == wt.WT_EINVAL
+
+
 def test_nomap_open_parses_without_mapping(L, tmp_path):
     ck = synth.build("many", str(tmp_path / "nm"), n_matrices=5)
     with wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY) as hm:
