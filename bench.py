@@ -57,9 +57,11 @@ def parse_args():
     p.add_argument("--workload", default="large")
     p.add_argument("--layers", type=int, default=None, help="override decoder layer count (small profiling cases)")
     p.add_argument("--mode", default="gather", choices=["gather", "ce", "staged"])
-    p.add_argument("--open", default="map", choices=["map", "nomap", "prefault", "register"],
+    p.add_argument("--open", default="map", choices=["map", "nomap", "prefault", "register", "maplarge"],
                    help="nomap: wt_open maps nothing (WT_OPEN_NOMAP) and --mode staged preads into the pinned ring; "
-                        "prefault: wt_open populates every mapping (WT_OPEN_PREFAULT)")
+                        "prefault: wt_open populates every mapping (WT_OPEN_PREFAULT); maplarge: only files of at "
+                        "least WT_MAP_MIN_BYTES are mapped, the rest adopted through the pinned ring "
+                        "(WT_OPEN_MAP_LARGE)")
     p.add_argument("--e2e-reps", type=int, default=5)
     p.add_argument("--skip-e2e", action="store_true", help="resident passes only (profiling runs)")
     p.add_argument("--arms", action="store_true", help="also time the ce/staged/stock-torch ingest arms")
@@ -416,6 +418,11 @@ def run_stamps(torch, wt, descs, s, args, gp):
     return out
 
 
+def open_flags(wt, name):
+    return {"map": 0, "nomap": wt.WT_OPEN_NOMAP, "prefault": wt.WT_OPEN_PREFAULT,
+            "register": wt.WT_ROUTE_REGISTER, "maplarge": wt.WT_OPEN_MAP_LARGE}[name]
+
+
 def consumer_stream(torch, args):
     """The stream of the event-gated GEMVs.  At high priority the block scheduler places a
     GEMV group's CTAs before those of the gather batch that becomes ready at the same moment."""
@@ -533,8 +540,7 @@ def run_wt(args, rank, world):
         dist.barrier()
     build.build()  # no-op when fresh; loads the same in-tree library on every rank
     mode = {"gather": wt.WT_ADOPT_GATHER, "ce": wt.WT_ADOPT_CE, "staged": wt.WT_ADOPT_STAGED}[args.mode]
-    oflags = {"map": 0, "nomap": wt.WT_OPEN_NOMAP, "prefault": wt.WT_OPEN_PREFAULT,
-              "register": wt.WT_ROUTE_REGISTER}[args.open]
+    oflags = open_flags(wt, args.open)
 
     probe = h2d_probe(torch)
     h2d = max(probe.values())
@@ -701,7 +707,9 @@ def run_wt(args, rank, world):
                    "files": len(ck.paths), "matrices": len(dev.gemv_mats()), "ingest_mode": args.mode,
                    "consumer_stream_priority": args.consumer_priority,
                    "open": {"map": "mapped", "nomap": "WT_OPEN_NOMAP (pread)", "prefault": "mapped, WT_OPEN_PREFAULT",
-                            "register": "mapped, WT_ROUTE_REGISTER"}[args.open],
+                            "register": "mapped, WT_ROUTE_REGISTER",
+                            "maplarge": "WT_OPEN_MAP_LARGE: files of >= %s bytes mapped, smaller ones read with pread"
+                                        % os.environ.get("WT_MAP_MIN_BYTES", wt.WT_MAP_MIN_BYTES)}[args.open],
                    "l2": ("inputs larger than L2 (no flush)" if weight_bytes > L2_BYTES else
                           "inputs smaller than L2, no flush: passes may hit L2 (a dispatch-overhead point)"),
                    "parallelism": "replicas" if world > 1 else "1 GPU",
@@ -930,8 +938,7 @@ def run_timeline(args):
     build.build()
     torch.cuda.set_device(0)
     mode = {"gather": wt.WT_ADOPT_GATHER, "ce": wt.WT_ADOPT_CE, "staged": wt.WT_ADOPT_STAGED}[args.mode]
-    oflags = {"map": 0, "nomap": wt.WT_OPEN_NOMAP, "prefault": wt.WT_OPEN_PREFAULT,
-              "register": wt.WT_ROUTE_REGISTER}[args.open]
+    oflags = open_flags(wt, args.open)
     h0 = wt.Handle(ck.paths, oflags)
     mats = pipeline.matrices(h0)
     slab = make_slab(torch, pipeline, h0, mats)

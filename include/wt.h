@@ -81,6 +81,18 @@ extern "C" {
  *              For checkpoints of many small files, where mapping every file costs
  *              more host time than their bytes take on the link (Sec. 5.3: the
  *              2506-file spine's map cost).  Not with REGISTER, DIRECT or PREFAULT.
+ * MAP_LARGE    map only the files of at least WT_MAP_MIN_BYTES (the environment variable
+ *              WT_MAP_MIN_BYTES, in bytes, overrides it); parse the smaller ones as NOMAP
+ *              does (no mapping, route NONE, host_ptr NULL).  wt_adopt in GATHER or CE
+ *              mode then moves the tensors of those small files as STAGED does (pread on
+ *              host threads into the pinned ring, gather from the slot).  It does so on an
+ *              internal stream, ordered after `stream`'s earlier work and concurrent with
+ *              the mapped files' transfer, and `stream` waits for it before wt_adopt
+ *              returns.  Each mapping costs an mmap and a page-table population, both
+ *              serialised on the process's address-space lock, while a pread costs host
+ *              copy bandwidth only.  So a checkpoint of many small files (Sec. 5.3)
+ *              splits its host cost over both.  Not with NOMAP; PREFAULT covers the mapped
+ *              files only.
  * TIMELINE     record a timing event before and after every ingest batch of
  *              wt_adopt and every GEMV group of wt_pass (outside stream capture),
  *              for wt_trace: the per-tensor overlap timeline of the first use.
@@ -101,6 +113,8 @@ extern "C" {
 #define WT_OPEN_TIMELINE (1u << 6)  /* timing events around every ingest batch and GEMV group (wt_trace) */
 #define WT_OPEN_NOMAP (1u << 7)     /* parse only; no mapping; staged adopt reads with pread */
 #define WT_OPEN_STAMPS (1u << 8)    /* per-CTA stamps of each one-column GEMV launch (wt_pass_stamps) */
+#define WT_OPEN_MAP_LARGE (1u << 9) /* map files of >= WT_MAP_MIN_BYTES only; adopt the rest via pread */
+#define WT_MAP_MIN_BYTES (1u << 18) /* WT_OPEN_MAP_LARGE's default threshold (file size, bytes) */
 
 /* ---- wt_adopt modes ---------------------------------------------------------
  *   GATHER   SM gather kernel: 16-byte vector loads from the device-readable
@@ -217,10 +231,11 @@ int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsign
  * endpoint: TMA-fed kernel streaming HBM) or lie inside one of this handle's file mappings
  * (the map endpoint of Sec. 8.1, contract C1: the kernel reads the mapped rows in place over
  * the host link, no copy; the rows are populated once when the plan is built and must stay
- * resident, Algorithm 2's precondition).  y must not lie inside a mapping.  Consecutive descriptors that
- * carry the same wait_event form one group: the stream waits on that event
- * (cudaStreamWaitEvent, never a host wait) and one persistent launch streams
- * every matrix of the group, rows split evenly across the SMs.  Repeated
+ * resident, Algorithm 2's precondition).  y must not lie inside a mapping.  Descriptors that
+ * carry the same wait_event form one group, wherever they stand in the list (those with
+ * none form one group too); groups are enqueued in order of their first descriptor.  For
+ * each group the stream waits on its event (cudaStreamWaitEvent, never a host wait) and one
+ * persistent launch streams every matrix of the group, rows split evenly across the SMs.  Repeated
  * calls with identical descriptors reuse a cached launch plan.  The result of
  * a row does not depend on how rows were grouped or split (deterministic, no
  * floating-point atomics).

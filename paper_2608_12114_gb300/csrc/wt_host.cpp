@@ -214,8 +214,9 @@ struct Tensor {
 
 struct File {
   std::string path;
-  uint8_t *base = nullptr;  // mapping (nullptr: opened with WT_OPEN_NOMAP)
+  uint8_t *base = nullptr;  // mapping (nullptr: opened with WT_OPEN_NOMAP, or small under MAP_LARGE)
   size_t size = 0;
+  bool small = false;       // WT_OPEN_MAP_LARGE left it unmapped: adopted through the pinned ring
   // identity at wt_open: a WT_OPEN_NOMAP file is opened again by a staged adopt, which checks
   // that the path still names the file whose index was validated
   uint64_t st_dev = 0, st_ino = 0;
@@ -290,6 +291,7 @@ struct Ring {
   static constexpr size_t kSlotBytes = 64ull << 20;
   std::mutex mu;
   bool ready = false;
+  cudaStream_t stream = nullptr;  // the staged half of a mixed adopt (WT_OPEN_MAP_LARGE)
   uint8_t *slot[kSlots] = {nullptr, nullptr, nullptr, nullptr};
   cudaEvent_t done[kSlots] = {nullptr, nullptr, nullptr, nullptr};
   bool used[kSlots] = {false, false, false, false};
@@ -317,7 +319,8 @@ struct wt_handle {
   };
   bool timeline = false;
   std::vector<TraceEv> trace;
-  uint64_t n_batches = 0, n_groups = 0;
+  std::atomic<uint64_t> n_batches{0};
+  uint64_t n_groups = 0;
   // WT_OPEN_STAMPS: one-column GEMV launches run the stamping kernel into stamp_dev
   // (stamp_cap CTAs of wt::kStampFields words); stamp_ctas is the grid of the latest one
   bool stamping = false;
@@ -328,8 +331,10 @@ struct wt_handle {
   int *status = nullptr;
   std::vector<cudaEvent_t> events;
   std::list<Plan *> plans;
-  uint64_t kernel_launches = 0;
+  std::atomic<uint64_t> kernel_launches{0};
   std::mutex mu;
+  // events and trace records: a mixed adopt (WT_OPEN_MAP_LARGE) adds them from two threads
+  std::mutex ev_mu;
 
   const Tensor &tensor(size_t i) const {
     return files[order[i].first].tensors[order[i].second];
@@ -425,8 +430,9 @@ void unmap_file(File &f) {
   }
 }
 
-// open, parse and map one file (not with `nomap`); closes the fd on every path.
-int open_one(File &f, bool nomap) {
+// open, parse and map one file (not with `nomap`, nor when it is smaller than `map_min`
+// bytes); closes the fd on every path.
+int open_one(File &f, bool nomap, uint64_t map_min) {
   if (wt::fault_injected("open")) return set_err(WT_EIO, "%s: open: injected fault", f.path.c_str());
   const int fd = open(f.path.c_str(), O_RDONLY | O_CLOEXEC);
   if (fd < 0) return set_err(WT_EIO, "%s: open: %s", f.path.c_str(), strerror(errno));
@@ -440,8 +446,10 @@ int open_one(File &f, bool nomap) {
   f.st_dev = (uint64_t)st.st_dev;
   f.st_ino = (uint64_t)st.st_ino;
   f.mtime_ns = (int64_t)st.st_mtim.tv_sec * 1000000000ll + st.st_mtim.tv_nsec;
-  if (rc == WT_OK && nomap) f.size = (size_t)st.st_size;
-  if (rc == WT_OK && !nomap) {
+  const bool skip = nomap || (uint64_t)st.st_size < map_min;
+  f.small = !nomap && skip;
+  if (rc == WT_OK && skip) f.size = (size_t)st.st_size;
+  if (rc == WT_OK && !skip) {
     f.size = (size_t)st.st_size;
     const bool injected = wt::fault_injected("mmap");
     void *p = injected ? MAP_FAILED : mmap(nullptr, f.size, PROT_READ, MAP_SHARED, fd, 0);
@@ -494,6 +502,7 @@ bool inside_mapping(const wt_handle *h, const void *p, uint64_t n) {
 
 int new_event(wt_handle *h, cudaEvent_t *ev) {
   CU(ev_create(ev, h->timeline ? cudaEventDefault : cudaEventDisableTiming));
+  std::lock_guard<std::mutex> g(h->ev_mu);
   h->events.push_back(*ev);
   return WT_OK;
 }
@@ -508,6 +517,11 @@ int trace_mark(cudaStream_t s, cudaEvent_t *ev) {
     return cuda_err(e, "cudaEventRecord (timeline)");
   }
   return WT_OK;
+}
+
+void trace_push(wt_handle *h, const wt_handle::TraceEv &t) {
+  std::lock_guard<std::mutex> g(h->ev_mu);
+  h->trace.push_back(t);
 }
 
 // ------------------------------------------------------------------ adopt
@@ -634,12 +648,12 @@ int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cuda
     }
     CU(cudaEventRecord(ev, s));
     for (size_t k = i; k < j; ++k) ready[ps[k].tensor] = ev;
+    const uint64_t bi = h->n_batches++;
     if (tb) {
       uint64_t bytes = 0;
       for (size_t k = i; k < j; ++k) bytes += ps[k].n;
-      h->trace.push_back({WT_TRACE_INGEST, h->n_batches, bytes, tb, ev, false, ev});
+      trace_push(h, {WT_TRACE_INGEST, bi, bytes, tb, ev, false, ev});
     }
-    h->n_batches++;
   }
   return WT_OK;
 }
@@ -650,6 +664,7 @@ int ring_setup(Ring &R) {
     if (!R.slot[k]) CU(pinned_alloc(reinterpret_cast<void **>(&R.slot[k]), Ring::kSlotBytes));
     if (!R.done[k]) CU(ev_create(&R.done[k], cudaEventDisableTiming));
   }
+  if (!R.stream) CU(cudaStreamCreateWithFlags(&R.stream, cudaStreamNonBlocking));
   R.ready = true;
   return WT_OK;
 }
@@ -677,15 +692,27 @@ int reopen_checked(const File &f) {
   return fd;
 }
 
+// The staged half of a mixed adopt runs on the ring's own stream: it starts after `after`
+// (recorded on the caller's stream) and records `last` once its final copy is enqueued.
+struct StagedJoin {
+  cudaEvent_t after = nullptr;
+  cudaEvent_t last = nullptr;
+};
+
 // Staged: page cache -> pinned slot (host threads: memcpy from the mapping, or pread for a
 // WT_OPEN_NOMAP file, which then needs no mapping at all) -> HBM (the gather kernel reading
 // the pinned slot over the host link: one launch per up to kMaxGather pieces, so a slot of many
 // small tensors costs one or two launches instead of one copy call per tensor).
-int adopt_staged(wt_handle *h, const std::vector<Range> &rs, cudaStream_t s, void **ready) {
+int adopt_staged(wt_handle *h, const std::vector<Range> &rs, cudaStream_t s, void **ready,
+                 StagedJoin *join = nullptr) {
   Ring &R = g_ring[h->device];
   std::lock_guard<std::mutex> ring_lock(R.mu);
   int rc = ring_setup(R);
   if (rc) return rc;
+  if (join) {
+    s = R.stream;
+    CU(cudaStreamWaitEvent(s, join->after, 0));
+  }
   // descriptors of the unmapped files this call reads, opened in parallel and closed on return
   std::vector<int> fds(h->files.size(), -1);
   std::vector<uint32_t> need;
@@ -823,10 +850,48 @@ int adopt_staged(wt_handle *h, const std::vector<Range> &rs, cudaStream_t s, voi
       }
       uint64_t bytes = 0;
       for (const PieceCopy &pc : pcs) bytes += pc.n;
-      h->trace.push_back({WT_TRACE_INGEST, h->n_batches, bytes, tb, te, true, ev});
+      trace_push(h, {WT_TRACE_INGEST, h->n_batches++, bytes, tb, te, true, ev});
+    } else {
+      h->n_batches++;
     }
-    h->n_batches++;
   }
+  if (join) {
+    rc = new_event(h, &join->last);
+    if (rc) return rc;
+    CU(cudaEventRecord(join->last, s));
+  }
+  return WT_OK;
+}
+
+// A GATHER or CE adopt over a WT_OPEN_MAP_LARGE handle whose call holds both mapped files
+// (`dv`, through the device route) and small unmapped ones (`st`, through the pinned ring):
+// the staged half runs on a helper thread and the ring's stream, ordered after the caller's
+// earlier work on `s`, while this thread enqueues the mapped half on `s`; `s` then waits
+// for the staged half, so the call keeps its stream semantics.
+int adopt_mixed(wt_handle *h, const std::vector<Range> &dv, const std::vector<Range> &st, unsigned mode,
+                cudaStream_t s, void **ready, uint64_t total_dev) {
+  StagedJoin join;
+  int rc = new_event(h, &join.after);
+  if (rc) return rc;
+  CU(cudaEventRecord(join.after, s));
+  int rc_st = WT_OK;
+  std::string err_st;
+  struct Joiner {
+    std::thread t;
+    ~Joiner() {
+      if (t.joinable()) t.join();
+    }
+  } helper;
+  helper.t = std::thread([&] {
+    const cudaError_t e = cudaSetDevice(h->device);
+    rc_st = e == cudaSuccess ? adopt_staged(h, st, s, ready, &join) : cuda_err(e, "cudaSetDevice");
+    if (rc_st) err_st = t_err;
+  });
+  rc = adopt_device(h, dv, mode, s, ready, total_dev);
+  helper.t.join();
+  if (rc) return rc;
+  if (rc_st) return set_err(rc_st, "%s", err_st.c_str());
+  CU(cudaStreamWaitEvent(s, join.last, 0));
   return WT_OK;
 }
 
@@ -1215,12 +1280,25 @@ const File *mapping_of(const wt_handle *h, const void *p, uint64_t n) {
 }
 
 int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
-  size_t i = 0;
-  while (i < n) {
-    size_t j = i;
-    while (j < n && d[j].wait_event == d[i].wait_event) ++j;
+  // One group per distinct wait_event (no event is a class of its own), in order of first
+  // appearance: each GEMV depends on its own event only, so descriptors of batches that
+  // interleave (two ingest streams, say) still make one wait and one launch per batch.
+  std::vector<std::vector<size_t>> members;
+  {
+    std::vector<std::pair<uintptr_t, size_t>> seen;  // (event, group), sorted by event
+    for (size_t k = 0; k < n; ++k) {
+      const uintptr_t e = reinterpret_cast<uintptr_t>(d[k].wait_event);
+      auto it = std::lower_bound(seen.begin(), seen.end(), std::make_pair(e, (size_t)0));
+      if (it == seen.end() || it->first != e) {
+        it = seen.insert(it, {e, members.size()});
+        members.emplace_back();
+      }
+      members[it->second].push_back(k);
+    }
+  }
+  for (const std::vector<size_t> &mem : members) {
     Plan::Group g;
-    g.first = i;
+    g.first = mem.front();
     // cols_dt: warp-MMA multi-column with T <= 8, colsw_dt: with 8 < T <= 16
     std::vector<wt::MatDesc> by_dt[4], mapped_dt[4], cols_dt[4], umma_dt[4], mcols_dt[4], colsw_dt[4], q8r_dt[4],
         q8r1_dt[4];  // row-owner int8 launches with two 8-column tiles (T > 8) and with one
@@ -1230,7 +1308,7 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
     std::vector<wt::SegReduce> reds;
     std::vector<size_t> red_ws;      // per reds entry: workspace float offset
     RangeCache rcw, rcx, rcy, rcs;
-    for (size_t k = i; k < j; ++k) {
+    for (const size_t k : mem) {
       const wt_gemv_desc &q = d[k];
       if (q.M == 0) continue;
       const int es = elem_bytes(q.dtype);
@@ -1422,7 +1500,6 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
         P->ws_patches.push_back({g.reduce + k * sizeof(wt::SegReduce) + offsetof(wt::SegReduce, ws), red_ws[k]});
     }
     P->groups.push_back(std::move(g));
-    i = j;
   }
   if (P->ws_floats) {
     CU(dev_alloc(reinterpret_cast<void **>(&P->ws), P->ws_floats * sizeof(float)));
@@ -1499,7 +1576,7 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
       ~TraceEnd() {
         if (!tb) return;
         cudaEvent_t te = nullptr;
-        if (trace_mark(s, &te) == WT_OK) h->trace.push_back({WT_TRACE_GEMV, h->n_groups, bytes, tb, te, true, wait});
+        if (trace_mark(s, &te) == WT_OK) trace_push(h, {WT_TRACE_GEMV, h->n_groups, bytes, tb, te, true, wait});
         else ev_destroy(tb);
       }
     } trace_end{h, s, tb, g.wbytes, wait};
@@ -1661,9 +1738,22 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
   *out = nullptr;
   if (n_paths < 0 || (n_paths > 0 && !paths)) return set_err(WT_EINVAL, "wt_open: bad path list");
   const unsigned route_req = flags & WT_ROUTE_MASK;
-  if (flags & ~(WT_ROUTE_MASK | WT_OPEN_HOST_ONLY | WT_OPEN_PREFAULT | WT_OPEN_TIMELINE | WT_OPEN_NOMAP | WT_OPEN_STAMPS))
+  if (flags & ~(WT_ROUTE_MASK | WT_OPEN_HOST_ONLY | WT_OPEN_PREFAULT | WT_OPEN_TIMELINE | WT_OPEN_NOMAP |
+                WT_OPEN_STAMPS | WT_OPEN_MAP_LARGE))
     return set_err(WT_EINVAL, "wt_open: unknown flag bits 0x%x", flags);
   const bool nomap = (flags & WT_OPEN_NOMAP) != 0;
+  if (nomap && (flags & WT_OPEN_MAP_LARGE))
+    return set_err(WT_EINVAL, "wt_open: WT_OPEN_NOMAP maps nothing: no WT_OPEN_MAP_LARGE");
+  uint64_t map_min = 0;
+  if (flags & WT_OPEN_MAP_LARGE) {
+    map_min = WT_MAP_MIN_BYTES;
+    if (const char *e = getenv("WT_MAP_MIN_BYTES")) {
+      char *end = nullptr;
+      const unsigned long long v = strtoull(e, &end, 10);
+      if (!end || end == e || *end) return set_err(WT_EINVAL, "wt_open: WT_MAP_MIN_BYTES=%s is not a byte count", e);
+      map_min = v;
+    }
+  }
   if (nomap && (route_req == WT_ROUTE_REGISTER || route_req == WT_ROUTE_DIRECT || (flags & WT_OPEN_PREFAULT)))
     return set_err(WT_EINVAL, "wt_open: WT_OPEN_NOMAP maps nothing: no REGISTER or DIRECT route, no PREFAULT");
   wt_handle *h = nullptr;
@@ -1686,7 +1776,7 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
     std::vector<int> rcs(n_paths, WT_OK);
     std::vector<std::string> errs(n_paths);
     host_pool().parallel_for((size_t)n_paths, [&](size_t i) {
-      rcs[i] = open_one(h->files[i], nomap);
+      rcs[i] = open_one(h->files[i], nomap, map_min);
       if (rcs[i]) errs[i] = t_err;
     });
     for (int i = 0; i < n_paths; ++i) {
@@ -1702,7 +1792,9 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
       if (h->files[f].base) h->by_base.push_back({reinterpret_cast<uintptr_t>(h->files[f].base), (uint32_t)f});
     std::sort(h->by_base.begin(), h->by_base.end());
     if (flags & WT_OPEN_PREFAULT) {
-      host_pool().parallel_for((size_t)n_paths, [&](size_t i) { prefault(h->files[i].base, h->files[i].size); });
+      host_pool().parallel_for((size_t)n_paths, [&](size_t i) {
+        if (h->files[i].base) prefault(h->files[i].base, h->files[i].size);
+      });
       h->prefaulted = true;
     }
     if (h->host_only) {
@@ -1723,7 +1815,7 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
     int ats = 0;
     cudaDeviceGetAttribute(&ats, cudaDevAttrPageableMemoryAccessUsesHostPageTables, h->device);
     for (File &f : h->files) {
-      unsigned want = nomap ? WT_ROUTE_NONE : route_req;
+      unsigned want = f.base ? route_req : WT_ROUTE_NONE;
       if (want == WT_ROUTE_AUTO) want = ats ? WT_ROUTE_DIRECT : WT_ROUTE_REGISTER;
       if (want == WT_ROUTE_DIRECT) {
         if (!ats) {
@@ -1879,7 +1971,7 @@ int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsign
   if (mode > WT_ADOPT_STAGED) return set_err(WT_EINVAL, "wt_adopt: unknown mode %u", mode);
   std::lock_guard<std::mutex> g(h->mu);
   try {
-    std::vector<Range> rs;
+    std::vector<Range> rs, st;  // st: small unmapped files of a MAP_LARGE handle (GATHER / CE)
     rs.reserve(n);
     uint64_t total = 0;
     RangeCache rc_dst;
@@ -1893,17 +1985,24 @@ int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsign
       if (!device_range_ok(dst[k], t.nbytes, rc_dst))
         return set_err(WT_EINVAL, "wt_adopt: dst[%zu] (%llu bytes) runs past the end of its device allocation", k,
                        (unsigned long long)t.nbytes);
-      if (mode != WT_ADOPT_STAGED && f.route == WT_ROUTE_NONE)
+      if (mode != WT_ADOPT_STAGED && f.route == WT_ROUTE_NONE && !f.small)
         return set_err(WT_ENOTSUP, "wt_adopt: %s has no device route; use WT_ADOPT_STAGED", f.path.c_str());
       ready[k] = nullptr;
-      rs.push_back({k, h->order[idx[k]].first, t.offset, f.base ? f.base + t.offset : nullptr,
+      const Range r{k, h->order[idx[k]].first, t.offset, f.base ? f.base + t.offset : nullptr,
                     f.dev ? f.dev + t.offset : nullptr, static_cast<uint8_t *>(dst[k]), t.nbytes,
-                    f.populated || h->prefaulted});
-      total += t.nbytes;
+                    f.populated || h->prefaulted};
+      if (mode != WT_ADOPT_STAGED && f.small) {
+        st.push_back(r);
+      } else {
+        rs.push_back(r);
+        total += t.nbytes;
+      }
     }
     const cudaStream_t s = static_cast<cudaStream_t>(stream);
-    int rc = mode == WT_ADOPT_STAGED ? adopt_staged(h, rs, s, ready) : adopt_device(h, rs, mode, s, ready, total);
-    return rc;
+    if (mode == WT_ADOPT_STAGED) return adopt_staged(h, rs, s, ready);
+    if (st.empty()) return adopt_device(h, rs, mode, s, ready, total);
+    if (rs.empty()) return adopt_staged(h, st, s, ready);
+    return adopt_mixed(h, rs, st, mode, s, ready, total);
   } catch (const std::bad_alloc &) {
     return set_err(WT_ENOMEM, "wt_adopt: out of host memory");
   }
@@ -1928,13 +2027,18 @@ int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream) {
   const bool capturing = cs == cudaStreamCaptureStatusActive;
   std::lock_guard<std::mutex> g(h->mu);
   try {
-    // Plans are keyed by the descriptors with each wait_event replaced by its group's
-    // ordinal: calls that differ only in which events they wait on share one plan.
+    // Plans are keyed by the descriptors with each wait_event replaced by the ordinal of its
+    // first appearance: calls that differ only in which events they wait on share one plan.
     std::vector<wt_gemv_desc> kd(d, d + n);
-    uintptr_t ordinal = 0;
-    for (size_t i = 0; i < n; ++i) {
-      if (i == 0 || d[i].wait_event != d[i - 1].wait_event) ++ordinal;
-      kd[i].wait_event = d[i].wait_event ? reinterpret_cast<void *>(ordinal) : nullptr;
+    {
+      std::vector<std::pair<uintptr_t, uintptr_t>> seen;  // (event, ordinal), sorted by event
+      for (size_t i = 0; i < n; ++i) {
+        const uintptr_t e = reinterpret_cast<uintptr_t>(d[i].wait_event);
+        if (!e) continue;
+        auto it = std::lower_bound(seen.begin(), seen.end(), std::make_pair(e, (uintptr_t)0));
+        if (it == seen.end() || it->first != e) it = seen.insert(it, {e, seen.size() + 1});
+        kd[i].wait_event = reinterpret_cast<void *>(it->second);
+      }
     }
     const uint8_t *kb = reinterpret_cast<const uint8_t *>(kd.data());
     std::vector<uint8_t> key(kb, kb + n * sizeof(wt_gemv_desc));
@@ -2038,7 +2142,7 @@ int wt_residency(const wt_handle *h, uint64_t *resident, uint64_t *total) {
   uint64_t res = 0, tot = 0;
   std::vector<unsigned char> vec;
   for (const File &f : h->files) {
-    if (!f.base) return set_err(WT_ENOTSUP, "wt_residency: %s is not mapped (WT_OPEN_NOMAP)", f.path.c_str());
+    if (!f.base) return set_err(WT_ENOTSUP, "wt_residency: %s is not mapped (WT_OPEN_NOMAP or MAP_LARGE)", f.path.c_str());
     const size_t pages = (f.size + pg - 1) / pg;
     vec.assign(pages, 0);
     if (pages && mincore(f.base, f.size, vec.data()) != 0)

@@ -11,7 +11,9 @@ Row blocks: a tensor named "<name>#r<k>" is row block k of matrix <name> (the
 many-small workload splits each matrix's rows across two files); its blocks are
 adopted into one contiguous [M, K] device buffer, in k order, and the GEMV of
 <name> waits on the event of its last-ingested block (the ingest stream is in
-order, so that event implies the earlier blocks).
+order, so that event implies the earlier blocks).  On a WT_OPEN_MAP_LARGE handle a
+matrix whose blocks lie in both small (unmapped) and large (mapped) files crosses two
+streams; it waits on an event recorded on the ingest stream after the wt_adopt call.
 """
 from __future__ import annotations
 
@@ -134,6 +136,30 @@ class DeviceCheckpoint:
     canary: int = 0
     _tables: Dict[tuple, object] = field(default_factory=dict)
     ptrs: List[int] = field(default_factory=list)  # device address of each MatrixRef's buffer
+    _joined: List[object] = field(default_factory=list)  # events of matrices that crossed two streams
+
+    def _join_mixed(self, h: wt.Handle, ks: Sequence[int], events: Dict[int, int], mode: int, stream: int):
+        """A matrix of `ks` whose tensors took both ways of one WT_OPEN_MAP_LARGE wt_adopt call
+        (mapped files on the device route, small unmapped files through the pinned ring on the
+        library's own stream) has no tensor event that implies the others: all its tensors get
+        one event recorded on `stream` after the call, which follows every byte of it."""
+        if mode == wt.WT_ADOPT_STAGED:
+            return
+        hp = h.tensors.host_ptrs
+        mixed = []
+        for k in ks:
+            ts = self.mats[k].parts + ([self.mats[k].scale] if self.mats[k].scale is not None else [])
+            if len({hp[i] == 0 for i in ts}) > 1:
+                mixed.append(ts)
+        if not mixed:
+            return
+        import torch
+        ev = torch.cuda.Event()
+        ev.record(torch.cuda.ExternalStream(stream) if stream else torch.cuda.default_stream())
+        self._joined.append(ev)
+        for ts in mixed:
+            for i in ts:
+                events[i] = ev.cuda_event
 
     @staticmethod
     def allocate(h: wt.Handle, mats: Sequence[MatrixRef], device="cuda", canary: int = 0,
@@ -214,14 +240,17 @@ class DeviceCheckpoint:
             idx.sort()
             if idx:
                 events.update(zip(idx, h.adopt(idx, [dc.dst[i] for i in idx], mode, stream)))
+                dc._join_mixed(h, range(a, b), events, mode, stream)
         return dc, events, alloc_s
 
     def adopt(self, h: wt.Handle, mode: int = wt.WT_ADOPT_GATHER, stream: int = 0,
               order: Optional[Sequence[int]] = None) -> Dict[int, int]:
         """wt_adopt every tensor (file/index order unless `order`); returns tensor -> event."""
         idx = list(order) if order is not None else sorted(self.dst)
-        evs = h.adopt(idx, [self.dst[i] for i in idx], mode, stream)
-        return dict(zip(idx, evs))
+        evs = dict(zip(idx, h.adopt(idx, [self.dst[i] for i in idx], mode, stream)))
+        got = set(idx)
+        self._join_mixed(h, [k for k, m in enumerate(self.mats) if got.issuperset(m.parts)], evs, mode, stream)
+        return evs
 
     def gemv_mats(self) -> List[int]:
         return [k for k, m in enumerate(self.mats) if m.gemv]

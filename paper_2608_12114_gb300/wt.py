@@ -22,7 +22,8 @@ WT_OK, WT_EINVAL, WT_EIO, WT_EFORMAT, WT_ENOMEM, WT_ECUDA, WT_ENOTSUP, WT_ETIMED
 WT_F32, WT_BF16, WT_F16, WT_I8, WT_U8 = 0, 1, 2, 3, 4
 WT_ROUTE_AUTO, WT_ROUTE_REGISTER, WT_ROUTE_DIRECT, WT_ROUTE_NONE = 0, 1, 2, 3
 WT_OPEN_HOST_ONLY, WT_OPEN_PREFAULT, WT_OPEN_TIMELINE, WT_OPEN_NOMAP = 1 << 4, 1 << 5, 1 << 6, 1 << 7
-WT_OPEN_STAMPS = 1 << 8
+WT_OPEN_STAMPS, WT_OPEN_MAP_LARGE = 1 << 8, 1 << 9
+WT_MAP_MIN_BYTES = 1 << 18
 # the per-CTA record of wt_pass_stamps, in field order
 STAMP_FIELDS = ("entry", "prologue", "operands", "first_copy", "first_full", "last_full", "exit", "sm")
 WT_TRACE_INGEST, WT_TRACE_GEMV = 0, 1

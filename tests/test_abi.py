@@ -174,12 +174,43 @@ def header_defines():
 def test_binding_constants_match_the_header():
     d = header_defines()
     for name in ("WT_OPEN_HOST_ONLY", "WT_OPEN_PREFAULT", "WT_OPEN_TIMELINE", "WT_OPEN_NOMAP", "WT_OPEN_STAMPS",
+                 "WT_OPEN_MAP_LARGE", "WT_MAP_MIN_BYTES",
                  "WT_TRACE_INGEST", "WT_TRACE_GEMV", "WT_ADOPT_GATHER", "WT_ADOPT_CE", "WT_ADOPT_STAGED"):
         assert d[name] == getattr(wt, name), name
     # the stamp record: field order and width
     assert d["WT_STAMP_FIELDS"] == len(wt.STAMP_FIELDS)
     for i, f in enumerate(wt.STAMP_FIELDS):
         assert d["WT_STAMP_" + f.upper()] == i, f
+
+
+def test_map_large_maps_only_the_large_files(L, tmp_path, monkeypatch):
+    ck = synth.build("many", str(tmp_path / "ml"), n_matrices=40)
+    sizes = [os.path.getsize(p) for p in ck.paths]
+    thr = sorted(sizes)[len(sizes) // 2]
+    monkeypatch.setenv("WT_MAP_MIN_BYTES", str(thr))
+    with wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY) as hm:
+        want = [(t.name, t.dtype, t.shape, t.nbytes, t.file, t.offset) for t in hm.tensors]
+    with wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY | wt.WT_OPEN_MAP_LARGE) as h:
+        assert [(t.name, t.dtype, t.shape, t.nbytes, t.file, t.offset) for t in h.tensors] == want
+        for t in h.tensors:
+            assert (t.host_ptr != 0) == (sizes[t.file] >= thr), (t.name, sizes[t.file])
+        maps = [l for l in open("/proc/self/maps") if str(tmp_path) in l]
+        assert len({l.split()[-1] for l in maps}) == sum(s >= thr for s in sizes)
+        # the mappings hold the files' bytes
+        import ctypes
+        for t in h.tensors:
+            if t.host_ptr and t.nbytes:
+                with open(ck.paths[t.file], "rb") as fh:
+                    fh.seek(t.offset)
+                    assert ctypes.string_at(t.host_ptr, min(4096, t.nbytes)) == fh.read(min(4096, t.nbytes))
+    for bad in (wt.WT_OPEN_NOMAP,):
+        with pytest.raises(wt.WtError) as ei:
+            wt.Handle(ck.paths, wt.WT_OPEN_MAP_LARGE | bad)
+        assert ei.value.code == wt.WT_EINVAL
+    monkeypatch.setenv("WT_MAP_MIN_BYTES", "1M")
+    with pytest.raises(wt.WtError) as ei:
+        wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY | wt.WT_OPEN_MAP_LARGE)
+    assert ei.value.code == wt.WT_EINVAL and "WT_MAP_MIN_BYTES" in str(ei.value)
 
 
 def test_stamps_query_on_host_only_handle(L, tmp_path):
@@ -190,7 +221,7 @@ def test_stamps_query_on_host_only_handle(L, tmp_path):
             h.pass_stamps()
         assert ei.value.code == wt.WT_EINVAL
     with pytest.raises(wt.WtError) as ei:
-        wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY | (1 << 9))  # unknown flag bit
+        wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY | (1 << 12))  # unknown flag bit
     assert ei.value.code == wt.WT_EINVAL
 
 

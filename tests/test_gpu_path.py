@@ -405,3 +405,88 @@ def test_nomap_refuses_device_routes_and_changed_files(torch, tmp_path):
     s.synchronize()
     check_bytes(torch, h, dev, co)
     h.close()
+
+
+# ----------------------------------------------------------------------------- mixed (WT_OPEN_MAP_LARGE)
+
+@pytest.mark.parametrize("mode", [wt.WT_ADOPT_GATHER, wt.WT_ADOPT_CE, wt.WT_ADOPT_STAGED], ids=["gather", "ce", "staged"])
+def test_map_large_mixed_ingest_matches_oracle(torch, tmp_path, monkeypatch, mode):
+    """WT_OPEN_MAP_LARGE maps only the files at or above the threshold (here the median file
+    size).  A GATHER or CE adopt moves the small files through the pinned ring on the library's
+    own stream, concurrently with the mapped files; the caller's stream is ordered after both
+    (digests taken on it with no host wait see every byte); bytes, canaries, digests and every
+    GEMV row match the oracle with the event-gated pass on another stream."""
+    ck = synth.build("many", str(tmp_path), workers=4, n_matrices=300)
+    import os
+    sizes = [os.path.getsize(p) for p in ck.paths]
+    thr = sorted(sizes)[len(sizes) // 2]
+    monkeypatch.setenv("WT_MAP_MIN_BYTES", str(thr))
+    co = oracle.CheckpointOracle(ck.paths)
+    h, dev, ev, s = ingest(torch, ck, mode, wt.WT_OPEN_MAP_LARGE)
+    mapped = {l.split()[-1] for l in open("/proc/self/maps") if str(tmp_path) in l}
+    assert len(mapped) == sum(n >= thr for n in sizes)
+    assert all((h.route(f) == wt.WT_ROUTE_NONE) == (sizes[f] < thr) for f in range(len(sizes)))
+    idx = sorted(dev.dst)
+    out = torch.zeros(len(idx), dtype=torch.int64, device="cuda")
+    h.checksum([dev.dst[i] for i in idx], [h.tensors[i].nbytes for i in idx], out.data_ptr(), s.cuda_stream)
+    xs, ys = dev.inputs(), dev.outputs()
+    for y in ys.values():
+        y.fill_(float("nan"))
+    c = torch.cuda.Stream()
+    h.pass_(dev.descs(xs, ys, ev), c.cuda_stream)
+    c.synchronize()
+    s.synchronize()
+    od = oracle_digests(h, co)
+    got = {i: int(v) & 0xFFFFFFFFFFFFFFFF for i, v in zip(idx, out.cpu().tolist())}
+    assert all(got[i] == od[i][1] for i in idx)
+    check_bytes(torch, h, dev, co)
+    check_gemv(h, dev, co, ys)
+    assert h.device_status() == 0
+    h.close()
+
+
+def test_map_large_matrix_across_both_ways(torch, tmp_path, monkeypatch):
+    """Matrices whose row blocks lie in a small (unmapped) and a large (mapped) file: the two
+    blocks cross two streams, so the pipeline gives the matrix one event recorded after the
+    wt_adopt call; every GEMV row matches the oracle with y NaN-filled first, for adopts issued
+    at once and segment by segment (stream_in)."""
+    T = []
+    mats = []
+    paths = []
+    K = 512
+    for m in range(12):
+        small_rows, large_rows = 1 + 3 * m, 200 + 17 * m  # 1 KB .. 34 KB and 200 KB .. 391 KB blocks
+        parts = []
+        for b, rows in enumerate((small_rows, large_rows) if m % 2 == 0 else (large_rows, small_rows)):
+            f = len(paths)
+            parts.append(len(T))
+            T.append(synth.TensorSpec(f"m{m}#r{b}", synth.DT_BF16, (rows, K), f, key=(5, 700 + f)))
+            paths.append(str(tmp_path / f"x{f:03d}.wt"))
+        mats.append(synth.Matrix(f"m{m}", synth.DT_BF16, small_rows + large_rows, K, parts))
+    ck = synth.write_files(synth.Checkpoint("split", paths, T, mats))
+    monkeypatch.setenv("WT_MAP_MIN_BYTES", str(100 << 10))
+    co = oracle.CheckpointOracle(ck.paths)
+    for how in ("adopt", "stream_in"):
+        h = wt.Handle(ck.paths, wt.WT_OPEN_MAP_LARGE)
+        hm = pipeline.matrices(h)
+        assert all(len({h.tensors.host_ptrs[i] == 0 for i in m.parts}) == 2 for m in hm)
+        s = torch.cuda.Stream()
+        if how == "adopt":
+            dev = pipeline.DeviceCheckpoint.allocate(h, hm)
+            ev = dev.adopt(h, wt.WT_ADOPT_GATHER, s.cuda_stream)
+        else:
+            dev, ev, _ = pipeline.DeviceCheckpoint.stream_in(h, hm, wt.WT_ADOPT_GATHER, s.cuda_stream,
+                                                             first_bytes=1 << 20, growth=1.0)
+        assert dev._joined  # one joint event per adopt call that held such matrices
+        for m in hm:
+            assert len({ev[i] for i in m.parts}) == 1
+        xs, ys = dev.inputs(), dev.outputs()
+        for y in ys.values():
+            y.fill_(float("nan"))
+        c = torch.cuda.Stream()
+        h.pass_(dev.descs(xs, ys, ev), c.cuda_stream)
+        c.synchronize()
+        s.synchronize()
+        check_gemv(h, dev, co, ys)
+        assert h.device_status() == 0
+        h.close()

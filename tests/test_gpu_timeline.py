@@ -76,3 +76,50 @@ def test_register_route_reports_its_registration(torch, tmp_path):
         assert flags & ~0x0A == 0  # and at most cudaHostRegisterReadOnly besides
     with wt.Handle(ck.paths, wt.WT_ROUTE_DIRECT) as h:
         assert h.registration(0) == 0
+
+
+def test_interleaved_wait_events_make_one_group_each(torch):
+    """Descriptors whose wait events interleave (A, B, none, A, B, none, ...) form one group per
+    distinct event, in order of first appearance: three GEMV records in the timeline, and the
+    same results, bit for bit, as one pass with no events; a later call with fresh events in
+    the same pattern reuses the plan."""
+    rng = np.random.default_rng(5)
+    K = 1024
+    Ws, ys, descs = [], [], []
+    x = torch.from_numpy(synth.make_x(K, wt.WT_BF16)).cuda()
+    for i in range(12):
+        M = 64 + 37 * i
+        W = torch.from_numpy(synth.f32_to_bf16_bits((0.02 * rng.standard_normal(M * K)).astype(np.float32))
+                             .view(np.uint8)).cuda()
+        y = torch.full((M,), float("nan"), dtype=torch.float32, device="cuda")
+        Ws.append(W)
+        ys.append(y)
+        descs.append(wt.gemv_desc(W.data_ptr(), wt.WT_BF16, M, K, x.data_ptr(), y.data_ptr()))
+    s = torch.cuda.Stream()
+    with wt.Handle([]) as h0:
+        h0.pass_(descs, s.cuda_stream)
+        s.synchronize()
+    ref = [y.clone() for y in ys]
+    other = torch.cuda.Stream()
+    with wt.Handle([], wt.WT_OPEN_TIMELINE) as h:
+        for rep in range(2):
+            a, b = torch.cuda.Event(), torch.cuda.Event()
+            a.record(other)
+            b.record(other)
+            pattern = [a.cuda_event, b.cuda_event, 0]
+            d = [wt.gemv_desc(q.W, q.dtype, q.M, q.K, q.x, q.y, wait_event=pattern[i % 3])
+                 for i, q in enumerate(descs)]
+            for y in ys:
+                y.fill_(float("nan"))
+            origin = torch.cuda.Event(enable_timing=True)
+            origin.record(s)
+            n0 = h.kernel_launches()
+            h.pass_(d, s.cuda_stream)
+            s.synchronize()
+            recs = [r for r in h.trace(origin.cuda_event) if r["kind"] == "gemv"]
+            assert len(recs) == 3
+            assert [r["event"] for r in recs] == pattern[:2] + [0]
+            assert h.kernel_launches() - n0 == 3
+            for y, r in zip(ys, ref):
+                assert torch.equal(y, r)
+        assert h.device_status() == 0
