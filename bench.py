@@ -459,6 +459,7 @@ def first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, 
     h = wt.Handle(ck.paths, flags | (wt.WT_OPEN_TIMELINE if trace is not None else 0))
     mats = pipeline.matrices(h)
     t1 = time.perf_counter()
+    ot = h.open_times() if phases is not None else None
     if origin is not None:
         origin.record(ingest_s)
     if slab is None:
@@ -485,6 +486,10 @@ def first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, 
         phases.setdefault("enqueue_ms", []).append((t2 - t1 - alloc_s) * 1e3)
         phases.setdefault("drain_ms", []).append((t0 + dt - t2) * 1e3)
         phases["route"] = wt.ROUTE_NAMES.get(h.route(0), "?") if h.n_files else None
+        for k in ("index_ms", "index_cpu_ms", "map_cpu_ms", "prefault_ms", "route_ms"):
+            phases.setdefault("wt_open_" + k, []).append(ot[k])
+        phases["files_mapped"] = ot["files_mapped"]
+        phases["files_registered"] = ot["files_registered"]
     if trace is not None:
         recs = h.trace(origin.cuda_event)
         batch_of = {r["event"]: r["index"] for r in recs if r["kind"] == "ingest"}
@@ -724,11 +729,14 @@ def run_wt(args, rank, world):
                         "torch.cuda.empty_cache; slabs allocated segment by segment between wt_adopt "
                         "calls) + wt_adopt + event-gated first pass + D2H of all y, page cache warm; "
                         "pinned_h2d_gbs is the highest of h2d_ceilings_gbs; phases: alloc_ms is host "
-                        "time in allocations, enqueue_ms the rest of the time to the last return",
+                        "time in allocations, enqueue_ms the rest of the time to the last return; "
+                        "wt_open_*: wt_open's own step times (wt_open_times: parallel index + map loop, "
+                        "summed per-file index and mmap time, prefault, route probe)",
                 "launches_per_run": e2e_launches,
                 "iqr_ms": [round(v * 1e3, 2) for v in quartiles(e2e_times)] if e2e_times else None,
                 "phases_ms_median": {k: round(statistics.median(v), 2) for k, v in phases.items() if k.endswith("_ms")},
                 "route": phases.get("route"),
+                "files_mapped": phases.get("files_mapped"), "files_registered": phases.get("files_registered"),
                 "buffers_reused": {"value": round(aggregate_gbs(data_bytes, world, reuse_s), 1), "unit": "GB/s",
                                    "ms": round(reuse_s * 1e3, 2),
                                    "frac_of_pinned_h2d": round(data_bytes / reuse_s / 1e9 / h2d, 4),

@@ -212,6 +212,28 @@ int wt_file_route(const wt_handle *h, size_t f, unsigned *route);
  * not by the registration).  Errors: WT_EINVAL. */
 int wt_file_registration(const wt_handle *h, size_t f, unsigned *flags);
 
+/* Host time wt_open spent in each of the hot path's first three steps (Sec. 5.3's map-and-
+ * wire cost, per phase), measured inside the call with a monotonic clock:
+ *   index_ms      wall time of the parallel loop that opens, parses and validates every file
+ *                 and maps those it maps (steps 1 and 2 together, on the host pool);
+ *   index_cpu_ms  summed over the files: open, fstat, index reads and validation (step 1);
+ *   map_cpu_ms    summed over the files: mmap (step 2; the calls serialise on the process's
+ *                 address-space lock, so this is close to their wall time);
+ *   prefault_ms   wall time of WT_OPEN_PREFAULT's population (0 without it);
+ *   route_ms      wall time of the route probe and any registration (step 3);
+ *   files_mapped, files_registered: how many files each step touched.
+ * Errors: WT_EINVAL (NULL argument). */
+typedef struct {
+  double index_ms;
+  double index_cpu_ms;
+  double map_cpu_ms;
+  double prefault_ms;
+  double route_ms;
+  uint64_t files_mapped;
+  uint64_t files_registered;
+} wt_open_phases;
+int wt_open_times(const wt_handle *h, wt_open_phases *out);
+
 /* Copy tensors idx[0..n) into device memory dst[0..n) (each at least nbytes of
  * that tensor, 16-byte aligned for the vector path) on `stream`, in order.
  * Tensors are grouped into batches of a few MB to a few hundred MB; one event

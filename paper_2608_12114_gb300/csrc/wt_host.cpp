@@ -18,6 +18,7 @@
 
 #include <algorithm>
 #include <atomic>
+#include <chrono>
 #include <cerrno>
 #include <condition_variable>
 #include <cstdarg>
@@ -217,6 +218,7 @@ struct File {
   uint8_t *base = nullptr;  // mapping (nullptr: opened with WT_OPEN_NOMAP, or small under MAP_LARGE)
   size_t size = 0;
   bool small = false;       // WT_OPEN_MAP_LARGE left it unmapped: adopted through the pinned ring
+  int64_t index_ns = 0, map_ns = 0;  // host time wt_open spent parsing and mapping it
   // identity at wt_open: a WT_OPEN_NOMAP file is opened again by a staged adopt, which checks
   // that the path still names the file whose index was validated
   uint64_t st_dev = 0, st_ino = 0;
@@ -332,6 +334,7 @@ struct wt_handle {
   std::vector<cudaEvent_t> events;
   std::list<Plan *> plans;
   std::atomic<uint64_t> kernel_launches{0};
+  wt_open_phases open_times{};
   std::mutex mu;
   // events and trace records: a mixed adopt (WT_OPEN_MAP_LARGE) adds them from two threads
   std::mutex ev_mu;
@@ -432,7 +435,13 @@ void unmap_file(File &f) {
 
 // open, parse and map one file (not with `nomap`, nor when it is smaller than `map_min`
 // bytes); closes the fd on every path.
+int64_t now_ns() {
+  return std::chrono::duration_cast<std::chrono::nanoseconds>(std::chrono::steady_clock::now().time_since_epoch())
+      .count();
+}
+
 int open_one(File &f, bool nomap, uint64_t map_min) {
+  const int64_t t0 = now_ns();
   if (wt::fault_injected("open")) return set_err(WT_EIO, "%s: open: injected fault", f.path.c_str());
   const int fd = open(f.path.c_str(), O_RDONLY | O_CLOEXEC);
   if (fd < 0) return set_err(WT_EIO, "%s: open: %s", f.path.c_str(), strerror(errno));
@@ -448,6 +457,8 @@ int open_one(File &f, bool nomap, uint64_t map_min) {
   f.mtime_ns = (int64_t)st.st_mtim.tv_sec * 1000000000ll + st.st_mtim.tv_nsec;
   const bool skip = nomap || (uint64_t)st.st_size < map_min;
   f.small = !nomap && skip;
+  const int64_t t1 = now_ns();
+  f.index_ns = t1 - t0;
   if (rc == WT_OK && skip) f.size = (size_t)st.st_size;
   if (rc == WT_OK && !skip) {
     f.size = (size_t)st.st_size;
@@ -455,6 +466,7 @@ int open_one(File &f, bool nomap, uint64_t map_min) {
     void *p = injected ? MAP_FAILED : mmap(nullptr, f.size, PROT_READ, MAP_SHARED, fd, 0);
     if (p == MAP_FAILED) rc = set_err(WT_EIO, "%s: mmap: %s", f.path.c_str(), injected ? "injected fault" : strerror(errno));
     else f.base = static_cast<uint8_t *>(p);
+    f.map_ns = now_ns() - t1;
   }
   close(fd);  // Algorithm 1: the mapping outlives the descriptor
   return rc;
@@ -1775,10 +1787,17 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
     // parse + map in parallel; keep the first failure in file order
     std::vector<int> rcs(n_paths, WT_OK);
     std::vector<std::string> errs(n_paths);
+    int64_t t0 = now_ns();
     host_pool().parallel_for((size_t)n_paths, [&](size_t i) {
       rcs[i] = open_one(h->files[i], nomap, map_min);
       if (rcs[i]) errs[i] = t_err;
     });
+    h->open_times.index_ms = (now_ns() - t0) * 1e-6;
+    for (const File &f : h->files) {
+      h->open_times.index_cpu_ms += f.index_ns * 1e-6;
+      h->open_times.map_cpu_ms += f.map_ns * 1e-6;
+      h->open_times.files_mapped += f.base ? 1 : 0;
+    }
     for (int i = 0; i < n_paths; ++i) {
       if (rcs[i]) {
         std::string msg = errs[i];
@@ -1792,10 +1811,12 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
       if (h->files[f].base) h->by_base.push_back({reinterpret_cast<uintptr_t>(h->files[f].base), (uint32_t)f});
     std::sort(h->by_base.begin(), h->by_base.end());
     if (flags & WT_OPEN_PREFAULT) {
+      t0 = now_ns();
       host_pool().parallel_for((size_t)n_paths, [&](size_t i) {
         if (h->files[i].base) prefault(h->files[i].base, h->files[i].size);
       });
       h->prefaulted = true;
+      h->open_times.prefault_ms = (now_ns() - t0) * 1e-6;
     }
     if (h->host_only) {
       for (File &f : h->files) f.route = WT_ROUTE_NONE;
@@ -1813,6 +1834,7 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
       return rc;
     }
     int ats = 0;
+    t0 = now_ns();
     cudaDeviceGetAttribute(&ats, cudaDevAttrPageableMemoryAccessUsesHostPageTables, h->device);
     for (File &f : h->files) {
       unsigned want = f.base ? route_req : WT_ROUTE_NONE;
@@ -1859,6 +1881,8 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
         f.route = WT_ROUTE_NONE;
       }
     }
+    h->open_times.route_ms = (now_ns() - t0) * 1e-6;
+    for (const File &f : h->files) h->open_times.files_registered += f.registered ? 1 : 0;
     ce = dev_alloc(reinterpret_cast<void **>(&h->status), 256);
     if (ce == cudaSuccess) ce = cudaMemset(h->status, 0, 256);
     if (ce != cudaSuccess) {
@@ -1959,6 +1983,12 @@ int wt_file_registration(const wt_handle *h, size_t f, unsigned *flags) {
   if (!h || !flags) return set_err(WT_EINVAL, "wt_file_registration: NULL argument");
   if (f >= h->files.size()) return set_err(WT_EINVAL, "wt_file_registration: file %zu out of range", f);
   *flags = h->files[f].registered ? h->files[f].reg_flags : 0u;
+  return WT_OK;
+}
+
+int wt_open_times(const wt_handle *h, wt_open_phases *out) {
+  if (!h || !out) return set_err(WT_EINVAL, "wt_open_times: NULL argument");
+  *out = h->open_times;
   return WT_OK;
 }
 

@@ -35,7 +35,7 @@ MODE_NAMES = {WT_ADOPT_GATHER: "gather", WT_ADOPT_CE: "ce", WT_ADOPT_STAGED: "st
 SYMBOLS = ("wt_last_error", "wt_abi_version", "wt_open", "wt_num_tensors", "wt_num_files",
            "wt_tensor_info", "wt_tensor_table", "wt_tensor_names", "wt_find", "wt_file_route", "wt_file_registration", "wt_adopt", "wt_pass", "wt_checksum",
            "wt_checksum_plain", "wt_checksum_noalloc", "wt_device_status", "wt_residency",
-           "wt_kernel_launches", "wt_trace", "wt_pass_stamps", "wt_live", "wt_close",
+           "wt_kernel_launches", "wt_trace", "wt_pass_stamps", "wt_open_times", "wt_live", "wt_close",
            # include/wt_dlpack.h
            "wt_dlpack_file", "wt_dlpack_tensor", "wt_dlpack_release", "wt_dlpack_live")
 WT_DLPACK_DEVICE, WT_DLPACK_HOST = 0, 1
@@ -115,6 +115,7 @@ def lib(path: str = LIB_PATH):
     L.wt_residency.argtypes = [vp, u64p, u64p]
     L.wt_trace.argtypes = [vp, vp, C.POINTER(TraceRec), sz, C.POINTER(sz)]
     L.wt_pass_stamps.argtypes = [vp, vp, sz, C.POINTER(sz)]
+    L.wt_open_times.argtypes = [vp, C.POINTER(OpenPhases)]
     L.wt_live.argtypes = [C.POINTER(LiveCounts)]
     L.wt_close.argtypes = [vp]
     L.wt_dlpack_file.argtypes = [C.c_char_p, C.c_int32, C.c_uint64, C.c_uint64, C.c_uint, C.POINTER(vp)]
@@ -144,6 +145,13 @@ class TensorInfo:
     file: int
     offset: int
     host_ptr: int
+
+
+class OpenPhases(C.Structure):
+    """wt_open_phases: wt_open's host time per hot-path step."""
+    _fields_ = [("index_ms", C.c_double), ("index_cpu_ms", C.c_double), ("map_cpu_ms", C.c_double),
+                ("prefault_ms", C.c_double), ("route_ms", C.c_double), ("files_mapped", C.c_uint64),
+                ("files_registered", C.c_uint64)]
 
 
 class TensorTable:
@@ -289,6 +297,13 @@ class Handle:
         return [dict(kind=kinds.get(buf[i].kind, "?"), index=buf[i].index, bytes=buf[i].bytes,
                      event=buf[i].event or 0, begin_ms=buf[i].begin_ms, end_ms=buf[i].end_ms)
                 for i in range(min(n.value, cap))]
+
+    def open_times(self) -> dict:
+        """wt_open_times: host ms wt_open spent per step (index, map, prefault, route) and the
+        counts of mapped and registered files."""
+        o = OpenPhases()
+        _check(lib().wt_open_times(self.ptr, C.byref(o)))
+        return {f: getattr(o, f) for f, _ in OpenPhases._fields_}
 
     def pass_stamps(self):
         """wt_pass_stamps (WT_OPEN_STAMPS handles): the per-CTA stamps of the latest one-column

@@ -203,6 +203,16 @@ def test_map_large_maps_only_the_large_files(L, tmp_path, monkeypatch):
                 with open(ck.paths[t.file], "rb") as fh:
                     fh.seek(t.offset)
                     assert ctypes.string_at(t.host_ptr, min(4096, t.nbytes)) == fh.read(min(4096, t.nbytes))
+        t = h.open_times()
+        assert t["files_mapped"] == sum(s >= thr for s in sizes) and t["files_registered"] == 0
+        assert t["index_ms"] > 0 and t["index_cpu_ms"] > 0 and t["map_cpu_ms"] > 0
+        assert t["prefault_ms"] == 0 and t["route_ms"] == 0  # host-only: no route probe
+    with wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY | wt.WT_OPEN_NOMAP) as h:
+        t = h.open_times()
+        assert t["files_mapped"] == 0 and t["map_cpu_ms"] == 0 and t["index_cpu_ms"] > 0
+    with wt.Handle(ck.paths, wt.WT_OPEN_HOST_ONLY | wt.WT_OPEN_PREFAULT) as h:
+        t = h.open_times()
+        assert t["files_mapped"] == len(sizes) and t["prefault_ms"] > 0
     for bad in (wt.WT_OPEN_NOMAP,):
         with pytest.raises(wt.WtError) as ei:
             wt.Handle(ck.paths, wt.WT_OPEN_MAP_LARGE | bad)
