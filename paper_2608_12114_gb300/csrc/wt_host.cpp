@@ -704,11 +704,10 @@ int reopen_checked(const File &f) {
   return fd;
 }
 
-// The staged half of a mixed adopt runs on the ring's own stream: it starts after `after`
-// (recorded on the caller's stream) and records `last` once its final copy is enqueued.
+// The staged half of a mixed adopt runs on the ring's own stream, after `after` (an event
+// recorded on the caller's stream).
 struct StagedJoin {
   cudaEvent_t after = nullptr;
-  cudaEvent_t last = nullptr;
 };
 
 // Staged: page cache -> pinned slot (host threads: memcpy from the mapping, or pread for a
@@ -867,11 +866,6 @@ int adopt_staged(wt_handle *h, const std::vector<Range> &rs, cudaStream_t s, voi
       h->n_batches++;
     }
   }
-  if (join) {
-    rc = new_event(h, &join->last);
-    if (rc) return rc;
-    CU(cudaEventRecord(join->last, s));
-  }
   return WT_OK;
 }
 
@@ -879,7 +873,8 @@ int adopt_staged(wt_handle *h, const std::vector<Range> &rs, cudaStream_t s, voi
 // (`dv`, through the device route) and small unmapped ones (`st`, through the pinned ring):
 // the staged half runs on a helper thread and the ring's stream, ordered after the caller's
 // earlier work on `s`, while this thread enqueues the mapped half on `s`; `s` then waits
-// for the staged half, so the call keeps its stream semantics.
+// for whatever the staged half enqueued, on success and on failure alike, so the call keeps
+// its stream semantics (later work on `s` never overlaps a copy of this call).
 int adopt_mixed(wt_handle *h, const std::vector<Range> &dv, const std::vector<Range> &st, unsigned mode,
                 cudaStream_t s, void **ready, uint64_t total_dev) {
   StagedJoin join;
@@ -901,9 +896,21 @@ int adopt_mixed(wt_handle *h, const std::vector<Range> &dv, const std::vector<Ra
   });
   rc = adopt_device(h, dv, mode, s, ready, total_dev);
   helper.t.join();
+  // The ring's stream is created once and never replaced, so it can be read here without
+  // the ring's lock; an event on it now follows every copy the staged half enqueued (and
+  // possibly later ones of other calls, which only adds order).
+  if (const cudaStream_t rs = g_ring[h->device].stream) {
+    cudaEvent_t done = nullptr;
+    int rc_j = new_event(h, &done);
+    if (rc_j == WT_OK) {
+      cudaError_t e = cudaEventRecord(done, rs);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(s, done, 0);
+      if (e != cudaSuccess) rc_j = cuda_err(e, "wt_adopt: joining the staged half");
+    }
+    if (rc_j && !rc && !rc_st) return rc_j;
+  }
   if (rc) return rc;
   if (rc_st) return set_err(rc_st, "%s", err_st.c_str());
-  CU(cudaStreamWaitEvent(s, join.last, 0));
   return WT_OK;
 }
 

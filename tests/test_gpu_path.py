@@ -490,3 +490,36 @@ def test_map_large_matrix_across_both_ways(torch, tmp_path, monkeypatch):
         check_gemv(h, dev, co, ys)
         assert h.device_status() == 0
         h.close()
+
+
+def test_map_large_staged_failure_is_reported_and_the_handle_recovers(torch, tmp_path, monkeypatch):
+    """The fifth pread of the staged half fails (WT_FAULT, made on the host) while the mapped
+    half is being enqueued: wt_adopt returns WT_EIO with the file named, the caller's stream is
+    still ordered after every copy the call issued, the pinned ring is free again, and the next
+    adopt on the same handle moves every byte (and leaves every canary) correctly."""
+    ck = synth.build("many", str(tmp_path), workers=4, n_matrices=120)
+    import os
+    sizes = [os.path.getsize(p) for p in ck.paths]
+    monkeypatch.setenv("WT_MAP_MIN_BYTES", str(sorted(sizes)[len(sizes) // 2]))
+    co = oracle.CheckpointOracle(ck.paths)
+    h = wt.Handle(ck.paths, wt.WT_OPEN_MAP_LARGE)
+    dev = pipeline.DeviceCheckpoint.allocate(h, pipeline.matrices(h), canary=CANARY)
+    for b in dev.bufs:
+        b.fill_(0xA5)
+    torch.cuda.synchronize()
+    s = torch.cuda.Stream()
+    monkeypatch.setenv("WT_FAULT", "pread:5")
+    with pytest.raises(wt.WtError) as ei:
+        dev.adopt(h, wt.WT_ADOPT_GATHER, s.cuda_stream)
+    monkeypatch.delenv("WT_FAULT")
+    assert ei.value.code == wt.WT_EIO and "injected" in str(ei.value)
+    s.synchronize()
+    for b in dev.bufs:
+        b.fill_(0xA5)
+    torch.cuda.synchronize()
+    ev = dev.adopt(h, wt.WT_ADOPT_GATHER, s.cuda_stream)
+    s.synchronize()
+    assert all(ev.values())
+    check_bytes(torch, h, dev, co)
+    assert h.device_status() == 0
+    h.close()
