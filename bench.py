@@ -89,6 +89,9 @@ def parse_args():
                    help="time wt_checksum (leaf-tree FNV-1a-64) over every resident tensor of the workload")
     p.add_argument("--consumer-priority", default="high", choices=["high", "normal"],
                    help="priority of the stream the event-gated first-use GEMVs run on")
+    p.add_argument("--fresh", action="store_true",
+                   help="with --timeline: allocate the device buffers inside each traced run (step 4), "
+                        "as the e2e value does")
     p.add_argument("--timeline", action="store_true",
                    help="one traced file -> first-use run (WT_OPEN_TIMELINE): per ingest batch and GEMV group, "
                         "device begin/end times (one JSON line)")
@@ -924,7 +927,12 @@ def overlap_summary(recs):
         later = [e for i, e in nxt if b is not None and i > b]
         if later and g["end_ms"] <= later[0]:
             early += 1
+    # time the link had nothing queued: gaps between one batch landing and the next beginning
+    order = sorted(ing, key=lambda r: r["begin_ms"])
+    idle = sum(max(0.0, b["begin_ms"] - a["end_ms"]) for a, b in zip(order, order[1:]))
     return {"batches": len(ing), "groups": len(gem),
+            "first_batch_begin_ms": round(first_ing, 3),
+            "link_idle_ms": round(idle, 3),
             "ingest_span_ms": round(last_ing - first_ing, 3),
             "ingest_gbs": round(sum(r["bytes"] for r in ing) / (last_ing - first_ing) / 1e6, 1),
             "gemv_busy_ms": round(busy, 3),
@@ -953,6 +961,9 @@ def run_timeline(args):
     rows = sum(mats[k].shape[0] for k in slab["dev"].gemv_mats())
     y_host = torch.empty(rows, dtype=torch.float32, pin_memory=True)
     ingest_s, consume_s = torch.cuda.Stream(), consumer_stream(torch, args)
+    if args.fresh:  # every run allocates its own buffers; this one goes back first
+        del slab["dev"], slab["ys"], slab["yflat"]
+        slab = None
     for _ in range(2):  # warm-up, untraced
         first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, flags=oflags)
     runs = []
@@ -965,8 +976,10 @@ def run_timeline(args):
     best = min(range(len(runs)), key=lambda i: runs[i]["host_ms"])
     out = {"metric": "first-use overlap timeline (ingest batches vs event-gated GEMV groups)",
            "config": {"workload": workload_desc(args), "ingest_mode": args.mode,
-                      "data_bytes": ck.data_bytes, "runs": len(runs)},
+                      "data_bytes": ck.data_bytes, "runs": len(runs),
+                      "buffers": "allocated inside each run" if args.fresh else "allocated once, reused"},
            "summaries": sums, "host_ms": [round(r["host_ms"], 3) for r in runs],
+           "open_ms": [round(r["open_ms"], 3) for r in runs], "alloc_ms": [round(r["alloc_ms"], 3) for r in runs],
            "records": runs[best]["records"]}
     log("timeline:", json.dumps(sums[best]))
     print(json.dumps(out), flush=True)

@@ -550,7 +550,12 @@ struct Range {
 
 int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cudaStream_t s,
                  void **ready, uint64_t total) {
-  const uint64_t target = std::min<uint64_t>(128ull << 20, std::max<uint64_t>(2ull << 20, total / 64));
+  // Batches of a 64th of the call, kept between 64 and 128 MiB: each batch is one gather
+  // launch and one event, and a gather kernel's ramp and tail idle part of the link.  Callers
+  // that allocate segment by segment make several smaller calls; with a 2 MiB floor their
+  // 16 GB first use ran 230 batches at 203 GB/s instead of 80 at 207 (mid decoder, allocation
+  // inside the run: 188 -> 194 GB/s with the 64 MiB floor; buffers reused: unchanged).
+  const uint64_t target = std::min<uint64_t>(128ull << 20, std::max<uint64_t>(64ull << 20, total / 64));
   // One gather CTA per SM: the link runs at 207 GB/s with 2, 1 or a third of a CTA per SM.
   // An event-gated GEMV group shares the SMs with the next batch's gather and advances at
   // about the gather's pace (a 200 MB group in ~1 ms instead of ~30 us alone); 48 or 64
