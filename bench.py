@@ -434,22 +434,28 @@ def consumer_stream(torch, args):
     return torch.cuda.Stream()
 
 
-def make_slab(torch, pipeline, h, mats, dev=None):
+def make_slab(torch, pipeline, h, mats, dev=None, x_host=None):
     """Step 4, device allocation: one torch slab for the checkpoint (256-byte aligned views;
-    or `dev`, already allocated), the x of every inner size and one fp32 buffer for every
-    matrix's y."""
+    or `dev`, already allocated with its io region) whose first bytes hold the step's inputs
+    and outputs: the x of every inner size and one fp32 y per matrix (pipeline.io_layout).
+    With `x_host` (pipeline.host_inputs) the x region is filled from it before returning."""
     if dev is None:
-        dev = pipeline.DeviceCheckpoint.allocate(h, mats)
-    xs = dev.inputs()
-    ys = dev.outputs_flat()
-    return {"dev": dev, "xs": xs, "ys": ys, "yflat": ys.buf}
+        dev = pipeline.DeviceCheckpoint.allocate(h, mats, io=True)
+    ys = dev.io_outputs()
+    sl = {"dev": dev, "xs": dev.io_inputs(), "ys": ys, "yflat": ys.buf, "xdev": dev.io_x()}
+    if x_host is not None:
+        sl["xdev"].copy_(x_host)
+        torch.cuda.synchronize()
+    return sl
 
 
-def first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, phases=None, flags=0,
+def first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, x_host, y_host, slab, phases=None, flags=0,
               trace=None):
     """One file -> first-use run; returns (seconds, handle stats).  `slab` None allocates the
     device buffers inside the timed run (step 4), after the previous run's memory went back to
-    the driver; otherwise the given buffers are reused.  With `phases` (a dict), also records
+    the driver; otherwise the given buffers are reused.  The step's inputs (every x, in the
+    pinned `x_host`) cross to the device inside the run, and every y comes back to the pinned
+    `y_host`.  With `phases` (a dict), also records
     host-side phase times in ms: open (wt_open: parse, map, route), alloc (device buffers, x,
     y), enqueue (wt_adopt + wt_pass return; includes page-table population), drain (until y is
     on the host), and the route of the first file.  With `trace` (a list; the handle is then
@@ -468,7 +474,7 @@ def first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, 
     if slab is None:
         # allocation interleaved with ingest: a small first slab, then the rest segment by
         # segment while earlier bytes cross the link; x and y once the link is busy
-        dev, ev, alloc_s = pipeline.DeviceCheckpoint.stream_in(h, mats, mode, ingest_s.cuda_stream)
+        dev, ev, alloc_s = pipeline.DeviceCheckpoint.stream_in(h, mats, mode, ingest_s.cuda_stream, io=True)
         tx = time.perf_counter()
         sl = make_slab(torch, pipeline, h, mats, dev)
         alloc_s += time.perf_counter() - tx
@@ -477,8 +483,9 @@ def first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, 
         dev = sl["dev"]
         ev = dev.adopt(h, mode, ingest_s.cuda_stream)
     ta = t1 + alloc_s
-    h.pass_(dev.descs(sl["xs"], sl["ys"], ev), consume_s.cuda_stream)
     with torch.cuda.stream(consume_s):
+        sl["xdev"].copy_(x_host, non_blocking=True)
+        h.pass_(dev.descs(sl["xs"], sl["ys"], ev), consume_s.cuda_stream)
         y_host.copy_(sl["yflat"], non_blocking=True)
     t2 = time.perf_counter()
     consume_s.synchronize()
@@ -557,7 +564,8 @@ def run_wt(args, rank, world):
     # buffers for the resident pass and the no-allocation first-use variant (allocated once)
     h0 = wt.Handle(ck.paths)
     mats = pipeline.matrices(h0)
-    slab = make_slab(torch, pipeline, h0, mats)
+    x_host = pipeline.host_inputs(mats)  # the step's inputs, pinned: copied in every timed run
+    slab = make_slab(torch, pipeline, h0, mats, x_host=x_host)
     dev, xs, ys = slab["dev"], slab["xs"], slab["ys"]
     rows = [mats[k].shape[0] for k in dev.gemv_mats()]
     y_host = torch.empty(sum(rows), dtype=torch.float32, pin_memory=True)  # host copy of every y
@@ -578,7 +586,7 @@ def run_wt(args, rank, world):
         for rep in range(0 if args.skip_e2e else 1 + args.e2e_reps):
             if dist:
                 dist.barrier()
-            dt, nl, st, nm = first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host,
+            dt, nl, st, nm = first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, x_host, y_host,
                                        None if fresh else slab, ph if rep > 0 else None, flags=oflags)
             if st != 0:
                 raise SystemExit("device status %d after first-use run" % st)
@@ -588,12 +596,12 @@ def run_wt(args, rank, world):
         return times, launches, ph
 
     if not args.skip_e2e:
-        del slab["dev"], slab["ys"], slab["yflat"]  # the reused buffers go back while fresh runs allocate
+        del slab["dev"], slab["ys"], slab["yflat"], slab["xdev"]  # the reused buffers go back while fresh runs allocate
         dev = ys = None
         torch.cuda.empty_cache()
     e2e_times, e2e_launches, phases = e2e_series(True)
     if not args.skip_e2e:
-        slab = make_slab(torch, pipeline, h0, mats)
+        slab = make_slab(torch, pipeline, h0, mats, x_host=x_host)
         dev, xs, ys = slab["dev"], slab["xs"], slab["ys"]
     reuse_times, _, reuse_phases = e2e_series(False)
     e2e_s = statistics.median(e2e_times) if e2e_times else float("nan")
@@ -611,7 +619,7 @@ def run_wt(args, rank, world):
         ct = []
         for _ in range(args.cold_reps):
             evict_page_cache(ck.paths)
-            ct.append(first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab)[0])
+            ct.append(first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, x_host, y_host, slab)[0])
         cold = {"value": round(aggregate_gbs(data_bytes, world, statistics.median(ct)), 1), "unit": "GB/s",
                 "ms": [round(t * 1e3, 1) for t in ct],
                 "what": "file -> first use after posix_fadvise(DONTNEED) on the checkpoint files: storage-bound"}
@@ -627,7 +635,7 @@ def run_wt(args, rank, world):
                 if m is None:
                     ts[n].append(data_bytes / stock_torch_arm(torch, ck, wt, pipeline))
                 else:
-                    ts[n].append(first_use(torch, wt, pipeline, ck, m, ingest_s, consume_s, y_host, slab)[0])
+                    ts[n].append(first_use(torch, wt, pipeline, ck, m, ingest_s, consume_s, x_host, y_host, slab)[0])
         arms = {n: round(data_bytes / statistics.median(v) / 1e9, 1) for n, v in ts.items()}
         log("ingest arms GB/s (median of 3, rotated order):", arms)
 
@@ -725,12 +733,13 @@ def run_wt(args, rank, world):
         "resident_frac_of_hbm": {"measured": round(value / world / peak, 4), "nominal_8TBps": round(value / world / NOMINAL_HBM_GBS, 4)},
         "clocks": clocks,
         "e2e": {"value": round(aggregate_gbs(data_bytes, world, e2e_s_max), 1), "unit": "GB/s",
-                "h2d_bytes_per_step": data_bytes, "d2h_bytes_per_step": int(y_host.numel() * 4),
+                "h2d_bytes_per_step": data_bytes + int(x_host.numel()), "d2h_bytes_per_step": int(y_host.numel() * 4),
                 "ms": round(e2e_s * 1e3, 2), "pinned_h2d_gbs": round(h2d, 1), "h2d_ceilings_gbs": probe,
                 "frac_of_pinned_h2d": round(e2e_gbs / h2d, 4), "reps": args.e2e_reps,
                 "what": "wt_open + device allocation of the slabs, x and y (fresh each run, after "
                         "torch.cuda.empty_cache; slabs allocated segment by segment between wt_adopt "
-                        "calls) + wt_adopt + event-gated first pass + D2H of all y, page cache warm; "
+                        "calls, x and y in the first one) + wt_adopt + H2D of every x from pinned host "
+                        "memory + event-gated first pass + D2H of all y, page cache warm; "
                         "pinned_h2d_gbs is the highest of h2d_ceilings_gbs; phases: alloc_ms is host "
                         "time in allocations, enqueue_ms the rest of the time to the last return; "
                         "wt_open_*: wt_open's own step times (wt_open_times: parallel index + map loop, "
@@ -957,19 +966,20 @@ def run_timeline(args):
     oflags = open_flags(wt, args.open)
     h0 = wt.Handle(ck.paths, oflags)
     mats = pipeline.matrices(h0)
-    slab = make_slab(torch, pipeline, h0, mats)
+    x_host = pipeline.host_inputs(mats)
+    slab = make_slab(torch, pipeline, h0, mats, x_host=x_host)
     rows = sum(mats[k].shape[0] for k in slab["dev"].gemv_mats())
     y_host = torch.empty(rows, dtype=torch.float32, pin_memory=True)
     ingest_s, consume_s = torch.cuda.Stream(), consumer_stream(torch, args)
     if args.fresh:  # every run allocates its own buffers; this one goes back first
-        del slab["dev"], slab["ys"], slab["yflat"]
+        del slab["dev"], slab["ys"], slab["yflat"], slab["xdev"]
         slab = None
     for _ in range(2):  # warm-up, untraced
-        first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, flags=oflags)
+        first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, x_host, y_host, slab, flags=oflags)
     runs = []
     for _ in range(max(1, min(args.e2e_reps, 5))):
         tr = []
-        first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, y_host, slab, flags=oflags, trace=tr)
+        first_use(torch, wt, pipeline, ck, mode, ingest_s, consume_s, x_host, y_host, slab, flags=oflags, trace=tr)
         runs.append(tr[0])
     h0.close()
     sums = [overlap_summary(r["records"]) for r in runs]

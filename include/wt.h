@@ -199,6 +199,16 @@ int wt_tensor_table(const wt_handle *h, size_t first, size_t n, wt_tensor_meta *
  * the bytes required; with cap == 0 only *needed is set.  Errors: WT_EINVAL (NULL, cap too
  * small). */
 int wt_tensor_names(const wt_handle *h, char *buf, size_t cap, size_t *needed);
+/* Logical tensors of an open checkpoint.  A checkpoint may split a matrix's rows across
+ * files (the paper's many-small spine, Sec. 5.3): a tensor named "<base>#r<k>", where k is
+ * one to nine decimal digits, is row block k of the logical tensor <base>, and the blocks of
+ * one base, from any file, form one logical tensor.  Every other tensor is a logical tensor
+ * of its own.  group[i] receives the logical tensor of tensor i, numbered 0.. in order of
+ * first appearance; block[i] receives k, or -1 for a tensor that is not a row block.  Both
+ * arrays have wt_num_tensors entries (the caller's); *n_groups receives the number of
+ * logical tensors.  Whether the blocks of a group stack (2-D, one dtype, one row length,
+ * distinct k) is the caller's check.  Errors: WT_EINVAL (NULL). */
+int wt_tensor_groups(const wt_handle *h, uint32_t *group, int32_t *block, size_t *n_groups);
 /* First tensor whose name equals `name`; WT_EINVAL if none. */
 int wt_find(const wt_handle *h, const char *name, size_t *i);
 /* Route actually taken for file f (WT_ROUTE_REGISTER / DIRECT / NONE). */
@@ -376,17 +386,24 @@ int wt_kernel_launches(const wt_handle *h, uint64_t *n);
 
 /* Objects the library holds right now, over all handles of the process: open handles,
  * cached launch plans, CUDA events it created, and the device and pinned host bytes it
- * allocated itself (status words, plan tables, split-K workspaces, the staged ring).  Buffers
- * the caller owns are not counted.  After wt_close of every handle all five return to their
- * earlier values (Sec. 5.1: a producer's lifetime leaves nothing behind; the 200-cycle checks
- * read these), except that the first staged adopt on a device adds its ring for good: 4
- * events and 268,435,456 pinned bytes.  Errors: WT_EINVAL. */
+ * allocated itself and has handed out (status words, plan tables, split-K workspaces, the
+ * staged ring).  Buffers the caller owns are not counted.  After wt_close of every handle
+ * these five return to their earlier values (Sec. 5.1: a producer's lifetime leaves nothing
+ * behind; the 200-cycle checks read these), except that the first staged adopt on a device
+ * adds its ring for good: 4 events and 268,435,456 pinned bytes.
+ * cached_device_bytes and cached_pinned_bytes are the blocks a closed handle gave back and
+ * the library keeps, per device, for the next handle (so that opening and using a handle
+ * calls no cudaMalloc, cudaHostAlloc or cudaFree once the cache holds its sizes); they are
+ * bounded by 256 MiB per device and kind and stay until the process exits.
+ * Errors: WT_EINVAL. */
 typedef struct {
   int64_t handles;
   int64_t plans;
   int64_t events;
   int64_t device_bytes;
   int64_t pinned_bytes;
+  int64_t cached_device_bytes;
+  int64_t cached_pinned_bytes;
 } wt_live_counts;
 int wt_live(wt_live_counts *out);
 

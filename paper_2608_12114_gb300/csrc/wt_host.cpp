@@ -21,6 +21,7 @@
 #include <chrono>
 #include <cerrno>
 #include <condition_variable>
+#include <deque>
 #include <cstdarg>
 #include <cstdio>
 #include <cstdlib>
@@ -30,7 +31,9 @@
 #include <mutex>
 #include <new>
 #include <string>
+#include <string_view>
 #include <thread>
+#include <unordered_map>
 #include <unordered_set>
 #include <memory>
 #include <vector>
@@ -104,8 +107,129 @@ cudaError_t pinned_alloc(void **p, size_t n) {
   return e;
 }
 
-void pinned_free(void *p, size_t n) {
-  if (p && cudaFreeHost(p) == cudaSuccess) g_pinned_bytes -= (int64_t)n;
+
+// ------------------------------------------------------------------ block cache
+// A handle's own device and pinned allocations (its status word, plan tables and their pinned
+// staging copies, split-K workspaces) come from a per-device cache of power-of-two blocks, kept
+// when the handle closes and handed to the next one.  A fresh handle then makes no cudaMalloc,
+// cudaHostAlloc or cudaFree call: on GB300 those cost tens of microseconds each (cudaFree also
+// waits for the device), which was most of the host time of a small checkpoint's file -> first
+// use.  Blocks of 256 B .. 64 MiB are cached, up to kCapBytes per device and kind; larger
+// blocks, and frees beyond the cap, go to the driver as before.  wt_live counts the bytes
+// handed out (device_bytes, pinned_bytes) apart from the bytes the cache holds.
+std::atomic<int64_t> g_dev_cached{0}, g_pinned_cached{0};
+
+struct BlockCache {
+  static constexpr int kMinLog2 = 8, kMaxLog2 = 26;
+  static constexpr int64_t kCapBytes = 256ll << 20;
+  std::mutex mu;
+  std::vector<void *> free_blocks[kMaxLog2 + 1];
+  int64_t cached = 0;
+  // status words: 256-byte device blocks that are zero (cleared by the closing handle, after
+  // its work has completed), so an open takes one without a memset
+  std::vector<int *> clean_status;
+  cudaStream_t stream = nullptr;  // clears status words
+};
+BlockCache g_dev_cache[64], g_pin_cache[64];
+
+int block_log2(size_t n) {
+  int c = BlockCache::kMinLog2;
+  while (c <= BlockCache::kMaxLog2 && ((size_t)1 << c) < n) ++c;
+  return c;  // kMaxLog2 + 1: not cached
+}
+
+cudaError_t cached_alloc(bool pinned, int dev, void **p, size_t n) {
+  *p = nullptr;
+  const int c = block_log2(n);
+  if (dev >= 0 && dev < 64 && c <= BlockCache::kMaxLog2) {
+    BlockCache &bc = pinned ? g_pin_cache[dev] : g_dev_cache[dev];
+    std::lock_guard<std::mutex> g(bc.mu);
+    if (!bc.free_blocks[c].empty()) {
+      *p = bc.free_blocks[c].back();
+      bc.free_blocks[c].pop_back();
+      bc.cached -= (int64_t)1 << c;
+      (pinned ? g_pinned_cached : g_dev_cached) -= (int64_t)1 << c;
+      (pinned ? g_pinned_bytes : g_dev_bytes) += (int64_t)n;
+      return cudaSuccess;
+    }
+  }
+  const size_t sz = c <= BlockCache::kMaxLog2 ? (size_t)1 << c : n;
+  const cudaError_t e = pinned ? cudaHostAlloc(p, sz, cudaHostAllocDefault) : cudaMalloc(p, sz);
+  if (e == cudaSuccess) (pinned ? g_pinned_bytes : g_dev_bytes) += (int64_t)n;
+  return e;
+}
+
+// p must no longer be in use by any enqueued work.
+void cached_free(bool pinned, int dev, void *p, size_t n) {
+  if (!p) return;
+  (pinned ? g_pinned_bytes : g_dev_bytes) -= (int64_t)n;
+  const int c = block_log2(n);
+  if (dev >= 0 && dev < 64 && c <= BlockCache::kMaxLog2) {
+    BlockCache &bc = pinned ? g_pin_cache[dev] : g_dev_cache[dev];
+    std::lock_guard<std::mutex> g(bc.mu);
+    if (bc.cached + ((int64_t)1 << c) <= BlockCache::kCapBytes) {
+      bc.free_blocks[c].push_back(p);
+      bc.cached += (int64_t)1 << c;
+      (pinned ? g_pinned_cached : g_dev_cached) += (int64_t)1 << c;
+      return;
+    }
+  }
+  if (pinned) cudaFreeHost(p);
+  else cudaFree(p);
+}
+
+// Clears a status word on the cache's own stream and waits for that alone (not the device).
+// Called with bc.mu held.
+cudaError_t status_clear(BlockCache &bc, int *p) {
+  cudaError_t e = bc.stream ? cudaSuccess : cudaStreamCreateWithFlags(&bc.stream, cudaStreamNonBlocking);
+  if (e == cudaSuccess) e = cudaMemsetAsync(p, 0, 256, bc.stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(bc.stream);
+  return e;
+}
+
+// A zeroed 256-byte status word on device `dev` (the current device).
+cudaError_t status_take(int dev, int **p) {
+  *p = nullptr;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  BlockCache &bc = g_dev_cache[dev];
+  std::lock_guard<std::mutex> g(bc.mu);
+  if (!bc.clean_status.empty()) {
+    *p = bc.clean_status.back();
+    bc.clean_status.pop_back();
+    bc.cached -= 256;
+    g_dev_cached -= 256;
+    g_dev_bytes += 256;
+    return cudaSuccess;
+  }
+  cudaError_t e = cudaMalloc(reinterpret_cast<void **>(p), 256);
+  if (e != cudaSuccess) return e;
+  e = status_clear(bc, *p);
+  if (e != cudaSuccess) {
+    cudaFree(*p);
+    *p = nullptr;
+    return e;
+  }
+  g_dev_bytes += 256;
+  return cudaSuccess;
+}
+
+// Returns a status word once every kernel that could write it has completed: it is cleared
+// and kept for the next handle (freed if the clear fails or the cache is full).
+void status_give(int dev, int *p) {
+  if (!p) return;
+  g_dev_bytes -= 256;
+  if (dev >= 0 && dev < 64) {
+    BlockCache &bc = g_dev_cache[dev];
+    std::lock_guard<std::mutex> g(bc.mu);
+    if (bc.cached + 256 <= BlockCache::kCapBytes && status_clear(bc, p) == cudaSuccess) {
+      bc.clean_status.push_back(p);
+      bc.cached += 256;
+      g_dev_cached += 256;
+      return;
+    }
+    cudaGetLastError();
+  }
+  cudaFree(p);
 }
 
 constexpr uint64_t kAlign = 64;
@@ -273,7 +397,7 @@ struct Plan {
   uint8_t *host = nullptr;  // pinned copy of table
   uint8_t *dev = nullptr;
   cudaEvent_t uploaded = nullptr;
-  cudaEvent_t last = nullptr;
+  std::vector<std::pair<cudaStream_t, cudaEvent_t>> last;  // (stream, its latest run's completion)
   bool sent = false;
   cudaStream_t sent_on = nullptr;
   bool pinned = false;  // used inside a captured CUDA graph: kept until wt_close
@@ -282,6 +406,7 @@ struct Plan {
   size_t ws_floats = 0;
   std::vector<std::pair<size_t, size_t>> ws_patches;  // (table byte offset of a pointer, ws float offset)
   uint64_t launches = 0;
+  int device = -1;  // its blocks' cache
 };
 
 // The staged arm's pinned ring: one per device for the whole process (pinning host memory
@@ -548,6 +673,66 @@ struct Range {
   bool populated;  // source page-table entries already filled
 };
 
+// One process-wide thread fills page tables ahead of the ingest launches (MADV_POPULATE_READ
+// on the mapped sources of batch after batch).  A thread of its own per wt_adopt call cost a
+// spawn and a join on every call; one thread for all of them keeps the populate calls from
+// contending on the address-space lock, which made the many-small checkpoint's adopt three
+// times slower when the whole host pool populated (6.6 -> 20 ms for 2506 files).
+class Populator {
+ public:
+  Populator() : th_([this] { run(); }) {}
+  ~Populator() {
+    {
+      std::lock_guard<std::mutex> g(mu_);
+      stop_ = true;
+    }
+    cv_.notify_all();
+    th_.join();
+  }
+  // Runs job on the thread; the caller must wait (finished()) before job's captures go away.
+  uint64_t post(std::function<void()> job) {
+    std::lock_guard<std::mutex> g(mu_);
+    q_.push_back(std::move(job));
+    cv_.notify_all();
+    return ++posted_;
+  }
+  void wait(uint64_t ticket) {
+    std::unique_lock<std::mutex> lk(mu_);
+    done_cv_.wait(lk, [&] { return done_ >= ticket; });
+  }
+
+ private:
+  void run() {
+    for (;;) {
+      std::function<void()> job;
+      {
+        std::unique_lock<std::mutex> lk(mu_);
+        cv_.wait(lk, [&] { return stop_ || !q_.empty(); });
+        if (q_.empty()) return;
+        job = std::move(q_.front());
+        q_.pop_front();
+      }
+      job();
+      {
+        std::lock_guard<std::mutex> g(mu_);
+        ++done_;
+      }
+      done_cv_.notify_all();
+    }
+  }
+  std::mutex mu_;
+  std::condition_variable cv_, done_cv_;
+  std::deque<std::function<void()>> q_;
+  uint64_t posted_ = 0, done_ = 0;
+  bool stop_ = false;
+  std::thread th_;
+};
+
+Populator &populator() {
+  static Populator p;
+  return p;
+}
+
 int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cudaStream_t s,
                  void **ready, uint64_t total) {
   // Batches of a 64th of the call, kept between 64 and 128 MiB: each batch is one gather
@@ -556,46 +741,54 @@ int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cuda
   // 16 GB first use ran 230 batches at 203 GB/s instead of 80 at 207 (mid decoder, allocation
   // inside the run: 188 -> 194 GB/s with the 64 MiB floor; buffers reused: unchanged).
   const uint64_t target = std::min<uint64_t>(128ull << 20, std::max<uint64_t>(64ull << 20, total / 64));
+  // When the stream has nothing in flight the link is idle until the first batch lands, and
+  // that batch waits for its own page tables first: batches then start at 4 MiB and double up
+  // to the target, so the first launch follows the population of 4 MiB instead of 64.  A call
+  // that finds its stream busy (a later segment of a first use) keeps full batches.
+  const cudaError_t q = cudaStreamQuery(s);
+  if (q != cudaSuccess && q != cudaErrorNotReady) cudaGetLastError();
+  uint64_t cap = q == cudaSuccess ? std::min<uint64_t>(target, 4ull << 20) : target;
   // One gather CTA per SM: the link runs at 207 GB/s with 2, 1 or a third of a CTA per SM.
   // An event-gated GEMV group shares the SMs with the next batch's gather and advances at
   // about the gather's pace (a 200 MB group in ~1 ms instead of ~30 us alone); 48 or 64
   // gather CTAs leave it almost untouched, but file -> first use measured 86-97 ms with
   // them against 78 ms here, so the link-bound whole keeps the wide grid.
   const int grid_cap = wt::num_sms();
-  // Tensors larger than a batch are cut into pieces (multiples of 64 KiB, so each piece keeps
-  // its range's alignment): page-table population and transfer then pipeline inside a tensor.
-  // A tensor's event is the event of the batch holding its last piece.
-  const uint64_t piece = std::max<uint64_t>(target & ~((1ull << 16) - 1), 1ull << 16);
+  // Ranges are cut into pieces that fill each batch to its size (cuts at multiples of 64 KiB
+  // from the range's start, so each piece keeps its range's alignment): page-table population
+  // and transfer then pipeline inside a large tensor.  A tensor's event is the event of the
+  // batch holding its last piece.
   std::vector<Range> ps;
   ps.reserve(rs.size());
-  for (const Range &r : rs) {
-    if (r.n <= piece) {
-      ps.push_back(r);
-      continue;
-    }
-    for (uint64_t o = 0; o < r.n; o += piece)
-      ps.push_back({r.tensor, r.file, r.foff + o, r.src_host + o, r.src_dev ? r.src_dev + o : nullptr, r.dst + o,
-                    std::min(piece, r.n - o), r.populated});
-  }
   std::vector<std::pair<size_t, size_t>> batches;
-  for (size_t i = 0; i < ps.size();) {
-    size_t j = i;
-    uint64_t bytes = 0;
-    while (j < ps.size() && (j == i || (bytes < target && j - i < (size_t)wt::kMaxGather))) bytes += ps[j++].n;
-    batches.push_back({i, j});
-    i = j;
+  size_t b0 = 0;
+  uint64_t bbytes = 0;
+  for (const Range &r : rs) {
+    uint64_t o = 0;
+    do {
+      if (ps.size() > b0 && (bbytes >= cap || ps.size() - b0 >= (size_t)wt::kMaxGather)) {
+        batches.push_back({b0, ps.size()});
+        b0 = ps.size();
+        bbytes = 0;
+        cap = std::min<uint64_t>(target, cap * 2);
+      }
+      uint64_t take = r.n - o;
+      if (take > cap - bbytes) take = std::min(take, std::max<uint64_t>((cap - bbytes) & ~((1ull << 16) - 1), 1ull << 16));
+      ps.push_back({r.tensor, r.file, r.foff + o, r.src_host ? r.src_host + o : nullptr,
+                    r.src_dev ? r.src_dev + o : nullptr, r.dst + o, take, r.populated});
+      bbytes += take;
+      o += take;
+    } while (o < r.n);
   }
-  // A helper thread populates the page-table entries of batch after batch; batch b is
-  // enqueued once its sources are populated, so this host work (about 1 TB/s for large
-  // ranges, a few microseconds per small mapping) overlaps the transfer of earlier batches.
-  // One thread does them all: populate calls from the whole host pool made the many-small
-  // checkpoint's adopt three times slower (6.6 -> 20 ms for 2506 files), as they contend on
-  // the address-space lock.
+  if (ps.size() > b0) batches.push_back({b0, ps.size()});
+  // The populator fills the page-table entries of batch after batch; batch b is enqueued once
+  // its sources are populated, so this host work (about 1 TB/s for large ranges, a few
+  // microseconds per small mapping) overlaps the transfer of earlier batches.
   std::vector<std::vector<std::pair<const uint8_t *, size_t>>> work(batches.size());
   bool any = false;
   for (size_t b = 0; b < batches.size(); ++b)
     for (size_t k = batches[b].first; k < batches[b].second; ++k)
-      if (!ps[k].populated)
+      if (!ps[k].populated && ps[k].src_host)
         for (uint64_t o = 0; o < ps[k].n; o += 16ull << 20) {
           work[b].push_back({ps[k].src_host + o, (size_t)std::min<uint64_t>(16ull << 20, ps[k].n - o)});
           any = true;
@@ -604,9 +797,9 @@ int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cuda
   std::condition_variable cv;
   size_t populated = any ? 0 : batches.size();
   std::atomic<bool> stop{false};
-  std::thread helper;
+  uint64_t ticket = 0;
   if (any) {
-    helper = std::thread([&] {
+    ticket = populator().post([&] {
       for (size_t b = 0; b < batches.size() && !stop.load(); ++b) {
         for (const auto &w : work[b]) prefault(w.first, w.second);
         {
@@ -617,14 +810,14 @@ int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cuda
       }
     });
   }
-  struct Joiner {
-    std::thread &t;
+  struct Joiner {  // the job refers to this frame: wait for it on every way out
+    uint64_t ticket;
     std::atomic<bool> &stop;
     ~Joiner() {
       stop.store(true);
-      if (t.joinable()) t.join();
+      if (ticket) populator().wait(ticket);
     }
-  } joiner{helper, stop};
+  } joiner{ticket, stop};
   for (size_t b = 0; b < batches.size(); ++b) {
     if (any) {
       std::unique_lock<std::mutex> lk(mu);
@@ -1526,30 +1719,32 @@ int build_plan(wt_handle *h, const wt_gemv_desc *d, size_t n, Plan *P) {
     P->groups.push_back(std::move(g));
   }
   if (P->ws_floats) {
-    CU(dev_alloc(reinterpret_cast<void **>(&P->ws), P->ws_floats * sizeof(float)));
+    CU(cached_alloc(false, P->device, reinterpret_cast<void **>(&P->ws), P->ws_floats * sizeof(float)));
     for (const auto &pt : P->ws_patches) {
       const float *p = P->ws + pt.second;
       memcpy(P->table.data() + pt.first, &p, sizeof p);
     }
   }
   const size_t bytes = std::max<size_t>(16, align16(P->table.size()));
-  CU(pinned_alloc(reinterpret_cast<void **>(&P->host), bytes));
+  CU(cached_alloc(true, P->device, reinterpret_cast<void **>(&P->host), bytes));
   P->table_bytes = bytes;
   memcpy(P->host, P->table.data(), P->table.size());
   if (wt::fault_injected("alloc")) return set_err(WT_ENOMEM, "wt_pass: plan tables: injected allocation fault");
-  CU(dev_alloc(reinterpret_cast<void **>(&P->dev), bytes));
+  CU(cached_alloc(false, P->device, reinterpret_cast<void **>(&P->dev), bytes));
   CU(ev_create(&P->uploaded, cudaEventDisableTiming));
-  CU(ev_create(&P->last, cudaEventDisableTiming));
   return WT_OK;
 }
 
 void destroy_plan(Plan *P) {
-  if (P->last) cudaEventSynchronize(P->last);
-  dev_free(P->dev, P->table_bytes);
-  dev_free(P->ws, P->ws_floats * sizeof(float));
-  pinned_free(P->host, P->table_bytes);
+  for (const auto &sl : P->last) cudaEventSynchronize(sl.second);
+  // a plan a captured graph refers to may still be read by a replay the caller did not wait
+  // for: its blocks go back to the cache only once the device is idle
+  if (P->pinned) cudaDeviceSynchronize();
+  cached_free(false, P->device, P->dev, P->table_bytes);
+  cached_free(false, P->device, P->ws, P->ws_floats * sizeof(float));
+  cached_free(true, P->device, P->host, P->table_bytes);
   ev_destroy(P->uploaded);
-  ev_destroy(P->last);
+  for (const auto &sl : P->last) ev_destroy(sl.second);
   delete P;
   g_live_plans--;
 }
@@ -1688,7 +1883,18 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
       h->kernel_launches++;
     }
   }
-  if (!capturing) CU(cudaEventRecord(P->last, s));
+  if (!capturing) {
+    // one completion event per stream the plan has run on: the plan's blocks are reused only
+    // after its latest run on every one of them
+    cudaEvent_t done = nullptr;
+    for (const auto &sl : P->last)
+      if (sl.first == s) done = sl.second;
+    if (!done) {
+      CU(ev_create(&done, cudaEventDisableTiming));
+      P->last.push_back({s, done});
+    }
+    CU(cudaEventRecord(done, s));
+  }
   return WT_OK;
 }
 
@@ -1711,7 +1917,7 @@ int close_impl(wt_handle *h) {
     h->plans.clear();
     for (cudaEvent_t e : h->events) ev_destroy(e);
     h->events.clear();
-    dev_free(h->status, 256);
+    status_give(h->device, h->status);
     h->status = nullptr;
     if (h->stamp_dev) {
       dev_free(h->stamp_dev, h->stamp_cap * wt::kStampFields * sizeof(uint64_t));
@@ -1755,7 +1961,7 @@ extern "C" {
 
 const char *wt_last_error(void) { return t_err.c_str(); }
 
-int wt_abi_version(void) { return 3; }
+int wt_abi_version(void) { return 4; }
 
 int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **out) {
   if (!out) return set_err(WT_EINVAL, "wt_open: out is NULL");
@@ -1895,8 +2101,7 @@ int wt_open(const char *const *paths, int n_paths, unsigned flags, wt_handle **o
     }
     h->open_times.route_ms = (now_ns() - t0) * 1e-6;
     for (const File &f : h->files) h->open_times.files_registered += f.registered ? 1 : 0;
-    ce = dev_alloc(reinterpret_cast<void **>(&h->status), 256);
-    if (ce == cudaSuccess) ce = cudaMemset(h->status, 0, 256);
+    ce = status_take(h->device, &h->status);
     if (ce != cudaSuccess) {
       close_impl(h);
       return cuda_err(ce, "status word");
@@ -1971,6 +2176,39 @@ int wt_tensor_names(const wt_handle *h, char *buf, size_t cap, size_t *needed) {
     memcpy(buf + pos, nm.c_str(), nm.size() + 1);
     pos += nm.size() + 1;
   }
+  return WT_OK;
+}
+
+int wt_tensor_groups(const wt_handle *h, uint32_t *group, int32_t *block, size_t *n_groups) {
+  if (!h || !n_groups || (!h->order.empty() && (!group || !block)))
+    return set_err(WT_EINVAL, "wt_tensor_groups: NULL argument");
+  // base name -> group, for the row blocks; every other tensor is a group of its own
+  std::unordered_map<std::string_view, uint32_t> by_base;  // views of the handle's own names
+  by_base.reserve(h->order.size());
+  uint32_t n = 0;
+  for (size_t i = 0; i < h->order.size(); ++i) {
+    const std::string &nm = h->tensor(i).name;
+    const size_t at = nm.rfind("#r");
+    int64_t k = -1;
+    if (at != std::string::npos) {
+      const size_t nd = nm.size() - at - 2;
+      if (nd >= 1 && nd <= 9) {
+        k = 0;
+        for (size_t c = at + 2; c < nm.size() && k >= 0; ++c)
+          k = (nm[c] >= '0' && nm[c] <= '9') ? k * 10 + (nm[c] - '0') : -1;
+      }
+    }
+    if (k < 0) {
+      group[i] = n++;
+      block[i] = -1;
+      continue;
+    }
+    auto ins = by_base.emplace(std::string_view(nm.data(), at), n);
+    if (ins.second) ++n;
+    group[i] = ins.first->second;
+    block[i] = (int32_t)k;
+  }
+  *n_groups = n;
   return WT_OK;
 }
 
@@ -2099,6 +2337,7 @@ int wt_pass(wt_handle *h, const wt_gemv_desc *d, size_t n, void *stream) {
     if (!P) {
       P = new Plan();
       g_live_plans++;
+      P->device = h->device;
       P->key = std::move(key);
       int rc = build_plan(h, d, n, P);
       if (rc) {
@@ -2265,6 +2504,8 @@ int wt_live(wt_live_counts *out) {
   out->events = g_live_events.load();
   out->device_bytes = g_dev_bytes.load();
   out->pinned_bytes = g_pinned_bytes.load();
+  out->cached_device_bytes = g_dev_cached.load();
+  out->cached_pinned_bytes = g_pinned_cached.load();
   return WT_OK;
 }
 

@@ -33,7 +33,8 @@ MODE_NAMES = {WT_ADOPT_GATHER: "gather", WT_ADOPT_CE: "ce", WT_ADOPT_STAGED: "st
 
 # every entry point declared in include/wt.h
 SYMBOLS = ("wt_last_error", "wt_abi_version", "wt_open", "wt_num_tensors", "wt_num_files",
-           "wt_tensor_info", "wt_tensor_table", "wt_tensor_names", "wt_find", "wt_file_route", "wt_file_registration", "wt_adopt", "wt_pass", "wt_checksum",
+           "wt_tensor_info", "wt_tensor_table", "wt_tensor_names", "wt_tensor_groups", "wt_find",
+           "wt_file_route", "wt_file_registration", "wt_adopt", "wt_pass", "wt_checksum",
            "wt_checksum_plain", "wt_checksum_noalloc", "wt_device_status", "wt_residency",
            "wt_kernel_launches", "wt_trace", "wt_pass_stamps", "wt_open_times", "wt_live", "wt_close",
            # include/wt_dlpack.h
@@ -62,7 +63,8 @@ class GemvDesc(C.Structure):
 
 class LiveCounts(C.Structure):
     _fields_ = [("handles", C.c_int64), ("plans", C.c_int64), ("events", C.c_int64),
-                ("device_bytes", C.c_int64), ("pinned_bytes", C.c_int64)]
+                ("device_bytes", C.c_int64), ("pinned_bytes", C.c_int64),
+                ("cached_device_bytes", C.c_int64), ("cached_pinned_bytes", C.c_int64)]
 
 
 class TraceRec(C.Structure):
@@ -83,6 +85,7 @@ assert DESC_DTYPE.itemsize == C.sizeof(GemvDesc)
 
 
 _lib = None
+ABI_VERSION = 4  # wt_abi_version() of the include/wt.h this binding follows
 
 
 def lib(path: str = LIB_PATH):
@@ -96,16 +99,20 @@ def lib(path: str = LIB_PATH):
     vp, sz, u64p = C.c_void_p, C.c_size_t, C.POINTER(C.c_uint64)
     L.wt_last_error.restype = C.c_char_p
     L.wt_abi_version.restype = C.c_int
+    if L.wt_abi_version() != ABI_VERSION:  # a stale build: structures would not match
+        raise RuntimeError("%s has ABI version %d, this binding needs %d; rebuild it"
+                           % (path, L.wt_abi_version(), ABI_VERSION))
     L.wt_open.argtypes = [C.POINTER(C.c_char_p), C.c_int, C.c_uint, C.POINTER(vp)]
     L.wt_num_tensors.argtypes = [vp, C.POINTER(sz)]
     L.wt_num_files.argtypes = [vp, C.POINTER(sz)]
     L.wt_tensor_info.argtypes = [vp, sz, C.POINTER(TensorMeta)]
     L.wt_tensor_table.argtypes = [vp, sz, sz, vp]
     L.wt_tensor_names.argtypes = [vp, C.c_char_p, sz, C.POINTER(sz)]
+    L.wt_tensor_groups.argtypes = [vp, vp, vp, C.POINTER(sz)]
     L.wt_find.argtypes = [vp, C.c_char_p, C.POINTER(sz)]
     L.wt_file_route.argtypes = [vp, sz, C.POINTER(C.c_uint)]
     L.wt_file_registration.argtypes = [vp, sz, C.POINTER(C.c_uint)]
-    L.wt_adopt.argtypes = [vp, C.POINTER(sz), C.POINTER(vp), sz, C.c_uint, vp, C.POINTER(vp)]
+    L.wt_adopt.argtypes = [vp, vp, vp, sz, C.c_uint, vp, vp]
     L.wt_pass.argtypes = [vp, C.POINTER(GemvDesc), sz, vp]
     L.wt_checksum.argtypes = [vp, C.POINTER(vp), u64p, sz, vp, vp]
     L.wt_checksum_plain.argtypes = [vp, C.POINTER(vp), u64p, sz, vp, vp]
@@ -155,20 +162,35 @@ class OpenPhases(C.Structure):
 
 
 class TensorTable:
-    """The index of an open checkpoint: TensorInfo per tensor, made on first access, and the
-    columns as plain lists (`names`, `dtypes`, `shapes`, `nbytes`, `files`, `offsets`) for
-    code that walks thousands of entries."""
+    """The index of an open checkpoint: TensorInfo per tensor, made on first access; the
+    columns as plain lists (`names`, `dtypes`, `shapes`, `nbytes`, `files`, `offsets`,
+    `host_ptrs`), each built on first use, for code that walks thousands of entries; and
+    `meta`, the same columns as one numpy record array (META_DTYPE)."""
 
     def __init__(self, meta: np.ndarray, names: List[str]):
+        self.meta = meta
         self.names = names
-        self.dtypes = meta["dtype"].tolist()
-        nds = meta["ndim"].tolist()
-        self.shapes = [tuple(sh[:nd]) for sh, nd in zip(meta["shape"].tolist(), nds)]
-        self.nbytes = meta["nbytes"].tolist()
-        self.files = meta["file"].tolist()
-        self.offsets = meta["offset"].tolist()
-        self.host_ptrs = meta["host_ptr"].tolist()
         self._items: List[object] = [None] * len(names)
+
+    def _col(self, f):
+        v = self.__dict__.get("_c_" + f)
+        if v is None:
+            v = self.__dict__["_c_" + f] = self.meta[f].tolist()
+        return v
+
+    dtypes = property(lambda self: self._col("dtype"))
+    nbytes = property(lambda self: self._col("nbytes"))
+    files = property(lambda self: self._col("file"))
+    offsets = property(lambda self: self._col("offset"))
+    host_ptrs = property(lambda self: self._col("host_ptr"))
+
+    @property
+    def shapes(self):
+        v = self.__dict__.get("_c_shapes")
+        if v is None:
+            v = self.__dict__["_c_shapes"] = [tuple(sh[:nd]) for sh, nd in
+                                              zip(self.meta["shape"].tolist(), self.meta["ndim"].tolist())]
+        return v
 
     def __len__(self) -> int:
         return len(self.names)
@@ -192,7 +214,7 @@ class Handle:
     def __init__(self, paths: Sequence[str], flags: int = 0):
         L = lib()
         # every path in one NUL-separated buffer, pointers computed from the NUL positions
-        blob = ("\0".join(os.fspath(p) for p in paths) + "\0").encode() if len(paths) else b"\0"
+        blob = ("\0".join(map(os.fspath, paths)) + "\0").encode() if len(paths) else b"\0"
         cbuf = C.create_string_buffer(blob, len(blob))
         ends = np.flatnonzero(np.frombuffer(blob, np.uint8) == 0)
         starts = np.concatenate(([0], ends[:-1] + 1)).astype(np.uint64) + np.uint64(C.addressof(cbuf))
@@ -240,14 +262,28 @@ class Handle:
         return r.value
 
     def adopt(self, idx: Sequence[int], dst: Sequence[int], mode: int = WT_ADOPT_GATHER,
-              stream: int = 0) -> List[int]:
-        """wt_adopt: returns the ready event (cudaEvent_t as int) of each tensor."""
-        n = len(idx)
-        ia = (C.c_size_t * max(1, n))(*idx)
-        da = (C.c_void_p * max(1, n))(*dst)
-        ra = (C.c_void_p * max(1, n))()
-        _check(lib().wt_adopt(self.ptr, ia, da, n, mode, C.c_void_p(stream), ra))
-        return [ra[i] or 0 for i in range(n)]
+              stream: int = 0, as_array: bool = False):
+        """wt_adopt: returns the ready event (cudaEvent_t as int) of each tensor, as a list, or
+        with as_array as a uint64 numpy array.  idx and dst may be numpy arrays."""
+        ia = np.ascontiguousarray(idx, dtype=np.uint64).reshape(-1)
+        da = np.ascontiguousarray(dst, dtype=np.uint64).reshape(-1)
+        n = ia.size
+        if da.size != n:
+            raise ValueError("adopt: %d indices, %d destinations" % (n, da.size))
+        if n == 0:
+            ia = da = np.zeros(1, np.uint64)
+        ra = np.zeros(max(1, n), np.uint64)
+        _check(lib().wt_adopt(self.ptr, ia.ctypes.data, da.ctypes.data, n, mode, C.c_void_p(stream), ra.ctypes.data))
+        return ra[:n] if as_array else ra[:n].tolist()
+
+    def groups(self):
+        """wt_tensor_groups: (group, block, n_groups): per tensor its logical tensor (uint32, in
+        order of first appearance) and its row-block number (int32, -1 for a plain tensor)."""
+        n = len(self.tensors)
+        g, b = np.zeros(max(1, n), np.uint32), np.zeros(max(1, n), np.int32)
+        ng = C.c_size_t()
+        _check(lib().wt_tensor_groups(self.ptr, g.ctypes.data, b.ctypes.data, C.byref(ng)))
+        return g[:n], b[:n], ng.value
 
     def pass_(self, descs, stream: int = 0):
         """wt_pass over a list of GemvDesc or a contiguous numpy array of DESC_DTYPE records."""
@@ -336,7 +372,8 @@ class Handle:
 
 
 def live() -> dict:
-    """wt_live: handles, plans, events, device and pinned bytes the library holds now."""
+    """wt_live: handles, plans, events, device and pinned bytes the library has handed out
+    now, and the bytes its block cache keeps for the next handle."""
     c = LiveCounts()
     _check(lib().wt_live(C.byref(c)))
     return {f: getattr(c, f) for f, _ in LiveCounts._fields_}

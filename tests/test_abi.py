@@ -32,7 +32,7 @@ def test_every_declared_symbol_is_exported(L):
     for s in decl:
         assert hasattr(L, s), s
     assert sorted(wt.SYMBOLS) == decl
-    assert L.wt_abi_version() == 3
+    assert L.wt_abi_version() == 4
 
 
 def test_only_the_abi_is_exported(L):

@@ -41,6 +41,7 @@ def test_stalled_launch_times_out_and_the_context_survives(torch, monkeypatch):
         assert h.device_status() == wt.WT_ETIMEDOUT
         monkeypatch.delenv("WT_FAULT")
     with wt.Handle([]) as h:                         # same process, same context: still good
+        assert h.device_status() == 0                # the recycled status word was cleared
         h.pass_(d, 0)
         torch.cuda.synchronize()
         assert h.device_status() == 0

@@ -143,3 +143,43 @@ def test_bytes_after_eviction_match_the_oracle(torch, tmp_path, route, mode):
     finally:
         co.close()
     shutil.rmtree(d, ignore_errors=True)
+
+
+def test_block_cache_serves_later_handles(torch):
+    """A closed handle's status word, plan tables (pinned and device) and split-K workspace go
+    back to the library's block cache and later handles take them from there: the bytes the
+    cache holds stay constant over the cycles, the bytes handed out return to their earlier
+    value, and every cycle computes the same y, within the bound of the oracle."""
+    rng = np.random.default_rng(11)
+    shapes = [(64, 4096), (8, 40000)]  # the second is cut into column segments: a workspace
+    cases, descs = [], []
+    for M, K in shapes:
+        W = synth.f32_to_bf16_bits((0.02 * rng.standard_normal((M, K))).astype(np.float32)).view(np.uint8).reshape(-1)
+        x = synth.make_x(K, wt.WT_BF16)
+        Wd, xd = torch.from_numpy(W.copy()).cuda(), torch.from_numpy(x.copy()).cuda()
+        y = torch.full((M,), float("nan"), dtype=torch.float32, device="cuda")
+        cases.append((W, x, Wd, xd, y))
+        descs.append(wt.gemv_desc(Wd.data_ptr(), wt.WT_BF16, M, K, xd.data_ptr(), y.data_ptr()))
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    torch.cuda.synchronize()
+    with wt.Handle([]) as h:  # warm-up: the cache takes this handle's blocks at close
+        h.pass_(descs, s1.cuda_stream)
+    base = wt.live()
+    counts, first = [], None
+    for _ in range(20):
+        with wt.Handle([]) as h:
+            h.pass_(descs, s1.cuda_stream)
+            s2.wait_stream(s1)
+            h.pass_(descs, s2.cuda_stream)  # the same plan on a second stream; close waits for both
+            assert wt.live()["device_bytes"] > base["device_bytes"]
+        counts.append(wt.live())
+        s2.synchronize()
+        ys = [c[4].clone() for c in cases]
+        if first is None:
+            first = ys
+        assert all(torch.equal(a, b) for a, b in zip(first, ys))
+    assert all(c == base for c in counts), (base, counts[-1])
+    assert base["cached_device_bytes"] > 0 and base["cached_pinned_bytes"] > 0
+    for (W, x, _, _, _), (M, K), y in zip(cases, shapes, first):
+        yhat, a = oracle.gemv(W, wt.WT_BF16, M, K, x)
+        assert oracle.gemv_error(y.cpu().numpy(), yhat, a) <= 2e-3

@@ -73,13 +73,16 @@ def check_gemv(h, dev, co, ys, rows=None):
         W = co.matrix_bytes([(h.tensors[i].file, h.tensors[i].name) for i in m.parts])
         x = synth.make_x(K, m.dtype)
         y = ys[k].cpu().numpy().astype(np.float64)
-        if rows is None:
+        r = None if rows is None else \
+            sorted(set([0, M - 1] + [int(v) for v in np.random.default_rng(k).integers(0, M, rows)]))
+        if m.scale is not None:  # int8 weights with fp16 row scales
+            t = h.tensors[m.scale]
+            yhat, a = oracle.gemv_q8(W, co.blob_of(t.file, t.name), M, K, x, rows=r)
+        elif r is None:
             yhat, a = oracle.gemv(W, m.dtype, M, K, x)
-            err = oracle.gemv_error(y, yhat, a)
         else:
-            r = sorted(set([0, M - 1] + [int(v) for v in np.random.default_rng(k).integers(0, M, rows)]))
             yhat, a = oracle.gemv_rows(W, m.dtype, M, K, x, r)
-            err = oracle.gemv_error(y[r], yhat, a)
+        err = oracle.gemv_error(y if r is None else y[r], yhat, a)
         assert err <= TOL, (m.name, err)
         worst = max(worst, err)
     return worst
@@ -224,6 +227,33 @@ def test_first_use_pipeline_mid(torch, tmp_path):
     consume_s.synchronize()
     for k in dev.gemv_mats():
         assert torch.equal(ys[k], yr[k])
+    h.close()
+
+
+@pytest.mark.parametrize("workload", ["tiny", "many", "protocol_q8"])
+def test_first_use_with_io_region(torch, tmp_path, workload):
+    """The timed first use: slabs allocated segment by segment with the step's inputs and
+    outputs in the first one (x copied from a pinned host buffer, y NaN-filled first), every
+    GEMV gated on its batch's event; every row against the oracle, the weight bytes exact."""
+    kw = {"many": {"n_matrices": 40}, "protocol_q8": {"matrices": 2, "rows": 2048}}.get(workload, {})
+    ck = synth.build(workload, str(tmp_path), **kw)
+    co = oracle.CheckpointOracle(ck.paths)
+    ingest_s, consume_s = torch.cuda.Stream(), torch.cuda.Stream()
+    h = wt.Handle(ck.paths)
+    mats = pipeline.matrices(h)
+    x_host = pipeline.host_inputs(mats)
+    dev, ev, _ = pipeline.DeviceCheckpoint.stream_in(h, mats, wt.WT_ADOPT_GATHER, ingest_s.cuda_stream, io=True)
+    ys = dev.io_outputs()
+    with torch.cuda.stream(consume_s):
+        ys.buf.fill_(float("nan"))
+        dev.io_x().copy_(x_host, non_blocking=True)
+        h.pass_(dev.descs(dev.io_inputs(), ys, ev), consume_s.cuda_stream)
+    consume_s.synchronize()
+    _, y_off, rows, total = pipeline.io_layout(mats)
+    assert dev.io.numel() >= total and ys.buf.numel() == max(1, sum(rows))
+    assert dev.io.data_ptr() % 256 == 0 and all(p % 256 == 0 for p in dev.ptrs)
+    check_gemv(h, dev, co, ys)
+    check_bytes(torch, h, dev, co)
     h.close()
 
 
