@@ -799,8 +799,14 @@ int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cuda
   std::atomic<bool> stop{false};
   uint64_t ticket = 0;
   if (any) {
+    // the first batch is populated here, on the calling thread: its launch then waits for no
+    // handoff to the populator and back; the populator starts at the second batch meanwhile
+    for (const auto &w : work[0]) prefault(w.first, w.second);
+    populated = 1;
+  }
+  if (any && batches.size() > 1) {
     ticket = populator().post([&] {
-      for (size_t b = 0; b < batches.size() && !stop.load(); ++b) {
+      for (size_t b = 1; b < batches.size() && !stop.load(); ++b) {
         for (const auto &w : work[b]) prefault(w.first, w.second);
         {
           std::lock_guard<std::mutex> g(mu);

@@ -466,7 +466,7 @@ class DeviceCheckpoint:
         (mapped files on the device route, small unmapped files through the pinned ring on the
         library's own stream) has no tensor event that implies the others: all its tensors get
         one event recorded on `stream` after the call, which follows every byte of it."""
-        if mode == wt.WT_ADOPT_STAGED or b <= a:
+        if mode == wt.WT_ADOPT_STAGED or b <= a or not h.flags & wt.WT_OPEN_MAP_LARGE:
             return
         m = self.mats
         small = h.tensors.meta["host_ptr"] == 0

@@ -223,6 +223,7 @@ class Handle:
         _check(L.wt_open(C.cast(arr.ctypes.data, C.POINTER(C.c_char_p)), len(paths), flags, C.byref(h)))
         del cbuf, arr
         self._h = h
+        self.flags = flags
         n = C.c_size_t()
         _check(L.wt_num_tensors(h, C.byref(n)))
         # two calls for the whole index (metadata table, then every name), not one per tensor
