@@ -739,7 +739,8 @@ def run_wt(args, rank, world):
                 "what": "wt_open + device allocation of the slabs, x and y (fresh each run, after "
                         "torch.cuda.empty_cache; slabs allocated segment by segment between wt_adopt "
                         "calls, x and y in the first one) + wt_adopt + H2D of every x from pinned host "
-                        "memory + event-gated first pass + D2H of all y, page cache warm; "
+                        "memory + event-gated first pass + D2H of all y, page cache warm; the library's "
+                        "own status word and plan tables come from its per-device block cache; "
                         "pinned_h2d_gbs is the highest of h2d_ceilings_gbs; phases: alloc_ms is host "
                         "time in allocations, enqueue_ms the rest of the time to the last return; "
                         "wt_open_*: wt_open's own step times (wt_open_times: parallel index + map loop, "
