@@ -689,7 +689,8 @@ class Populator {
     cv_.notify_all();
     th_.join();
   }
-  // Runs job on the thread; the caller must wait (finished()) before job's captures go away.
+  // Queues job for the thread and returns its ticket; the caller must wait(ticket) before
+  // anything the job refers to goes away.
   uint64_t post(std::function<void()> job) {
     std::lock_guard<std::mutex> g(mu_);
     q_.push_back(std::move(job));
@@ -1891,11 +1892,18 @@ int run_plan(wt_handle *h, Plan *P, const wt_gemv_desc *d, cudaStream_t s, bool 
   }
   if (!capturing) {
     // one completion event per stream the plan has run on: the plan's blocks are reused only
-    // after its latest run on every one of them
+    // after its latest run on every one of them.  Past kPlanStreams streams, the oldest entry
+    // is waited for and taken over, so a caller that cycles through streams holds few events.
+    constexpr size_t kPlanStreams = 8;
     cudaEvent_t done = nullptr;
     for (const auto &sl : P->last)
       if (sl.first == s) done = sl.second;
-    if (!done) {
+    if (!done && P->last.size() >= kPlanStreams) {
+      done = P->last.front().second;
+      CU(cudaEventSynchronize(done));
+      P->last.erase(P->last.begin());
+      P->last.push_back({s, done});
+    } else if (!done) {
       CU(ev_create(&done, cudaEventDisableTiming));
       P->last.push_back({s, done});
     }

@@ -183,3 +183,33 @@ def test_block_cache_serves_later_handles(torch):
     for (W, x, _, _, _), (M, K), y in zip(cases, shapes, first):
         yhat, a = oracle.gemv(W, wt.WT_BF16, M, K, x)
         assert oracle.gemv_error(y.cpu().numpy(), yhat, a) <= 2e-3
+
+
+def test_plan_run_on_many_streams_holds_few_events(torch):
+    """A plan keeps one completion event per stream it ran on, at most eight: a caller that
+    runs one pass on ever-new streams holds a bounded number of events, and closing the handle
+    releases them."""
+    rng = np.random.default_rng(12)
+    M, K = 96, 2048
+    W = synth.f32_to_bf16_bits((0.02 * rng.standard_normal((M, K))).astype(np.float32)).view(np.uint8).reshape(-1)
+    x = synth.make_x(K, wt.WT_BF16)
+    Wd, xd = torch.from_numpy(W.copy()).cuda(), torch.from_numpy(x.copy()).cuda()
+    y = torch.full((M,), float("nan"), dtype=torch.float32, device="cuda")
+    d = [wt.gemv_desc(Wd.data_ptr(), wt.WT_BF16, M, K, xd.data_ptr(), y.data_ptr())]
+    torch.cuda.synchronize()
+    base = wt.live()
+    streams = [torch.cuda.Stream() for _ in range(12)]
+    with wt.Handle([]) as h:
+        prev = None
+        for s in streams:
+            if prev is not None:
+                s.wait_stream(prev)  # one run at a time: they all write the same y
+            h.pass_(d, s.cuda_stream)
+            prev = s
+        live = wt.live()
+        assert live["plans"] == base["plans"] + 1
+        assert live["events"] <= base["events"] + 1 + 8, (base, live)  # the upload event and 8 streams
+    torch.cuda.synchronize()
+    assert wt.live() == base
+    yhat, a = oracle.gemv(W, wt.WT_BF16, M, K, x)
+    assert oracle.gemv_error(y.cpu().numpy(), yhat, a) <= 2e-3
