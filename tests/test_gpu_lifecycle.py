@@ -196,6 +196,8 @@ def test_plan_run_on_many_streams_holds_few_events(torch):
     Wd, xd = torch.from_numpy(W.copy()).cuda(), torch.from_numpy(x.copy()).cuda()
     y = torch.full((M,), float("nan"), dtype=torch.float32, device="cuda")
     d = [wt.gemv_desc(Wd.data_ptr(), wt.WT_BF16, M, K, xd.data_ptr(), y.data_ptr())]
+    with wt.Handle([]) as h:  # warm-up: the block cache takes this plan's blocks at close
+        h.pass_(d, 0)
     torch.cuda.synchronize()
     base = wt.live()
     streams = [torch.cuda.Stream() for _ in range(12)]
