@@ -85,7 +85,7 @@ class Matrices:
         two = (ndim[first] == 2) | self.stacked
         self.dtype = dt[first]
         self.K = np.where(two, shp[first, 1], 0)
-        if ng != n and bool(self.stacked.any()):
+        if bool(self.stacked.any()):
             # row blocks stack: 2-D, one dtype, one row length, distinct block numbers; each
             # part is compared with the first part of its logical tensor
             g_p = group[order]
@@ -136,7 +136,6 @@ class Matrices:
                 blocks = [bi for bi, _ in p]
                 if any(len(shs[i]) != 2 or dts[i] != dts[f] or shs[i][1] != shs[f][1] for i in idx) or \
                         len(set(blocks)) != len(blocks):
-                    self._names = T.names
                     raise ValueError("row blocks of %s do not stack" % T.names[f].rpartition("#r")[0])
             t2 = st or len(shs[f]) == 2
             order += idx
@@ -157,6 +156,7 @@ class Matrices:
         self.scale = np.full(ng, -1, np.int64)
         self._find_scales([k for k in range(ng) if two[k] and dtype[k] == wt.WT_I8 and ptr[k + 1] - ptr[k] == 1])
         self.gemv_idx = np.flatnonzero(self.gemv)
+
     def __len__(self) -> int:
         return len(self.part_ptr) - 1
 

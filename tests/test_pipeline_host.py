@@ -70,8 +70,10 @@ def test_matrices_columns_match_the_reference_grouping(tmp_path):
         assert got[0] == ("w", (6, 8), [5, 0, 8], True, None) and ("q", (4, 16), [6], True, 7) in got
         assert ("t#r1234567890", (2, 8), [4], True, None) in got
     # row blocks that do not stack are refused, as by the reference grouping
+    lone = [("a#r0", 1, (16,))] + [("p%d" % i, 1, (4,)) for i in range(40)]  # no two joined, numpy branch
     for bad in ([("a#r0", 1, (2, 8)), ("a#r1", 1, (2, 9))], [("a#r0", 1, (2, 8)), ("a#r1", 2, (2, 8))],
-                [("a#r0", 1, (2, 8)), ("a#r1", 1, (16,))]):
+                [("a#r0", 1, (2, 8)), ("a#r1", 1, (16,))], [("a#r0", 1, (16,))], lone,
+                lone + [("a#r1", 1, (2, 8))]):
         p = str(tmp_path / "bad.wt")
         write_entries(p, bad)
         with wt.Handle([p], wt.WT_OPEN_HOST_ONLY) as h:
