@@ -735,13 +735,14 @@ Populator &populator() {
 }
 
 int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cudaStream_t s,
-                 void **ready, uint64_t total) {
-  // Batches of a 64th of the call, kept between 64 and 128 MiB: each batch is one gather
-  // launch and one event, and a gather kernel's ramp and tail idle part of the link.  Callers
-  // that allocate segment by segment make several smaller calls; with a 2 MiB floor their
-  // 16 GB first use ran 230 batches at 203 GB/s instead of 80 at 207 (mid decoder, allocation
-  // inside the run: 188 -> 194 GB/s with the 64 MiB floor; buffers reused: unchanged).
-  const uint64_t target = std::min<uint64_t>(128ull << 20, std::max<uint64_t>(64ull << 20, total / 64));
+                 void **ready) {
+  // Batches of 128 MiB: each batch is one gather launch and one event, and a gather kernel's
+  // ramp and tail idle part of the link (a 64 MiB batch ran at a median 204 GB/s of the
+  // link's 210).  Callers that allocate segment by segment make several smaller calls, which
+  // keep full batches too.  Measured with the allocation inside the run: batches of at least
+  // 2 MiB -> 64 MiB took the mid decoder from 188 to 194 GB/s, and 64 -> 128 MiB the large
+  // decoder from 197.9 to 198.6 and the mid decoder from 195.5 to 196.8 GB/s.
+  const uint64_t target = 128ull << 20;
   // When the stream has nothing in flight the link is idle until the first batch lands, and
   // that batch waits for its own page tables first: batches then start at 4 MiB and double up
   // to the target, so the first launch follows the population of 4 MiB instead of 64.  A call
@@ -1081,7 +1082,7 @@ int adopt_staged(wt_handle *h, const std::vector<Range> &rs, cudaStream_t s, voi
 // for whatever the staged half enqueued, on success and on failure alike, so the call keeps
 // its stream semantics (later work on `s` never overlaps a copy of this call).
 int adopt_mixed(wt_handle *h, const std::vector<Range> &dv, const std::vector<Range> &st, unsigned mode,
-                cudaStream_t s, void **ready, uint64_t total_dev) {
+                cudaStream_t s, void **ready) {
   StagedJoin join;
   int rc = new_event(h, &join.after);
   if (rc) return rc;
@@ -1099,7 +1100,7 @@ int adopt_mixed(wt_handle *h, const std::vector<Range> &dv, const std::vector<Ra
     rc_st = e == cudaSuccess ? adopt_staged(h, st, s, ready, &join) : cuda_err(e, "cudaSetDevice");
     if (rc_st) err_st = t_err;
   });
-  rc = adopt_device(h, dv, mode, s, ready, total_dev);
+  rc = adopt_device(h, dv, mode, s, ready);
   helper.t.join();
   // The ring's stream is created once and never replaced, so it can be read here without
   // the ring's lock; an event on it now follows every copy the staged half enqueued (and
@@ -2267,7 +2268,6 @@ int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsign
   try {
     std::vector<Range> rs, st;  // st: small unmapped files of a MAP_LARGE handle (GATHER / CE)
     rs.reserve(n);
-    uint64_t total = 0;
     RangeCache rc_dst;
     for (size_t k = 0; k < n; ++k) {
       if (idx[k] >= h->order.size()) return set_err(WT_EINVAL, "wt_adopt: tensor index %zu out of range", idx[k]);
@@ -2289,14 +2289,13 @@ int wt_adopt(wt_handle *h, const size_t *idx, void *const *dst, size_t n, unsign
         st.push_back(r);
       } else {
         rs.push_back(r);
-        total += t.nbytes;
       }
     }
     const cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (mode == WT_ADOPT_STAGED) return adopt_staged(h, rs, s, ready);
-    if (st.empty()) return adopt_device(h, rs, mode, s, ready, total);
+    if (st.empty()) return adopt_device(h, rs, mode, s, ready);
     if (rs.empty()) return adopt_staged(h, st, s, ready);
-    return adopt_mixed(h, rs, st, mode, s, ready, total);
+    return adopt_mixed(h, rs, st, mode, s, ready);
   } catch (const std::bad_alloc &) {
     return set_err(WT_ENOMEM, "wt_adopt: out of host memory");
   }
