@@ -1,11 +1,19 @@
 """File -> first use, on top of the C ABI (torch supplies device memory and streams only).
 
     h = wt.Handle(paths)                       # wt_open: parse, map, route
-    mats = matrices(h)                         # 2-D tensors, row blocks joined
+    mats = matrices(h)                         # logical tensors as columns, row blocks joined
     dev = DeviceCheckpoint.allocate(h, mats)   # one caller-owned buffer per matrix/vector
     events = dev.adopt(h, mode, stream)        # wt_adopt: per-tensor ready events
     xs, ys = dev.inputs(), dev.outputs()       # x per inner size K, fp32 y per matrix
     h.pass_(dev.descs(xs, ys, events), stream) # wt_pass: each GEMV waits on its bytes only
+
+The timed first use allocates while it ingests, with the step's inputs and outputs in the
+first slab:
+
+    x_host = host_inputs(mats)                                  # every x, pinned, once
+    dev, events, _ = DeviceCheckpoint.stream_in(h, mats, mode, ingest, io=True)
+    dev.io_x().copy_(x_host, non_blocking=True)                 # on the consumer stream
+    h.pass_(dev.descs(dev.io_inputs(), dev.io_outputs(), events), consumer)
 
 Row blocks: a tensor named "<name>#r<k>" is row block k of matrix <name> (the
 many-small workload splits each matrix's rows across two files); its blocks are
