@@ -153,3 +153,57 @@ def test_descs_and_addresses_follow_the_adoption_order(tmp_path):
             # the same events as a plain mapping give the same waits
             d2 = dc.descs(xs, ys, dict(ev.items()))
             assert np.array_equal(d["wait_event"], d2["wait_event"])
+
+
+def test_random_checkpoints_group_like_the_reference(tmp_path):
+    """Random multi-file checkpoints (row blocks spread over files in any order, plain 1-D and
+    2-D tensors, int8 matrices with and without row scales, names that only look like
+    blocks): the columnar grouping, the io layout and the buffer offsets equal the plain-Python
+    reference's, on both branches (up to 32 tensors and above)."""
+    build.build()
+    rng = np.random.default_rng(21)
+    for trial in range(24):
+        specs = []  # (name, dtype, shape)
+        for m in range(int(rng.integers(1, 30))):
+            kind = rng.integers(0, 5)
+            K = int(rng.choice([8, 16, 64, 256]))
+            dt = int(rng.choice([0, 1, 2]))
+            if kind == 0:    # a matrix split into row blocks
+                nb = int(rng.integers(1, 4))
+                for b in rng.permutation(nb).tolist():
+                    specs.append(("m%d#r%d" % (m, b), dt, (int(rng.integers(1, 5)), K)))
+            elif kind == 1:  # a plain 2-D matrix
+                specs.append(("p%d" % m, dt, (int(rng.integers(1, 6)), K)))
+            elif kind == 2:  # a vector, or a name that only looks like a block
+                specs.append(("v%d#r%s" % (m, rng.choice(["x", "", "1234567890"])), dt, (K,)))
+            elif kind == 3:  # int8 with fp16 row scales
+                M = int(rng.integers(1, 6))
+                specs.append(("q%d" % m, 3, (M, K)))
+                specs.append(("q%d.scale" % m, 2, (M,)))
+            else:            # int8 without scales, and scales of the wrong length
+                specs.append(("r%d" % m, 3, (3, K)))
+                specs.append(("r%d.scale" % m, 2, (2,)))
+        order = rng.permutation(len(specs)).tolist()
+        nf = int(rng.integers(1, 4))
+        files = [[] for _ in range(nf)]
+        for j, i in enumerate(order):
+            files[j % nf].append(specs[i])
+        paths = []
+        for f, fs in enumerate(files):
+            if fs:
+                p = str(tmp_path / ("t%d_%d.wt" % (trial, f)))
+                write_entries(p, fs)
+                paths.append(p)
+        with wt.Handle(paths, wt.WT_OPEN_HOST_ONLY) as h:
+            m, ref = pipeline.matrices(h), pipeline._matrices_list(h)
+            got = [(r.name, r.dtype, tuple(r.shape), r.parts, r.gemv, r.scale) for r in m]
+            assert got == [(r.name, r.dtype, tuple(r.shape), r.parts, r.gemv, r.scale) for r in ref], trial
+            assert pipeline.io_layout(m) == pipeline.io_layout(ref), trial
+            dc = pipeline.DeviceCheckpoint._new(h, m, None)
+            dc.ptrs[:] = (1 << 40) + np.arange(len(m), dtype=np.uint64) * (1 << 20)
+            dc._set_dst(h)
+            for k, r in enumerate(ref):
+                off = 0
+                for i in r.parts:
+                    assert dc.dst[i] == (1 << 40) + k * (1 << 20) + off
+                    off += h.tensors.nbytes[i]
