@@ -736,13 +736,15 @@ Populator &populator() {
 
 int adopt_device(wt_handle *h, const std::vector<Range> &rs, unsigned mode, cudaStream_t s,
                  void **ready) {
-  // Batches of 128 MiB: each batch is one gather launch and one event, and a gather kernel's
+  // Batches of 256 MiB: each batch is one gather launch and one event, and a gather kernel's
   // ramp and tail idle part of the link (a 64 MiB batch ran at a median 204 GB/s of the
-  // link's 210).  Callers that allocate segment by segment make several smaller calls, which
-  // keep full batches too.  Measured with the allocation inside the run: batches of at least
-  // 2 MiB -> 64 MiB took the mid decoder from 188 to 194 GB/s, and 64 -> 128 MiB the large
-  // decoder from 197.9 to 198.6 and the mid decoder from 195.5 to 196.8 GB/s.
-  const uint64_t target = 128ull << 20;
+  // link's 210, a 128 MiB one at 207).  Callers that allocate segment by segment make several
+  // smaller calls, which keep full batches too.  Measured with the allocation inside the run:
+  // batches of at least 2 MiB -> 64 MiB took the mid decoder from 188 to 194 GB/s; 64 -> 128
+  // MiB the large decoder from 197.9 to 198.6 and the mid decoder from 195.5 to 196.8 GB/s;
+  // 128 -> 256 MiB the large decoder from 198.3 to 199.9 and the mid from 196.6 to 197.9 GB/s,
+  // with many-small unchanged.
+  const uint64_t target = 256ull << 20;
   // When the stream has nothing in flight the link is idle until the first batch lands, and
   // that batch waits for its own page tables first: batches then start at 4 MiB and double up
   // to the target, so the first launch follows the population of 4 MiB instead of 64.  A call
